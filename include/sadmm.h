@@ -1,0 +1,200 @@
+/*
+ * sadmm.h -- C ABI of libsadmm: the forward pass of a CONV layer whose weights
+ * are structurally pruned (StructADMM, arXiv 1807.11091), on one sm_103a GPU.
+ *
+ * Three calls make up the path, in the paper's order:
+ *
+ *   sadmm_project_groups  Euclidean projection of V = W (+U) onto a structured
+ *                         sparsity set: squared Frobenius norm of every group,
+ *                         then the k largest (Sec. 4, the Z-subproblem, Eq. 4,
+ *                         and its filter-, channel- and shape-wise solutions).
+ *   sadmm_pack            Compacts the kept rows (filters) and columns
+ *                         ((channel, kt, kh, kw) taps) of the lowered GEMM
+ *                         matrix into a dense bf16 matrix plus a gather table
+ *                         (Sec. 3, "Combination of structured sparsities":
+ *                         filter-wise = row pruning, channel-/shape-wise =
+ *                         column pruning; the result is a smaller full matrix).
+ *   sadmm_conv_fwd        Implicit GEMM over only the kept rows and columns,
+ *                         bias + ReLU fused, written to the full NCHW / NCDHW
+ *                         output with every pruned filter's plane set to zero.
+ *
+ * Conventions for every call:
+ *  - All tensor pointers are DEVICE pointers owned by the caller.  The library
+ *    never allocates device memory and never synchronises the stream, except
+ *    sadmm_last_device_status, which synchronises to read the device flag.
+ *  - `stream` is a cudaStream_t (NULL = legacy default stream).  All work is
+ *    enqueued on it, in order, asynchronously.
+ *  - Arguments are validated on the host before any launch; a bad argument
+ *    returns SADMM_EINVAL and enqueues nothing.  A failed launch returns
+ *    SADMM_ECUDA.  Shapes the kernels do not support (see each call) return
+ *    SADMM_EUNSUPPORTED.  There is no CPU fallback.
+ *  - Layouts are dense row-major (C order): W is [F][Cg][KT][KH][KW]
+ *    (OIDHW, KT = 1 for 2-D, Cg = C / groups), x is [N][C][T][H][W], y is
+ *    [N][F][OT][OH][OW].  Dilation is 1.
+ */
+#ifndef SADMM_H
+#define SADMM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SADMM_ABI_VERSION 1
+
+typedef enum {
+    SADMM_OK = 0,
+    SADMM_EINVAL = -1,       /* bad argument, shape or buffer size          */
+    SADMM_ECUDA = -2,        /* a CUDA runtime call or launch failed        */
+    SADMM_ETIMEOUT = -3,     /* a device-side wait ran past its limit       */
+    SADMM_EUNSUPPORTED = -4  /* valid request outside what the kernels do   */
+} sadmm_status;
+
+typedef enum { SADMM_BF16 = 0, SADMM_FP32 = 1 } sadmm_dtype;
+
+/* Column (GEMM-column) pruning kind.  Filter (row) pruning is always
+ * available through k_filters / n_filt and combines with any of these. */
+typedef enum {
+    SADMM_COL_NONE = 0,    /* keep every column                                  */
+    SADMM_COL_SHAPE = 1,   /* shape-wise: groups are single (c,kt,kh,kw) columns */
+    SADMM_COL_CHANNEL = 2  /* channel-wise: groups are whole channels c          */
+} sadmm_colkind;
+
+/* A CONV layer.  t = kt = st = 1 and pt = 0 for 2-D layers. */
+typedef struct {
+    int n, c, t, h, w;   /* input: batch, channels, depth, height, width */
+    int f, groups;       /* filters (output channels), conv groups       */
+    int kt, kh, kw;      /* kernel extent                                */
+    int st, sh, sw;      /* strides                                      */
+    int pt, ph, pw;      /* zero padding on each side                    */
+} sadmm_conv_desc;
+
+/* Execution plan of one pruned layer.  Filled on the host by sadmm_plan_init
+ * (sizes) and sadmm_pack (device buffer, TMA descriptor); read-only after.
+ * The device buffer `dev` is caller-owned and must stay alive while any
+ * sadmm_conv_fwd that uses the plan is in flight.  The struct itself is plain
+ * host memory and may be copied. */
+typedef struct {
+    sadmm_conv_desc desc;
+    int n_filt;       /* F': kept filters over all conv groups                */
+    int colkind;      /* sadmm_colkind                                        */
+    int n_colgroups;  /* kept column groups (columns, or channels)           */
+    int n_cols;       /* K': kept GEMM columns (channels x taps if channel)  */
+    int k_pad;        /* K' rounded up to a multiple of 64 (at least 64)     */
+    int bn;           /* filter rows per tile: multiple of 16, at most 256    */
+    int n_tiles;      /* filter tiles per conv group                          */
+    int n_pad;        /* rows per conv group in the packed matrix = bn*n_tiles */
+    size_t dev_bytes; /* device bytes the plan needs (see sadmm_plan_init)    */
+    void* dev;        /* device buffer bound by sadmm_pack                    */
+    size_t off_wp, off_gather, off_rowmap, off_zeromap, off_counts, off_colidx;
+    uint64_t tmap[16];/* 128-byte TMA tensor map of the packed matrix         */
+} sadmm_plan;
+
+/* ------------------------------------------------------------------------ */
+
+/* Library ABI version (SADMM_ABI_VERSION) and sizeof(sadmm_plan), so that
+ * bindings can check their mirror of the struct. */
+int sadmm_abi_version(void);
+size_t sadmm_plan_struct_size(void);
+
+/* Human-readable name of a status code (static string). */
+const char* sadmm_status_string(int status);
+
+/* Device bytes of scratch sadmm_project_groups needs for this layer and
+ * column kind (keys, counters).  0 on a bad descriptor. */
+size_t sadmm_workspace_size(const sadmm_conv_desc* d, int colkind);
+
+/*
+ * Euclidean projection onto the structured-sparsity set (Sec. 4, Eq. 4):
+ * V = W (+U when U != NULL, the scaled ADMM dual; Sec. 4 projects W + U),
+ * squared Frobenius norm O_g of every group, keep the k largest.
+ *
+ *   W, U       device, dtype `wdt` (bf16 or fp32), layout OIDHW ([F][K] as a
+ *              GEMM matrix, K = Cg*KT*KH*KW).  U may be NULL.
+ *   k_filters  filters to keep, 0..F (F = no filter pruning).
+ *   colkind    SADMM_COL_NONE / SHAPE / CHANNEL.
+ *   k_cols     column groups to keep: 0..K (shape) or 0..Cg (channel); ignored
+ *              for SADMM_COL_NONE.
+ *   filt_idx   device int32 [k_filters]: kept filters, ascending.
+ *   col_idx    device int32 [k_cols]: kept columns (shape) or channels
+ *              (channel), ascending.  May be NULL for SADMM_COL_NONE.
+ *   keys_out   optional device fp64 [F + G]: filter keys, then column-group
+ *              keys (G = K or Cg; 0 for SADMM_COL_NONE).
+ *   workspace  device scratch of at least sadmm_workspace_size() bytes.
+ *
+ * Combined row and column pruning: filters are chosen first on the full
+ * tensor, then column keys are summed over the kept filters only.  Equal keys
+ * go to the lower group index.  Keys are fp64 sums of exact fp64 squares;
+ * the order of equal-key groups is resolved by index, so the index lists are
+ * deterministic.  Grouped convs: a filter group is one filter among all F; a
+ * column group spans all F filters (the same column set serves every conv
+ * group).
+ */
+sadmm_status sadmm_project_groups(const sadmm_conv_desc* d, const void* W, const void* U,
+                                  int wdt, int k_filters, int colkind, int k_cols,
+                                  int* filt_idx, int* col_idx, double* keys_out,
+                                  void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * Sizes a plan for `n_filt` kept filters and `n_colgroups` kept column groups
+ * (columns or channels) of kind `colkind`.  Fills every size field of `plan`,
+ * including plan->dev_bytes, the device buffer sadmm_pack needs.  Host only;
+ * enqueues nothing.  SADMM_EUNSUPPORTED when the packed row count per conv
+ * group would exceed 4096 or K' would exceed 65536.
+ */
+sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d,
+                             int n_filt, int colkind, int n_colgroups);
+
+/*
+ * Compacts the kept weights (Sec. 3, row/column pruning of the GEMM matrix):
+ *   Wp[g][i][j] = bf16(W[f_i][col_j]) for the i-th kept filter f_i of conv
+ *   group g and the j-th kept column, zero beyond the kept counts;
+ *   a gather table entry per kept column (its channel offset in x and its
+ *   (kt,kh,kw) tap); per conv group the list of kept and of pruned filters.
+ *
+ *   filt_idx  device int32 [plan->n_filt], ascending, in [0,F); NULL when
+ *             n_filt == F (all filters).
+ *   col_idx   device int32 [plan->n_colgroups], ascending: columns in [0,K)
+ *             (shape) or channels in [0,Cg) (channel); NULL for COL_NONE.
+ *   dev       device buffer of >= plan->dev_bytes bytes, 1024-byte aligned;
+ *             becomes plan->dev.
+ * Writes the TMA descriptor of Wp into plan->tmap.  Index lists that are not
+ * ascending or out of range give undefined (but in-bounds) plans.
+ */
+sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt,
+                        const int* filt_idx, const int* col_idx,
+                        void* dev, size_t dev_bytes, void* stream);
+
+/*
+ * Pruned CONV forward (Sec. 3: the pruned layer is a smaller full GEMM):
+ *   y[n, f, o] = ReLU(bias[f] + sum_{j < K'} Wp[f][j] * x[n, g*Cg + c_j,
+ *                ot*st-pt+kt_j, oh*sh-ph+kh_j, ow*sw-pw+kw_j])   f kept,
+ *   y[n, f, o] = 0                                                f pruned,
+ * x outside the input reads as zero.  bf16 x bf16 products accumulate in fp32
+ * (tcgen05 MMA, TMEM accumulator).
+ *
+ *   x     device bf16 [N][C][T][H][W]; 16-byte aligned.
+ *   bias  device fp32 [F] or NULL (zero).
+ *   relu  nonzero: apply ReLU.
+ *   y     device [N][F][OT][OH][OW] of dtype `ydt` (fp32 or bf16, rounded
+ *         to nearest even); every element is written.
+ * Requires sm_100-family tensor cores (SADMM_EUNSUPPORTED otherwise) and
+ * N*C*T*H*W < 2^31.
+ */
+sadmm_status sadmm_conv_fwd(const sadmm_plan* plan, const void* x, const float* bias,
+                            int relu, void* y, int ydt, void* stream);
+
+/*
+ * Synchronises `stream`, then reports and clears the device status word that
+ * the kernels set when a bounded wait expires (SADMM_ETIMEOUT) or a
+ * device-side check fails (SADMM_EINVAL).  SADMM_OK when clear.
+ */
+sadmm_status sadmm_last_device_status(void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SADMM_H */

@@ -1,0 +1,248 @@
+// abi.cu -- the extern "C" entry points of libsadmm: host-side validation,
+// plan sizing and the device status word.  Every entry point checks its
+// arguments before enqueuing anything and never synchronises, except
+// sadmm_last_device_status.
+#include <string.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace sadmm {
+
+__device__ int g_status_word;
+
+namespace {
+constexpr int kMaxDevices = 64;
+int* g_status_ptr[kMaxDevices];
+int g_sm_count[kMaxDevices];
+int g_cc_major[kMaxDevices];
+
+int current_device()
+{
+    int d = 0;
+    if (cudaGetDevice(&d) != cudaSuccess || d < 0 || d >= kMaxDevices) return 0;
+    return d;
+}
+}  // namespace
+
+int* device_status_ptr()
+{
+    const int d = current_device();
+    if (!g_status_ptr[d]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_status_word) == cudaSuccess) g_status_ptr[d] = static_cast<int*>(p);
+    }
+    return g_status_ptr[d];
+}
+
+int device_sm_count()
+{
+    const int d = current_device();
+    if (!g_sm_count[d]) {
+        int v = 0;
+        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, d);
+        g_sm_count[d] = v > 0 ? v : 1;
+    }
+    return g_sm_count[d];
+}
+
+int device_cc_major()
+{
+    const int d = current_device();
+    if (!g_cc_major[d]) {
+        int v = 0;
+        cudaDeviceGetAttribute(&v, cudaDevAttrComputeCapabilityMajor, d);
+        g_cc_major[d] = v;
+    }
+    return g_cc_major[d];
+}
+
+sadmm_status check_desc(const sadmm_conv_desc* d, Geometry* g)
+{
+    if (!d || !g) return SADMM_EINVAL;
+    const long long v[16] = {d->n,  d->c,  d->t,  d->h,  d->w,  d->f,  d->groups, d->kt,
+                             d->kh, d->kw, d->st, d->sh, d->sw, d->pt, d->ph,     d->pw};
+    for (int i = 0; i < 13; ++i)
+        if (v[i] < 1) return SADMM_EINVAL;
+    for (int i = 13; i < 16; ++i)
+        if (v[i] < 0) return SADMM_EINVAL;
+    Geometry r;
+    r.n = d->n; r.c = d->c; r.t = d->t; r.h = d->h; r.w = d->w; r.f = d->f; r.groups = d->groups;
+    r.kt = d->kt; r.kh = d->kh; r.kw = d->kw; r.st = d->st; r.sh = d->sh; r.sw = d->sw;
+    r.pt = d->pt; r.ph = d->ph; r.pw = d->pw;
+    if (r.c % r.groups != 0 || r.f % r.groups != 0) return SADMM_EINVAL;
+    r.cg = r.c / r.groups;
+    r.fg = r.f / r.groups;
+    r.taps = r.kt * r.kh * r.kw;
+    r.k = r.cg * r.taps;
+    if (r.t + 2 * r.pt < r.kt || r.h + 2 * r.ph < r.kh || r.w + 2 * r.pw < r.kw) return SADMM_EINVAL;
+    r.ot = (r.t + 2 * r.pt - r.kt) / r.st + 1;
+    r.oh = (r.h + 2 * r.ph - r.kh) / r.sh + 1;
+    r.ow = (r.w + 2 * r.pw - r.kw) / r.sw + 1;
+    r.plane = r.ot * r.oh * r.ow;
+    r.m = r.n * r.plane;
+    // index arithmetic limits of the kernels (32-bit offsets inside a tensor)
+    if (r.n * r.c * r.t * r.h * r.w >= (1ll << 31)) return SADMM_EUNSUPPORTED;
+    if (r.f * r.k >= (1ll << 31) || r.plane >= (1ll << 31) || r.m >= (1ll << 40)) return SADMM_EUNSUPPORTED;
+    if (r.kt * r.kh > 32 || r.kw > 32) return SADMM_EUNSUPPORTED;
+    if (r.groups > 64) return SADMM_EUNSUPPORTED;
+    *g = r;
+    return SADMM_OK;
+}
+
+}  // namespace sadmm
+
+using namespace sadmm;
+
+extern "C" {
+
+int sadmm_abi_version(void) { return SADMM_ABI_VERSION; }
+
+size_t sadmm_plan_struct_size(void) { return sizeof(sadmm_plan); }
+
+const char* sadmm_status_string(int status)
+{
+    switch (status) {
+    case SADMM_OK: return "ok";
+    case SADMM_EINVAL: return "invalid argument";
+    case SADMM_ECUDA: return "CUDA error";
+    case SADMM_ETIMEOUT: return "device wait timed out";
+    case SADMM_EUNSUPPORTED: return "unsupported";
+    default: return "unknown status";
+    }
+}
+
+size_t sadmm_workspace_size(const sadmm_conv_desc* d, int colkind)
+{
+    Geometry g;
+    if (check_desc(d, &g) != SADMM_OK) return 0;
+    return project_workspace_bytes(g, colkind);
+}
+
+sadmm_status sadmm_project_groups(const sadmm_conv_desc* d, const void* W, const void* U, int wdt,
+                                  int k_filters, int colkind, int k_cols, int* filt_idx, int* col_idx,
+                                  double* keys_out, void* workspace, size_t ws_bytes, void* stream)
+{
+    Geometry g;
+    sadmm_status st = check_desc(d, &g);
+    if (st != SADMM_OK) return st;
+    if (!W || !filt_idx || !workspace) return SADMM_EINVAL;
+    if (wdt != SADMM_BF16 && wdt != SADMM_FP32) return SADMM_EINVAL;
+    if (colkind != SADMM_COL_NONE && colkind != SADMM_COL_SHAPE && colkind != SADMM_COL_CHANNEL)
+        return SADMM_EINVAL;
+    if (k_filters < 0 || k_filters > g.f) return SADMM_EINVAL;
+    if (colkind != SADMM_COL_NONE) {
+        const long long G = (colkind == SADMM_COL_SHAPE) ? g.k : g.cg;
+        if (k_cols < 0 || k_cols > G || !col_idx) return SADMM_EINVAL;
+    }
+    if (ws_bytes < project_workspace_bytes(g, colkind)) return SADMM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 7) != 0) return SADMM_EINVAL;
+    if (keys_out && (reinterpret_cast<uintptr_t>(keys_out) & 7) != 0) return SADMM_EINVAL;
+    return launch_project(g, W, U, wdt, k_filters, colkind, k_cols, filt_idx, col_idx, keys_out, workspace,
+                          static_cast<cudaStream_t>(stream));
+}
+
+sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d, int n_filt, int colkind,
+                             int n_colgroups)
+{
+    if (!plan) return SADMM_EINVAL;
+    Geometry g;
+    sadmm_status st = check_desc(d, &g);
+    if (st != SADMM_OK) return st;
+    if (n_filt < 0 || n_filt > g.f) return SADMM_EINVAL;
+    long long n_cols;
+    if (colkind == SADMM_COL_SHAPE) {
+        if (n_colgroups < 0 || n_colgroups > g.k) return SADMM_EINVAL;
+        n_cols = n_colgroups;
+    } else if (colkind == SADMM_COL_CHANNEL) {
+        if (n_colgroups < 0 || n_colgroups > g.cg) return SADMM_EINVAL;
+        n_cols = (long long)n_colgroups * g.taps;
+    } else if (colkind == SADMM_COL_NONE) {
+        n_colgroups = (int)g.k;
+        n_cols = g.k;
+    } else {
+        return SADMM_EINVAL;
+    }
+    if (n_cols > 65536) return SADMM_EUNSUPPORTED;
+    sadmm_plan p;
+    memset(&p, 0, sizeof(p));
+    p.desc = *d;
+    p.n_filt = n_filt;
+    p.colkind = colkind;
+    p.n_colgroups = n_colgroups;
+    p.n_cols = (int)n_cols;
+    p.k_pad = (int)(n_cols < 64 ? 64 : round_up(n_cols, 64));
+    // rows of the packed matrix per conv group: the most kept filters any group
+    // can have, in tiles of at most 256 rows (multiples of 16)
+    long long rmax = n_filt < g.fg ? n_filt : g.fg;
+    if (rmax < 16) rmax = 16;
+    rmax = round_up(rmax, 16);
+    p.n_tiles = (int)((rmax + 255) / 256);
+    p.bn = (int)round_up((rmax + p.n_tiles - 1) / p.n_tiles, 16);
+    p.n_pad = p.bn * p.n_tiles;
+    if (p.n_pad > 4096) return SADMM_EUNSUPPORTED;
+    size_t off = 0;
+    auto take = [&off](size_t bytes) {
+        const size_t at = off;
+        off += (size_t)round_up((long long)bytes, 1024);
+        return at;
+    };
+    p.off_wp = take((size_t)g.groups * p.n_pad * p.k_pad * 2);
+    p.off_gather = take((size_t)p.k_pad * 16);
+    p.off_colidx = take((size_t)p.k_pad * 4);
+    p.off_rowmap = take((size_t)g.groups * p.n_pad * 4);
+    p.off_zeromap = take((size_t)g.f * 4);
+    p.off_counts = take((size_t)g.groups * 2 * 4);
+    p.dev_bytes = off;
+    p.dev = nullptr;
+    *plan = p;
+    return SADMM_OK;
+}
+
+sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt, const int* filt_idx, const int* col_idx,
+                        void* dev, size_t dev_bytes, void* stream)
+{
+    if (!plan || !W || !dev) return SADMM_EINVAL;
+    Geometry g;
+    sadmm_status st = check_desc(&plan->desc, &g);
+    if (st != SADMM_OK) return st;
+    if (wdt != SADMM_BF16 && wdt != SADMM_FP32) return SADMM_EINVAL;
+    if (dev_bytes < plan->dev_bytes) return SADMM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(dev) & 255) != 0) return SADMM_EINVAL;
+    if (plan->n_filt < (int)g.f && plan->n_filt > 0 && !filt_idx) return SADMM_EINVAL;
+    if (plan->colkind != SADMM_COL_NONE && plan->n_colgroups > 0 && !col_idx) return SADMM_EINVAL;
+    if (device_cc_major() < 10) return SADMM_EUNSUPPORTED;
+    plan->dev = dev;
+    return launch_pack(plan, g, W, wdt, filt_idx, col_idx, static_cast<cudaStream_t>(stream));
+}
+
+sadmm_status sadmm_conv_fwd(const sadmm_plan* plan, const void* x, const float* bias, int relu, void* y,
+                            int ydt, void* stream)
+{
+    if (!plan || !x || !y || !plan->dev) return SADMM_EINVAL;
+    Geometry g;
+    sadmm_status st = check_desc(&plan->desc, &g);
+    if (st != SADMM_OK) return st;
+    if (ydt != SADMM_BF16 && ydt != SADMM_FP32) return SADMM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(x) & 1) != 0) return SADMM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(y) & (ydt == SADMM_FP32 ? 3 : 1)) != 0) return SADMM_EINVAL;
+    if (bias && (reinterpret_cast<uintptr_t>(bias) & 3) != 0) return SADMM_EINVAL;
+    if (device_cc_major() < 10) return SADMM_EUNSUPPORTED;
+    return launch_conv_fwd(plan, g, x, bias, relu, y, ydt, static_cast<cudaStream_t>(stream));
+}
+
+sadmm_status sadmm_last_device_status(void* stream)
+{
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return SADMM_ECUDA;
+    int v = 0;
+    if (cudaMemcpyFromSymbol(&v, g_status_word, sizeof(int)) != cudaSuccess) return SADMM_ECUDA;
+    if (v != 0) {
+        const int zero = 0;
+        cudaMemcpyToSymbol(g_status_word, &zero, sizeof(int));
+    }
+    if (v == kDevTimeout) return SADMM_ETIMEOUT;
+    if (v != 0) return SADMM_EINVAL;
+    return SADMM_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,455 @@
+// conv_fwd.cu -- pruned CONV forward as an implicit GEMM on the sm_103a tensor
+// cores (Sec. 3: after filter-wise (row) and channel-/shape-wise (column)
+// pruning the layer is a smaller full GEMM).
+//
+//   D[m, i] = sum_{j < K'} A[m, j] * Wp[i, j]
+//   A[m, j] = x[n, g*Cg + c_j, ot*st-pt+kt_j, oh*sh-ph+kh_j, ow*sw-pw+kw_j]
+//
+// m runs over output pixels (N*OT*OH*OW), i over the kept filters of conv group
+// g, j over the kept (channel, tap) columns.  Pixels are the MMA M side (128 per
+// tile, one TMEM lane each), kept filters the N side (bn <= 256 per tile), so a
+// gathered pixel tile is reused by every kept filter of the tile.
+//
+// One persistent CTA per SM, warp-specialised (512 threads):
+//   warp 0      TMA producer: 64-column x bn-row boxes of Wp (128-byte swizzle)
+//   warp 1      TMEM allocator and MMA issuer (tcgen05.mma kind::f16, bf16 in,
+//               fp32 accumulate, 128 x n x 16 per instruction)
+//   warps 4-7   epilogue: tcgen05.ld of the accumulator (lane = pixel), bias,
+//               ReLU, coalesced stores to the NCHW output (consecutive lanes
+//               write consecutive pixels of one filter plane), and zero-fill of
+//               the pruned filters' planes for the tile's pixels
+//   warps 8-15  gather: each thread owns one pixel of the tile and builds 16-byte
+//               K-major chunks of A through the gather table, with zero fill
+//               outside the input, into the 128-byte-swizzled stage buffer
+// Shared-memory stages are guarded by mbarriers; the accumulator is double
+// buffered in TMEM so the epilogue of one tile overlaps the MMAs of the next.
+#include <cuda.h>
+#include <string.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace sadmm {
+namespace {
+
+constexpr int kBM = 128;           // pixels per tile
+constexpr int kBK = 64;            // GEMM columns per stage
+constexpr int kGatherWarps = 8;
+constexpr int kEpiWarps = 4;
+constexpr int kThreads = (4 + kEpiWarps + kGatherWarps) * 32;
+constexpr int kGatherThreads = kGatherWarps * 32;
+constexpr int kATileBytes = kBM * kBK * 2;  // 16 KB
+constexpr int kMaxStages = 8;
+constexpr int kMaxGroups = 64;
+constexpr int kSmemTail = 2048;  // barriers, TMEM address, counts
+
+struct ConvArgs {
+    const __nv_bfloat16* x;
+    void* y;
+    const float* bias;
+    const int4* gather;
+    const int* rowmap;
+    const int* zeromap;
+    const int* counts;
+    int* status;
+    long long M;      // N * plane
+    long long x_chw;  // elements per input image
+    long long thw;    // elements per input channel
+    long long units;  // m_tiles * groups * n_tiles
+    int hw, W, H, T;
+    int F, groups, Cg, Fg;
+    int OW, OHW, plane;
+    int st, sh, sw, pt, ph, pw;
+    int KT, KH, KW;
+    int nks;  // k_pad / 64
+    int bn, n_tiles, n_pad;
+    int stages;
+    int tmem_stride;
+    int tmem_cols;
+    int relu;
+};
+
+SADMM_DEV void decode_unit(const ConvArgs& a, long long u, int& nt, int& g, long long& mt)
+{
+    nt = (int)(u % a.n_tiles);
+    const long long t = u / a.n_tiles;
+    g = (int)(t % a.groups);
+    mt = t / a.groups;
+}
+
+// Tap-validity masks of one output pixel: bit set where the tap reads inside
+// the input.  MODE 0: bit (kt*KH + kh)*KW + kw.  MODE 1: rmask bit kt*KH + kh,
+// cmask bit kw.
+template <int MODE>
+SADMM_DEV void pixel_masks(const ConvArgs& a, int it0, int ih0, int iw0, uint32_t& m0, uint32_t& m1)
+{
+    uint32_t rm = 0, cm = 0;
+    for (int kt = 0; kt < a.KT; ++kt) {
+        const bool vt = (unsigned)(it0 + kt) < (unsigned)a.T;
+        for (int kh = 0; kh < a.KH; ++kh)
+            if (vt && (unsigned)(ih0 + kh) < (unsigned)a.H) rm |= 1u << (kt * a.KH + kh);
+    }
+    for (int kw = 0; kw < a.KW; ++kw)
+        if ((unsigned)(iw0 + kw) < (unsigned)a.W) cm |= 1u << kw;
+    if (MODE == 0) {
+        uint32_t m = 0;
+        for (int r = 0; r < a.KT * a.KH; ++r)
+            if (rm & (1u << r)) m |= cm << (r * a.KW);
+        m0 = m;
+        m1 = 0;
+    } else {
+        m0 = rm;
+        m1 = cm;
+    }
+}
+
+template <int MODE>
+SADMM_DEV bool tap_ok(const int4& e, uint32_t m0, uint32_t m1)
+{
+    if (MODE == 0) return (m0 & (uint32_t)e.y) != 0u;
+    return ((m0 & (uint32_t)e.y) != 0u) & ((m1 & (uint32_t)e.z) != 0u);
+}
+
+template <int MODE, bool OUT_BF16>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_conv_fwd(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ ConvArgs a)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int S = a.stages;
+    const uint32_t b_bytes = (uint32_t)a.bn * 128u;
+    uint8_t* sA = smem;
+    uint8_t* sB = smem + (size_t)S * kATileBytes;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sB + (size_t)S * b_bytes);
+    uint64_t* full_a = bars;
+    uint64_t* full_b = bars + S;
+    uint64_t* empty = bars + 2 * S;
+    uint64_t* acc_full = bars + 3 * S;
+    uint64_t* acc_empty = acc_full + 2;
+    uint64_t* drain = acc_empty + 2;
+    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+    int* s_counts = reinterpret_cast<int*>(tmem_holder + 2);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full_a[s], kGatherThreads);
+            mbar_init(&full_b[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], kEpiWarps * 32);
+        }
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    for (int i = threadIdx.x; i < 2 * a.groups; i += blockDim.x) s_counts[i] = a.counts[i];
+    if (warp == 0 && lane == 0) tma_prefetch_desc(&tmap);
+    if (warp == 1) {
+        tmem_alloc(tmem_holder, (uint32_t)a.tmem_cols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_holder;
+
+    if (warp == 0) {
+        // ------------------------------------------------ TMA producer (Wp)
+        if (lane == 0) {
+            int s = 0;
+            uint32_t ph = 0;
+            uint32_t issued_parity[kMaxStages];
+            uint32_t issued_mask = 0;
+            bool ok = true;
+            for (long long u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
+                int nt, g;
+                long long mt;
+                decode_unit(a, u, nt, g, mt);
+                if (s_counts[2 * g] <= nt * a.bn) continue;
+                const int row0 = g * a.n_pad + nt * a.bn;
+                for (int ks = 0; ks < a.nks; ++ks) {
+                    if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, a.status)) { ok = false; break; }
+                    mbar_arrive_expect_tx(&full_b[s], b_bytes);
+                    tma_load_2d(sB + (size_t)s * b_bytes, &tmap, &full_b[s], ks * kBK, row0);
+                    issued_parity[s] = ph;
+                    issued_mask |= 1u << s;
+                    if (++s == S) { s = 0; ph ^= 1u; }
+                }
+            }
+            // Every box this thread issued has landed before the CTA retires
+            // (normally already true: the MMA consumed them).
+            for (int q = 0; q < S; ++q) {
+                if (!(issued_mask & (1u << q))) continue;
+                const unsigned long long t0 = globaltimer();
+                while (!mbar_try_wait(&full_b[q], issued_parity[q]) && globaltimer() - t0 < kWaitLimitNs) {}
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            int s = 0;
+            uint32_t ph = 0;
+            int ab = 0;
+            uint32_t acc_ph = 0;
+            bool ok = true;
+            for (long long u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
+                int nt, g;
+                long long mt;
+                decode_unit(a, u, nt, g, mt);
+                const int cnt = s_counts[2 * g] - nt * a.bn;
+                if (cnt <= 0) continue;
+                const int n_rt = min(a.bn, (cnt + 15) & ~15);
+                const uint32_t idesc = idesc_bf16_f32(kBM, n_rt);
+                if (!mbar_wait(&acc_empty[ab], acc_ph ^ 1u, abort_flag, a.status)) break;
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + (uint32_t)(ab * a.tmem_stride);
+                for (int ks = 0; ks < a.nks; ++ks) {
+                    if (!mbar_wait(&full_a[s], ph, abort_flag, a.status) ||
+                        !mbar_wait(&full_b[s], ph, abort_flag, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a0 = smem_u32(sA + (size_t)s * kATileBytes);
+                    const uint32_t b0 = smem_u32(sB + (size_t)s * b_bytes);
+#pragma unroll
+                    for (int kk = 0; kk < kBK / 16; ++kk) {
+                        mma_bf16_ss(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32), sdesc_kmajor_sw128(b0 + kk * 32),
+                                    idesc, (ks | kk) != 0 ? 1u : 0u);
+                    }
+                    mma_commit(&empty[s]);
+                    if (++s == S) { s = 0; ph ^= 1u; }
+                }
+                if (!ok) break;
+                mma_commit(&acc_full[ab]);
+                ab ^= 1;
+                if (ab == 0) acc_ph ^= 1u;
+            }
+            // Every MMA this thread issued has completed before TMEM is freed.
+            mma_commit(drain);
+            const unsigned long long t0 = globaltimer();
+            while (!mbar_try_wait(drain, 0) && globaltimer() - t0 < kWaitLimitNs) {}
+        }
+        __syncwarp();
+    } else if (warp >= 4 && warp < 4 + kEpiWarps) {
+        // --------------------------------------------------------- epilogue
+        const int q = warp & 3;  // TMEM lane quadrant this warp may access
+        const int row = q * 32 + lane;
+        int ab = 0;
+        uint32_t acc_ph = 0;
+        for (long long u = blockIdx.x; u < a.units; u += gridDim.x) {
+            int nt, g;
+            long long mt;
+            decode_unit(a, u, nt, g, mt);
+            const int cnt = s_counts[2 * g] - nt * a.bn;
+            const long long m = mt * kBM + row;
+            const bool valid = m < a.M;
+            const long long n_img = valid ? m / a.plane : 0;
+            const long long p = valid ? m - n_img * a.plane : 0;
+            const long long ybase = n_img * (long long)a.F * a.plane + p;
+            if (cnt > 0) {
+                const int nrows = min(a.bn, cnt);
+                // warp-uniform outcome: the TMEM loads below are .sync.aligned
+                if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[ab], acc_ph, abort_flag, a.status))) break;
+                tc_fence_after();
+                const uint32_t taddr = tmem_base + (uint32_t)(ab * a.tmem_stride) + ((uint32_t)(q * 32) << 16);
+                const int* rmap = a.rowmap + (long long)g * a.n_pad + (long long)nt * a.bn;
+                for (int c0 = 0; c0 < nrows; c0 += 32) {
+                    uint32_t r[32];
+                    tmem_ld_32x32b_x32(taddr + (uint32_t)c0, r);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        if (c0 + j < nrows) {
+                            const int f = __ldg(rmap + c0 + j);
+                            float v = __uint_as_float(r[j]);
+                            if (a.bias) v += __ldg(a.bias + f);
+                            if (a.relu) v = fmaxf(v, 0.0f);
+                            if (valid) {
+                                const long long off = ybase + (long long)f * a.plane;
+                                if (OUT_BF16)
+                                    reinterpret_cast<__nv_bfloat16*>(a.y)[off] = __float2bfloat16_rn(v);
+                                else
+                                    __stcs(reinterpret_cast<float*>(a.y) + off, v);
+                            }
+                        }
+                    }
+                }
+                tc_fence_before();
+                mbar_arrive(&acc_empty[ab]);
+                ab ^= 1;
+                if (ab == 0) acc_ph ^= 1u;
+            }
+            if (nt == 0 && valid) {
+                // pruned filters of this conv group: their planes are zero
+                const int zc = s_counts[2 * g + 1];
+                const int* zmap = a.zeromap + (long long)g * a.Fg;
+                for (int z = 0; z < zc; ++z) {
+                    const long long off = ybase + (long long)__ldg(zmap + z) * a.plane;
+                    if (OUT_BF16)
+                        reinterpret_cast<__nv_bfloat16*>(a.y)[off] = __float2bfloat16_rn(0.0f);
+                    else
+                        __stcs(reinterpret_cast<float*>(a.y) + off, 0.0f);
+                }
+            }
+        }
+    } else if (warp >= 4 + kEpiWarps) {
+        // ----------------------------------------------------------- gather
+        const int gt = threadIdx.x - (4 + kEpiWarps) * 32;
+        const int prow = gt & (kBM - 1);
+        const int chunk0 = gt >> 7;  // 0 or 1: this thread builds chunks chunk0, +2, +4, +6
+        const unsigned short* xs = reinterpret_cast<const unsigned short*>(a.x);
+        int s = 0;
+        uint32_t ph = 0;
+        bool ok = true;
+        for (long long u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
+            int nt, g;
+            long long mt;
+            decode_unit(a, u, nt, g, mt);
+            if (s_counts[2 * g] <= nt * a.bn) continue;
+            const long long m = mt * kBM + prow;
+            uint32_t m0 = 0, m1 = 0;
+            const unsigned short* xb = xs;
+            if (m < a.M) {
+                const long long n_img = m / a.plane;
+                const int p = (int)(m - n_img * a.plane);
+                const int ot = p / a.OHW;
+                const int r2 = p - ot * a.OHW;
+                const int oh = r2 / a.OW;
+                const int ow = r2 - oh * a.OW;
+                const int it0 = ot * a.st - a.pt, ih0 = oh * a.sh - a.ph, iw0 = ow * a.sw - a.pw;
+                pixel_masks<MODE>(a, it0, ih0, iw0, m0, m1);
+                xb = xs + (n_img * a.x_chw + (long long)g * a.Cg * a.thw + (long long)it0 * a.hw +
+                           (long long)ih0 * a.W + iw0);
+            }
+            for (int ks = 0; ks < a.nks; ++ks) {
+                if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, a.status)) { ok = false; break; }
+                const int4* ge = a.gather + (size_t)ks * kBK;
+                uint8_t* tile = sA + (size_t)s * kATileBytes;
+#pragma unroll
+                for (int ci = 0; ci < 4; ++ci) {
+                    const int c = chunk0 + 2 * ci;
+                    uint32_t w[4];
+#pragma unroll
+                    for (int e2 = 0; e2 < 4; ++e2) {
+                        const int4 e0 = __ldg(ge + c * 8 + 2 * e2);
+                        const int4 e1 = __ldg(ge + c * 8 + 2 * e2 + 1);
+                        const uint32_t v0 = tap_ok<MODE>(e0, m0, m1) ? (uint32_t)__ldg(xb + e0.x) : 0u;
+                        const uint32_t v1 = tap_ok<MODE>(e1, m0, m1) ? (uint32_t)__ldg(xb + e1.x) : 0u;
+                        w[e2] = v0 | (v1 << 16);
+                    }
+                    *reinterpret_cast<uint4*>(tile + sw128_offset((uint32_t)prow, (uint32_t)c)) =
+                        make_uint4(w[0], w[1], w[2], w[3]);
+                }
+                fence_proxy_async_smem();
+                mbar_arrive(&full_a[s]);
+                if (++s == S) { s = 0; ph ^= 1u; }
+            }
+        }
+    }
+
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, (uint32_t)a.tmem_cols);
+    }
+}
+
+template <int MODE, bool OUT_BF16>
+cudaError_t launch(const CUtensorMap& map, const ConvArgs& a, int grid, size_t smem, cudaStream_t s)
+{
+    auto kern = k_conv_fwd<MODE, OUT_BF16>;
+    static int configured_dev = -1;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (configured_dev != dev) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
+        if (e != cudaSuccess) return e;
+        configured_dev = dev;
+    }
+    kern<<<grid, kThreads, smem, s>>>(map, a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const void* x, const float* bias,
+                             int relu, void* y, int ydt, cudaStream_t s)
+{
+    if (g.groups > kMaxGroups) return SADMM_EUNSUPPORTED;
+    const char* base = static_cast<const char*>(plan->dev);
+    ConvArgs a;
+    memset(&a, 0, sizeof(a));
+    a.x = static_cast<const __nv_bfloat16*>(x);
+    a.y = y;
+    a.bias = bias;
+    a.gather = reinterpret_cast<const int4*>(base + plan->off_gather);
+    a.rowmap = reinterpret_cast<const int*>(base + plan->off_rowmap);
+    a.zeromap = reinterpret_cast<const int*>(base + plan->off_zeromap);
+    a.counts = reinterpret_cast<const int*>(base + plan->off_counts);
+    a.status = device_status_ptr();
+    a.M = g.m;
+    a.x_chw = g.c * g.t * g.h * g.w;
+    a.thw = g.t * g.h * g.w;
+    a.hw = (int)(g.h * g.w);
+    a.W = (int)g.w;
+    a.H = (int)g.h;
+    a.T = (int)g.t;
+    a.F = (int)g.f;
+    a.groups = (int)g.groups;
+    a.Cg = (int)g.cg;
+    a.Fg = (int)g.fg;
+    a.OW = (int)g.ow;
+    a.OHW = (int)(g.oh * g.ow);
+    a.plane = (int)g.plane;
+    a.st = (int)g.st;
+    a.sh = (int)g.sh;
+    a.sw = (int)g.sw;
+    a.pt = (int)g.pt;
+    a.ph = (int)g.ph;
+    a.pw = (int)g.pw;
+    a.KT = (int)g.kt;
+    a.KH = (int)g.kh;
+    a.KW = (int)g.kw;
+    a.nks = plan->k_pad / kBK;
+    a.bn = plan->bn;
+    a.n_tiles = plan->n_tiles;
+    a.n_pad = plan->n_pad;
+    a.relu = relu ? 1 : 0;
+    const long long m_tiles = (g.m + kBM - 1) / kBM;
+    a.units = m_tiles * g.groups * plan->n_tiles;
+
+    const int stage_bytes = kATileBytes + plan->bn * 128;
+    const int budget = 232448 - 1024 - kSmemTail;
+    a.stages = budget / stage_bytes;
+    if (a.stages > kMaxStages) a.stages = kMaxStages;
+    if (a.stages < 2) return SADMM_EUNSUPPORTED;
+    a.tmem_stride = (plan->bn + 31) & ~31;
+    int cols = 32;
+    while (cols < 2 * a.tmem_stride) cols <<= 1;
+    a.tmem_cols = cols;
+    const size_t smem = 1024 + (size_t)a.stages * stage_bytes + kSmemTail;
+
+    long long grid = device_sm_count();
+    if (grid > a.units) grid = a.units;
+    if (grid < 1) grid = 1;
+
+    CUtensorMap map;
+    memcpy(&map, plan->tmap, sizeof(map));
+    const int mode = tap_mask_mode(g);
+    cudaError_t e;
+    if (mode == 0)
+        e = (ydt == SADMM_BF16) ? launch<0, true>(map, a, (int)grid, smem, s)
+                                : launch<0, false>(map, a, (int)grid, smem, s);
+    else
+        e = (ydt == SADMM_BF16) ? launch<1, true>(map, a, (int)grid, smem, s)
+                                : launch<1, false>(map, a, (int)grid, smem, s);
+    return e == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
+}
+
+}  // namespace sadmm

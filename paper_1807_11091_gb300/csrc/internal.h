@@ -1,0 +1,52 @@
+// internal.h -- host-side declarations shared by the libsadmm translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/sadmm.h"
+
+namespace sadmm {
+
+// Derived sizes of a validated descriptor.
+struct Geometry {
+    long long n, c, t, h, w, f, groups, kt, kh, kw, st, sh, sw, pt, ph, pw;
+    long long cg, fg, taps, k;      // K = Cg * taps GEMM columns
+    long long ot, oh, ow, plane, m; // output extents, pixels per image, N * plane
+};
+
+// Checks a descriptor; fills `g` on success.
+sadmm_status check_desc(const sadmm_conv_desc* d, Geometry* g);
+
+// Address of the device status word on the current device (cached per device).
+int* device_status_ptr();
+
+// Number of SMs of the current device (cached per device).
+int device_sm_count();
+
+// Compute capability major of the current device (cached per device).
+int device_cc_major();
+
+// Rounds x up to a multiple of a.
+inline long long round_up(long long x, long long a) { return (x + a - 1) / a * a; }
+
+// ---- projection (project.cu) ----
+size_t project_workspace_bytes(const Geometry& g, int colkind);
+sadmm_status launch_project(const Geometry& g, const void* W, const void* U, int wdt, int k_filters,
+                            int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out,
+                            void* ws, cudaStream_t s);
+
+// ---- pack (pack.cu) ----
+sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* filt_idx,
+                         const int* col_idx, cudaStream_t s);
+
+// ---- forward (conv_fwd.cu) ----
+sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const void* x, const float* bias,
+                             int relu, void* y, int ydt, cudaStream_t s);
+
+// Tap-mask mode of the gather table: 0 = one 32-bit mask over all taps
+// (KT*KH*KW <= 32), 1 = a (kt,kh) row mask and a kw column mask.
+inline int tap_mask_mode(const Geometry& g) { return g.taps <= 32 ? 0 : 1; }
+
+}  // namespace sadmm

@@ -1,0 +1,250 @@
+// pack.cu -- compaction of the kept rows and columns of the lowered GEMM matrix
+// (Sec. 3, "Combination of structured sparsities": filter-wise sparsity is row
+// pruning and channel-/shape-wise sparsity is column pruning; what remains is a
+// smaller full matrix).
+//
+//   k_pack_meta  one block: per conv group the kept and pruned filter lists and
+//                counts, the kept-column list and the gather table (channel
+//                offset of each kept column in x plus its tap bits).
+//   k_pack_wp    one block per packed row: Wp[g][i][j] = bf16(W[f_i][col_j]),
+//                zero outside the kept counts, 16-byte stores.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <string.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace sadmm {
+namespace {
+
+struct PackArgs {
+    const int* filt_idx;  // kept filters, ascending (unused when all_kept)
+    int all_kept;         // n_filt == F
+    const int* col_idx;   // NULL: all columns
+    int n_filt, colkind, n_colgroups, n_cols;
+    int F, groups, Fg, K, taps, KT, KH, KW;
+    long long thw;  // T*H*W
+    int hw, W;
+    int k_pad, n_pad;
+    int mask_mode;
+    int4* gather;
+    int* colidx;
+    int* rowmap;
+    int* zeromap;
+    int* counts;
+};
+
+// First position p in the ascending list a[0..n) with a[p] >= v.
+SADMM_DEV int lower_bound(const int* a, int n, int v)
+{
+    int lo = 0, hi = n;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (a[mid] < v) lo = mid + 1;
+        else hi = mid;
+    }
+    return lo;
+}
+
+__global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status)
+{
+    __shared__ int s_start[65];
+    __shared__ int s_bad;
+    const int tid = threadIdx.x;
+    // Index lists must be strictly ascending and in range.  A list that is not
+    // gives a plan with every filter pruned and every column dropped (an
+    // all-zero output) and raises the device status word.
+    if (tid == 0) s_bad = 0;
+    __syncthreads();
+    if (!a.all_kept) {
+        for (int i = tid; i < a.n_filt; i += blockDim.x) {
+            const int v = a.filt_idx[i];
+            if (v < 0 || v >= a.F || (i + 1 < a.n_filt && a.filt_idx[i + 1] <= v)) s_bad = 1;
+        }
+    }
+    if (a.col_idx && a.colkind != SADMM_COL_NONE) {
+        const int lim = (a.colkind == SADMM_COL_CHANNEL) ? a.K / a.taps : a.K;
+        for (int i = tid; i < a.n_colgroups; i += blockDim.x) {
+            const int v = a.col_idx[i];
+            if (v < 0 || v >= lim || (i + 1 < a.n_colgroups && a.col_idx[i + 1] <= v)) s_bad = 1;
+        }
+    }
+    __syncthreads();
+    if (s_bad) {
+        if (tid == 0) raise_status(status, kDevBadIndex);
+        for (int g = tid; g < a.groups; g += blockDim.x) {
+            a.counts[2 * g] = 0;
+            a.counts[2 * g + 1] = a.Fg;
+        }
+        for (int r = tid; r < a.groups * a.n_pad; r += blockDim.x) a.rowmap[r] = -1;
+        for (int f = tid; f < a.F; f += blockDim.x) a.zeromap[f] = f;
+        for (int j = tid; j < a.k_pad; j += blockDim.x) {
+            a.colidx[j] = -1;
+            a.gather[j] = make_int4(0, 0, 0, 0);
+        }
+        return;
+    }
+    // kept-filter range of each conv group in the ascending filter list
+    for (int g = tid; g <= a.groups; g += blockDim.x)
+        s_start[g] = a.all_kept ? g * a.Fg : lower_bound(a.filt_idx, a.n_filt, g * a.Fg);
+    __syncthreads();
+    for (int g = tid; g < a.groups; g += blockDim.x) {
+        const int kept = s_start[g + 1] - s_start[g];
+        a.counts[2 * g] = kept;
+        a.counts[2 * g + 1] = a.Fg - kept;
+    }
+    // rows of the packed matrix -> output filter (or -1 for padding rows)
+    for (int r = tid; r < a.groups * a.n_pad; r += blockDim.x) {
+        const int g = r / a.n_pad, i = r % a.n_pad;
+        const int kept = s_start[g + 1] - s_start[g];
+        int f = -1;
+        if (i < kept) f = a.all_kept ? g * a.Fg + i : a.filt_idx[s_start[g] + i];
+        a.rowmap[r] = f;
+    }
+    // pruned filters of each group, ascending
+    if (!a.all_kept) {
+        for (int f = tid; f < a.F; f += blockDim.x) {
+            const int pos = lower_bound(a.filt_idx, a.n_filt, f);
+            const bool kept = pos < a.n_filt && a.filt_idx[pos] == f;
+            if (!kept) {
+                const int g = f / a.Fg;
+                const int z = (f - g * a.Fg) - (pos - s_start[g]);
+                a.zeromap[g * a.Fg + z] = f;
+            }
+        }
+    }
+    // kept GEMM columns and their gather entries
+    for (int j = tid; j < a.k_pad; j += blockDim.x) {
+        int col = -1;
+        if (j < a.n_cols) {
+            if (a.colkind == SADMM_COL_SHAPE) col = a.col_idx[j];
+            else if (a.colkind == SADMM_COL_CHANNEL) col = a.col_idx[j / a.taps] * a.taps + j % a.taps;
+            else col = j;
+        }
+        a.colidx[j] = col;
+        int4 e = make_int4(0, 0, 0, 0);
+        if (col >= 0) {
+            const int c = col / a.taps, r = col % a.taps;
+            const int kt = r / (a.KH * a.KW), kh = (r / a.KW) % a.KH, kw = r % a.KW;
+            e.x = (int)(c * a.thw + (long long)kt * a.hw + kh * a.W + kw);
+            if (a.mask_mode == 0) {
+                e.y = (int)(1u << r);
+            } else {
+                e.y = (int)(1u << (kt * a.KH + kh));
+                e.z = (int)(1u << kw);
+            }
+        }
+        a.gather[j] = e;
+    }
+}
+
+template <typename T>
+SADMM_DEV float load_f32(const T* p);
+template <>
+SADMM_DEV float load_f32<__nv_bfloat16>(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+template <>
+SADMM_DEV float load_f32<float>(const float* p) { return *p; }
+
+template <typename T>
+__global__ void __launch_bounds__(128) k_pack_wp(const T* __restrict__ W, int K, const int* __restrict__ rowmap,
+                                                 const int* __restrict__ colidx, int k_pad,
+                                                 __nv_bfloat16* __restrict__ wp)
+{
+    const long long r = blockIdx.x;
+    const int f = rowmap[r];
+    uint4* dst = reinterpret_cast<uint4*>(wp + r * k_pad);
+    for (int j8 = threadIdx.x; j8 < k_pad / 8; j8 += blockDim.x) {
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int j0 = j8 * 8 + 2 * e;
+            const int c0 = colidx[j0], c1 = colidx[j0 + 1];
+            const float v0 = (f >= 0 && c0 >= 0) ? load_f32<T>(W + (long long)f * K + c0) : 0.0f;
+            const float v1 = (f >= 0 && c1 >= 0) ? load_f32<T>(W + (long long)f * K + c1) : 0.0f;
+            const __nv_bfloat162 p = __floats2bfloat162_rn(v0, v1);  // .x = v0 (low half)
+            w[e] = *reinterpret_cast<const uint32_t*>(&p);
+        }
+        dst[j8] = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            return nullptr;
+        fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }
+    return fn;
+}
+
+}  // namespace
+
+sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* filt_idx,
+                         const int* col_idx, cudaStream_t s)
+{
+    char* base = static_cast<char*>(plan->dev);
+    PackArgs a;
+    a.all_kept = (plan->n_filt == (int)g.f) ? 1 : 0;
+    a.filt_idx = a.all_kept ? nullptr : filt_idx;
+    a.col_idx = col_idx;
+    a.n_filt = plan->n_filt;
+    a.colkind = plan->colkind;
+    a.n_colgroups = plan->n_colgroups;
+    a.n_cols = plan->n_cols;
+    a.F = (int)g.f;
+    a.groups = (int)g.groups;
+    a.Fg = (int)g.fg;
+    a.K = (int)g.k;
+    a.taps = (int)g.taps;
+    a.KT = (int)g.kt;
+    a.KH = (int)g.kh;
+    a.KW = (int)g.kw;
+    a.thw = g.t * g.h * g.w;
+    a.hw = (int)(g.h * g.w);
+    a.W = (int)g.w;
+    a.k_pad = plan->k_pad;
+    a.n_pad = plan->n_pad;
+    a.mask_mode = tap_mask_mode(g);
+    a.gather = reinterpret_cast<int4*>(base + plan->off_gather);
+    a.colidx = reinterpret_cast<int*>(base + plan->off_colidx);
+    a.rowmap = reinterpret_cast<int*>(base + plan->off_rowmap);
+    a.zeromap = reinterpret_cast<int*>(base + plan->off_zeromap);
+    a.counts = reinterpret_cast<int*>(base + plan->off_counts);
+    k_pack_meta<<<1, 1024, 0, s>>>(a, device_status_ptr());
+
+    __nv_bfloat16* wp = reinterpret_cast<__nv_bfloat16*>(base + plan->off_wp);
+    const unsigned rows = (unsigned)(g.groups * plan->n_pad);
+    if (wdt == SADMM_BF16)
+        k_pack_wp<__nv_bfloat16><<<rows, 128, 0, s>>>((const __nv_bfloat16*)W, (int)g.k, a.rowmap, a.colidx,
+                                                       plan->k_pad, wp);
+    else
+        k_pack_wp<float><<<rows, 128, 0, s>>>((const float*)W, (int)g.k, a.rowmap, a.colidx, plan->k_pad, wp);
+    if (cudaGetLastError() != cudaSuccess) return SADMM_ECUDA;
+
+    // TMA descriptor of Wp: [groups*n_pad rows][k_pad bf16], boxes of 64 x bn,
+    // 128-byte swizzle (the layout the tensor-core operand descriptor expects).
+    PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
+    if (!enc) return SADMM_ECUDA;
+    alignas(64) CUtensorMap map;
+    memset(&map, 0, sizeof(map));
+    const cuuint64_t gdim[2] = {(cuuint64_t)plan->k_pad, (cuuint64_t)rows};
+    const cuuint64_t gstride[1] = {(cuuint64_t)plan->k_pad * 2};
+    const cuuint32_t box[2] = {64u, (cuuint32_t)plan->bn};
+    const cuuint32_t estride[2] = {1u, 1u};
+    const CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, wp, gdim, gstride, box, estride,
+                           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return SADMM_ECUDA;
+    static_assert(sizeof(CUtensorMap) == sizeof(plan->tmap), "tensor map size");
+    memcpy(plan->tmap, &map, sizeof(map));
+    return SADMM_OK;
+}
+
+}  // namespace sadmm

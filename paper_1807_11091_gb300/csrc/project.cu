@@ -1,0 +1,249 @@
+// project.cu -- Euclidean projection onto a structured-sparsity set (Sec. 4,
+// solution of the Z-subproblem, Eq. 4): squared Frobenius norms of the filter,
+// channel or shape groups of V = W (+U), then an exact top-k.
+//
+// Kernels:
+//   k_filter_keys   one warp per GEMM row (filter): fp64 sum of squares,
+//                   warp-shuffle reduction.
+//   k_column_keys   32 columns per block, 8 warps over the (kept) rows, fixed
+//                   order shared-memory reduction: one key per GEMM column.
+//   k_select        one block: optional channel sums of column keys, an MSB-
+//                   first radix select over the fp64 key bit patterns (exact
+//                   k-th largest key), then an ordered compaction that keeps
+//                   every key above it and the lowest-index keys equal to it.
+//
+// Keys are non-negative fp64 values, so their IEEE bit patterns order like the
+// values; selection compares bit patterns (a NaN key would rank above +Inf).
+#include "common.cuh"
+#include "internal.h"
+
+namespace sadmm {
+namespace {
+
+template <typename T>
+SADMM_DEV double to_f64(T v);
+template <>
+SADMM_DEV double to_f64<__nv_bfloat16>(__nv_bfloat16 v) { return (double)__bfloat162float(v); }
+template <>
+SADMM_DEV double to_f64<float>(float v) { return (double)v; }
+
+// V = W (+U) element, exactly in fp64.
+template <typename T>
+SADMM_DEV double v_elem(const T* __restrict__ W, const T* __restrict__ U, long long i)
+{
+    double v = to_f64<T>(W[i]);
+    if (U) v += to_f64<T>(U[i]);
+    return v;
+}
+
+// O_a = sum_k V[a,k]^2 for every row a (filter-wise groups).
+template <typename T>
+__global__ void k_filter_keys(const T* __restrict__ W, const T* __restrict__ U, int F, int K,
+                              double* __restrict__ keys)
+{
+    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (warp >= F) return;
+    const long long base = (long long)warp * K;
+    double s = 0.0;
+    for (int k = lane; k < K; k += 32) {
+        const double v = v_elem(W, U, base + k);
+        s += v * v;
+    }
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_down_sync(0xffffffffu, s, o);
+    if (lane == 0) keys[warp] = s;
+}
+
+// O_j = sum over kept rows a of V[a,j]^2 for every column j.  rows == NULL
+// means rows 0..nrows-1.
+template <typename T>
+__global__ void __launch_bounds__(256) k_column_keys(const T* __restrict__ W, const T* __restrict__ U, int K,
+                                                     const int* __restrict__ rows, int nrows,
+                                                     double* __restrict__ keys)
+{
+    __shared__ double part[8][33];
+    const int lane = threadIdx.x & 31;
+    const int wy = threadIdx.x >> 5;
+    const int j = blockIdx.x * 32 + lane;
+    double s = 0.0;
+    if (j < K) {
+        for (int r = wy; r < nrows; r += 8) {
+            const int a = rows ? rows[r] : r;
+            const double v = v_elem(W, U, (long long)a * K + j);
+            s += v * v;
+        }
+    }
+    part[wy][lane] = s;
+    __syncthreads();
+    if (wy == 0 && j < K) {
+        double t = 0.0;
+        for (int q = 0; q < 8; ++q) t += part[q][lane];
+        keys[j] = t;
+    }
+}
+
+constexpr int kSelThreads = 1024;
+
+// Exclusive block-wide prefix count of a predicate (1024 threads).  Returns
+// the exclusive count for this thread; *total gets the block total.
+SADMM_DEV int block_excl_count(bool pred, int* warp_tot, int* total)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const unsigned b = __ballot_sync(0xffffffffu, pred);
+    const int in_warp = __popc(b & ((1u << lane) - 1u));
+    if (lane == 0) warp_tot[warp] = __popc(b);
+    __syncthreads();
+    if (warp == 0) {
+        const int v = warp_tot[lane];
+        int inc = v;
+        for (int o = 1; o < 32; o <<= 1) {
+            const int t = __shfl_up_sync(0xffffffffu, inc, o);
+            if (lane >= o) inc += t;
+        }
+        warp_tot[lane] = inc - v;  // exclusive
+        if (lane == 31) warp_tot[32] = inc;
+    }
+    __syncthreads();
+    const int r = warp_tot[warp] + in_warp;
+    *total = warp_tot[32];
+    __syncthreads();  // warp_tot is reused by the next call
+    return r;
+}
+
+// Exact top-k of G fp64 keys (ties to the lower index), ascending index list.
+// When taps > 1 the keys are first formed as sums of `taps` consecutive source
+// keys (channel-wise groups from column keys).
+__global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict__ src, int G, int taps, int k,
+                                                        double* __restrict__ keys, double* __restrict__ keys_out,
+                                                        int* __restrict__ out_idx)
+{
+    __shared__ unsigned int hist[256];
+    __shared__ unsigned long long s_prefix;
+    __shared__ int s_kk;
+    __shared__ int warp_tot[33];
+    const int tid = threadIdx.x;
+
+    // 1. keys (channel sums when taps > 1) and the optional copy for the caller
+    for (int i = tid; i < G; i += kSelThreads) {
+        double v;
+        if (taps > 1) {
+            v = 0.0;
+            for (int t = 0; t < taps; ++t) v += src[(long long)i * taps + t];
+            keys[i] = v;
+        } else {
+            v = src[i];
+        }
+        if (keys_out) keys_out[i] = v;
+    }
+    const double* kv = (taps > 1) ? keys : src;
+    __syncthreads();
+
+    if (k <= 0) return;
+    if (k >= G) {
+        for (int i = tid; i < G; i += kSelThreads) out_idx[i] = i;
+        return;
+    }
+
+    // 2. radix select, 8 bits per pass from the most significant digit
+    if (tid == 0) { s_prefix = 0ull; s_kk = k; }
+    unsigned long long mask = 0ull;
+    for (int shift = 56; shift >= 0; shift -= 8) {
+        for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0u;
+        __syncthreads();
+        const unsigned long long prefix = s_prefix;
+        for (int i = tid; i < G; i += kSelThreads) {
+            const unsigned long long u = (unsigned long long)__double_as_longlong(kv[i]);
+            if ((u & mask) == prefix) atomicAdd(&hist[(u >> shift) & 255u], 1u);
+        }
+        __syncthreads();
+        if (tid < 32) {
+            // lane l owns digits 255-8l .. 248-8l, highest first
+            unsigned c[8];
+            unsigned tot = 0;
+            for (int j = 0; j < 8; ++j) { c[j] = hist[255 - 8 * tid - j]; tot += c[j]; }
+            unsigned inc = tot;
+            for (int o = 1; o < 32; o <<= 1) {
+                const unsigned t = __shfl_up_sync(0xffffffffu, inc, o);
+                if (tid >= o) inc += t;
+            }
+            unsigned cum = inc - tot;  // keys with a higher digit than this lane's
+            const unsigned kk = (unsigned)s_kk;
+            if (cum < kk && kk <= cum + tot) {
+                for (int j = 0; j < 8; ++j) {
+                    if (cum + c[j] >= kk) {
+                        const unsigned d = 255u - 8u * tid - j;
+                        s_prefix = prefix | ((unsigned long long)d << shift);
+                        s_kk = (int)(kk - cum);
+                        break;
+                    }
+                    cum += c[j];
+                }
+            }
+        }
+        mask |= 0xFFull << shift;
+        __syncthreads();
+    }
+    const unsigned long long T = s_prefix;  // exact k-th largest key
+    const int take_eq = s_kk;               // how many keys equal to T are kept
+
+    // 3. ordered compaction
+    int run_out = 0, run_eq = 0;
+    for (int base = 0; base < G; base += kSelThreads) {
+        const int i = base + tid;
+        const bool valid = i < G;
+        const unsigned long long u = valid ? (unsigned long long)__double_as_longlong(kv[i]) : 0ull;
+        const bool gt = valid && u > T;
+        const bool eq = valid && u == T;
+        int eq_tot, take_tot;
+        const int eq_before = block_excl_count(eq, warp_tot, &eq_tot);
+        const bool take = gt || (eq && run_eq + eq_before < take_eq);
+        const int pos = block_excl_count(take, warp_tot, &take_tot);
+        if (take) out_idx[run_out + pos] = i;
+        run_eq += eq_tot;
+        run_out += take_tot;
+    }
+}
+
+template <typename T>
+sadmm_status run_project(const Geometry& g, const T* W, const T* U, int k_filters, int colkind, int k_cols,
+                         int* filt_idx, int* col_idx, double* keys_out, void* ws, cudaStream_t s)
+{
+    const int F = (int)g.f, K = (int)g.k;
+    double* fkeys = reinterpret_cast<double*>(ws);
+    double* ckeys = fkeys + round_up(F, 32);
+    double* chkeys = ckeys + round_up(K, 32);
+
+    k_filter_keys<T><<<(F * 32 + 255) / 256, 256, 0, s>>>(W, U, F, K, fkeys);
+    k_select<<<1, kSelThreads, 0, s>>>(fkeys, F, 1, k_filters, fkeys, keys_out, filt_idx);
+    if (colkind != SADMM_COL_NONE) {
+        const bool all_rows = (k_filters == F);
+        k_column_keys<T><<<(K + 31) / 32, 256, 0, s>>>(W, U, K, all_rows ? nullptr : filt_idx,
+                                                       all_rows ? F : k_filters, ckeys);
+        const int taps = (colkind == SADMM_COL_CHANNEL) ? (int)g.taps : 1;
+        const int G = (colkind == SADMM_COL_CHANNEL) ? (int)g.cg : K;
+        k_select<<<1, kSelThreads, 0, s>>>(ckeys, G, taps, k_cols, chkeys, keys_out ? keys_out + F : nullptr,
+                                           col_idx);
+    }
+    return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
+}
+
+}  // namespace
+
+size_t project_workspace_bytes(const Geometry& g, int colkind)
+{
+    (void)colkind;
+    return (size_t)(round_up(g.f, 32) + round_up(g.k, 32) + round_up(g.cg, 32)) * sizeof(double) + 256;
+}
+
+sadmm_status launch_project(const Geometry& g, const void* W, const void* U, int wdt, int k_filters,
+                            int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out,
+                            void* ws, cudaStream_t s)
+{
+    if (wdt == SADMM_BF16)
+        return run_project<__nv_bfloat16>(g, (const __nv_bfloat16*)W, (const __nv_bfloat16*)U, k_filters,
+                                          colkind, k_cols, filt_idx, col_idx, keys_out, ws, s);
+    return run_project<float>(g, (const float*)W, (const float*)U, k_filters, colkind, k_cols, filt_idx,
+                              col_idx, keys_out, ws, s);
+}
+
+}  // namespace sadmm

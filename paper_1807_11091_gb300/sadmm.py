@@ -1,0 +1,265 @@
+"""ctypes binding of libsadmm (include/sadmm.h).
+
+The functions named like the C entry points (``sadmm_*``) marshal arguments and
+nothing else: every step of the path runs in the CUDA library.  The torch
+helpers at the end (``project_groups``, ``PrunedConv``) only allocate device
+memory with torch and pass raw pointers and the current stream through.
+
+There is no CPU fallback: when the library cannot be built or loaded, every
+call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence, Tuple
+
+from . import build as _build
+
+SADMM_OK, SADMM_EINVAL, SADMM_ECUDA, SADMM_ETIMEOUT, SADMM_EUNSUPPORTED = 0, -1, -2, -3, -4
+SADMM_BF16, SADMM_FP32 = 0, 1
+SADMM_COL_NONE, SADMM_COL_SHAPE, SADMM_COL_CHANNEL = 0, 1, 2
+
+DESC_FIELDS = ("n", "c", "t", "h", "w", "f", "groups", "kt", "kh", "kw", "st", "sh", "sw", "pt", "ph", "pw")
+
+
+class SadmmError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} ({status})")
+
+
+class ConvDesc(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int) for n in DESC_FIELDS]
+
+
+class Plan(ctypes.Structure):
+    _fields_ = [
+        ("desc", ConvDesc),
+        ("n_filt", ctypes.c_int),
+        ("colkind", ctypes.c_int),
+        ("n_colgroups", ctypes.c_int),
+        ("n_cols", ctypes.c_int),
+        ("k_pad", ctypes.c_int),
+        ("bn", ctypes.c_int),
+        ("n_tiles", ctypes.c_int),
+        ("n_pad", ctypes.c_int),
+        ("dev_bytes", ctypes.c_size_t),
+        ("dev", ctypes.c_void_p),
+        ("off_wp", ctypes.c_size_t),
+        ("off_gather", ctypes.c_size_t),
+        ("off_rowmap", ctypes.c_size_t),
+        ("off_zeromap", ctypes.c_size_t),
+        ("off_counts", ctypes.c_size_t),
+        ("off_colidx", ctypes.c_size_t),
+        ("tmap", ctypes.c_uint64 * 16),
+    ]
+
+
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load():
+    """Loads libsadmm.so, building it first when it is missing or stale."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.build()
+    lib = ctypes.CDLL(path)
+    vp, sz, ci = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int
+    P = ctypes.POINTER
+    lib.sadmm_abi_version.restype = ci
+    lib.sadmm_abi_version.argtypes = []
+    lib.sadmm_plan_struct_size.restype = sz
+    lib.sadmm_plan_struct_size.argtypes = []
+    lib.sadmm_status_string.restype = ctypes.c_char_p
+    lib.sadmm_status_string.argtypes = [ci]
+    lib.sadmm_workspace_size.restype = sz
+    lib.sadmm_workspace_size.argtypes = [P(ConvDesc), ci]
+    lib.sadmm_project_groups.restype = ci
+    lib.sadmm_project_groups.argtypes = [P(ConvDesc), vp, vp, ci, ci, ci, ci, vp, vp, vp, vp, sz, vp]
+    lib.sadmm_plan_init.restype = ci
+    lib.sadmm_plan_init.argtypes = [P(Plan), P(ConvDesc), ci, ci, ci]
+    lib.sadmm_pack.restype = ci
+    lib.sadmm_pack.argtypes = [P(Plan), vp, ci, vp, vp, vp, sz, vp]
+    lib.sadmm_conv_fwd.restype = ci
+    lib.sadmm_conv_fwd.argtypes = [P(Plan), vp, vp, ci, vp, ci, vp]
+    lib.sadmm_last_device_status.restype = ci
+    lib.sadmm_last_device_status.argtypes = [vp]
+    if lib.sadmm_plan_struct_size() != ctypes.sizeof(Plan):
+        raise RuntimeError("sadmm_plan layout differs between the library and this binding")
+    _lib = lib
+    return lib
+
+
+def _check(status: int, where: str) -> None:
+    if status != SADMM_OK:
+        raise SadmmError(status, where)
+
+
+def status_string(status: int) -> str:
+    try:
+        return load().sadmm_status_string(int(status)).decode()
+    except Exception:  # pragma: no cover - only when the library is absent
+        return "status"
+
+
+def make_desc(values: Sequence[int]) -> ConvDesc:
+    """ConvDesc from the 16 fields n c t h w f groups kt kh kw st sh sw pt ph pw."""
+    return ConvDesc(*[int(v) for v in values])
+
+
+# --------------------------------------------------------------------------
+# C entry points (argument marshalling only; pointers are plain ints)
+# --------------------------------------------------------------------------
+
+def sadmm_abi_version() -> int:
+    return load().sadmm_abi_version()
+
+
+def sadmm_plan_struct_size() -> int:
+    return load().sadmm_plan_struct_size()
+
+
+def sadmm_status_string(status: int) -> str:
+    return status_string(status)
+
+
+def sadmm_workspace_size(desc: ConvDesc, colkind: int) -> int:
+    return load().sadmm_workspace_size(ctypes.byref(desc), int(colkind))
+
+
+def sadmm_project_groups(desc: ConvDesc, W: int, U: Optional[int], wdt: int, k_filters: int, colkind: int,
+                         k_cols: int, filt_idx: int, col_idx: Optional[int], keys_out: Optional[int],
+                         workspace: int, ws_bytes: int, stream: Optional[int]) -> int:
+    return load().sadmm_project_groups(ctypes.byref(desc), W, U, int(wdt), int(k_filters), int(colkind),
+                                       int(k_cols), filt_idx, col_idx, keys_out, workspace, int(ws_bytes),
+                                       stream)
+
+
+def sadmm_plan_init(desc: ConvDesc, n_filt: int, colkind: int, n_colgroups: int) -> Tuple[int, Plan]:
+    plan = Plan()
+    st = load().sadmm_plan_init(ctypes.byref(plan), ctypes.byref(desc), int(n_filt), int(colkind),
+                                int(n_colgroups))
+    return st, plan
+
+
+def sadmm_pack(plan: Plan, W: int, wdt: int, filt_idx: Optional[int], col_idx: Optional[int], dev: int,
+               dev_bytes: int, stream: Optional[int]) -> int:
+    return load().sadmm_pack(ctypes.byref(plan), W, int(wdt), filt_idx, col_idx, dev, int(dev_bytes), stream)
+
+
+def sadmm_conv_fwd(plan: Plan, x: int, bias: Optional[int], relu: int, y: int, ydt: int,
+                   stream: Optional[int]) -> int:
+    return load().sadmm_conv_fwd(ctypes.byref(plan), x, bias, int(relu), y, int(ydt), stream)
+
+
+def sadmm_last_device_status(stream: Optional[int]) -> int:
+    return load().sadmm_last_device_status(stream)
+
+
+# --------------------------------------------------------------------------
+# torch helpers: device memory and streams only
+# --------------------------------------------------------------------------
+
+def _torch():
+    import torch
+    return torch
+
+
+def _ptr(t) -> Optional[int]:
+    return None if t is None else int(t.data_ptr())
+
+
+def _stream(stream=None) -> int:
+    torch = _torch()
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return int(s.cuda_stream)
+
+
+def _wdt(t) -> int:
+    torch = _torch()
+    if t.dtype == torch.bfloat16:
+        return SADMM_BF16
+    if t.dtype == torch.float32:
+        return SADMM_FP32
+    raise TypeError(f"weights must be bf16 or fp32, got {t.dtype}")
+
+
+def project_groups(desc16: Sequence[int], W, k_filters: int, colkind: int, k_cols: int, U=None,
+                   with_keys: bool = False, stream=None, workspace=None):
+    """Runs sadmm_project_groups; returns (filt_idx, col_idx, keys or None) as device tensors."""
+    torch = _torch()
+    desc = make_desc(desc16)
+    dev = W.device
+    ws_bytes = sadmm_workspace_size(desc, colkind)
+    if ws_bytes == 0:
+        raise SadmmError(SADMM_EINVAL, "sadmm_workspace_size")
+    if workspace is None or workspace.numel() < ws_bytes:
+        workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    f = int(desc16[5])
+    cg = int(desc16[1]) // int(desc16[6])
+    taps = int(desc16[7]) * int(desc16[8]) * int(desc16[9])
+    G = 0 if colkind == SADMM_COL_NONE else (cg * taps if colkind == SADMM_COL_SHAPE else cg)
+    filt_idx = torch.empty(max(k_filters, 1), dtype=torch.int32, device=dev)
+    col_idx = torch.empty(max(k_cols, 1), dtype=torch.int32, device=dev) if colkind != SADMM_COL_NONE else None
+    keys = torch.empty(f + G, dtype=torch.float64, device=dev) if with_keys else None
+    st = sadmm_project_groups(desc, _ptr(W), _ptr(U), _wdt(W), k_filters, colkind, k_cols, _ptr(filt_idx),
+                              _ptr(col_idx), _ptr(keys), _ptr(workspace), ws_bytes, _stream(stream))
+    _check(st, "sadmm_project_groups")
+    fi = filt_idx[:k_filters]
+    ci = col_idx[:k_cols] if col_idx is not None else None
+    return fi, ci, keys
+
+
+class PrunedConv:
+    """A packed pruned layer: plan plus its device buffer (sadmm_plan_init + sadmm_pack)."""
+
+    def __init__(self, desc16: Sequence[int], W, filt_idx, colkind: int, col_idx, n_filt: int,
+                 n_colgroups: int, stream=None):
+        torch = _torch()
+        self.desc16 = [int(v) for v in desc16]
+        desc = make_desc(self.desc16)
+        st, plan = sadmm_plan_init(desc, n_filt, colkind, n_colgroups)
+        _check(st, "sadmm_plan_init")
+        self.plan = plan
+        self.buf = torch.empty(plan.dev_bytes, dtype=torch.uint8, device=W.device)
+        self.W = W
+        self.repack(W, filt_idx, col_idx, stream)
+
+    def repack(self, W, filt_idx, col_idx, stream=None):
+        st = sadmm_pack(self.plan, _ptr(W), _wdt(W), _ptr(filt_idx), _ptr(col_idx), _ptr(self.buf),
+                        self.plan.dev_bytes, _stream(stream))
+        _check(st, "sadmm_pack")
+
+    def out_shape(self):
+        n, c, t, h, w, f, g, kt, kh, kw, st_, sh, sw, pt, ph, pw = self.desc16
+        ot = (t + 2 * pt - kt) // st_ + 1
+        oh = (h + 2 * ph - kh) // sh + 1
+        ow = (w + 2 * pw - kw) // sw + 1
+        if t == 1 and kt == 1:
+            return (n, f, oh, ow)
+        return (n, f, ot, oh, ow)
+
+    def forward(self, x, bias=None, relu: bool = True, out_dtype=None, out=None, stream=None):
+        torch = _torch()
+        if x.dtype != torch.bfloat16 or not x.is_contiguous():
+            raise TypeError("x must be a contiguous bf16 tensor")
+        if out is None:
+            out_dtype = out_dtype or torch.float32
+            out = torch.empty(self.out_shape(), dtype=out_dtype, device=x.device)
+        ydt = SADMM_BF16 if out.dtype == torch.bfloat16 else SADMM_FP32
+        if bias is not None and (bias.dtype != torch.float32 or not bias.is_contiguous()):
+            raise TypeError("bias must be a contiguous fp32 tensor")
+        st = sadmm_conv_fwd(self.plan, _ptr(x), _ptr(bias), 1 if relu else 0, _ptr(out), ydt, _stream(stream))
+        _check(st, "sadmm_conv_fwd")
+        return out
+
+
+def device_status(stream=None) -> int:
+    """Synchronises the stream and returns (and clears) the device status word."""
+    return sadmm_last_device_status(_stream(stream))

@@ -1,0 +1,96 @@
+"""The C ABI without a GPU: the library builds for sm_103a, loads, exports every
+entry point include/*.h declares, and rejects bad arguments on the host before
+any launch."""
+import ctypes
+import glob
+import os
+import re
+
+import pytest
+
+from paper_1807_11091_gb300 import sadmm
+import workloads as wl
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    names = set()
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        text = open(h).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        for m in re.finditer(r"\b(sadmm_[a-z0-9_]+)\s*\(", text):
+            names.add(m.group(1))
+    return sorted(names)
+
+
+def test_library_exports_every_declared_entry_point():
+    lib = sadmm.load()
+    names = _declared()
+    assert {"sadmm_project_groups", "sadmm_pack", "sadmm_conv_fwd"} <= set(names)
+    for n in names:
+        assert hasattr(lib, n), f"{n} not exported"
+
+
+def test_struct_layout_and_version():
+    assert sadmm.sadmm_abi_version() == 1
+    assert sadmm.sadmm_plan_struct_size() == ctypes.sizeof(sadmm.Plan)
+    assert sadmm.sadmm_status_string(-1) == "invalid argument"
+
+
+def test_plan_sizes():
+    L = wl.alexnet()[3]  # conv4: groups 2, 77 filters, 346 columns
+    st, p = sadmm.sadmm_plan_init(sadmm.make_desc(L.shape.desc16()), L.k_filters, wl.COL_SHAPE, L.k_cols)
+    assert st == 0
+    assert p.n_cols == 346 and p.k_pad == 384
+    assert p.bn % 16 == 0 and p.bn <= 256 and p.n_pad == p.bn * p.n_tiles >= 77
+    assert p.dev_bytes >= 2 * p.n_pad * p.k_pad * 2
+    # channel-wise expands to taps columns per channel
+    st, p = sadmm.sadmm_plan_init(sadmm.make_desc(L.shape.desc16()), 10, wl.COL_CHANNEL, 7)
+    assert st == 0 and p.n_cols == 7 * 9
+    # more than 256 kept rows per group -> several filter tiles
+    s = wl.sweep()[0].shape
+    st, p = sadmm.sadmm_plan_init(sadmm.make_desc(s.desc16()), 512, wl.COL_SHAPE, 2304)
+    assert st == 0 and p.n_tiles == 2 and p.bn == 256 and p.k_pad == 2304
+
+
+@pytest.mark.parametrize("field,value", [("n", 0), ("groups", 3), ("kh", 40), ("st", 0), ("ph", -1)])
+def test_bad_descriptors_rejected(field, value):
+    d = wl.single2d()[0].shape.desc16()
+    d[sadmm.DESC_FIELDS.index(field)] = value
+    st, _ = sadmm.sadmm_plan_init(sadmm.make_desc(d), 10, wl.COL_SHAPE, 10)
+    assert st in (sadmm.SADMM_EINVAL, sadmm.SADMM_EUNSUPPORTED)
+
+
+def test_bad_counts_rejected_on_host():
+    s = wl.single2d()[0].shape
+    d = sadmm.make_desc(s.desc16())
+    assert sadmm.sadmm_plan_init(d, s.f + 1, wl.COL_SHAPE, 1)[0] == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_plan_init(d, 1, wl.COL_SHAPE, s.k + 1)[0] == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_plan_init(d, 1, wl.COL_CHANNEL, s.cg + 1)[0] == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_plan_init(d, 1, 7, 1)[0] == sadmm.SADMM_EINVAL
+    ws = sadmm.sadmm_workspace_size(d, wl.COL_SHAPE)
+    assert ws > 0
+    fake = 1 << 20  # never dereferenced: validation fails first
+    args = dict(W=fake, U=None, wdt=0, k_filters=1, colkind=wl.COL_SHAPE, k_cols=1, filt_idx=fake,
+                col_idx=fake, keys_out=None, workspace=fake, ws_bytes=ws, stream=None)
+    for bad in (dict(k_filters=-1), dict(k_filters=s.f + 1), dict(k_cols=s.k + 1), dict(wdt=5),
+                dict(ws_bytes=ws - 1), dict(W=None), dict(col_idx=None), dict(colkind=9)):
+        a = dict(args, **bad)
+        assert sadmm.sadmm_project_groups(d, **a) == sadmm.SADMM_EINVAL, bad
+
+
+def test_conv_rejects_unbound_plan_and_nulls():
+    s = wl.single2d()[0].shape
+    st, p = sadmm.sadmm_plan_init(sadmm.make_desc(s.desc16()), s.f, wl.COL_SHAPE, 100)
+    assert st == 0
+    fake = 1 << 20
+    # plan never packed: no device buffer
+    assert sadmm.sadmm_conv_fwd(p, fake, None, 1, fake, 1, None) == sadmm.SADMM_EINVAL
+    p.dev = fake
+    assert sadmm.sadmm_conv_fwd(p, None, None, 1, fake, 1, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_conv_fwd(p, fake, None, 1, None, 1, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_conv_fwd(p, fake + 1, None, 1, fake, 1, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_conv_fwd(p, fake, None, 1, fake, 7, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_pack(p, fake, 0, None, fake, fake, p.dev_bytes - 1, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_pack(p, fake, 0, None, fake, fake + 8, p.dev_bytes, None) == sadmm.SADMM_EINVAL

@@ -1,0 +1,82 @@
+"""GPU parity of sadmm_project_groups against the oracle (index lists bit-exact,
+keys to fp64 rounding)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads as wl
+from workloads import ConvShape
+
+from _helpers import gpu_project
+
+pytestmark = pytest.mark.gpu
+
+TINY = [
+    ConvShape(n=1, c=3, h=4, w=4, f=6, kh=2, kw=2),
+    ConvShape(n=1, c=4, h=4, w=4, f=4, kh=3, kw=1, groups=2),
+    ConvShape(n=1, c=2, t=3, h=3, w=3, f=5, kt=2, kh=1, kw=3),
+    ConvShape(n=1, c=33, h=5, w=5, f=70, kh=3, kw=3, ph=1, pw=1),
+]
+
+
+def _check(shape, W, kf, ck, kc, U=None):
+    fi, ci, keys = gpu_project(shape, W.cuda(), kf, ck, kc, U=None if U is None else U.cuda())
+    rows, cols, fk, ckeys = oracle.project(W, shape.taps, kf, ck, kc, U=U)
+    assert np.array_equal(fi, rows), "filter index list"
+    if ck != wl.COL_NONE:
+        assert np.array_equal(ci, cols), "column index list"
+    F = shape.f
+    assert np.allclose(keys[:F], fk, rtol=1e-12, atol=0), "filter keys"
+    if ckeys is not None:
+        assert np.allclose(keys[F:], ckeys, rtol=1e-12, atol=1e-300), "column keys"
+
+
+@pytest.mark.parametrize("si", range(len(TINY)))
+@pytest.mark.parametrize("ck", [wl.COL_NONE, wl.COL_SHAPE, wl.COL_CHANNEL])
+def test_tiny_all_k(si, ck):
+    s = TINY[si]
+    t = wl.gen_tensors(s, seed=40 + si)
+    G = s.k if ck == wl.COL_SHAPE else s.cg
+    for kf in sorted({0, 1, s.f // 2, s.f}):
+        for kc in sorted({0, 1, G // 3, G}):
+            _check(s, t["W"], kf, ck, kc if ck != wl.COL_NONE else 0)
+
+
+def test_dual_and_fp32_weights():
+    s = TINY[3]
+    t = wl.gen_tensors(s, seed=3)
+    U = wl.gen_dual(s, seed=3, scale=0.05)
+    _check(s, t["W"], 35, wl.COL_SHAPE, 100, U=U)
+    W32 = t["W"].float() * 1.37
+    _check(s, W32, 20, wl.COL_CHANNEL, 9)
+
+
+def test_ties_resolved_by_index():
+    """Integer weights: every key is an exact small integer on both sides, so
+    equal keys are common and the lower index must win."""
+    s = ConvShape(n=1, c=40, h=5, w=5, f=300, kh=3, kw=3, ph=1, pw=1)
+    W = wl.gen_integer_weights(s, seed=5, lo=-1, hi=1)
+    for kf, kc in ((150, 100), (7, 359), (299, 1)):
+        _check(s, W, kf, wl.COL_SHAPE, kc)
+        _check(s, W, kf, wl.COL_CHANNEL, min(kc, s.cg))
+    Wz = torch.zeros(s.w_shape(), dtype=torch.bfloat16)
+    _check(s, Wz, 10, wl.COL_SHAPE, 17)  # all keys zero: lowest indices
+
+
+ALL = wl.single2d() + wl.alexnet() + wl.resnet50() + wl.c3d() + wl.sweep()
+
+
+@pytest.mark.parametrize("layer", ALL, ids=lambda l: l.name)
+def test_workload_layers(layer):
+    s = layer.shape
+    t = wl.gen_tensors(s.with_batch(1), seed=layer.seed)
+    _check(s, t["W"], layer.k_filters, layer.colkind, layer.k_cols)
+
+
+def test_large_group_count():
+    """More groups than one block pass of the select (several compaction chunks)."""
+    s = ConvShape(n=1, c=512, h=3, w=3, f=1500, kh=3, kw=3, ph=1, pw=1)
+    t = wl.gen_tensors(s, seed=77)
+    _check(s, t["W"], 1499, wl.COL_SHAPE, 2345)
+    _check(s, t["W"], 1, wl.COL_SHAPE, s.k - 1)
