@@ -1,0 +1,484 @@
+#!/usr/bin/env python3
+"""Benchmark of the structured-pruned CONV forward path on GB300.
+
+One step = the whole path over one batch of every layer of the workload:
+sadmm_project_groups (group norms + exact top-k) -> sadmm_pack -> sadmm_conv_fwd
+(implicit GEMM on the kept filters and columns, bias + ReLU, zero planes).
+
+Default workload: AlexNet CONV1-5 at batch 128 (bf16 inputs, fp32 output),
+filter-wise plus shape-wise pruning at retained fractions 1.0/0.5/0.25/0.2/0.2
+(each applied to filters and columns), seeded synthetic tensors.
+
+Metric: TFLOP/s on retained MACs (2 * M * F' * K' per layer) over the step,
+plus the fraction of the measured bf16 tensor peak and the speedup over the
+same step at 0% sparsity.  Timing: CUDA events on the launching stream, L2
+flushed (256 MiB write) before every timed step, outside the timed window; a
+short device sleep before each step's start event lets the host enqueue ahead,
+so the window holds only GPU work.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+                       [--workload alexnet|single2d|c3d|resnet50|sweep]
+                       [--out-dtype fp32|bf16]
+Under torchrun (N > 1) every rank runs its own batch (weak scaling, no
+collective on the data path); rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import workloads as wl  # noqa: E402
+
+METRIC = "pruned-conv TFLOP/s (retained MACs) & % bf16 peak; speedup vs dense"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as fh:
+            d = json.load(fh)
+        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def workload_name(name, layers, out_dtype):
+    desc = {
+        "alexnet": "AlexNet CONV1-5, batch 128, filter-wise + shape-wise pruning, retained 1.0/0.5/0.25/0.2/0.2",
+        "single2d": "single 2-D CONV N8 C64 32x32 F64 3x3, shape-wise 50%",
+        "c3d": "C3D layer N8 C128 T8 28x28 F256 3x3x3, shape-wise 30%",
+        "resnet50": "ResNet-50 bottleneck CONV layers, batch 64, filter-wise 50% + channel-wise 50%",
+        "sweep": "N128 C256 28x28 F512 3x3, shape-wise {1,.5,.25,.1,.05} x filter-wise {1,.5}",
+    }[name]
+    return f"{desc} ({out_dtype} output)"
+
+
+# --------------------------------------------------------------------------
+# Reference arm: the CPU oracle as it stands
+# --------------------------------------------------------------------------
+
+def oracle_sample_step(layers, tensors, nimg):
+    """The path through the oracle on images 0..nimg-1 of every layer; returns
+    the retained FLOPs of that sample."""
+    import oracle
+    flops = 0.0
+    for L, t in zip(layers, tensors):
+        s = L.shape
+        rows, cols, _, _ = oracle.project(t["W"], s.taps, L.k_filters, L.colkind, L.k_cols)
+        d = s.with_batch(int(t["x"].shape[0])).desc16()
+        oracle.pruned_conv(t["x"], t["W"], t["bias"], d, s.taps, rows, L.colkind, cols,
+                           relu=True, n0=0, n1=nimg)
+        flops += L.retained_flops() * nimg / s.n
+    return flops
+
+
+def oracle_threads():
+    try:
+        import oracle
+        lib = oracle._load()
+        import ctypes
+        omp = ctypes.CDLL(lib._name)
+        f = getattr(omp, "omp_get_max_threads", None)
+        if f is not None:
+            return int(f())
+    except Exception:
+        pass
+    return os.cpu_count() or 1
+
+
+def cpu_baseline(layers, tensors, target_s=10.0, max_img=16):
+    """Times the oracle on a bounded sample (images 0..n-1 of every layer)."""
+    t0 = time.perf_counter()
+    f1 = oracle_sample_step(layers, tensors, 1)
+    dt1 = time.perf_counter() - t0
+    nimg = max(1, min(max_img, min(L.shape.n for L in layers), int(target_s / max(dt1, 1e-3))))
+    if nimg > 1:
+        t0 = time.perf_counter()
+        f = oracle_sample_step(layers, tensors, nimg)
+        dt = time.perf_counter() - t0
+    else:
+        f, dt = f1, dt1
+    return {"value": f / dt / 1e12, "unit": "TFLOP/s", "cores": oracle_threads(), "kind": "oracle",
+            "sample": f"images 0..{nimg - 1} of every layer through oracle.project + oracle.pruned_conv "
+                      f"(fp64 direct convolution over the full masked weights), {dt:.1f} s"}
+
+
+def run_reference(args):
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    layers = wl.get(args.workload)
+    tensors = [wl.gen_tensors(L.shape.with_batch(1), seed=L.seed) for L in layers]
+    # each step is one image of every layer (a bounded sample of the workload)
+    for _ in range(args.warmup):
+        oracle_sample_step(layers, tensors, 1)
+    times, flops = [], 0.0
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        flops = oracle_sample_step(layers, tensors, 1)
+        times.append(time.perf_counter() - t0)
+    tot = sum(times)
+    value = flops * args.steps / tot / 1e12
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": tot / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": workload_name(args.workload, layers, "fp64"),
+                   "sample": "image 0 of every layer per step"},
+        "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": oracle_threads(), "kind": "oracle",
+                         "sample": "image 0 of every layer per step"},
+        "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# --------------------------------------------------------------------------
+# GPU arm
+# --------------------------------------------------------------------------
+
+class LayerRun:
+    """Device buffers and raw-pointer arguments of one layer's path."""
+
+    def __init__(self, L, t, dev, out_dtype, dense=False):
+        import torch
+        from paper_1807_11091_gb300 import sadmm
+        self.L = L
+        s = L.shape
+        self.s = s
+        self.dense = dense
+        self.k_filters = s.f if dense else L.k_filters
+        self.colkind = L.colkind
+        G = s.cg if L.colkind == wl.COL_CHANNEL else s.k
+        self.k_cols = (G if dense else L.k_cols) if L.colkind != wl.COL_NONE else 0
+        self.n_cg = self.k_cols if L.colkind != wl.COL_NONE else s.k
+        self.W = t["W"].to(dev)
+        self.x = t["x"].to(dev)
+        self.bias = t["bias"].to(dev)
+        self.desc = sadmm.make_desc(s.desc16())
+        self.ws_bytes = sadmm.sadmm_workspace_size(self.desc, self.colkind)
+        self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=dev)
+        self.fi = torch.empty(max(s.f, 1), dtype=torch.int32, device=dev)
+        self.ci = torch.empty(max(G, 1), dtype=torch.int32, device=dev)
+        st, self.plan = sadmm.sadmm_plan_init(self.desc, self.k_filters, self.colkind, self.n_cg)
+        assert st == 0, st
+        self.buf = torch.empty(self.plan.dev_bytes, dtype=torch.uint8, device=dev)
+        self.ydt = sadmm.SADMM_BF16 if out_dtype == "bf16" else sadmm.SADMM_FP32
+        ytype = torch.bfloat16 if out_dtype == "bf16" else torch.float32
+        self.y = torch.empty(s.y_shape(), dtype=ytype, device=dev)
+        self.out_bytes = 2 if out_dtype == "bf16" else 4
+        self.launches = (2 + (2 if self.colkind != wl.COL_NONE else 0)) + 2 + 1
+
+    def flops(self):
+        s = self.s
+        return 2.0 * s.m * self.k_filters * (self.k_cols * (s.taps if self.colkind == wl.COL_CHANNEL else 1)
+                                            if self.colkind != wl.COL_NONE else s.k)
+
+    def conv_bytes(self):
+        """Algorithmic HBM bytes of one conv launch: x once, packed weights once,
+        the full output once, the bias."""
+        s = self.s
+        kc = self.flops() / (2.0 * s.m * max(self.k_filters, 1)) if self.k_filters else 0
+        return (s.n * s.c * s.t * s.h * s.w * 2 + self.k_filters * kc * 2
+                + s.n * s.f * s.plane * self.out_bytes + s.f * 4)
+
+    def project(self, stream):
+        from paper_1807_11091_gb300 import sadmm
+        st = sadmm.sadmm_project_groups(self.desc, self.W.data_ptr(), None, sadmm.SADMM_BF16, self.k_filters,
+                                        self.colkind, self.k_cols, self.fi.data_ptr(),
+                                        self.ci.data_ptr() if self.colkind != wl.COL_NONE else None, None,
+                                        self.ws.data_ptr(), self.ws_bytes, stream)
+        assert st == 0, st
+
+    def pack(self, stream):
+        from paper_1807_11091_gb300 import sadmm
+        st = sadmm.sadmm_pack(self.plan, self.W.data_ptr(), sadmm.SADMM_BF16,
+                              self.fi.data_ptr() if self.k_filters < self.s.f else None,
+                              self.ci.data_ptr() if self.colkind != wl.COL_NONE else None,
+                              self.buf.data_ptr(), self.plan.dev_bytes, stream)
+        assert st == 0, st
+
+    def conv(self, stream):
+        from paper_1807_11091_gb300 import sadmm
+        st = sadmm.sadmm_conv_fwd(self.plan, self.x.data_ptr(), self.bias.data_ptr(), 1, self.y.data_ptr(),
+                                  self.ydt, stream)
+        assert st == 0, st
+
+
+def enqueue_step(runs, stream, conv_events=None):
+    for i, r in enumerate(runs):
+        r.project(stream)
+        r.pack(stream)
+        if conv_events is not None:
+            conv_events[i][0].record()
+        r.conv(stream)
+        if conv_events is not None:
+            conv_events[i][1].record()
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clock, power and throttle reasons."""
+
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index, path=None):
+        self.index = index
+        self.proc = None
+        self.lines = []
+        self.path = path
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-i",
+                 str(self.index), "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        self.lines = [ln for ln in out.splitlines() if ln.strip()]
+        if self.path:
+            try:
+                with open(self.path, "w") as fh:
+                    fh.write(self.FIELDS + "\n" + "\n".join(self.lines) + "\n")
+            except Exception:
+                pass
+
+    def summary(self):
+        sm, mx, reasons, power = [], None, set(), []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 10:
+                continue
+            try:
+                clk = float(f[2])
+                mx = float(f[3])
+            except ValueError:
+                continue
+            try:
+                power.append(float(f[4]))
+            except ValueError:
+                pass
+            sm.append(clk)
+            for nm, v in zip(names, f[6:10]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        loaded = [c for c, p in zip(sm, power)] if power else sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm), "power_w_max": max(power) if power else None}
+
+
+def run_gpu(args):
+    import torch
+    ws, rank, local = dist_env()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_1807_11091_gb300 import sadmm
+    sadmm.load()
+    stream = torch.cuda.current_stream()
+    sp = int(stream.cuda_stream)
+
+    layers = wl.get(args.workload)
+    tensors = [wl.gen_tensors(L.shape, seed=L.seed + 1000 * rank) for L in layers]
+    runs = [LayerRun(L, t, dev, args.out_dtype) for L, t in zip(layers, tensors)]
+    dense = [LayerRun(L, t, dev, args.out_dtype, dense=True) for L, t in zip(layers, tensors)]
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    peaks, peak_src = load_peaks()
+
+    def timed_steps(rs, k, with_conv_events):
+        step_ms, conv_ms = [], [[] for _ in rs]
+        for _ in range(k):
+            flush.fill_(1)
+            torch.cuda._sleep(3_000_000)  # ~1.5-2 ms: host enqueues the step meanwhile
+            ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in rs] \
+                if with_conv_events else None
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+            enqueue_step(rs, sp, ev)
+            e1.record()
+            torch.cuda.synchronize()
+            step_ms.append(e0.elapsed_time(e1))
+            if ev:
+                for i, (a, b) in enumerate(ev):
+                    conv_ms[i].append(a.elapsed_time(b))
+        return step_ms, conv_ms
+
+    # warm-up (also the first-call setup of every kernel)
+    for _ in range(max(args.warmup, 3)):
+        enqueue_step(runs, sp)
+        enqueue_step(dense, sp)
+    torch.cuda.synchronize()
+    st = sadmm.sadmm_last_device_status(sp)
+    if st != 0:
+        raise RuntimeError(f"device status {st} after warm-up")
+
+    os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
+    clocks = ClockSampler(local, os.path.join(ROOT, "gpurun_out", f"bench_clocks_rank{rank}.csv"))
+    clocks.start()
+    # clock soak: the same steps, untimed, so the sampler sees the load before the window
+    t_end = time.time() + 1.0
+    while time.time() < t_end:
+        enqueue_step(runs, sp)
+        torch.cuda.synchronize()
+
+    if ws > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    step_ms, conv_ms = timed_steps(runs, args.steps, True)
+    torch.cuda.synchronize()
+    if ws > 1:
+        torch.distributed.barrier()
+    clocks.stop()
+    dense_ms, dense_conv_ms = timed_steps(dense, max(3, min(args.steps, 10)), True)
+
+    # end to end through the C ABI with host buffers: pinned H2D of every input,
+    # the step, D2H of every output
+    h_x = [r.x.cpu().pin_memory() for r in runs]
+    h_w = [r.W.cpu().pin_memory() for r in runs]
+    h_b = [r.bias.cpu().pin_memory() for r in runs]
+    h_y = [torch.empty(r.y.shape, dtype=r.y.dtype).pin_memory() for r in runs]
+    h2d = sum(a.numel() * a.element_size() for a in h_x + h_w + h_b)
+    d2h = sum(a.numel() * a.element_size() for a in h_y)
+    e2e_ms = []
+    for _ in range(max(2, min(args.steps, 10))):
+        flush.fill_(1)
+        torch.cuda._sleep(3_000_000)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for r, a, b, c in zip(runs, h_x, h_w, h_b):
+            r.x.copy_(a, non_blocking=True)
+            r.W.copy_(b, non_blocking=True)
+            r.bias.copy_(c, non_blocking=True)
+        enqueue_step(runs, sp)
+        for r, hy in zip(runs, h_y):
+            hy.copy_(r.y, non_blocking=True)
+        e1.record()
+        torch.cuda.synchronize()
+        e2e_ms.append(e0.elapsed_time(e1))
+    st = sadmm.sadmm_last_device_status(sp)
+    if st != 0:
+        raise RuntimeError(f"device status {st} after the timed steps")
+
+    # max over ranks of the timed totals
+    tot_ms = sum(step_ms)
+    if ws > 1:
+        t = torch.tensor([tot_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        tot_ms = float(t.item())
+
+    flops_step = sum(r.flops() for r in runs)
+    value = flops_step * ws * args.steps / (tot_ms * 1e-3) / 1e12
+    ms_per_step = tot_ms / args.steps
+    dense_step = statistics.median(dense_ms)
+    pruned_step_med = statistics.median(step_ms)
+    conv_avg = [statistics.mean(c) for c in conv_ms]
+    dense_conv_avg = [statistics.mean(c) for c in dense_conv_ms]
+
+    # roofline of the dominant kernel (sadmm_conv_fwd over the step's launches)
+    conv_bytes = [r.conv_bytes() for r in runs]
+    conv_flops = [r.flops() for r in runs]
+    t_conv = sum(conv_avg) * 1e-3
+    t_mem = sum(conv_bytes) / (peaks["hbm_gbs"] * 1e9)
+    t_cmp = sum(conv_flops) / (peaks["bf16_tflops"] * 1e12)
+    if t_mem >= t_cmp:
+        achieved = sum(conv_bytes) / len(runs) / (t_conv / len(runs)) / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / peaks["hbm_gbs"]}
+    else:
+        achieved = sum(conv_flops) / t_conv / 1e12
+        roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                "frac": achieved / peaks["bf16_tflops"]}
+    roof["traffic"] = None
+    roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
+    roof["kernel"] = "k_conv_fwd (sadmm_conv_fwd), averaged over the step's launches"
+    roof["combined_roofline_frac"] = max(t_mem, t_cmp) / t_conv
+
+    e2e_value = flops_step * ws / (statistics.median(e2e_ms) * 1e-3) / 1e12
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": workload_name(args.workload, layers, args.out_dtype),
+                   "layers": [L.name for L in layers],
+                   "out_dtype": args.out_dtype,
+                   "l2": "flushed before every timed step (256 MiB write, outside the timed window)",
+                   "parallelism": "one replica per GPU, batch per GPU fixed, no collective"},
+        "pct_bf16_peak": value / peaks["bf16_tflops"],
+        "speedup_vs_dense": dense_step / pruned_step_med,
+        "conv_speedup_vs_dense": sum(dense_conv_avg) / sum(conv_avg),
+        "conv_tflops": sum(conv_flops) / t_conv / 1e12,
+        "breakdown_us": {L.name: {"conv": c * 1e3, "dense_conv": d * 1e3}
+                         for L, c, d in zip(layers, conv_avg, dense_conv_avg)},
+        "roofline": roof,
+        "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": statistics.median(e2e_ms)},
+        "gpu_launches": sum(r.launches for r in runs) * args.steps,
+        "clocks": clocks.summary(),
+    }
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(layers, [wl.gen_tensors(L.shape.with_batch(16), seed=L.seed)
+                                                     for L in layers])
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="alexnet", choices=sorted(wl.WORKLOADS))
+    ap.add_argument("--out-dtype", default="fp32", choices=["fp32", "bf16"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())
