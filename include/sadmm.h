@@ -142,7 +142,7 @@ sadmm_status sadmm_project_groups(const sadmm_conv_desc* d, const void* W, const
  * (columns or channels) of kind `colkind`.  Fills every size field of `plan`,
  * including plan->dev_bytes, the device buffer sadmm_pack needs.  Host only;
  * enqueues nothing.  SADMM_EUNSUPPORTED when the packed row count per conv
- * group would exceed 4096 or K' would exceed 65536.
+ * group would exceed 4096 or K' would exceed 8192.
  */
 sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d,
                              int n_filt, int colkind, int n_colgroups);
@@ -158,7 +158,7 @@ sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d,
  *             n_filt == F (all filters).
  *   col_idx   device int32 [plan->n_colgroups], ascending: columns in [0,K)
  *             (shape) or channels in [0,Cg) (channel); NULL for COL_NONE.
- *   dev       device buffer of >= plan->dev_bytes bytes, 1024-byte aligned;
+ *   dev       device buffer of >= plan->dev_bytes bytes, 256-byte aligned;
  *             becomes plan->dev.
  * Writes the TMA descriptor of Wp into plan->tmap.  Index lists that are not
  * ascending or out of range give undefined (but in-bounds) plans.

@@ -163,7 +163,7 @@ sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d, int n_f
     } else {
         return SADMM_EINVAL;
     }
-    if (n_cols > 65536) return SADMM_EUNSUPPORTED;
+    if (n_cols > 8192) return SADMM_EUNSUPPORTED;
     sadmm_plan p;
     memset(&p, 0, sizeof(p));
     p.desc = *d;
@@ -188,7 +188,7 @@ sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d, int n_f
         return at;
     };
     p.off_wp = take((size_t)g.groups * p.n_pad * p.k_pad * 2);
-    p.off_gather = take((size_t)p.k_pad * 16);
+    p.off_gather = take((size_t)p.k_pad * 8);
     p.off_colidx = take((size_t)p.k_pad * 4);
     p.off_rowmap = take((size_t)g.groups * p.n_pad * 4);
     p.off_zeromap = take((size_t)g.f * 4);

@@ -39,7 +39,7 @@ constexpr int kEpiWarps = 4;
 constexpr int kThreads = (4 + kEpiWarps + kGatherWarps) * 32;
 constexpr int kGatherThreads = kGatherWarps * 32;
 constexpr int kATileBytes = kBM * kBK * 2;  // 16 KB
-constexpr int kMaxStages = 8;
+constexpr int kMaxStages = 4;
 constexpr int kMaxGroups = 64;
 constexpr int kSmemTail = 2048;  // barriers, TMEM address, counts
 
@@ -47,7 +47,7 @@ struct ConvArgs {
     const __nv_bfloat16* x;
     void* y;
     const float* bias;
-    const int4* gather;
+    const uint2* gather;  // [k_pad] {channel/tap offset in x, tap bits}
     const int* rowmap;
     const int* zeromap;
     const int* counts;
@@ -64,6 +64,7 @@ struct ConvArgs {
     int nks;  // k_pad / 64
     int bn, n_tiles, n_pad;
     int stages;
+    int k_pad;
     int tmem_stride;
     int tmem_cols;
     int relu;
@@ -103,11 +104,14 @@ SADMM_DEV void pixel_masks(const ConvArgs& a, int it0, int ih0, int iw0, uint32_
     }
 }
 
+// Whether gather entry `e` reads inside the input for the pixel whose masks are
+// (m0, m1).  MODE 0: e.y = 1 << tap.  MODE 1: e.y = row | kw << 8 | 1 << 16
+// (0 for a padding column).
 template <int MODE>
-SADMM_DEV bool tap_ok(const int4& e, uint32_t m0, uint32_t m1)
+SADMM_DEV bool tap_ok(const uint2& e, uint32_t m0, uint32_t m1)
 {
-    if (MODE == 0) return (m0 & (uint32_t)e.y) != 0u;
-    return ((m0 & (uint32_t)e.y) != 0u) & ((m1 & (uint32_t)e.z) != 0u);
+    if (MODE == 0) return (m0 & e.y) != 0u;
+    return (((m0 >> (e.y & 31u)) & (m1 >> ((e.y >> 8) & 31u)) & (e.y >> 16)) & 1u) != 0u;
 }
 
 template <int MODE, bool OUT_BF16>
@@ -120,7 +124,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t b_bytes = (uint32_t)a.bn * 128u;
     uint8_t* sA = smem;
     uint8_t* sB = smem + (size_t)S * kATileBytes;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sB + (size_t)S * b_bytes);
+    uint2* s_table = reinterpret_cast<uint2*>(sB + (size_t)S * b_bytes);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(s_table + a.k_pad);
     uint64_t* full_a = bars;
     uint64_t* full_b = bars + S;
     uint64_t* empty = bars + 2 * S;
@@ -148,6 +153,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         fence_mbar_init();
     }
     for (int i = threadIdx.x; i < 2 * a.groups; i += blockDim.x) s_counts[i] = a.counts[i];
+    {
+        // the gather table is the same for every tile: keep it in shared memory
+        const uint4* src = reinterpret_cast<const uint4*>(a.gather);
+        uint4* dst = reinterpret_cast<uint4*>(s_table);
+        for (int i = threadIdx.x; i < a.k_pad / 2; i += blockDim.x) dst[i] = __ldg(src + i);
+    }
     if (warp == 0 && lane == 0) tma_prefetch_desc(&tmap);
     if (warp == 1) {
         tmem_alloc(tmem_holder, (uint32_t)a.tmem_cols);
@@ -328,23 +339,28 @@ __global__ void __launch_bounds__(kThreads, 1)
                            (long long)ih0 * a.W + iw0);
             }
             for (int ks = 0; ks < a.nks; ++ks) {
+                // Issue every load of this thread's 32 columns first (they read
+                // only x), then wait for the stage buffer and store.
+                const uint2* te = s_table + (size_t)ks * kBK;
+                uint32_t v[32];
+#pragma unroll
+                for (int ci = 0; ci < 4; ++ci) {
+                    const int c = chunk0 + 2 * ci;
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const uint2 t = te[c * 8 + e];
+                        v[ci * 8 + e] = tap_ok<MODE>(t, m0, m1) ? (uint32_t)__ldg(xb + (int)t.x) : 0u;
+                    }
+                }
                 if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, a.status)) { ok = false; break; }
-                const int4* ge = a.gather + (size_t)ks * kBK;
                 uint8_t* tile = sA + (size_t)s * kATileBytes;
 #pragma unroll
                 for (int ci = 0; ci < 4; ++ci) {
                     const int c = chunk0 + 2 * ci;
-                    uint32_t w[4];
-#pragma unroll
-                    for (int e2 = 0; e2 < 4; ++e2) {
-                        const int4 e0 = __ldg(ge + c * 8 + 2 * e2);
-                        const int4 e1 = __ldg(ge + c * 8 + 2 * e2 + 1);
-                        const uint32_t v0 = tap_ok<MODE>(e0, m0, m1) ? (uint32_t)__ldg(xb + e0.x) : 0u;
-                        const uint32_t v1 = tap_ok<MODE>(e1, m0, m1) ? (uint32_t)__ldg(xb + e1.x) : 0u;
-                        w[e2] = v0 | (v1 << 16);
-                    }
+                    const uint32_t* q = v + ci * 8;
                     *reinterpret_cast<uint4*>(tile + sw128_offset((uint32_t)prow, (uint32_t)c)) =
-                        make_uint4(w[0], w[1], w[2], w[3]);
+                        make_uint4(q[0] | (q[1] << 16), q[2] | (q[3] << 16), q[4] | (q[5] << 16),
+                                   q[6] | (q[7] << 16));
                 }
                 fence_proxy_async_smem();
                 mbar_arrive(&full_a[s]);
@@ -388,7 +404,7 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     a.x = static_cast<const __nv_bfloat16*>(x);
     a.y = y;
     a.bias = bias;
-    a.gather = reinterpret_cast<const int4*>(base + plan->off_gather);
+    a.gather = reinterpret_cast<const uint2*>(base + plan->off_gather);
     a.rowmap = reinterpret_cast<const int*>(base + plan->off_rowmap);
     a.zeromap = reinterpret_cast<const int*>(base + plan->off_zeromap);
     a.counts = reinterpret_cast<const int*>(base + plan->off_counts);
@@ -424,8 +440,11 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     const long long m_tiles = (g.m + kBM - 1) / kBM;
     a.units = m_tiles * g.groups * plan->n_tiles;
 
+    a.k_pad = plan->k_pad;
     const int stage_bytes = kATileBytes + plan->bn * 128;
-    const int budget = 232448 - 1024 - kSmemTail;
+    const int table_bytes = plan->k_pad * 8;
+    const int budget = 232448 - 1024 - kSmemTail - table_bytes;
+    // At most kMaxStages: what shared memory leaves over serves as L1 for x.
     a.stages = budget / stage_bytes;
     if (a.stages > kMaxStages) a.stages = kMaxStages;
     if (a.stages < 2) return SADMM_EUNSUPPORTED;
@@ -433,7 +452,7 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     int cols = 32;
     while (cols < 2 * a.tmem_stride) cols <<= 1;
     a.tmem_cols = cols;
-    const size_t smem = 1024 + (size_t)a.stages * stage_bytes + kSmemTail;
+    const size_t smem = 1024 + (size_t)a.stages * stage_bytes + table_bytes + kSmemTail;
 
     long long grid = device_sm_count();
     if (grid > a.units) grid = a.units;

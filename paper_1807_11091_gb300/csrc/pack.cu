@@ -28,7 +28,7 @@ struct PackArgs {
     int hw, W;
     int k_pad, n_pad;
     int mask_mode;
-    int4* gather;
+    uint2* gather;
     int* colidx;
     int* rowmap;
     int* zeromap;
@@ -81,7 +81,7 @@ __global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status)
         for (int f = tid; f < a.F; f += blockDim.x) a.zeromap[f] = f;
         for (int j = tid; j < a.k_pad; j += blockDim.x) {
             a.colidx[j] = -1;
-            a.gather[j] = make_int4(0, 0, 0, 0);
+            a.gather[j] = make_uint2(0u, 0u);
         }
         return;
     }
@@ -123,17 +123,15 @@ __global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status)
             else col = j;
         }
         a.colidx[j] = col;
-        int4 e = make_int4(0, 0, 0, 0);
+        uint2 e = make_uint2(0u, 0u);
         if (col >= 0) {
             const int c = col / a.taps, r = col % a.taps;
             const int kt = r / (a.KH * a.KW), kh = (r / a.KW) % a.KH, kw = r % a.KW;
-            e.x = (int)(c * a.thw + (long long)kt * a.hw + kh * a.W + kw);
-            if (a.mask_mode == 0) {
-                e.y = (int)(1u << r);
-            } else {
-                e.y = (int)(1u << (kt * a.KH + kh));
-                e.z = (int)(1u << kw);
-            }
+            e.x = (uint32_t)(c * a.thw + (long long)kt * a.hw + kh * a.W + kw);
+            if (a.mask_mode == 0)
+                e.y = 1u << r;
+            else
+                e.y = (uint32_t)(kt * a.KH + kh) | ((uint32_t)kw << 8) | (1u << 16);
         }
         a.gather[j] = e;
     }
@@ -212,7 +210,7 @@ sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int
     a.k_pad = plan->k_pad;
     a.n_pad = plan->n_pad;
     a.mask_mode = tap_mask_mode(g);
-    a.gather = reinterpret_cast<int4*>(base + plan->off_gather);
+    a.gather = reinterpret_cast<uint2*>(base + plan->off_gather);
     a.colidx = reinterpret_cast<int*>(base + plan->off_colidx);
     a.rowmap = reinterpret_cast<int*>(base + plan->off_rowmap);
     a.zeromap = reinterpret_cast<int*>(base + plan->off_zeromap);
