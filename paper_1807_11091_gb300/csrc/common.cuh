@@ -11,7 +11,7 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
-#include "../../include/sadmm.h"
+#include "sadmm.h"
 
 #define SADMM_DEV __device__ __forceinline__
 

@@ -65,6 +65,9 @@ struct ConvArgs {
     int bn, n_tiles, n_pad;
     int stages;
     int k_pad;
+    int n_cols;          // K' (columns past it are padding)
+    int split_mask;      // tap-mask encoding: 0 one bit per tap, 1 row bits + kw bits
+    uint32_t full_mask;  // the mask of a pixel whose every tap is inside the input
     int tmem_stride;
     int tmem_cols;
     int relu;
@@ -78,11 +81,11 @@ SADMM_DEV void decode_unit(const ConvArgs& a, long long u, int& nt, int& g, long
     mt = t / a.groups;
 }
 
-// Tap-validity masks of one output pixel: bit set where the tap reads inside
-// the input.  MODE 0: bit (kt*KH + kh)*KW + kw.  MODE 1: rmask bit kt*KH + kh,
-// cmask bit kw.
-template <int MODE>
-SADMM_DEV void pixel_masks(const ConvArgs& a, int it0, int ih0, int iw0, uint32_t& m0, uint32_t& m1)
+// Tap-validity mask of one output pixel: a bit is set where a tap reads inside
+// the input.  One bit per tap t = (kt*KH + kh)*KW + kw when the kernel has at
+// most 31 taps; otherwise bits 0..15 mark valid rows kt*KH + kh and bits
+// 16..30 valid kw.  Bit 31 is never set (it marks padding columns).
+SADMM_DEV uint32_t pixel_mask(const ConvArgs& a, int it0, int ih0, int iw0)
 {
     uint32_t rm = 0, cm = 0;
     for (int kt = 0; kt < a.KT; ++kt) {
@@ -92,29 +95,18 @@ SADMM_DEV void pixel_masks(const ConvArgs& a, int it0, int ih0, int iw0, uint32_
     }
     for (int kw = 0; kw < a.KW; ++kw)
         if ((unsigned)(iw0 + kw) < (unsigned)a.W) cm |= 1u << kw;
-    if (MODE == 0) {
-        uint32_t m = 0;
-        for (int r = 0; r < a.KT * a.KH; ++r)
-            if (rm & (1u << r)) m |= cm << (r * a.KW);
-        m0 = m;
-        m1 = 0;
-    } else {
-        m0 = rm;
-        m1 = cm;
-    }
+    if (a.split_mask) return rm | (cm << 16);
+    uint32_t m = 0;
+    for (int r = 0; r < a.KT * a.KH; ++r)
+        if (rm & (1u << r)) m |= cm << (r * a.KW);
+    return m;
 }
 
-// Whether gather entry `e` reads inside the input for the pixel whose masks are
-// (m0, m1).  MODE 0: e.y = 1 << tap.  MODE 1: e.y = row | kw << 8 | 1 << 16
-// (0 for a padding column).
-template <int MODE>
-SADMM_DEV bool tap_ok(const uint2& e, uint32_t m0, uint32_t m1)
-{
-    if (MODE == 0) return (m0 & e.y) != 0u;
-    return (((m0 >> (e.y & 31u)) & (m1 >> ((e.y >> 8) & 31u)) & (e.y >> 16)) & 1u) != 0u;
-}
+// Gather entry e = {offset in x, tap bits}: the column reads inside the input
+// for a pixel of mask M when every tap bit of the entry is set in M.
+SADMM_DEV bool tap_ok(uint32_t bits, uint32_t M) { return (M & bits) == bits; }
 
-template <int MODE, bool OUT_BF16>
+template <bool OUT_BF16>
 __global__ void __launch_bounds__(kThreads, 1)
     k_conv_fwd(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ ConvArgs a)
 {
@@ -271,15 +263,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t taddr = tmem_base + (uint32_t)(ab * a.tmem_stride) + ((uint32_t)(q * 32) << 16);
                 const int* rmap = a.rowmap + (long long)g * a.n_pad + (long long)nt * a.bn;
                 for (int c0 = 0; c0 < nrows; c0 += 32) {
+                    // filter index and bias of column c0 + lane, shared by shuffles
+                    const bool live = c0 + lane < nrows;
+                    const int f_l = live ? __ldg(rmap + c0 + lane) : 0;
+                    const float b_l = (live && a.bias) ? __ldg(a.bias + f_l) : 0.0f;
                     uint32_t r[32];
                     tmem_ld_32x32b_x32(taddr + (uint32_t)c0, r);
                     tmem_ld_wait();
 #pragma unroll
                     for (int j = 0; j < 32; ++j) {
+                        const int f = __shfl_sync(0xffffffffu, f_l, j);
+                        const float b = __shfl_sync(0xffffffffu, b_l, j);
                         if (c0 + j < nrows) {
-                            const int f = __ldg(rmap + c0 + j);
-                            float v = __uint_as_float(r[j]);
-                            if (a.bias) v += __ldg(a.bias + f);
+                            float v = __uint_as_float(r[j]) + b;
                             if (a.relu) v = fmaxf(v, 0.0f);
                             if (valid) {
                                 const long long off = ybase + (long long)f * a.plane;
@@ -324,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             decode_unit(a, u, nt, g, mt);
             if (s_counts[2 * g] <= nt * a.bn) continue;
             const long long m = mt * kBM + prow;
-            uint32_t m0 = 0, m1 = 0;
+            uint32_t M = 0;
             const unsigned short* xb = xs;
             if (m < a.M) {
                 const long long n_img = m / a.plane;
@@ -334,22 +330,33 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int oh = r2 / a.OW;
                 const int ow = r2 - oh * a.OW;
                 const int it0 = ot * a.st - a.pt, ih0 = oh * a.sh - a.ph, iw0 = ow * a.sw - a.pw;
-                pixel_masks<MODE>(a, it0, ih0, iw0, m0, m1);
+                M = pixel_mask(a, it0, ih0, iw0);
                 xb = xs + (n_img * a.x_chw + (long long)g * a.Cg * a.thw + (long long)it0 * a.hw +
                            (long long)ih0 * a.W + iw0);
             }
+            // Every lane's pixel sees every tap: no bounds test is needed.
+            const bool interior = __all_sync(0xffffffffu, M == a.full_mask);
             for (int ks = 0; ks < a.nks; ++ks) {
                 // Issue every load of this thread's 32 columns first (they read
                 // only x), then wait for the stage buffer and store.
                 const uint2* te = s_table + (size_t)ks * kBK;
                 uint32_t v[32];
+                if (interior && (ks + 1) * kBK <= a.n_cols) {
 #pragma unroll
-                for (int ci = 0; ci < 4; ++ci) {
-                    const int c = chunk0 + 2 * ci;
+                    for (int ci = 0; ci < 4; ++ci) {
+                        const int c = chunk0 + 2 * ci;
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const uint2 t = te[c * 8 + e];
-                        v[ci * 8 + e] = tap_ok<MODE>(t, m0, m1) ? (uint32_t)__ldg(xb + (int)t.x) : 0u;
+                        for (int e = 0; e < 8; ++e) v[ci * 8 + e] = __ldg(xb + (int)te[c * 8 + e].x);
+                    }
+                } else {
+#pragma unroll
+                    for (int ci = 0; ci < 4; ++ci) {
+                        const int c = chunk0 + 2 * ci;
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            const uint2 t = te[c * 8 + e];
+                            v[ci * 8 + e] = tap_ok(t.y, M) ? (uint32_t)__ldg(xb + (int)t.x) : 0u;
+                        }
                     }
                 }
                 if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, a.status)) { ok = false; break; }
@@ -376,10 +383,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-template <int MODE, bool OUT_BF16>
+template <bool OUT_BF16>
 cudaError_t launch(const CUtensorMap& map, const ConvArgs& a, int grid, size_t smem, cudaStream_t s)
 {
-    auto kern = k_conv_fwd<MODE, OUT_BF16>;
+    auto kern = k_conv_fwd<OUT_BF16>;
     static int configured_dev = -1;
     int dev = 0;
     cudaGetDevice(&dev);
@@ -441,6 +448,12 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     a.units = m_tiles * g.groups * plan->n_tiles;
 
     a.k_pad = plan->k_pad;
+    a.n_cols = plan->n_cols;
+    a.split_mask = tap_mask_mode(g);
+    if (a.split_mask)
+        a.full_mask = ((1u << (g.kt * g.kh)) - 1u) | (((1u << g.kw) - 1u) << 16);
+    else
+        a.full_mask = (uint32_t)((1ull << g.taps) - 1ull);
     const int stage_bytes = kATileBytes + plan->bn * 128;
     const int table_bytes = plan->k_pad * 8;
     const int budget = 232448 - 1024 - kSmemTail - table_bytes;
@@ -460,14 +473,8 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
 
     CUtensorMap map;
     memcpy(&map, plan->tmap, sizeof(map));
-    const int mode = tap_mask_mode(g);
-    cudaError_t e;
-    if (mode == 0)
-        e = (ydt == SADMM_BF16) ? launch<0, true>(map, a, (int)grid, smem, s)
-                                : launch<0, false>(map, a, (int)grid, smem, s);
-    else
-        e = (ydt == SADMM_BF16) ? launch<1, true>(map, a, (int)grid, smem, s)
-                                : launch<1, false>(map, a, (int)grid, smem, s);
+    const cudaError_t e = (ydt == SADMM_BF16) ? launch<true>(map, a, (int)grid, smem, s)
+                                              : launch<false>(map, a, (int)grid, smem, s);
     return e == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
 }
 

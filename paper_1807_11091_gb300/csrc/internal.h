@@ -5,7 +5,7 @@
 #include <stddef.h>
 #include <stdint.h>
 
-#include "../../include/sadmm.h"
+#include "sadmm.h"
 
 namespace sadmm {
 
@@ -45,8 +45,9 @@ sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int
 sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const void* x, const float* bias,
                              int relu, void* y, int ydt, cudaStream_t s);
 
-// Tap-mask mode of the gather table: 0 = one 32-bit mask over all taps
-// (KT*KH*KW <= 32), 1 = a (kt,kh) row mask and a kw column mask.
-inline int tap_mask_mode(const Geometry& g) { return g.taps <= 32 ? 0 : 1; }
+// Tap-mask encoding of the gather table: 0 = one bit per tap (at most 31
+// taps), 1 = (kt,kh) row bits 0..15 and kw bits 16..30.  Bit 31 marks padding
+// columns and is never valid.
+inline int tap_mask_mode(const Geometry& g) { return g.taps <= 31 ? 0 : 1; }
 
 }  // namespace sadmm

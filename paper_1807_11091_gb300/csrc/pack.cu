@@ -81,7 +81,7 @@ __global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status)
         for (int f = tid; f < a.F; f += blockDim.x) a.zeromap[f] = f;
         for (int j = tid; j < a.k_pad; j += blockDim.x) {
             a.colidx[j] = -1;
-            a.gather[j] = make_uint2(0u, 0u);
+            a.gather[j] = make_uint2(0u, 1u << 31);
         }
         return;
     }
@@ -123,7 +123,7 @@ __global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status)
             else col = j;
         }
         a.colidx[j] = col;
-        uint2 e = make_uint2(0u, 0u);
+        uint2 e = make_uint2(0u, 1u << 31);  // padding column: never inside the input
         if (col >= 0) {
             const int c = col / a.taps, r = col % a.taps;
             const int kt = r / (a.KH * a.KW), kh = (r / a.KW) % a.KH, kw = r % a.KW;
@@ -131,7 +131,7 @@ __global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status)
             if (a.mask_mode == 0)
                 e.y = 1u << r;
             else
-                e.y = (uint32_t)(kt * a.KH + kh) | ((uint32_t)kw << 8) | (1u << 16);
+                e.y = (1u << (kt * a.KH + kh)) | (1u << (16 + kw));
         }
         a.gather[j] = e;
     }

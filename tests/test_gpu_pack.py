@@ -67,14 +67,14 @@ def test_pack_matches_index_lists(case, wdtype):
     gt = _view(pc, p.off_gather, k_pad * 8, torch.int32).numpy().reshape(k_pad, 2).view(np.uint32)
     for j in range(k_pad):
         if j >= len(kcols):
-            assert gt[j, 1] == 0
+            assert int(gt[j, 1]) == 1 << 31
             continue
         col = int(kcols[j])
         c, r = divmod(col, s.taps)
         kt, rem = divmod(r, s.kh * s.kw)
         kh, kw = divmod(rem, s.kw)
         assert gt[j, 0] == c * s.t * s.h * s.w + kt * s.h * s.w + kh * s.w + kw
-        if s.taps <= 32:
+        if s.taps <= 31:
             assert int(gt[j, 1]) == (1 << r)
         else:
-            assert int(gt[j, 1]) == (kt * s.kh + kh) | (kw << 8) | (1 << 16)
+            assert int(gt[j, 1]) == (1 << (kt * s.kh + kh)) | (1 << (16 + kw))
