@@ -83,7 +83,7 @@ sadmm_status check_desc(const sadmm_conv_desc* d, Geometry* g)
     r.m = r.n * r.plane;
     // index arithmetic limits of the kernels (32-bit offsets inside a tensor)
     if (r.n * r.c * r.t * r.h * r.w >= (1ll << 31)) return SADMM_EUNSUPPORTED;
-    if (r.f * r.k >= (1ll << 31) || r.plane >= (1ll << 31) || r.m >= (1ll << 40)) return SADMM_EUNSUPPORTED;
+    if (r.f * r.k >= (1ll << 31) || r.f * r.plane >= (1ll << 31) || r.m >= (1ll << 40)) return SADMM_EUNSUPPORTED;
     // tap-validity masks: one bit per tap, or 16 row bits + 15 kw bits
     if (r.taps > 31 && (r.kt * r.kh > 16 || r.kw > 15)) return SADMM_EUNSUPPORTED;
     if (r.groups > 64) return SADMM_EUNSUPPORTED;

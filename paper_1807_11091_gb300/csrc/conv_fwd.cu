@@ -35,13 +35,14 @@ namespace {
 constexpr int kBM = 128;           // pixels per tile
 constexpr int kBK = 64;            // GEMM columns per stage
 constexpr int kGatherWarps = 8;
-constexpr int kEpiWarps = 4;
+constexpr int kEpiWarps = 8;
 constexpr int kThreads = (4 + kEpiWarps + kGatherWarps) * 32;
 constexpr int kGatherThreads = kGatherWarps * 32;
 constexpr int kATileBytes = kBM * kBK * 2;  // 16 KB
 constexpr int kMaxStages = 4;
 constexpr int kMaxGroups = 64;
-constexpr int kSmemTail = 2048;  // barriers, TMEM address, counts
+constexpr int kPrefetchAhead = 2;  // stages of x the gather prefetches into L1 ahead
+constexpr int kSmemTail = 6144;  // barriers, TMEM address, counts, epilogue tables
 
 struct ConvArgs {
     const __nv_bfloat16* x;
@@ -106,6 +107,71 @@ SADMM_DEV uint32_t pixel_mask(const ConvArgs& a, int it0, int ih0, int iw0)
 // for a pixel of mask M when every tap bit of the entry is set in M.
 SADMM_DEV bool tap_ok(uint32_t bits, uint32_t M) { return (M & bits) == bits; }
 
+// Input rows one 128-pixel tile reads: image n, depth slices [t0, t0+nt),
+// rows [r0, r0+nr) of every channel of conv group g (clamped to the input).
+struct Footprint {
+    const char* base;  // x[n, g*Cg, 0, 0, 0]
+    int t0, nt, r0, nr;
+};
+
+SADMM_DEV Footprint tile_footprint(const ConvArgs& a, long long u)
+{
+    Footprint fp{nullptr, 0, 0, 0, 0};
+    if (u >= a.units) return fp;
+    int nt_, g;
+    long long mt;
+    decode_unit(a, u, nt_, g, mt);
+    const long long m0 = mt * kBM;
+    if (m0 >= a.M) return fp;
+    const long long n = m0 / a.plane;
+    long long m1 = min(m0 + kBM - 1, a.M - 1);
+    m1 = min(m1, (n + 1) * (long long)a.plane - 1);
+    const int p0 = (int)(m0 - n * a.plane), p1 = (int)(m1 - n * a.plane);
+    const int ot0 = p0 / a.OHW, ot1 = p1 / a.OHW;
+    int oh0 = 0, oh1 = a.OHW / a.OW - 1;
+    if (ot0 == ot1) {
+        oh0 = (p0 - ot0 * a.OHW) / a.OW;
+        oh1 = (p1 - ot1 * a.OHW) / a.OW;
+    }
+    const int r0 = max(0, oh0 * a.sh - a.ph), r1 = min(a.H - 1, oh1 * a.sh - a.ph + a.KH - 1);
+    const int t0 = max(0, ot0 * a.st - a.pt), t1 = min(a.T - 1, ot1 * a.st - a.pt + a.KT - 1);
+    if (r1 < r0 || t1 < t0) return fp;
+    fp.base = reinterpret_cast<const char*>(a.x) + 2 * (n * a.x_chw + (long long)g * a.Cg * a.thw);
+    fp.t0 = t0;
+    fp.nt = t1 - t0 + 1;
+    fp.r0 = r0;
+    fp.nr = r1 - r0 + 1;
+    return fp;
+}
+
+// Prefetches into L1 the 128-byte lines of x that stage ks of a tile with
+// footprint fp reads: every channel between the stage's first and last kept
+// column, the footprint's slices and rows.  Thread `t` of `nthr` takes every
+// nthr-th line.
+SADMM_DEV void prefetch_stage(const ConvArgs& a, const Footprint& fp, const uint2* table, int ks, int t,
+                              int nthr)
+{
+    if (!fp.base) return;
+    const int j0 = ks * kBK;
+    const int j1 = min(j0 + kBK, a.n_cols) - 1;
+    if (j1 < j0) return;
+    const int c_lo = (int)(table[j0].x / (uint32_t)a.thw);
+    const int c_hi = (int)(table[j1].x / (uint32_t)a.thw);
+    const long long bytes = 2ll * fp.nr * a.W;
+    const int per = (int)((bytes + 127) >> 7) + 1;
+    const int pairs = (c_hi - c_lo + 1) * fp.nt;
+    const int jobs = min(pairs * per, 4096);
+    for (int job = t; job < jobs; job += nthr) {
+        const int pr = job / per, i = job - pr * per;
+        const int c = c_lo + pr / fp.nt, it = fp.t0 + pr % fp.nt;
+        const char* start = fp.base + 2 * ((long long)c * a.thw + (long long)it * a.hw + (long long)fp.r0 * a.W);
+        const uintptr_t first = reinterpret_cast<uintptr_t>(start) >> 7;
+        const uintptr_t last = (reinterpret_cast<uintptr_t>(start) + bytes - 1) >> 7;
+        if (first + i <= last)
+            asm volatile("prefetch.global.L1 [%0];" ::"l"((first + i) << 7));
+    }
+}
+
 template <bool OUT_BF16>
 __global__ void __launch_bounds__(kThreads, 1)
     k_conv_fwd(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ ConvArgs a)
@@ -127,6 +193,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
     int* s_counts = reinterpret_cast<int*>(tmem_holder + 2);
+    int* s_eoff = s_counts + 2 * kMaxGroups;          // [2][256] output-plane offsets
+    float* s_ebias = reinterpret_cast<float*>(s_eoff + 512);  // [2][256] biases
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -241,10 +309,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else if (warp >= 4 && warp < 4 + kEpiWarps) {
         // --------------------------------------------------------- epilogue
+        // kEpiWarps / 4 warps share each TMEM lane quadrant and split its
+        // 32-column chunks.  Per unit, the output-plane offset and bias of every
+        // packed row go to shared memory before the accumulator wait, so the
+        // store loop reads them with broadcast loads.
+        constexpr int kHalves = kEpiWarps / 4;
         const int q = warp & 3;  // TMEM lane quadrant this warp may access
+        const int h = (warp - 4) >> 2;
+        const int et = threadIdx.x - 4 * 32;  // 0 .. kEpiWarps*32-1
         const int row = q * 32 + lane;
         int ab = 0;
         uint32_t acc_ph = 0;
+        int ub = 0;  // double-buffered per-unit tables
         for (long long u = blockIdx.x; u < a.units; u += gridDim.x) {
             int nt, g;
             long long mt;
@@ -254,35 +330,39 @@ __global__ void __launch_bounds__(kThreads, 1)
             const bool valid = m < a.M;
             const long long n_img = valid ? m / a.plane : 0;
             const long long p = valid ? m - n_img * a.plane : 0;
-            const long long ybase = n_img * (long long)a.F * a.plane + p;
+            float* yf = reinterpret_cast<float*>(a.y) + (n_img * (long long)a.F * a.plane + p);
+            __nv_bfloat16* yh = reinterpret_cast<__nv_bfloat16*>(a.y) + (n_img * (long long)a.F * a.plane + p);
+            int* u_off = s_eoff + ub * 256;
+            float* u_bias = s_ebias + ub * 256;
+            if (cnt > 0) {
+                const int* rmap = a.rowmap + (long long)g * a.n_pad + (long long)nt * a.bn;
+                for (int i = et; i < a.bn; i += kEpiWarps * 32) {
+                    const int f = __ldg(rmap + i);
+                    u_off[i] = f >= 0 ? f * a.plane : 0;
+                    u_bias[i] = (f >= 0 && a.bias) ? __ldg(a.bias + f) : 0.0f;
+                }
+            }
+            asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
             if (cnt > 0) {
                 const int nrows = min(a.bn, cnt);
                 // warp-uniform outcome: the TMEM loads below are .sync.aligned
                 if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[ab], acc_ph, abort_flag, a.status))) break;
                 tc_fence_after();
                 const uint32_t taddr = tmem_base + (uint32_t)(ab * a.tmem_stride) + ((uint32_t)(q * 32) << 16);
-                const int* rmap = a.rowmap + (long long)g * a.n_pad + (long long)nt * a.bn;
-                for (int c0 = 0; c0 < nrows; c0 += 32) {
-                    // filter index and bias of column c0 + lane, shared by shuffles
-                    const bool live = c0 + lane < nrows;
-                    const int f_l = live ? __ldg(rmap + c0 + lane) : 0;
-                    const float b_l = (live && a.bias) ? __ldg(a.bias + f_l) : 0.0f;
+                for (int c0 = 32 * h; c0 < nrows; c0 += 32 * kHalves) {
                     uint32_t r[32];
                     tmem_ld_32x32b_x32(taddr + (uint32_t)c0, r);
                     tmem_ld_wait();
+                    if (valid) {
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        const int f = __shfl_sync(0xffffffffu, f_l, j);
-                        const float b = __shfl_sync(0xffffffffu, b_l, j);
-                        if (c0 + j < nrows) {
-                            float v = __uint_as_float(r[j]) + b;
-                            if (a.relu) v = fmaxf(v, 0.0f);
-                            if (valid) {
-                                const long long off = ybase + (long long)f * a.plane;
+                        for (int j = 0; j < 32; ++j) {
+                            if (c0 + j < nrows) {
+                                float v = __uint_as_float(r[j]) + u_bias[c0 + j];
+                                if (a.relu) v = fmaxf(v, 0.0f);
                                 if (OUT_BF16)
-                                    reinterpret_cast<__nv_bfloat16*>(a.y)[off] = __float2bfloat16_rn(v);
+                                    yh[u_off[c0 + j]] = __float2bfloat16_rn(v);
                                 else
-                                    __stcs(reinterpret_cast<float*>(a.y) + off, v);
+                                    __stcs(yf + u_off[c0 + j], v);
                             }
                         }
                     }
@@ -292,18 +372,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ab ^= 1;
                 if (ab == 0) acc_ph ^= 1u;
             }
-            if (nt == 0 && valid) {
+            if (nt == 0) {
                 // pruned filters of this conv group: their planes are zero
                 const int zc = s_counts[2 * g + 1];
                 const int* zmap = a.zeromap + (long long)g * a.Fg;
-                for (int z = 0; z < zc; ++z) {
-                    const long long off = ybase + (long long)__ldg(zmap + z) * a.plane;
-                    if (OUT_BF16)
-                        reinterpret_cast<__nv_bfloat16*>(a.y)[off] = __float2bfloat16_rn(0.0f);
-                    else
-                        __stcs(reinterpret_cast<float*>(a.y) + off, 0.0f);
+                for (int z0 = 32 * h; z0 < zc; z0 += 32 * kHalves) {
+                    const int zo = (z0 + lane < zc) ? __ldg(zmap + z0 + lane) * a.plane : 0;
+                    const int zn = min(32, zc - z0);
+                    for (int j = 0; j < zn; ++j) {
+                        const int off = __shfl_sync(0xffffffffu, zo, j);
+                        if (valid) {
+                            if (OUT_BF16)
+                                yh[off] = __float2bfloat16_rn(0.0f);
+                            else
+                                __stcs(yf + off, 0.0f);
+                        }
+                    }
                 }
             }
+            ub ^= 1;
         }
     } else if (warp >= 4 + kEpiWarps) {
         // ----------------------------------------------------------- gather
@@ -314,11 +401,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         int s = 0;
         uint32_t ph = 0;
         bool ok = true;
+        bool primed = false;  // the first stages of this unit were prefetched
         for (long long u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
             int nt, g;
             long long mt;
             decode_unit(a, u, nt, g, mt);
-            if (s_counts[2 * g] <= nt * a.bn) continue;
+            if (s_counts[2 * g] <= nt * a.bn) {
+                primed = false;
+                continue;
+            }
+            const Footprint fp_cur = tile_footprint(a, u);
+            const Footprint fp_next = tile_footprint(a, u + gridDim.x);
+            if (!primed)
+                for (int q = 0; q < kPrefetchAhead && q < a.nks; ++q)
+                    prefetch_stage(a, fp_cur, s_table, q, gt, kGatherThreads);
+            primed = true;
             const long long m = mt * kBM + prow;
             uint32_t M = 0;
             const unsigned short* xb = xs;
@@ -337,6 +434,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             // Every lane's pixel sees every tap: no bounds test is needed.
             const bool interior = __all_sync(0xffffffffu, M == a.full_mask);
             for (int ks = 0; ks < a.nks; ++ks) {
+                // Lines of the stage kPrefetchAhead ahead (of the next tile when
+                // this one ends) go to L1 while this stage's loads run.
+                if (ks + kPrefetchAhead < a.nks)
+                    prefetch_stage(a, fp_cur, s_table, ks + kPrefetchAhead, gt, kGatherThreads);
+                else
+                    prefetch_stage(a, fp_next, s_table, ks + kPrefetchAhead - a.nks, gt, kGatherThreads);
                 // Issue every load of this thread's 32 columns first (they read
                 // only x), then wait for the stage buffer and store.
                 const uint2* te = s_table + (size_t)ks * kBK;
