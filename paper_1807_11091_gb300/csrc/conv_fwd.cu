@@ -41,7 +41,6 @@ constexpr int kGatherThreads = kGatherWarps * 32;
 constexpr int kATileBytes = kBM * kBK * 2;  // 16 KB
 constexpr int kMaxStages = 4;
 constexpr int kMaxGroups = 64;
-constexpr int kPrefetchAhead = 2;  // stages of x the gather prefetches into L1 ahead
 constexpr int kSmemTail = 6144;  // barriers, TMEM address, counts, epilogue tables
 
 struct ConvArgs {
@@ -106,71 +105,6 @@ SADMM_DEV uint32_t pixel_mask(const ConvArgs& a, int it0, int ih0, int iw0)
 // Gather entry e = {offset in x, tap bits}: the column reads inside the input
 // for a pixel of mask M when every tap bit of the entry is set in M.
 SADMM_DEV bool tap_ok(uint32_t bits, uint32_t M) { return (M & bits) == bits; }
-
-// Input rows one 128-pixel tile reads: image n, depth slices [t0, t0+nt),
-// rows [r0, r0+nr) of every channel of conv group g (clamped to the input).
-struct Footprint {
-    const char* base;  // x[n, g*Cg, 0, 0, 0]
-    int t0, nt, r0, nr;
-};
-
-SADMM_DEV Footprint tile_footprint(const ConvArgs& a, long long u)
-{
-    Footprint fp{nullptr, 0, 0, 0, 0};
-    if (u >= a.units) return fp;
-    int nt_, g;
-    long long mt;
-    decode_unit(a, u, nt_, g, mt);
-    const long long m0 = mt * kBM;
-    if (m0 >= a.M) return fp;
-    const long long n = m0 / a.plane;
-    long long m1 = min(m0 + kBM - 1, a.M - 1);
-    m1 = min(m1, (n + 1) * (long long)a.plane - 1);
-    const int p0 = (int)(m0 - n * a.plane), p1 = (int)(m1 - n * a.plane);
-    const int ot0 = p0 / a.OHW, ot1 = p1 / a.OHW;
-    int oh0 = 0, oh1 = a.OHW / a.OW - 1;
-    if (ot0 == ot1) {
-        oh0 = (p0 - ot0 * a.OHW) / a.OW;
-        oh1 = (p1 - ot1 * a.OHW) / a.OW;
-    }
-    const int r0 = max(0, oh0 * a.sh - a.ph), r1 = min(a.H - 1, oh1 * a.sh - a.ph + a.KH - 1);
-    const int t0 = max(0, ot0 * a.st - a.pt), t1 = min(a.T - 1, ot1 * a.st - a.pt + a.KT - 1);
-    if (r1 < r0 || t1 < t0) return fp;
-    fp.base = reinterpret_cast<const char*>(a.x) + 2 * (n * a.x_chw + (long long)g * a.Cg * a.thw);
-    fp.t0 = t0;
-    fp.nt = t1 - t0 + 1;
-    fp.r0 = r0;
-    fp.nr = r1 - r0 + 1;
-    return fp;
-}
-
-// Prefetches into L1 the 128-byte lines of x that stage ks of a tile with
-// footprint fp reads: every channel between the stage's first and last kept
-// column, the footprint's slices and rows.  Thread `t` of `nthr` takes every
-// nthr-th line.
-SADMM_DEV void prefetch_stage(const ConvArgs& a, const Footprint& fp, const uint2* table, int ks, int t,
-                              int nthr)
-{
-    if (!fp.base) return;
-    const int j0 = ks * kBK;
-    const int j1 = min(j0 + kBK, a.n_cols) - 1;
-    if (j1 < j0) return;
-    const int c_lo = (int)(table[j0].x / (uint32_t)a.thw);
-    const int c_hi = (int)(table[j1].x / (uint32_t)a.thw);
-    const long long bytes = 2ll * fp.nr * a.W;
-    const int per = (int)((bytes + 127) >> 7) + 1;
-    const int pairs = (c_hi - c_lo + 1) * fp.nt;
-    const int jobs = min(pairs * per, 4096);
-    for (int job = t; job < jobs; job += nthr) {
-        const int pr = job / per, i = job - pr * per;
-        const int c = c_lo + pr / fp.nt, it = fp.t0 + pr % fp.nt;
-        const char* start = fp.base + 2 * ((long long)c * a.thw + (long long)it * a.hw + (long long)fp.r0 * a.W);
-        const uintptr_t first = reinterpret_cast<uintptr_t>(start) >> 7;
-        const uintptr_t last = (reinterpret_cast<uintptr_t>(start) + bytes - 1) >> 7;
-        if (first + i <= last)
-            asm volatile("prefetch.global.L1 [%0];" ::"l"((first + i) << 7));
-    }
-}
 
 template <bool OUT_BF16>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -401,21 +335,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         int s = 0;
         uint32_t ph = 0;
         bool ok = true;
-        bool primed = false;  // the first stages of this unit were prefetched
         for (long long u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
             int nt, g;
             long long mt;
             decode_unit(a, u, nt, g, mt);
-            if (s_counts[2 * g] <= nt * a.bn) {
-                primed = false;
-                continue;
-            }
-            const Footprint fp_cur = tile_footprint(a, u);
-            const Footprint fp_next = tile_footprint(a, u + gridDim.x);
-            if (!primed)
-                for (int q = 0; q < kPrefetchAhead && q < a.nks; ++q)
-                    prefetch_stage(a, fp_cur, s_table, q, gt, kGatherThreads);
-            primed = true;
+            if (s_counts[2 * g] <= nt * a.bn) continue;
             const long long m = mt * kBM + prow;
             uint32_t M = 0;
             const unsigned short* xb = xs;
@@ -434,12 +358,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             // Every lane's pixel sees every tap: no bounds test is needed.
             const bool interior = __all_sync(0xffffffffu, M == a.full_mask);
             for (int ks = 0; ks < a.nks; ++ks) {
-                // Lines of the stage kPrefetchAhead ahead (of the next tile when
-                // this one ends) go to L1 while this stage's loads run.
-                if (ks + kPrefetchAhead < a.nks)
-                    prefetch_stage(a, fp_cur, s_table, ks + kPrefetchAhead, gt, kGatherThreads);
-                else
-                    prefetch_stage(a, fp_next, s_table, ks + kPrefetchAhead - a.nks, gt, kGatherThreads);
                 // Issue every load of this thread's 32 columns first (they read
                 // only x), then wait for the stage buffer and store.
                 const uint2* te = s_table + (size_t)ks * kBK;
