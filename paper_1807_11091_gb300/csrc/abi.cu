@@ -189,7 +189,7 @@ sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d, int n_f
         return at;
     };
     p.off_wp = take((size_t)g.groups * p.n_pad * p.k_pad * 2);
-    p.off_gather = take((size_t)p.k_pad * 8);
+    p.off_gather = take((size_t)p.k_pad * 8 + (size_t)(p.k_pad / 64) * 8);  // entries + stage channel ranges
     p.off_colidx = take((size_t)p.k_pad * 4);
     p.off_rowmap = take((size_t)g.groups * p.n_pad * 4);
     p.off_zeromap = take((size_t)g.f * 4);

@@ -41,6 +41,7 @@ constexpr int kGatherThreads = kGatherWarps * 32;
 constexpr int kATileBytes = kBM * kBK * 2;  // 16 KB
 constexpr int kMaxStages = 4;
 constexpr int kMaxGroups = 64;
+constexpr int kTouchAhead = 2;  // stages ahead whose input lines the gather touches
 constexpr int kSmemTail = 6144;  // barriers, TMEM address, counts, epilogue tables
 
 struct ConvArgs {
@@ -48,6 +49,7 @@ struct ConvArgs {
     void* y;
     const float* bias;
     const uint2* gather;  // [k_pad] {channel/tap offset in x, tap bits}
+    const int2* stage_chan;  // [k_pad/64] first and last channel of each stage
     const int* rowmap;
     const int* zeromap;
     const int* counts;
@@ -105,6 +107,66 @@ SADMM_DEV uint32_t pixel_mask(const ConvArgs& a, int it0, int ih0, int iw0)
 // Gather entry e = {offset in x, tap bits}: the column reads inside the input
 // for a pixel of mask M when every tap bit of the entry is set in M.
 SADMM_DEV bool tap_ok(uint32_t bits, uint32_t M) { return (M & bits) == bits; }
+
+// Input lines one tile reads, for touching them ahead of the gather: image n,
+// depth slices [t0, t0+nt), rows [r0, r0+nr) (clamped), and this thread's
+// share: line `li` of (channel, slice) pair `pr` of a stage.
+struct TouchPlan {
+    const char* base;  // x[n, g*Cg, 0, 0, 0]
+    int t0, nt, r0, nr;
+    int pr, li;
+};
+
+SADMM_DEV TouchPlan touch_plan(const ConvArgs& a, long long u, int t)
+{
+    TouchPlan tp{nullptr, 0, 0, 0, 0, 0, 0};
+    int nt_, g;
+    long long mt;
+    decode_unit(a, u, nt_, g, mt);
+    const long long m0 = mt * kBM;
+    if (m0 >= a.M) return tp;
+    const long long n = m0 / a.plane;
+    long long m1 = min(m0 + kBM - 1, a.M - 1);
+    m1 = min(m1, (n + 1) * (long long)a.plane - 1);
+    const int p0 = (int)(m0 - n * a.plane), p1 = (int)(m1 - n * a.plane);
+    const int ot0 = p0 / a.OHW, ot1 = p1 / a.OHW;
+    int oh0 = 0, oh1 = a.OHW / a.OW - 1;
+    if (ot0 == ot1) {
+        oh0 = (p0 - ot0 * a.OHW) / a.OW;
+        oh1 = (p1 - ot1 * a.OHW) / a.OW;
+    }
+    const int r0 = max(0, oh0 * a.sh - a.ph), r1 = min(a.H - 1, oh1 * a.sh - a.ph + a.KH - 1);
+    const int t0 = max(0, ot0 * a.st - a.pt), t1 = min(a.T - 1, ot1 * a.st - a.pt + a.KT - 1);
+    if (r1 < r0 || t1 < t0) return tp;
+    tp.base = reinterpret_cast<const char*>(a.x) + 2 * (n * a.x_chw + (long long)g * a.Cg * a.thw);
+    tp.t0 = t0;
+    tp.nt = t1 - t0 + 1;
+    tp.r0 = r0;
+    tp.nr = r1 - r0 + 1;
+    const int per = (2 * tp.nr * a.W + 127) / 128 + 1;  // lines a (channel, slice) range can touch
+    tp.pr = t / per;
+    tp.li = t - tp.pr * per;
+    return tp;
+}
+
+// Issues this thread's touch load (a 2-byte load that lands the line in L1;
+// nothing waits for it) for stage ks of the tile of `tp`.
+SADMM_DEV void touch_stage(const ConvArgs& a, const TouchPlan& tp, int ks)
+{
+    if (!tp.base || ks >= a.nks) return;
+    const int2 cr = __ldg(a.stage_chan + ks);
+    const int pairs = (cr.y - cr.x + 1) * tp.nt;
+    if (tp.pr >= pairs) return;
+    const int c = cr.x + tp.pr / tp.nt, it = tp.t0 + tp.pr % tp.nt;
+    const char* start = tp.base + 2 * ((long long)c * a.thw + (long long)it * a.hw + (long long)tp.r0 * a.W);
+    const char* end = start + 2ll * tp.nr * a.W;  // exclusive
+    const char* addr = reinterpret_cast<const char*>(((reinterpret_cast<uintptr_t>(start) >> 7) + tp.li) << 7);
+    if (addr >= end) return;
+    if (addr < start) addr = start;
+    unsigned short sink;
+    asm volatile("ld.global.nc.b16 %0, [%1];" : "=h"(sink) : "l"(addr));
+    (void)sink;
+}
 
 template <bool OUT_BF16>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -335,11 +397,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         int s = 0;
         uint32_t ph = 0;
         bool ok = true;
+        int touched = 0;  // leading stages of the current unit already touched
         for (long long u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
             int nt, g;
             long long mt;
             decode_unit(a, u, nt, g, mt);
-            if (s_counts[2 * g] <= nt * a.bn) continue;
+            if (s_counts[2 * g] <= nt * a.bn) {
+                touched = 0;
+                continue;
+            }
+            const TouchPlan tp_cur = touch_plan(a, u, gt);
+            const TouchPlan tp_next = touch_plan(a, u + gridDim.x, gt);
+            for (int q = touched; q < kTouchAhead; ++q) touch_stage(a, tp_cur, q);
             const long long m = mt * kBM + prow;
             uint32_t M = 0;
             const unsigned short* xb = xs;
@@ -358,6 +427,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             // Every lane's pixel sees every tap: no bounds test is needed.
             const bool interior = __all_sync(0xffffffffu, M == a.full_mask);
             for (int ks = 0; ks < a.nks; ++ks) {
+                // Land the input lines of the stage kTouchAhead ahead (of the
+                // next tile near the end of this one) in L1.
+                if (ks + kTouchAhead < a.nks)
+                    touch_stage(a, tp_cur, ks + kTouchAhead);
+                else
+                    touch_stage(a, tp_next, ks + kTouchAhead - a.nks);
                 // Issue every load of this thread's 32 columns first (they read
                 // only x), then wait for the stage buffer and store.
                 const uint2* te = s_table + (size_t)ks * kBK;
@@ -394,6 +469,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_arrive(&full_a[s]);
                 if (++s == S) { s = 0; ph ^= 1u; }
             }
+            touched = min(kTouchAhead, a.nks);
         }
     }
 
@@ -433,6 +509,7 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     a.y = y;
     a.bias = bias;
     a.gather = reinterpret_cast<const uint2*>(base + plan->off_gather);
+    a.stage_chan = reinterpret_cast<const int2*>(a.gather + plan->k_pad);
     a.rowmap = reinterpret_cast<const int*>(base + plan->off_rowmap);
     a.zeromap = reinterpret_cast<const int*>(base + plan->off_zeromap);
     a.counts = reinterpret_cast<const int*>(base + plan->off_counts);

@@ -29,6 +29,7 @@ struct PackArgs {
     int k_pad, n_pad;
     int mask_mode;
     uint2* gather;
+    int2* stage_chan;  // [k_pad/64] first and last channel of each stage
     int* colidx;
     int* rowmap;
     int* zeromap;
@@ -83,6 +84,7 @@ __global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status)
             a.colidx[j] = -1;
             a.gather[j] = make_uint2(0u, 1u << 31);
         }
+        for (int st = tid; st < a.k_pad / 64; st += blockDim.x) a.stage_chan[st] = make_int2(0, -1);
         return;
     }
     // kept-filter range of each conv group in the ascending filter list
@@ -134,6 +136,12 @@ __global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status)
                 e.y = (1u << (kt * a.KH + kh)) | (1u << (16 + kw));
         }
         a.gather[j] = e;
+    }
+    __syncthreads();
+    // channel range (first, last kept column's channel) of every 64-column stage
+    for (int st = tid; st < a.k_pad / 64; st += blockDim.x) {
+        const int j0 = st * 64, j1 = min(j0 + 63, a.n_cols - 1);
+        a.stage_chan[st] = (j1 < j0) ? make_int2(0, -1) : make_int2(a.colidx[j0] / a.taps, a.colidx[j1] / a.taps);
     }
 }
 
@@ -211,6 +219,7 @@ sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int
     a.n_pad = plan->n_pad;
     a.mask_mode = tap_mask_mode(g);
     a.gather = reinterpret_cast<uint2*>(base + plan->off_gather);
+    a.stage_chan = reinterpret_cast<int2*>(a.gather + plan->k_pad);
     a.colidx = reinterpret_cast<int*>(base + plan->off_colidx);
     a.rowmap = reinterpret_cast<int*>(base + plan->off_rowmap);
     a.zeromap = reinterpret_cast<int*>(base + plan->off_zeromap);
