@@ -44,6 +44,9 @@ extern "C" {
 
 #define SADMM_ABI_VERSION 1
 
+/* Bytes of the fixed device array of sadmm_project_groups_noalloc. */
+#define SADMM_NOALLOC_SCRATCH_BYTES (256 * 1024)
+
 typedef enum {
     SADMM_OK = 0,
     SADMM_EINVAL = -1,       /* bad argument, shape or buffer size          */
@@ -185,6 +188,33 @@ sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt,
  */
 sadmm_status sadmm_conv_fwd(const sadmm_plan* plan, const void* x, const float* bias,
                             int relu, void* y, int ydt, void* stream);
+
+/*
+ * sadmm_project_groups without a caller-provided workspace.  The paper has no
+ * counterpart: this exists for callers that cannot hand the library device
+ * scratch memory -- a plugin or host framework that passes only its input and
+ * output tensors and keeps every allocation to itself, or a serving loop that
+ * must not allocate (nor risk running out of memory) once it is running.
+ *
+ * Arguments and results are those of sadmm_project_groups without
+ * `workspace` / `ws_bytes`.  The group keys go to one fixed device array
+ * compiled into the library, SADMM_NOALLOC_SCRATCH_BYTES (256 KiB) on every
+ * GPU that loads the library, held until the process exits.  A layer
+ * whose keys need more (sadmm_workspace_size() above that) is rejected with
+ * SADMM_EUNSUPPORTED before anything is enqueued; this holds F + K + Cg up to
+ * about 32000 groups.  The call allocates nothing: no cudaMalloc, no cudaFree.
+ *
+ * The first call on a device looks up the array's device address (a host-side
+ * CUDA runtime query, once per device, with that device current); make that
+ * first call before any stream capture.  Every call shares the array.  Nothing
+ * in it needs to start at zero (each key is written before it is read), but
+ * calls that overlap on the GPU -- on different streams with no ordering
+ * between them -- race on it and can return wrong index lists.
+ */
+sadmm_status sadmm_project_groups_noalloc(const sadmm_conv_desc* d, const void* W, const void* U,
+                                          int wdt, int k_filters, int colkind, int k_cols,
+                                          int* filt_idx, int* col_idx, double* keys_out,
+                                          void* stream);
 
 /*
  * Synchronises `stream`, then reports and clears the device status word that

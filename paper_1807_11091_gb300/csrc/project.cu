@@ -246,4 +246,72 @@ sadmm_status launch_project(const Geometry& g, const void* W, const void* U, int
                               col_idx, keys_out, ws, s);
 }
 
+// ---------------------------------------------------------------------------
+// Projection without caller-provided scratch.
+//
+// Some callers cannot hand this library a device workspace: a plugin or host
+// framework that passes only its input and output tensors and owns every
+// allocation itself, or a serving loop that must not allocate (or risk an
+// out-of-memory failure) once it is running.  For them the keys live in one
+// fixed device array compiled into the library instead.  The array is
+// kNoAllocScratchBytes on every GPU that loads the library and stays there
+// until the process exits.  All calls share it: nothing in it has to start at
+// zero (every key is written before it is read), but two calls that run at the
+// same time on the GPU (different streams, no ordering between them) overwrite
+// each other's keys and give wrong index lists.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = SADMM_NOALLOC_SCRATCH_BYTES;
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+constexpr int kNoAllocMaxDevices = 64;
+void* g_noalloc_ptr[kNoAllocMaxDevices];
+
+// Device address of the array on the current device; looked up once per device
+// (host code only sees a stand-in for the array, never its device address).
+cudaError_t noalloc_scratch(void** out)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return cudaErrorInvalidDevice;
+    if (!g_noalloc_ptr[dev]) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess) return e;
+        g_noalloc_ptr[dev] = p;
+    }
+    *out = g_noalloc_ptr[dev];
+    return cudaSuccess;
+}
+
+}  // namespace
 }  // namespace sadmm
+
+extern "C" sadmm_status sadmm_project_groups_noalloc(const sadmm_conv_desc* d, const void* W, const void* U,
+                                                     int wdt, int k_filters, int colkind, int k_cols,
+                                                     int* filt_idx, int* col_idx, double* keys_out,
+                                                     void* stream)
+{
+    using namespace sadmm;
+    Geometry g;
+    sadmm_status st = check_desc(d, &g);
+    if (st != SADMM_OK) return st;
+    if (!W || !filt_idx) return SADMM_EINVAL;
+    if (wdt != SADMM_BF16 && wdt != SADMM_FP32) return SADMM_EINVAL;
+    if (colkind != SADMM_COL_NONE && colkind != SADMM_COL_SHAPE && colkind != SADMM_COL_CHANNEL)
+        return SADMM_EINVAL;
+    if (k_filters < 0 || k_filters > g.f) return SADMM_EINVAL;
+    if (colkind != SADMM_COL_NONE) {
+        const long long G = (colkind == SADMM_COL_SHAPE) ? g.k : g.cg;
+        if (k_cols < 0 || k_cols > G || !col_idx) return SADMM_EINVAL;
+    }
+    if (keys_out && (reinterpret_cast<uintptr_t>(keys_out) & 7) != 0) return SADMM_EINVAL;
+    // the layer's keys must fit the fixed array
+    if (project_workspace_bytes(g, colkind) > kNoAllocScratchBytes) return SADMM_EUNSUPPORTED;
+    void* ws = nullptr;
+    if (noalloc_scratch(&ws) != cudaSuccess) return SADMM_ECUDA;
+    return launch_project(g, W, U, wdt, k_filters, colkind, k_cols, filt_idx, col_idx, keys_out, ws,
+                          static_cast<cudaStream_t>(stream));
+}

@@ -20,6 +20,8 @@ SADMM_OK, SADMM_EINVAL, SADMM_ECUDA, SADMM_ETIMEOUT, SADMM_EUNSUPPORTED = 0, -1,
 SADMM_BF16, SADMM_FP32 = 0, 1
 SADMM_COL_NONE, SADMM_COL_SHAPE, SADMM_COL_CHANNEL = 0, 1, 2
 
+SADMM_NOALLOC_SCRATCH_BYTES = 256 * 1024  # include/sadmm.h
+
 DESC_FIELDS = ("n", "c", "t", "h", "w", "f", "groups", "kt", "kh", "kw", "st", "sh", "sw", "pt", "ph", "pw")
 
 
@@ -90,6 +92,8 @@ def load():
     lib.sadmm_conv_fwd.argtypes = [P(Plan), vp, vp, ci, vp, ci, vp]
     lib.sadmm_last_device_status.restype = ci
     lib.sadmm_last_device_status.argtypes = [vp]
+    lib.sadmm_project_groups_noalloc.restype = ci
+    lib.sadmm_project_groups_noalloc.argtypes = [P(ConvDesc), vp, vp, ci, ci, ci, ci, vp, vp, vp, vp]
     if lib.sadmm_plan_struct_size() != ctypes.sizeof(Plan):
         raise RuntimeError("sadmm_plan layout differs between the library and this binding")
     _lib = lib
@@ -139,6 +143,15 @@ def sadmm_project_groups(desc: ConvDesc, W: int, U: Optional[int], wdt: int, k_f
     return load().sadmm_project_groups(ctypes.byref(desc), W, U, int(wdt), int(k_filters), int(colkind),
                                        int(k_cols), filt_idx, col_idx, keys_out, workspace, int(ws_bytes),
                                        stream)
+
+
+def sadmm_project_groups_noalloc(desc: ConvDesc, W: int, U: Optional[int], wdt: int, k_filters: int,
+                                 colkind: int, k_cols: int, filt_idx: int, col_idx: Optional[int],
+                                 keys_out: Optional[int], stream: Optional[int]) -> int:
+    """The projection for callers that cannot pass device scratch memory: the
+    keys live in a fixed array inside the library (see include/sadmm.h)."""
+    return load().sadmm_project_groups_noalloc(ctypes.byref(desc), W, U, int(wdt), int(k_filters),
+                                               int(colkind), int(k_cols), filt_idx, col_idx, keys_out, stream)
 
 
 def sadmm_plan_init(desc: ConvDesc, n_filt: int, colkind: int, n_colgroups: int) -> Tuple[int, Plan]:
