@@ -201,8 +201,8 @@ sadmm_status sadmm_conv_fwd(const sadmm_plan* plan, const void* x, const float* 
  * compiled into the library, SADMM_NOALLOC_SCRATCH_BYTES (256 KiB) on every
  * GPU that loads the library, held until the process exits.  A layer
  * whose keys need more (sadmm_workspace_size() above that) is rejected with
- * SADMM_EUNSUPPORTED before anything is enqueued; this holds F + K + Cg up to
- * about 32000 groups.  The call allocates nothing: no cudaMalloc, no cudaFree.
+ * SADMM_EUNSUPPORTED before anything is enqueued; F + K up to about 16000
+ * groups fit.  The call allocates nothing: no cudaMalloc, no cudaFree.
  *
  * The first call on a device looks up the array's device address (a host-side
  * CUDA runtime query, once per device, with that device current); make that

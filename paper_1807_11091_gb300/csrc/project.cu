@@ -14,6 +14,8 @@
 //
 // Keys are non-negative fp64 values, so their IEEE bit patterns order like the
 // values; selection compares bit patterns (a NaN key would rank above +Inf).
+#include <algorithm>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -36,41 +38,51 @@ SADMM_DEV double v_elem(const T* __restrict__ W, const T* __restrict__ U, long l
     return v;
 }
 
-// O_a = sum_k V[a,k]^2 for every row a (filter-wise groups).
+// O_a = sum_k V[a,k]^2 for every row a (filter-wise groups): one block per
+// row, strided fp64 partial sums, fixed-order block reduction.
 template <typename T>
-__global__ void k_filter_keys(const T* __restrict__ W, const T* __restrict__ U, int F, int K,
-                              double* __restrict__ keys)
+__global__ void __launch_bounds__(256) k_filter_keys(const T* __restrict__ W, const T* __restrict__ U, int F,
+                                                     int K, double* __restrict__ keys)
 {
-    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    if (warp >= F) return;
-    const long long base = (long long)warp * K;
+    __shared__ double part[8];
+    const int a = blockIdx.x;
+    const int lane = threadIdx.x & 31, wy = threadIdx.x >> 5;
+    const long long base = (long long)a * K;
     double s = 0.0;
-    for (int k = lane; k < K; k += 32) {
+    for (int k = threadIdx.x; k < K; k += 256) {
         const double v = v_elem(W, U, base + k);
-        s += v * v;
+        s = fma(v, v, s);
     }
     for (int o = 16; o > 0; o >>= 1) s += __shfl_down_sync(0xffffffffu, s, o);
-    if (lane == 0) keys[warp] = s;
+    if (lane == 0) part[wy] = s;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int q = 0; q < 8; ++q) t += part[q];
+        keys[a] = t;
+    }
 }
 
-// O_j = sum over kept rows a of V[a,j]^2 for every column j.  rows == NULL
-// means rows 0..nrows-1.
+// Partial column keys: block (bx, by) sums V[a,j]^2 over rows by, by + R, ...
+// of the kept-row list for the 32 columns j of bx, and writes
+// part[by][j].  rows == NULL means rows 0..nrows-1.  The select kernel adds the
+// R partials of a column in fixed order.
 template <typename T>
 __global__ void __launch_bounds__(256) k_column_keys(const T* __restrict__ W, const T* __restrict__ U, int K,
                                                      const int* __restrict__ rows, int nrows,
-                                                     double* __restrict__ keys)
+                                                     double* __restrict__ part_out)
 {
     __shared__ double part[8][33];
     const int lane = threadIdx.x & 31;
     const int wy = threadIdx.x >> 5;
     const int j = blockIdx.x * 32 + lane;
+    const int R = gridDim.y;
     double s = 0.0;
     if (j < K) {
-        for (int r = wy; r < nrows; r += 8) {
+        for (int r = blockIdx.y + R * wy; r < nrows; r += 8 * R) {
             const int a = rows ? rows[r] : r;
             const double v = v_elem(W, U, (long long)a * K + j);
-            s += v * v;
+            s = fma(v, v, s);
         }
     }
     part[wy][lane] = s;
@@ -78,7 +90,7 @@ __global__ void __launch_bounds__(256) k_column_keys(const T* __restrict__ W, co
     if (wy == 0 && j < K) {
         double t = 0.0;
         for (int q = 0; q < 8; ++q) t += part[q][lane];
-        keys[j] = t;
+        part_out[(long long)blockIdx.y * K + j] = t;
     }
 }
 
@@ -114,6 +126,7 @@ SADMM_DEV int block_excl_count(bool pred, int* warp_tot, int* total)
 // When taps > 1 the keys are first formed as sums of `taps` consecutive source
 // keys (channel-wise groups from column keys).
 __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict__ src, int G, int taps, int k,
+                                                        int nparts, long long part_stride,
                                                         double* __restrict__ keys, double* __restrict__ keys_out,
                                                         int* __restrict__ out_idx)
 {
@@ -123,19 +136,21 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
     __shared__ int warp_tot[33];
     const int tid = threadIdx.x;
 
-    // 1. keys (channel sums when taps > 1) and the optional copy for the caller
+    // 1. keys: the sum of the nparts partial sums of each source key, then of
+    //    `taps` consecutive source keys (channel-wise groups); and the optional
+    //    copy for the caller
     for (int i = tid; i < G; i += kSelThreads) {
-        double v;
-        if (taps > 1) {
-            v = 0.0;
-            for (int t = 0; t < taps; ++t) v += src[(long long)i * taps + t];
-            keys[i] = v;
-        } else {
-            v = src[i];
+        double v = 0.0;
+        for (int t = 0; t < taps; ++t) {
+            const long long si = (long long)i * taps + t;
+            double w = 0.0;
+            for (int q = 0; q < nparts; ++q) w += src[q * part_stride + si];
+            v += w;
         }
+        if (taps > 1 || nparts > 1) keys[i] = v;
         if (keys_out) keys_out[i] = v;
     }
-    const double* kv = (taps > 1) ? keys : src;
+    const double* kv = (taps > 1 || nparts > 1) ? keys : src;
     __syncthreads();
 
     if (k <= 0) return;
@@ -204,25 +219,37 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
     }
 }
 
+// Row chunks of the column-key pass: enough blocks to fill the GPU, with the
+// partial sums bounded to 16384 doubles.
+int column_parts(long long K, long long nrows)
+{
+    long long r = (304 + (K + 31) / 32 - 1) / ((K + 31) / 32);
+    r = std::min(r, 16384 / std::max(K, 1ll));
+    r = std::min(r, std::max(nrows / 32, 1ll));
+    return (int)std::max(r, 1ll);
+}
+
 template <typename T>
 sadmm_status run_project(const Geometry& g, const T* W, const T* U, int k_filters, int colkind, int k_cols,
                          int* filt_idx, int* col_idx, double* keys_out, void* ws, cudaStream_t s)
 {
     const int F = (int)g.f, K = (int)g.k;
     double* fkeys = reinterpret_cast<double*>(ws);
-    double* ckeys = fkeys + round_up(F, 32);
-    double* chkeys = ckeys + round_up(K, 32);
+    double* ckeys = fkeys + round_up(F, 32);                   // column keys
+    double* parts = ckeys + round_up(K, 32);                   // [R][K] partial column keys
 
-    k_filter_keys<T><<<(F * 32 + 255) / 256, 256, 0, s>>>(W, U, F, K, fkeys);
-    k_select<<<1, kSelThreads, 0, s>>>(fkeys, F, 1, k_filters, fkeys, keys_out, filt_idx);
+    k_filter_keys<T><<<F, 256, 0, s>>>(W, U, F, K, fkeys);
+    k_select<<<1, kSelThreads, 0, s>>>(fkeys, F, 1, k_filters, 1, 0, fkeys, keys_out, filt_idx);
     if (colkind != SADMM_COL_NONE) {
         const bool all_rows = (k_filters == F);
-        k_column_keys<T><<<(K + 31) / 32, 256, 0, s>>>(W, U, K, all_rows ? nullptr : filt_idx,
-                                                       all_rows ? F : k_filters, ckeys);
+        const int nrows = all_rows ? F : k_filters;
+        const int R = column_parts(K, nrows);
+        k_column_keys<T><<<dim3((K + 31) / 32, R), 256, 0, s>>>(W, U, K, all_rows ? nullptr : filt_idx, nrows,
+                                                                parts);
         const int taps = (colkind == SADMM_COL_CHANNEL) ? (int)g.taps : 1;
         const int G = (colkind == SADMM_COL_CHANNEL) ? (int)g.cg : K;
-        k_select<<<1, kSelThreads, 0, s>>>(ckeys, G, taps, k_cols, chkeys, keys_out ? keys_out + F : nullptr,
-                                           col_idx);
+        k_select<<<1, kSelThreads, 0, s>>>(parts, G, taps, k_cols, R, K, ckeys,
+                                           keys_out ? keys_out + F : nullptr, col_idx);
     }
     return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
 }
@@ -232,7 +259,10 @@ sadmm_status run_project(const Geometry& g, const T* W, const T* U, int k_filter
 size_t project_workspace_bytes(const Geometry& g, int colkind)
 {
     (void)colkind;
-    return (size_t)(round_up(g.f, 32) + round_up(g.k, 32) + round_up(g.cg, 32)) * sizeof(double) + 256;
+    // filter keys, column keys, and the partial column keys (at most 16384,
+    // at least one row chunk of K)
+    const long long parts = std::max(16384ll, round_up(g.k, 32));
+    return (size_t)(round_up(g.f, 32) + round_up(g.k, 32) + parts) * sizeof(double) + 256;
 }
 
 sadmm_status launch_project(const Geometry& g, const void* W, const void* U, int wdt, int k_filters,
