@@ -112,14 +112,15 @@ SADMM_DEV bool tap_ok(uint32_t bits, uint32_t M) { return (M & bits) == bits; }
 // depth slices [t0, t0+nt), rows [r0, r0+nr) (clamped), and this thread's
 // share: line `li` of (channel, slice) pair `pr` of a stage.
 struct TouchPlan {
-    const char* base;  // x[n, g*Cg, 0, 0, 0]
-    int t0, nt, r0, nr;
-    int pr, li;
+    const char* base;  // x[n, g*Cg, 0, 0, 0] plus this thread's (slice, first row, line) offset
+    int pc;            // channel offset of this thread's pair from the stage's first channel
+    int end_off;       // bytes from the plane's range start to its end (exclusive)
+    int line_off;      // this thread's line within the range (0 = the range start)
 };
 
 SADMM_DEV TouchPlan touch_plan(const ConvArgs& a, long long u, int t)
 {
-    TouchPlan tp{nullptr, 0, 0, 0, 0, 0, 0};
+    TouchPlan tp{nullptr, 0, 0, 0};
     int nt_, g;
     long long mt;
     decode_unit(a, u, nt_, g, mt);
@@ -138,34 +139,44 @@ SADMM_DEV TouchPlan touch_plan(const ConvArgs& a, long long u, int t)
     const int r0 = max(0, oh0 * a.sh - a.ph), r1 = min(a.H - 1, oh1 * a.sh - a.ph + a.KH - 1);
     const int t0 = max(0, ot0 * a.st - a.pt), t1 = min(a.T - 1, ot1 * a.st - a.pt + a.KT - 1);
     if (r1 < r0 || t1 < t0) return tp;
-    tp.base = reinterpret_cast<const char*>(a.x) + 2 * (n * a.x_chw + (long long)g * a.Cg * a.thw);
-    tp.t0 = t0;
-    tp.nt = t1 - t0 + 1;
-    tp.r0 = r0;
-    tp.nr = r1 - r0 + 1;
-    const int per = (2 * tp.nr * a.W + 127) / 128 + 1;  // lines a (channel, slice) range can touch
-    tp.pr = t / per;
-    tp.li = t - tp.pr * per;
+    // this thread's share: line li of (channel, slice) pair pr of a stage
+    const int nt2 = t1 - t0 + 1, nr = r1 - r0 + 1;
+    const int per = (2 * nr * a.W + 127) / 128 + 1;  // lines a (channel, slice) range can touch
+    const int pr = t / per, li = t - pr * per;
+    tp.pc = pr / nt2;
+    const int it = t0 + pr % nt2;
+    tp.base = reinterpret_cast<const char*>(a.x) +
+              2 * (n * a.x_chw + (long long)g * a.Cg * a.thw + (long long)it * a.hw + (long long)r0 * a.W);
+    tp.end_off = 2 * nr * a.W;
+    tp.line_off = li;
     return tp;
 }
 
-// Issues this thread's touch load (a 2-byte load that lands the line in L1;
-// nothing waits for it) for stage ks of the tile of `tp`.
 SADMM_DEV void touch_stage(const ConvArgs& a, const TouchPlan& tp, int ks)
 {
     if (!tp.base || ks >= a.nks) return;
     const int2 cr = __ldg(a.stage_chan + ks);
-    const int pairs = (cr.y - cr.x + 1) * tp.nt;
-    if (tp.pr >= pairs) return;
-    const int c = cr.x + tp.pr / tp.nt, it = tp.t0 + tp.pr % tp.nt;
-    const char* start = tp.base + 2 * ((long long)c * a.thw + (long long)it * a.hw + (long long)tp.r0 * a.W);
-    const char* end = start + 2ll * tp.nr * a.W;  // exclusive
-    const char* addr = reinterpret_cast<const char*>(((reinterpret_cast<uintptr_t>(start) >> 7) + tp.li) << 7);
-    if (addr >= end) return;
+    if (cr.x + tp.pc > cr.y) return;
+    const char* start = tp.base + 2 * (long long)(cr.x + tp.pc) * a.thw;
+    const char* addr = reinterpret_cast<const char*>(((reinterpret_cast<uintptr_t>(start) >> 7) + tp.line_off) << 7);
+    if (addr >= start + tp.end_off) return;
     if (addr < start) addr = start;
-    unsigned short sink;
-    asm volatile("ld.global.nc.b16 %0, [%1];" : "=h"(sink) : "l"(addr));
-    (void)sink;
+    asm volatile("{\n\t.reg .b16 t;\n\tld.global.nc.b16 t, [%0];\n\t}" ::"l"(addr));
+}
+
+// Branch-free conditional gather: the 16-bit element at p when every tap bit
+// of `bits` is set in the pixel mask M, else 0 (a predicated load).
+SADMM_DEV uint32_t ldg_u16_if(const unsigned short* p, uint32_t bits, uint32_t M)
+{
+    uint32_t v;
+    asm("{\n\t.reg .pred q;\n\t.reg .b32 t;\n\t"
+        "and.b32 t, %2, %3;\n\t"
+        "setp.eq.b32 q, t, %3;\n\t"
+        "mov.b32 %0, 0;\n\t"
+        "@q ld.global.nc.u16 %0, [%1];\n\t}"
+        : "=r"(v)
+        : "l"(p), "r"(M), "r"(bits));
+    return v;
 }
 
 template <bool OUT_BF16>
@@ -437,21 +448,28 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // only x), then wait for the stage buffer and store.
                 const uint2* te = s_table + (size_t)ks * kBK;
                 uint32_t v[32];
+                // two table entries per 16-byte shared-memory load
+                const uint4* te4 = reinterpret_cast<const uint4*>(te);
                 if (interior && (ks + 1) * kBK <= a.n_cols) {
 #pragma unroll
                     for (int ci = 0; ci < 4; ++ci) {
                         const int c = chunk0 + 2 * ci;
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) v[ci * 8 + e] = __ldg(xb + (int)te[c * 8 + e].x);
+                        for (int e = 0; e < 8; e += 2) {
+                            const uint4 t = te4[(c * 8 + e) >> 1];
+                            v[ci * 8 + e] = __ldg(xb + (int)t.x);
+                            v[ci * 8 + e + 1] = __ldg(xb + (int)t.z);
+                        }
                     }
                 } else {
 #pragma unroll
                     for (int ci = 0; ci < 4; ++ci) {
                         const int c = chunk0 + 2 * ci;
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            const uint2 t = te[c * 8 + e];
-                            v[ci * 8 + e] = tap_ok(t.y, M) ? (uint32_t)__ldg(xb + (int)t.x) : 0u;
+                        for (int e = 0; e < 8; e += 2) {
+                            const uint4 t = te4[(c * 8 + e) >> 1];
+                            v[ci * 8 + e] = ldg_u16_if(xb + (int)t.x, t.y, M);
+                            v[ci * 8 + e + 1] = ldg_u16_if(xb + (int)t.z, t.w, M);
                         }
                     }
                 }
@@ -462,8 +480,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int c = chunk0 + 2 * ci;
                     const uint32_t* q = v + ci * 8;
                     *reinterpret_cast<uint4*>(tile + sw128_offset((uint32_t)prow, (uint32_t)c)) =
-                        make_uint4(q[0] | (q[1] << 16), q[2] | (q[3] << 16), q[4] | (q[5] << 16),
-                                   q[6] | (q[7] << 16));
+                        make_uint4(__byte_perm(q[0], q[1], 0x5410), __byte_perm(q[2], q[3], 0x5410),
+                                   __byte_perm(q[4], q[5], 0x5410), __byte_perm(q[6], q[7], 0x5410));
                 }
                 fence_proxy_async_smem();
                 mbar_arrive(&full_a[s]);

@@ -138,3 +138,34 @@ def test_repeated_calls_reuse_the_plan():
 def test_status_word_clear_after_runs():
     from paper_1807_11091_gb300 import sadmm
     assert sadmm.device_status() == 0
+
+
+def test_slab_and_direct_stages_in_one_launch():
+    """Wide input rows make each slab slot large, so stages whose columns span
+    many channels take the direct gather while the others read the slab."""
+    s = ConvShape(n=2, c=16, h=227, w=227, f=24, kh=11, kw=11, sh=4, sw=4)
+    t = wl.gen_tensors(s, seed=61)
+    cols = list(range(0, 121)) + [c * 121 + (7 * c) % 121 for c in range(1, 16)] + list(range(15 * 121, 15 * 121 + 40))
+    cols = np.array(sorted(set(cols)), dtype=np.int64)
+    rows = np.array([0, 3, 4, 9, 10, 11, 20, 23], dtype=np.int64)
+    fi, ci, y, _ = gpu_layer(s, t, len(rows), wl.COL_SHAPE, len(cols), project=False, filt_idx=rows, col_idx=cols)
+    ref = oracle_layer(s, t, rows, wl.COL_SHAPE, cols)
+    assert_close(y, ref, what="mixed stages")
+    assert np.all(y[:, pruned_filters(s.f, rows)] == 0.0)
+
+
+@pytest.mark.parametrize("case", [
+    ("odd_plane_3x3", ConvShape(n=3, c=20, h=13, w=13, f=40, kh=3, kw=3, ph=1, pw=1), 0.5, wl.COL_SHAPE, 0.3),
+    ("tiny_plane_7x7", ConvShape(n=5, c=16, h=7, w=7, f=32, kh=3, kw=3, ph=1, pw=1), 1.0, wl.COL_CHANNEL, 0.5),
+    ("c3d_two_slices", ConvShape(n=2, c=6, t=4, h=12, w=12, f=16, kt=3, kh=3, kw=3, pt=1, ph=1, pw=1), 1.0,
+     wl.COL_SHAPE, 0.5),
+], ids=lambda c: c[0])
+def test_slab_tiling_edge_planes(case):
+    """Planes smaller than or not a multiple of a 128-pixel tile (ragged last tile
+    of every slice), and 3-D slices."""
+    name, s, ff, ck, cf = case
+    kf, kc = _k(s, ff, ck, cf)
+    t = wl.gen_tensors(s, seed=71)
+    fi, ci, y, _ = gpu_layer(s, t, kf, ck, kc)
+    ref = oracle_layer(s, t, fi, ck, ci)
+    assert_close(y, ref, what=name)
