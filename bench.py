@@ -321,6 +321,78 @@ class ClockSampler:
                 "samples": len(sm), "power_w_max": max(power) if power else None}
 
 
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "conv_fwd_alexnet_b128_dram.txt")
+CONV_SRC = os.path.join(ROOT, "paper_1807_11091_gb300", "csrc", "conv_fwd.cu")
+
+
+def conv_traffic(workload, out_dtype):
+    """DRAM bytes per sadmm_conv_fwd launch (read + write, averaged over the
+    step's launches) from the committed ncu summary, or None when that summary
+    is for another workload or the kernel source changed since it was taken."""
+    import hashlib
+    if workload != "alexnet" or out_dtype != "fp32":
+        return None
+    try:
+        fields = {}
+        with open(TRAFFIC_FILE) as fh:
+            for ln in fh:
+                if ":" in ln and not ln.startswith("#"):
+                    k, v = ln.split(":", 1)
+                    fields[k.strip()] = v.strip()
+        with open(CONV_SRC, "rb") as fh:
+            sha = hashlib.sha1(fh.read()).hexdigest()
+        if fields.get("kernel_source_sha1") != sha:
+            return None
+        return float(fields["dram_bytes_per_launch_avg"])
+    except Exception:
+        return None
+
+
+def sweep_report(dev, out_dtype, reps=5):
+    """sadmm_conv_fwd alone on the large sweep layer (N128 C256 28x28 F512 3x3)
+    at every retained fraction, against the same kernel at 0% sparsity."""
+    import torch
+    layers = wl.sweep()
+    s = layers[0].shape
+    t = wl.gen_tensors(s, seed=layers[0].seed)
+    dense = wl.Layer("sweep_dense", s, 1.0, wl.COL_SHAPE, 1.0, seed=layers[0].seed)
+    runs = [LayerRun(L, t, dev, out_dtype) for L in [dense] + layers]
+    for r in runs[1:]:  # one input and output buffer for all variants
+        r.x, r.y = runs[0].x, runs[0].y
+    sp = int(torch.cuda.current_stream().cuda_stream)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    for r in runs:
+        r.project(sp)
+        r.pack(sp)
+        r.conv(sp)
+    torch.cuda.synchronize()
+    times = []
+    for r in runs:
+        ms = []
+        for _ in range(reps):
+            flush.fill_(1)
+            torch.cuda._sleep(1_000_000)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+            r.conv(sp)
+            e1.record()
+            torch.cuda.synchronize()
+            ms.append(e0.elapsed_time(e1))
+        times.append(statistics.median(ms))
+    dense_us = times[0] * 1e3
+    out = {"layer": "N128 C256 28x28 F512 3x3 p1, shape-wise x filter-wise", "dense_conv_us": dense_us,
+           "dense_tflops": runs[0].flops() / (times[0] * 1e-3) / 1e12, "variants": []}
+    for L, r, ms in zip(layers, runs[1:], times[1:]):
+        out["variants"].append({"filters": L.filt_frac, "columns": L.col_frac, "conv_us": ms * 1e3,
+                                "tflops_retained": r.flops() / (ms * 1e-3) / 1e12,
+                                "speedup_vs_dense": times[0] / ms,
+                                "retained_fraction": r.flops() / runs[0].flops()})
+    del runs, flush
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_gpu(args):
     import torch
     ws, rank, local = dist_env()
@@ -447,7 +519,7 @@ def run_gpu(args):
         achieved = sum(conv_flops) / t_conv / 1e12
         roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
                 "frac": achieved / peaks["bf16_tflops"]}
-    roof["traffic"] = None
+    roof["traffic"] = conv_traffic(args.workload, args.out_dtype)
     roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
     roof["kernel"] = "k_conv_fwd (sadmm_conv_fwd), averaged over the step's launches"
     roof["combined_roofline_frac"] = max(t_mem, t_cmp) / t_conv
@@ -475,6 +547,8 @@ def run_gpu(args):
         "gpu_launches": sum(r.launches for r in runs) * args.steps,
         "clocks": clocks.summary(),
     }
+    if rank == 0 and not args.no_sweep:
+        line["sweep"] = sweep_report(dev, args.out_dtype)
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(layers, [wl.gen_tensors(L.shape.with_batch(16), seed=L.seed)
                                                      for L in layers])
@@ -494,6 +568,7 @@ def main():
     ap.add_argument("--workload", default="alexnet", choices=sorted(wl.WORKLOADS))
     ap.add_argument("--out-dtype", default="fp32", choices=["fp32", "bf16"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-sweep", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -1,0 +1,66 @@
+"""Runs one pruned layer of a seeded workload through the C ABI and times it.
+
+    python -m paper_1807_11091_gb300.run_layer --workload sweep --layer 0 --reps 3
+
+Projection and pack run once; sadmm_conv_fwd runs `reps` times, each timed with
+CUDA events on the launching stream.  Prints one line per run: time, TFLOP/s on
+retained MACs and the plan's tile sizes.  This is the program the per-kernel
+profiles run under ncu.
+"""
+from __future__ import annotations
+
+import argparse
+import os
+import sys
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+
+def main(argv=None) -> int:
+    import torch
+
+    import workloads as wl
+    from paper_1807_11091_gb300 import sadmm
+
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--workload", default="alexnet", choices=sorted(wl.WORKLOADS))
+    ap.add_argument("--layer", type=int, default=0)
+    ap.add_argument("--batch", type=int, default=0, help="override the workload's batch")
+    ap.add_argument("--reps", type=int, default=3)
+    ap.add_argument("--out-dtype", default="fp32", choices=["fp32", "bf16"])
+    ap.add_argument("--dense", action="store_true", help="keep every filter and column")
+    args = ap.parse_args(argv)
+
+    L = wl.get(args.workload)[args.layer]
+    s = L.shape if args.batch == 0 else L.shape.with_batch(args.batch)
+    t = wl.gen_tensors(s, seed=L.seed, device="cuda")
+    kf = s.f if args.dense else L.k_filters
+    G = s.cg if L.colkind == wl.COL_CHANNEL else s.k
+    kc = (G if args.dense else L.k_cols) if L.colkind != wl.COL_NONE else 0
+    fi, ci, _ = sadmm.project_groups(s.desc16(), t["W"], kf, L.colkind, kc)
+    pc = sadmm.PrunedConv(s.desc16(), t["W"], fi if kf < s.f else None, L.colkind, ci, kf,
+                          kc if L.colkind != wl.COL_NONE else s.k)
+    ydt = torch.bfloat16 if args.out_dtype == "bf16" else torch.float32
+    y = torch.empty(pc.out_shape(), dtype=ydt, device="cuda")
+    flops = 2.0 * s.m * kf * pc.plan.n_cols
+    for i in range(args.reps):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        pc.forward(t["x"], t["bias"], out=y)
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        print(f"{L.name} N={s.n} run {i}: {ms * 1e3:.1f} us  {flops / ms / 1e9:.1f} TFLOP/s  "
+              f"bn={pc.plan.bn} n_tiles={pc.plan.n_tiles} k_pad={pc.plan.k_pad}")
+    st = sadmm.device_status()
+    if st != 0:
+        print(f"device status {st}")
+        return 1
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())
