@@ -42,7 +42,7 @@ constexpr int kATileBytes = kBM * kBK * 2;  // 16 KB
 constexpr int kMaxStages = 4;
 constexpr int kMaxGroups = 64;
 constexpr int kTouchAhead = 2;  // stages ahead whose input lines the gather touches
-constexpr int kSmemTail = 6144;  // barriers, TMEM address, counts, epilogue tables
+constexpr int kSmemTail = 10240;  // barriers, TMEM address, counts, epilogue tables
 
 struct ConvArgs {
     const __nv_bfloat16* x;
@@ -57,7 +57,7 @@ struct ConvArgs {
     long long M;      // N * plane
     long long x_chw;  // elements per input image
     long long thw;    // elements per input channel
-    long long units;  // m_tiles * groups * n_tiles
+    long long units;  // m_tiles * groups * upairs
     int hw, W, H, T;
     int F, groups, Cg, Fg;
     int OW, OHW, plane;
@@ -65,6 +65,9 @@ struct ConvArgs {
     int KT, KH, KW;
     int nks;  // k_pad / 64
     int bn, n_tiles, n_pad;
+    int nacc;      // filter tiles per unit (TMEM accumulators sharing one A tile)
+    int upairs;    // units per (pixel tile, group): ceil(n_tiles / nacc)
+    int acc_bufs;  // accumulator sets in TMEM (2: the epilogue overlaps the next unit's MMAs)
     int stages;
     int k_pad;
     int n_cols;          // K' (columns past it are padding)
@@ -75,10 +78,12 @@ struct ConvArgs {
     int relu;
 };
 
-SADMM_DEV void decode_unit(const ConvArgs& a, long long u, int& nt, int& g, long long& mt)
+// Unit u covers filter tiles p*nacc .. p*nacc+nacc-1 of conv group g for pixel
+// tile mt.
+SADMM_DEV void decode_unit(const ConvArgs& a, long long u, int& p, int& g, long long& mt)
 {
-    nt = (int)(u % a.n_tiles);
-    const long long t = u / a.n_tiles;
+    p = (int)(u % a.upairs);
+    const long long t = u / a.upairs;
     g = (int)(t % a.groups);
     mt = t / a.groups;
 }
@@ -186,10 +191,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = a.stages;
-    const uint32_t b_bytes = (uint32_t)a.bn * 128u;
+    const uint32_t b_bytes = (uint32_t)a.bn * 128u;      // one Wp box (bn rows x 64 columns)
+    const uint32_t bstage = b_bytes * (uint32_t)a.nacc;  // a B stage holds nacc boxes
     uint8_t* sA = smem;
     uint8_t* sB = smem + (size_t)S * kATileBytes;
-    uint2* s_table = reinterpret_cast<uint2*>(sB + (size_t)S * b_bytes);
+    uint2* s_table = reinterpret_cast<uint2*>(sB + (size_t)S * bstage);
     uint64_t* bars = reinterpret_cast<uint64_t*>(s_table + a.k_pad);
     uint64_t* full_a = bars;
     uint64_t* full_b = bars + S;
@@ -200,8 +206,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
     int* s_counts = reinterpret_cast<int*>(tmem_holder + 2);
-    int* s_eoff = s_counts + 2 * kMaxGroups;          // [2][256] output-plane offsets
-    float* s_ebias = reinterpret_cast<float*>(s_eoff + 512);  // [2][256] biases
+    int* s_eoff = s_counts + 2 * kMaxGroups;                   // [2][512] output-plane offsets
+    float* s_ebias = reinterpret_cast<float*>(s_eoff + 1024);  // [2][512] biases
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -211,7 +217,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&full_b[s], 1);
             mbar_init(&empty[s], 1);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < a.acc_bufs; ++b) {
             mbar_init(&acc_full[b], 1);
             mbar_init(&acc_empty[b], kEpiWarps * 32);
         }
@@ -245,15 +251,21 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t issued_mask = 0;
             bool ok = true;
             for (long long u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-                int nt, g;
+                int p, g;
                 long long mt;
-                decode_unit(a, u, nt, g, mt);
-                if (s_counts[2 * g] <= nt * a.bn) continue;
-                const int row0 = g * a.n_pad + nt * a.bn;
+                decode_unit(a, u, p, g, mt);
+                const int nt0 = p * a.nacc;
+                if (s_counts[2 * g] <= nt0 * a.bn) continue;
+                int nbox = 0;  // filter tiles of this unit with kept rows
+                for (int i = 0; i < a.nacc; ++i)
+                    if (nt0 + i < a.n_tiles && s_counts[2 * g] > (nt0 + i) * a.bn) nbox = i + 1;
+                const int row0 = g * a.n_pad + nt0 * a.bn;
                 for (int ks = 0; ks < a.nks; ++ks) {
                     if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, a.status)) { ok = false; break; }
-                    mbar_arrive_expect_tx(&full_b[s], b_bytes);
-                    tma_load_2d(sB + (size_t)s * b_bytes, &tmap, &full_b[s], ks * kBK, row0);
+                    mbar_arrive_expect_tx(&full_b[s], b_bytes * (uint32_t)nbox);
+                    for (int i = 0; i < nbox; ++i)
+                        tma_load_2d(sB + (size_t)s * bstage + (size_t)i * b_bytes, &tmap, &full_b[s], ks * kBK,
+                                    row0 + i * a.bn);
                     issued_parity[s] = ph;
                     issued_mask |= 1u << s;
                     if (++s == S) { s = 0; ph ^= 1u; }
@@ -276,16 +288,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t acc_ph = 0;
             bool ok = true;
             for (long long u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-                int nt, g;
+                int p, g;
                 long long mt;
-                decode_unit(a, u, nt, g, mt);
-                const int cnt = s_counts[2 * g] - nt * a.bn;
+                decode_unit(a, u, p, g, mt);
+                const int cnt = s_counts[2 * g] - p * a.nacc * a.bn;  // kept rows from the unit's first tile
                 if (cnt <= 0) continue;
-                const int n_rt = min(a.bn, (cnt + 15) & ~15);
-                const uint32_t idesc = idesc_bf16_f32(kBM, n_rt);
+                // one accumulator per filter tile with kept rows, N rounded up to 16
+                const int rows1 = (a.nacc == 2 && p * 2 + 1 < a.n_tiles) ? min(a.bn, cnt - a.bn) : 0;
+                const uint32_t idesc0 = idesc_bf16_f32(kBM, min(a.bn, (cnt + 15) & ~15));
+                const uint32_t idesc1 = idesc_bf16_f32(kBM, min(a.bn, (max(rows1, 16) + 15) & ~15));
+                const bool two = rows1 > 0;
                 if (!mbar_wait(&acc_empty[ab], acc_ph ^ 1u, abort_flag, a.status)) break;
                 tc_fence_after();
-                const uint32_t d_tmem = tmem_base + (uint32_t)(ab * a.tmem_stride);
+                const uint32_t d_tmem = tmem_base + (uint32_t)(ab * a.nacc * a.tmem_stride);
                 for (int ks = 0; ks < a.nks; ++ks) {
                     if (!mbar_wait(&full_a[s], ph, abort_flag, a.status) ||
                         !mbar_wait(&full_b[s], ph, abort_flag, a.status)) {
@@ -294,19 +309,31 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     tc_fence_after();
                     const uint32_t a0 = smem_u32(sA + (size_t)s * kATileBytes);
-                    const uint32_t b0 = smem_u32(sB + (size_t)s * b_bytes);
+                    const uint32_t b0 = smem_u32(sB + (size_t)s * bstage);
+                    // The issuing thread is on the critical path: straight-line
+                    // code, descriptors in registers.
+                    if (!two) {
 #pragma unroll
-                    for (int kk = 0; kk < kBK / 16; ++kk) {
-                        mma_bf16_ss(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32), sdesc_kmajor_sw128(b0 + kk * 32),
-                                    idesc, (ks | kk) != 0 ? 1u : 0u);
+                        for (int kk = 0; kk < kBK / 16; ++kk)
+                            mma_bf16_ss(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32), sdesc_kmajor_sw128(b0 + kk * 32),
+                                        idesc0, (ks | kk) != 0 ? 1u : 0u);
+                    } else {
+                        const uint32_t d1 = d_tmem + (uint32_t)a.tmem_stride;
+                        const uint32_t b1 = b0 + b_bytes;
+#pragma unroll
+                        for (int kk = 0; kk < kBK / 16; ++kk) {
+                            const uint64_t adesc = sdesc_kmajor_sw128(a0 + kk * 32);
+                            const uint32_t acc = (ks | kk) != 0 ? 1u : 0u;
+                            mma_bf16_ss(d_tmem, adesc, sdesc_kmajor_sw128(b0 + kk * 32), idesc0, acc);
+                            mma_bf16_ss(d1, adesc, sdesc_kmajor_sw128(b1 + kk * 32), idesc1, acc);
+                        }
                     }
                     mma_commit(&empty[s]);
                     if (++s == S) { s = 0; ph ^= 1u; }
                 }
                 if (!ok) break;
                 mma_commit(&acc_full[ab]);
-                ab ^= 1;
-                if (ab == 0) acc_ph ^= 1u;
+                if (++ab == a.acc_bufs) { ab = 0; acc_ph ^= 1u; }
             }
             // Every MMA this thread issued has completed before TMEM is freed.
             mma_commit(drain);
@@ -329,21 +356,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t acc_ph = 0;
         int ub = 0;  // double-buffered per-unit tables
         for (long long u = blockIdx.x; u < a.units; u += gridDim.x) {
-            int nt, g;
+            int p, g;
             long long mt;
-            decode_unit(a, u, nt, g, mt);
-            const int cnt = s_counts[2 * g] - nt * a.bn;
+            decode_unit(a, u, p, g, mt);
+            const int nt0 = p * a.nacc;
+            const int cnt = s_counts[2 * g] - nt0 * a.bn;  // kept rows from the unit's first tile
             const long long m = mt * kBM + row;
             const bool valid = m < a.M;
             const long long n_img = valid ? m / a.plane : 0;
-            const long long p = valid ? m - n_img * a.plane : 0;
-            float* yf = reinterpret_cast<float*>(a.y) + (n_img * (long long)a.F * a.plane + p);
-            __nv_bfloat16* yh = reinterpret_cast<__nv_bfloat16*>(a.y) + (n_img * (long long)a.F * a.plane + p);
-            int* u_off = s_eoff + ub * 256;
-            float* u_bias = s_ebias + ub * 256;
+            const long long pix = valid ? m - n_img * a.plane : 0;
+            float* yf = reinterpret_cast<float*>(a.y) + (n_img * (long long)a.F * a.plane + pix);
+            __nv_bfloat16* yh = reinterpret_cast<__nv_bfloat16*>(a.y) + (n_img * (long long)a.F * a.plane + pix);
+            int* u_off = s_eoff + ub * 512;
+            float* u_bias = s_ebias + ub * 512;
             if (cnt > 0) {
-                const int* rmap = a.rowmap + (long long)g * a.n_pad + (long long)nt * a.bn;
-                for (int i = et; i < a.bn; i += kEpiWarps * 32) {
+                // column i of the unit = row i % bn of filter tile nt0 + i / bn
+                const int* rmap = a.rowmap + (long long)g * a.n_pad + (long long)nt0 * a.bn;
+                const int ncol = min(a.nacc, a.n_tiles - nt0) * a.bn;
+                for (int i = et; i < ncol; i += kEpiWarps * 32) {
                     const int f = __ldg(rmap + i);
                     u_off[i] = f >= 0 ? f * a.plane : 0;
                     u_bias[i] = (f >= 0 && a.bias) ? __ldg(a.bias + f) : 0.0f;
@@ -351,35 +381,40 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
             if (cnt > 0) {
-                const int nrows = min(a.bn, cnt);
                 // warp-uniform outcome: the TMEM loads below are .sync.aligned
                 if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[ab], acc_ph, abort_flag, a.status))) break;
                 tc_fence_after();
-                const uint32_t taddr = tmem_base + (uint32_t)(ab * a.tmem_stride) + ((uint32_t)(q * 32) << 16);
-                for (int c0 = 32 * h; c0 < nrows; c0 += 32 * kHalves) {
-                    uint32_t r[32];
-                    tmem_ld_32x32b_x32(taddr + (uint32_t)c0, r);
-                    tmem_ld_wait();
-                    if (valid) {
+                for (int ti = 0; ti < a.nacc && nt0 + ti < a.n_tiles; ++ti) {
+                    const int nrows = min(a.bn, cnt - ti * a.bn);
+                    if (nrows <= 0) break;
+                    const uint32_t taddr = tmem_base + (uint32_t)((ab * a.nacc + ti) * a.tmem_stride) +
+                                           ((uint32_t)(q * 32) << 16);
+                    const int* t_off = u_off + ti * a.bn;
+                    const float* t_bias = u_bias + ti * a.bn;
+                    for (int c0 = 32 * h; c0 < nrows; c0 += 32 * kHalves) {
+                        uint32_t r[32];
+                        tmem_ld_32x32b_x32(taddr + (uint32_t)c0, r);
+                        tmem_ld_wait();
+                        if (valid) {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) {
-                            if (c0 + j < nrows) {
-                                float v = __uint_as_float(r[j]) + u_bias[c0 + j];
-                                if (a.relu) v = fmaxf(v, 0.0f);
-                                if (OUT_BF16)
-                                    yh[u_off[c0 + j]] = __float2bfloat16_rn(v);
-                                else
-                                    __stcs(yf + u_off[c0 + j], v);
+                            for (int j = 0; j < 32; ++j) {
+                                if (c0 + j < nrows) {
+                                    float v = __uint_as_float(r[j]) + t_bias[c0 + j];
+                                    if (a.relu) v = fmaxf(v, 0.0f);
+                                    if (OUT_BF16)
+                                        yh[t_off[c0 + j]] = __float2bfloat16_rn(v);
+                                    else
+                                        __stcs(yf + t_off[c0 + j], v);
+                                }
                             }
                         }
                     }
                 }
                 tc_fence_before();
                 mbar_arrive(&acc_empty[ab]);
-                ab ^= 1;
-                if (ab == 0) acc_ph ^= 1u;
+                if (++ab == a.acc_bufs) { ab = 0; acc_ph ^= 1u; }
             }
-            if (nt == 0) {
+            if (p == 0) {
                 // pruned filters of this conv group: their planes are zero
                 const int zc = s_counts[2 * g + 1];
                 const int* zmap = a.zeromap + (long long)g * a.Fg;
@@ -410,10 +445,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = true;
         int touched = 0;  // leading stages of the current unit already touched
         for (long long u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-            int nt, g;
+            int p, g;
             long long mt;
-            decode_unit(a, u, nt, g, mt);
-            if (s_counts[2 * g] <= nt * a.bn) {
+            decode_unit(a, u, p, g, mt);
+            if (s_counts[2 * g] <= p * a.nacc * a.bn) {
                 touched = 0;
                 continue;
             }
@@ -558,10 +593,12 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     a.nks = plan->k_pad / kBK;
     a.bn = plan->bn;
     a.n_tiles = plan->n_tiles;
+    a.nacc = plan->n_tiles >= 2 ? 2 : 1;
+    a.upairs = (plan->n_tiles + a.nacc - 1) / a.nacc;
     a.n_pad = plan->n_pad;
     a.relu = relu ? 1 : 0;
     const long long m_tiles = (g.m + kBM - 1) / kBM;
-    a.units = m_tiles * g.groups * plan->n_tiles;
+    a.units = m_tiles * g.groups * a.upairs;
 
     a.k_pad = plan->k_pad;
     a.n_cols = plan->n_cols;
@@ -570,7 +607,7 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
         a.full_mask = ((1u << (g.kt * g.kh)) - 1u) | (((1u << g.kw) - 1u) << 16);
     else
         a.full_mask = (uint32_t)((1ull << g.taps) - 1ull);
-    const int stage_bytes = kATileBytes + plan->bn * 128;
+    const int stage_bytes = kATileBytes + a.nacc * plan->bn * 128;
     const int table_bytes = plan->k_pad * 8;
     const int budget = 232448 - 1024 - kSmemTail - table_bytes;
     // At most kMaxStages: what shared memory leaves over serves as L1 for x.
@@ -578,8 +615,9 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     if (a.stages > kMaxStages) a.stages = kMaxStages;
     if (a.stages < 2) return SADMM_EUNSUPPORTED;
     a.tmem_stride = (plan->bn + 31) & ~31;
+    a.acc_bufs = (2 * a.nacc * a.tmem_stride <= 512) ? 2 : 1;
     int cols = 32;
-    while (cols < 2 * a.tmem_stride) cols <<= 1;
+    while (cols < a.acc_bufs * a.nacc * a.tmem_stride) cols <<= 1;
     a.tmem_cols = cols;
     const size_t smem = 1024 + (size_t)a.stages * stage_bytes + table_bytes + kSmemTail;
 
