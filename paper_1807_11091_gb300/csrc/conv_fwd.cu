@@ -10,17 +10,17 @@
 // tile, one TMEM lane each), kept filters the N side (bn <= 256 per tile), so a
 // gathered pixel tile is reused by every kept filter of the tile.
 //
-// One persistent CTA per SM, warp-specialised (512 threads):
+// One persistent CTA per SM, warp-specialised (896 threads):
 //   warp 0      TMA producer: 64-column x bn-row boxes of Wp (128-byte swizzle)
 //   warp 1      TMEM allocator and MMA issuer (tcgen05.mma kind::f16, bf16 in,
 //               fp32 accumulate, 128 x n x 16 per instruction)
-//   warps 4-7   epilogue: tcgen05.ld of the accumulator (lane = pixel), bias,
+//   warps 4-11  epilogue (two warps per TMEM lane quadrant): tcgen05.ld of the accumulator (lane = pixel), bias,
 //               ReLU, coalesced stores to the NCHW output (consecutive lanes
 //               write consecutive pixels of one filter plane), and zero-fill of
 //               the pruned filters' planes for the tile's pixels
-//   warps 8-15  gather: each thread owns one pixel of the tile and builds 16-byte
-//               K-major chunks of A through the gather table, with zero fill
-//               outside the input, into the 128-byte-swizzled stage buffer
+//   warps 12-27 gather: four threads per pixel of the tile, each building two
+//               16-byte K-major chunks of A through the gather table, with zero
+//               fill outside the input, into the 128-byte-swizzled stage buffer
 // Shared-memory stages are guarded by mbarriers; the accumulator is double
 // buffered in TMEM so the epilogue of one tile overlaps the MMAs of the next.
 #include <cuda.h>
@@ -34,10 +34,13 @@ namespace {
 
 constexpr int kBM = 128;           // pixels per tile
 constexpr int kBK = 64;            // GEMM columns per stage
-constexpr int kGatherWarps = 8;
+constexpr int kGatherWarps = 16;
 constexpr int kEpiWarps = 8;
 constexpr int kThreads = (4 + kEpiWarps + kGatherWarps) * 32;
 constexpr int kGatherThreads = kGatherWarps * 32;
+constexpr int kGatherGroups = kGatherThreads / kBM;     // threads per pixel
+constexpr int kChunksPerThread = 8 / kGatherGroups;     // 16-byte chunks of a stage row per thread
+static_assert(kGatherThreads % kBM == 0 && 8 % kGatherGroups == 0, "gather threads must split a 64-column row evenly");
 constexpr int kATileBytes = kBM * kBK * 2;  // 16 KB
 constexpr int kMaxStages = 4;
 constexpr int kMaxGroups = 64;
@@ -438,7 +441,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ----------------------------------------------------------- gather
         const int gt = threadIdx.x - (4 + kEpiWarps) * 32;
         const int prow = gt & (kBM - 1);
-        const int chunk0 = gt >> 7;  // 0 or 1: this thread builds chunks chunk0, +2, +4, +6
+        const int chunk0 = gt >> 7;  // this thread builds chunks chunk0 + kGatherGroups * i
         const unsigned short* xs = reinterpret_cast<const unsigned short*>(a.x);
         int s = 0;
         uint32_t ph = 0;
@@ -479,16 +482,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                     touch_stage(a, tp_cur, ks + kTouchAhead);
                 else
                     touch_stage(a, tp_next, ks + kTouchAhead - a.nks);
-                // Issue every load of this thread's 32 columns first (they read
+                // Issue every load of this thread's columns first (they read
                 // only x), then wait for the stage buffer and store.
                 const uint2* te = s_table + (size_t)ks * kBK;
-                uint32_t v[32];
+                uint32_t v[8 * kChunksPerThread];
                 // two table entries per 16-byte shared-memory load
                 const uint4* te4 = reinterpret_cast<const uint4*>(te);
                 if (interior && (ks + 1) * kBK <= a.n_cols) {
 #pragma unroll
-                    for (int ci = 0; ci < 4; ++ci) {
-                        const int c = chunk0 + 2 * ci;
+                    for (int ci = 0; ci < kChunksPerThread; ++ci) {
+                        const int c = chunk0 + kGatherGroups * ci;
 #pragma unroll
                         for (int e = 0; e < 8; e += 2) {
                             const uint4 t = te4[(c * 8 + e) >> 1];
@@ -498,8 +501,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 } else {
 #pragma unroll
-                    for (int ci = 0; ci < 4; ++ci) {
-                        const int c = chunk0 + 2 * ci;
+                    for (int ci = 0; ci < kChunksPerThread; ++ci) {
+                        const int c = chunk0 + kGatherGroups * ci;
 #pragma unroll
                         for (int e = 0; e < 8; e += 2) {
                             const uint4 t = te4[(c * 8 + e) >> 1];
@@ -511,8 +514,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, a.status)) { ok = false; break; }
                 uint8_t* tile = sA + (size_t)s * kATileBytes;
 #pragma unroll
-                for (int ci = 0; ci < 4; ++ci) {
-                    const int c = chunk0 + 2 * ci;
+                for (int ci = 0; ci < kChunksPerThread; ++ci) {
+                    const int c = chunk0 + kGatherGroups * ci;
                     const uint32_t* q = v + ci * 8;
                     *reinterpret_cast<uint4*>(tile + sw128_offset((uint32_t)prow, (uint32_t)c)) =
                         make_uint4(__byte_perm(q[0], q[1], 0x5410), __byte_perm(q[2], q[3], 0x5410),
