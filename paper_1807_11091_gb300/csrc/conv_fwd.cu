@@ -18,9 +18,10 @@
 //               ReLU, coalesced stores to the NCHW output (consecutive lanes
 //               write consecutive pixels of one filter plane), and zero-fill of
 //               the pruned filters' planes for the tile's pixels
-//   warps 12-27 gather: four threads per pixel of the tile, each building two
-//               16-byte K-major chunks of A through the gather table, with zero
-//               fill outside the input, into the 128-byte-swizzled stage buffer
+//   warps 12-27 gather, in two sets that fill alternate stages: in a set, two
+//               threads per pixel of the tile, each building four 16-byte
+//               K-major chunks of A through the gather table, with zero fill
+//               outside the input, into the 128-byte-swizzled stage buffer
 // Shared-memory stages are guarded by mbarriers; the accumulator is double
 // buffered in TMEM so the epilogue of one tile overlaps the MMAs of the next.
 #include <cuda.h>
@@ -38,21 +39,33 @@ constexpr int kGatherWarps = 16;
 constexpr int kEpiWarps = 8;
 constexpr int kThreads = (4 + kEpiWarps + kGatherWarps) * 32;
 constexpr int kGatherThreads = kGatherWarps * 32;
-constexpr int kGatherGroups = kGatherThreads / kBM;     // threads per pixel
-constexpr int kChunksPerThread = 8 / kGatherGroups;     // 16-byte chunks of a stage row per thread
-static_assert(kGatherThreads % kBM == 0 && 8 % kGatherGroups == 0, "gather threads must split a 64-column row evenly");
+// The gather warps form kGatherSets independent sets; set i fills the stages
+// whose running index is i modulo kGatherSets, so the load latency of one
+// stage overlaps the loads of the next.
+constexpr int kGatherSets = 2;
+constexpr int kSetThreads = kGatherThreads / kGatherSets;
+constexpr int kSetGroups = kSetThreads / kBM;       // threads of a set per pixel
+constexpr int kChunksPerThread = 8 / kSetGroups;    // 16-byte chunks of a stage row per thread
+static_assert(kSetThreads % kBM == 0 && 8 % kSetGroups == 0, "a gather set must split a 64-column row evenly");
 constexpr int kATileBytes = kBM * kBK * 2;  // 16 KB
 constexpr int kMaxStages = 4;
 constexpr int kMaxGroups = 64;
-constexpr int kTouchAhead = 2;  // stages ahead whose input lines the gather touches
-constexpr int kSmemTail = 10240;  // barriers, TMEM address, counts, epilogue tables
+constexpr int kEpiCols = 16;       // accumulator columns per epilogue TMEM load
+constexpr int kTabCap = 512;       // kept-row entries of an epilogue table buffer
+// Fixed shared-memory tail: epilogue tables [2][kTabCap] offsets and biases,
+// per-group counts, barriers and the TMEM address.  The zero-plane table
+// [2][zcap] follows it.
+constexpr int kTailOffBias = 0;
+constexpr int kTailCounts = kTailOffBias + 2 * 2 * kTabCap * 4;
+constexpr int kTailBars = kTailCounts + 2 * kMaxGroups * 4;
+constexpr int kTailZero = kTailBars + 512;
+constexpr int kSmemTail = kTailZero;
 
 struct ConvArgs {
     const __nv_bfloat16* x;
     void* y;
     const float* bias;
     const uint2* gather;  // [k_pad] {channel/tap offset in x, tap bits}
-    const int2* stage_chan;  // [k_pad/64] first and last channel of each stage
     const int* rowmap;
     const int* zeromap;
     const int* counts;
@@ -78,6 +91,7 @@ struct ConvArgs {
     uint32_t full_mask;  // the mask of a pixel whose every tap is inside the input
     int tmem_stride;
     int tmem_cols;
+    int zcap;  // zero-plane offsets per table buffer kept in shared memory
     int relu;
 };
 
@@ -116,62 +130,6 @@ SADMM_DEV uint32_t pixel_mask(const ConvArgs& a, int it0, int ih0, int iw0)
 // for a pixel of mask M when every tap bit of the entry is set in M.
 SADMM_DEV bool tap_ok(uint32_t bits, uint32_t M) { return (M & bits) == bits; }
 
-// Input lines one tile reads, for touching them ahead of the gather: image n,
-// depth slices [t0, t0+nt), rows [r0, r0+nr) (clamped), and this thread's
-// share: line `li` of (channel, slice) pair `pr` of a stage.
-struct TouchPlan {
-    const char* base;  // x[n, g*Cg, 0, 0, 0] plus this thread's (slice, first row, line) offset
-    int pc;            // channel offset of this thread's pair from the stage's first channel
-    int end_off;       // bytes from the plane's range start to its end (exclusive)
-    int line_off;      // this thread's line within the range (0 = the range start)
-};
-
-SADMM_DEV TouchPlan touch_plan(const ConvArgs& a, long long u, int t)
-{
-    TouchPlan tp{nullptr, 0, 0, 0};
-    int nt_, g;
-    long long mt;
-    decode_unit(a, u, nt_, g, mt);
-    const long long m0 = mt * kBM;
-    if (m0 >= a.M) return tp;
-    const long long n = m0 / a.plane;
-    long long m1 = min(m0 + kBM - 1, a.M - 1);
-    m1 = min(m1, (n + 1) * (long long)a.plane - 1);
-    const int p0 = (int)(m0 - n * a.plane), p1 = (int)(m1 - n * a.plane);
-    const int ot0 = p0 / a.OHW, ot1 = p1 / a.OHW;
-    int oh0 = 0, oh1 = a.OHW / a.OW - 1;
-    if (ot0 == ot1) {
-        oh0 = (p0 - ot0 * a.OHW) / a.OW;
-        oh1 = (p1 - ot1 * a.OHW) / a.OW;
-    }
-    const int r0 = max(0, oh0 * a.sh - a.ph), r1 = min(a.H - 1, oh1 * a.sh - a.ph + a.KH - 1);
-    const int t0 = max(0, ot0 * a.st - a.pt), t1 = min(a.T - 1, ot1 * a.st - a.pt + a.KT - 1);
-    if (r1 < r0 || t1 < t0) return tp;
-    // this thread's share: line li of (channel, slice) pair pr of a stage
-    const int nt2 = t1 - t0 + 1, nr = r1 - r0 + 1;
-    const int per = (2 * nr * a.W + 127) / 128 + 1;  // lines a (channel, slice) range can touch
-    const int pr = t / per, li = t - pr * per;
-    tp.pc = pr / nt2;
-    const int it = t0 + pr % nt2;
-    tp.base = reinterpret_cast<const char*>(a.x) +
-              2 * (n * a.x_chw + (long long)g * a.Cg * a.thw + (long long)it * a.hw + (long long)r0 * a.W);
-    tp.end_off = 2 * nr * a.W;
-    tp.line_off = li;
-    return tp;
-}
-
-SADMM_DEV void touch_stage(const ConvArgs& a, const TouchPlan& tp, int ks)
-{
-    if (!tp.base || ks >= a.nks) return;
-    const int2 cr = __ldg(a.stage_chan + ks);
-    if (cr.x + tp.pc > cr.y) return;
-    const char* start = tp.base + 2 * (long long)(cr.x + tp.pc) * a.thw;
-    const char* addr = reinterpret_cast<const char*>(((reinterpret_cast<uintptr_t>(start) >> 7) + tp.line_off) << 7);
-    if (addr >= start + tp.end_off) return;
-    if (addr < start) addr = start;
-    asm volatile("{\n\t.reg .b16 t;\n\tld.global.nc.b16 t, [%0];\n\t}" ::"l"(addr));
-}
-
 // Branch-free conditional gather: the 16-bit element at p when every tap bit
 // of `bits` is set in the pixel mask M, else 0 (a predicated load).
 SADMM_DEV uint32_t ldg_u16_if(const unsigned short* p, uint32_t bits, uint32_t M)
@@ -199,7 +157,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t* sA = smem;
     uint8_t* sB = smem + (size_t)S * kATileBytes;
     uint2* s_table = reinterpret_cast<uint2*>(sB + (size_t)S * bstage);
-    uint64_t* bars = reinterpret_cast<uint64_t*>(s_table + a.k_pad);
+    uint8_t* tail = reinterpret_cast<uint8_t*>(s_table + a.k_pad);  // 512-byte aligned
+    int* s_eoff = reinterpret_cast<int*>(tail + kTailOffBias);                   // [2][kTabCap] plane offsets
+    float* s_ebias = reinterpret_cast<float*>(tail + kTailOffBias) + 2 * kTabCap;  // [2][kTabCap] biases
+    int* s_counts = reinterpret_cast<int*>(tail + kTailCounts);
+    int* s_zoff = reinterpret_cast<int*>(tail + kTailZero);  // [2][zcap] zero-plane offsets
+    uint64_t* bars = reinterpret_cast<uint64_t*>(tail + kTailBars);
     uint64_t* full_a = bars;
     uint64_t* full_b = bars + S;
     uint64_t* empty = bars + 2 * S;
@@ -208,15 +171,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* drain = acc_empty + 2;
     uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
-    int* s_counts = reinterpret_cast<int*>(tmem_holder + 2);
-    int* s_eoff = s_counts + 2 * kMaxGroups;                   // [2][512] output-plane offsets
-    float* s_ebias = reinterpret_cast<float*>(s_eoff + 1024);  // [2][512] biases
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
-            mbar_init(&full_a[s], kGatherThreads);
+            mbar_init(&full_a[s], kSetThreads);
             mbar_init(&full_b[s], 1);
             mbar_init(&empty[s], 1);
         }
@@ -346,10 +306,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else if (warp >= 4 && warp < 4 + kEpiWarps) {
         // --------------------------------------------------------- epilogue
-        // kEpiWarps / 4 warps share each TMEM lane quadrant and split its
-        // 32-column chunks.  Per unit, the output-plane offset and bias of every
-        // packed row go to shared memory before the accumulator wait, so the
-        // store loop reads them with broadcast loads.
+        // kEpiWarps / 4 warps share each TMEM lane quadrant and take its
+        // 16-column chunks in turn, then the zero planes.  The output-plane
+        // offset and bias of every packed row, and the offsets of the pruned
+        // filters' planes, sit in shared memory; they are reloaded only when
+        // a unit's (conv group, filter tiles) differ from the previous one's.
         constexpr int kHalves = kEpiWarps / 4;
         const int q = warp & 3;  // TMEM lane quadrant this warp may access
         const int h = (warp - 4) >> 2;
@@ -357,76 +318,131 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int row = q * 32 + lane;
         int ab = 0;
         uint32_t acc_ph = 0;
-        int ub = 0;  // double-buffered per-unit tables
+        int ub = 1;         // table buffer of the current unit
+        long long tab_key = -1;  // (group, filter tiles) the tables hold
+        // After a failed wait (another role aborted) the warp keeps walking the
+        // units, without TMEM or stores, so the named barrier stays balanced.
+        bool alive = true;
         for (long long u = blockIdx.x; u < a.units; u += gridDim.x) {
             int p, g;
             long long mt;
             decode_unit(a, u, p, g, mt);
             const int nt0 = p * a.nacc;
             const int cnt = s_counts[2 * g] - nt0 * a.bn;  // kept rows from the unit's first tile
+            const int zc = (p == 0) ? s_counts[2 * g + 1] : 0;  // pruned filters whose planes this unit zeroes
+            const long long key = (long long)g * a.upairs + p;
+            if (key != tab_key) {
+                ub ^= 1;
+                int* u_off = s_eoff + ub * kTabCap;
+                float* u_bias = s_ebias + ub * kTabCap;
+                if (cnt > 0) {
+                    // column i of the unit = row i % bn of filter tile nt0 + i / bn
+                    const int* rmap = a.rowmap + (long long)g * a.n_pad + (long long)nt0 * a.bn;
+                    const int ncol = min(a.nacc, a.n_tiles - nt0) * a.bn;
+                    for (int i = et; i < ncol; i += kEpiWarps * 32) {
+                        const int f = __ldg(rmap + i);
+                        u_off[i] = f >= 0 ? f * a.plane : 0;
+                        u_bias[i] = (f >= 0 && a.bias) ? __ldg(a.bias + f) : 0.0f;
+                    }
+                }
+                const int* zmap = a.zeromap + (long long)g * a.Fg;
+                int* u_zero = s_zoff + ub * a.zcap;
+                for (int i = et; i < min(zc, a.zcap); i += kEpiWarps * 32) u_zero[i] = __ldg(zmap + i) * a.plane;
+                asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+                tab_key = key;
+            }
+            const int* u_off = s_eoff + ub * kTabCap;
+            const float* u_bias = s_ebias + ub * kTabCap;
             const long long m = mt * kBM + row;
             const bool valid = m < a.M;
             const long long n_img = valid ? m / a.plane : 0;
             const long long pix = valid ? m - n_img * a.plane : 0;
             float* yf = reinterpret_cast<float*>(a.y) + (n_img * (long long)a.F * a.plane + pix);
             __nv_bfloat16* yh = reinterpret_cast<__nv_bfloat16*>(a.y) + (n_img * (long long)a.F * a.plane + pix);
-            int* u_off = s_eoff + ub * 512;
-            float* u_bias = s_ebias + ub * 512;
-            if (cnt > 0) {
-                // column i of the unit = row i % bn of filter tile nt0 + i / bn
-                const int* rmap = a.rowmap + (long long)g * a.n_pad + (long long)nt0 * a.bn;
-                const int ncol = min(a.nacc, a.n_tiles - nt0) * a.bn;
-                for (int i = et; i < ncol; i += kEpiWarps * 32) {
-                    const int f = __ldg(rmap + i);
-                    u_off[i] = f >= 0 ? f * a.plane : 0;
-                    u_bias[i] = (f >= 0 && a.bias) ? __ldg(a.bias + f) : 0.0f;
-                }
-            }
-            asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
-            if (cnt > 0) {
-                // warp-uniform outcome: the TMEM loads below are .sync.aligned
-                if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[ab], acc_ph, abort_flag, a.status))) break;
+            int chunks = 0;  // accumulator chunks of this unit, over all its tiles
+            // warp-uniform outcome: the TMEM loads below are .sync.aligned
+            if (cnt > 0 && alive && !__all_sync(0xffffffffu, mbar_wait(&acc_full[ab], acc_ph, abort_flag, a.status)))
+                alive = false;
+            if (cnt > 0 && alive) {
                 tc_fence_after();
                 for (int ti = 0; ti < a.nacc && nt0 + ti < a.n_tiles; ++ti) {
                     const int nrows = min(a.bn, cnt - ti * a.bn);
                     if (nrows <= 0) break;
+                    const int nch = (nrows + kEpiCols - 1) / kEpiCols;
                     const uint32_t taddr = tmem_base + (uint32_t)((ab * a.nacc + ti) * a.tmem_stride) +
                                            ((uint32_t)(q * 32) << 16);
                     const int* t_off = u_off + ti * a.bn;
                     const float* t_bias = u_bias + ti * a.bn;
-                    for (int c0 = 32 * h; c0 < nrows; c0 += 32 * kHalves) {
-                        uint32_t r[32];
-                        tmem_ld_32x32b_x32(taddr + (uint32_t)c0, r);
+                    // chunk k of this tile is the unit's chunk chunks + k; warp h takes those = h mod kHalves
+                    for (int k = (h - chunks % kHalves + kHalves) % kHalves; k < nch; k += kHalves) {
+                        const int c0 = k * kEpiCols;
+                        uint32_t r[kEpiCols];
+                        tmem_ld_32x32b_x16(taddr + (uint32_t)c0, r);
                         tmem_ld_wait();
                         if (valid) {
+                            if (c0 + kEpiCols <= nrows) {
 #pragma unroll
-                            for (int j = 0; j < 32; ++j) {
-                                if (c0 + j < nrows) {
-                                    float v = __uint_as_float(r[j]) + t_bias[c0 + j];
-                                    if (a.relu) v = fmaxf(v, 0.0f);
-                                    if (OUT_BF16)
-                                        yh[t_off[c0 + j]] = __float2bfloat16_rn(v);
-                                    else
-                                        __stcs(yf + t_off[c0 + j], v);
+                                for (int j = 0; j < kEpiCols; j += 4) {
+                                    const int4 o = *reinterpret_cast<const int4*>(t_off + c0 + j);
+                                    const float4 b = *reinterpret_cast<const float4*>(t_bias + c0 + j);
+                                    float v0 = __uint_as_float(r[j]) + b.x, v1 = __uint_as_float(r[j + 1]) + b.y;
+                                    float v2 = __uint_as_float(r[j + 2]) + b.z, v3 = __uint_as_float(r[j + 3]) + b.w;
+                                    if (a.relu) {
+                                        v0 = fmaxf(v0, 0.0f); v1 = fmaxf(v1, 0.0f);
+                                        v2 = fmaxf(v2, 0.0f); v3 = fmaxf(v3, 0.0f);
+                                    }
+                                    if (OUT_BF16) {
+                                        yh[o.x] = __float2bfloat16_rn(v0); yh[o.y] = __float2bfloat16_rn(v1);
+                                        yh[o.z] = __float2bfloat16_rn(v2); yh[o.w] = __float2bfloat16_rn(v3);
+                                    } else {
+                                        __stcs(yf + o.x, v0); __stcs(yf + o.y, v1);
+                                        __stcs(yf + o.z, v2); __stcs(yf + o.w, v3);
+                                    }
+                                }
+                            } else {
+#pragma unroll
+                                for (int j = 0; j < kEpiCols; ++j) {
+                                    if (c0 + j < nrows) {
+                                        float v = __uint_as_float(r[j]) + t_bias[c0 + j];
+                                        if (a.relu) v = fmaxf(v, 0.0f);
+                                        if (OUT_BF16)
+                                            yh[t_off[c0 + j]] = __float2bfloat16_rn(v);
+                                        else
+                                            __stcs(yf + t_off[c0 + j], v);
+                                    }
                                 }
                             }
                         }
                     }
+                    chunks += nch;
                 }
                 tc_fence_before();
                 mbar_arrive(&acc_empty[ab]);
                 if (++ab == a.acc_bufs) { ab = 0; acc_ph ^= 1u; }
             }
-            if (p == 0) {
-                // pruned filters of this conv group: their planes are zero
-                const int zc = s_counts[2 * g + 1];
+            if (zc > 0 && valid && alive) {
+                // pruned filters of this conv group: their planes are zero.
+                // Chunks of 16 planes continue the unit's chunk sequence.
                 const int* zmap = a.zeromap + (long long)g * a.Fg;
-                for (int z0 = 32 * h; z0 < zc; z0 += 32 * kHalves) {
-                    const int zo = (z0 + lane < zc) ? __ldg(zmap + z0 + lane) * a.plane : 0;
-                    const int zn = min(32, zc - z0);
-                    for (int j = 0; j < zn; ++j) {
-                        const int off = __shfl_sync(0xffffffffu, zo, j);
-                        if (valid) {
+                const int* u_zero = s_zoff + ub * a.zcap;
+                const int nzc = (zc + kEpiCols - 1) / kEpiCols;
+                for (int k = (h - chunks % kHalves + kHalves) % kHalves; k < nzc; k += kHalves) {
+                    const int z0 = k * kEpiCols;
+                    if (z0 + kEpiCols <= a.zcap && z0 + kEpiCols <= zc) {
+#pragma unroll
+                        for (int j = 0; j < kEpiCols; j += 4) {
+                            const int4 o = *reinterpret_cast<const int4*>(u_zero + z0 + j);
+                            if (OUT_BF16) {
+                                const __nv_bfloat16 zb = __float2bfloat16_rn(0.0f);
+                                yh[o.x] = zb; yh[o.y] = zb; yh[o.z] = zb; yh[o.w] = zb;
+                            } else {
+                                __stcs(yf + o.x, 0.0f); __stcs(yf + o.y, 0.0f);
+                                __stcs(yf + o.z, 0.0f); __stcs(yf + o.w, 0.0f);
+                            }
+                        }
+                    } else {
+                        for (int z = z0; z < min(z0 + kEpiCols, zc); ++z) {
+                            const int off = z < a.zcap ? u_zero[z] : __ldg(zmap + z) * a.plane;
                             if (OUT_BF16)
                                 yh[off] = __float2bfloat16_rn(0.0f);
                             else
@@ -435,29 +451,24 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
             }
-            ub ^= 1;
         }
     } else if (warp >= 4 + kEpiWarps) {
         // ----------------------------------------------------------- gather
         const int gt = threadIdx.x - (4 + kEpiWarps) * 32;
-        const int prow = gt & (kBM - 1);
-        const int chunk0 = gt >> 7;  // this thread builds chunks chunk0 + kGatherGroups * i
+        const int set = gt / kSetThreads;
+        const int st = gt - set * kSetThreads;
+        const int prow = st & (kBM - 1);
+        const int chunk0 = st >> 7;  // this thread builds chunks chunk0 + kSetGroups * i
         const unsigned short* xs = reinterpret_cast<const unsigned short*>(a.x);
         int s = 0;
         uint32_t ph = 0;
+        int turn = 0;  // running stage index modulo kGatherSets
         bool ok = true;
-        int touched = 0;  // leading stages of the current unit already touched
         for (long long u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
             int p, g;
             long long mt;
             decode_unit(a, u, p, g, mt);
-            if (s_counts[2 * g] <= p * a.nacc * a.bn) {
-                touched = 0;
-                continue;
-            }
-            const TouchPlan tp_cur = touch_plan(a, u, gt);
-            const TouchPlan tp_next = touch_plan(a, u + gridDim.x, gt);
-            for (int q = touched; q < kTouchAhead; ++q) touch_stage(a, tp_cur, q);
+            if (s_counts[2 * g] <= p * a.nacc * a.bn) continue;
             const long long m = mt * kBM + prow;
             uint32_t M = 0;
             const unsigned short* xb = xs;
@@ -476,56 +487,52 @@ __global__ void __launch_bounds__(kThreads, 1)
             // Every lane's pixel sees every tap: no bounds test is needed.
             const bool interior = __all_sync(0xffffffffu, M == a.full_mask);
             for (int ks = 0; ks < a.nks; ++ks) {
-                // Land the input lines of the stage kTouchAhead ahead (of the
-                // next tile near the end of this one) in L1.
-                if (ks + kTouchAhead < a.nks)
-                    touch_stage(a, tp_cur, ks + kTouchAhead);
-                else
-                    touch_stage(a, tp_next, ks + kTouchAhead - a.nks);
-                // Issue every load of this thread's columns first (they read
-                // only x), then wait for the stage buffer and store.
-                const uint2* te = s_table + (size_t)ks * kBK;
-                uint32_t v[8 * kChunksPerThread];
-                // two table entries per 16-byte shared-memory load
-                const uint4* te4 = reinterpret_cast<const uint4*>(te);
-                if (interior && (ks + 1) * kBK <= a.n_cols) {
+                if (turn == set) {
+                    // Issue every load of this thread's columns first (they
+                    // read only x), then wait for the stage buffer and store.
+                    const uint2* te = s_table + (size_t)ks * kBK;
+                    uint32_t v[8 * kChunksPerThread];
+                    // two table entries per 16-byte shared-memory load
+                    const uint4* te4 = reinterpret_cast<const uint4*>(te);
+                    if (interior && (ks + 1) * kBK <= a.n_cols) {
 #pragma unroll
-                    for (int ci = 0; ci < kChunksPerThread; ++ci) {
-                        const int c = chunk0 + kGatherGroups * ci;
+                        for (int ci = 0; ci < kChunksPerThread; ++ci) {
+                            const int c = chunk0 + kSetGroups * ci;
 #pragma unroll
-                        for (int e = 0; e < 8; e += 2) {
-                            const uint4 t = te4[(c * 8 + e) >> 1];
-                            v[ci * 8 + e] = __ldg(xb + (int)t.x);
-                            v[ci * 8 + e + 1] = __ldg(xb + (int)t.z);
+                            for (int e = 0; e < 8; e += 2) {
+                                const uint4 t = te4[(c * 8 + e) >> 1];
+                                v[ci * 8 + e] = __ldg(xb + (int)t.x);
+                                v[ci * 8 + e + 1] = __ldg(xb + (int)t.z);
+                            }
+                        }
+                    } else {
+#pragma unroll
+                        for (int ci = 0; ci < kChunksPerThread; ++ci) {
+                            const int c = chunk0 + kSetGroups * ci;
+#pragma unroll
+                            for (int e = 0; e < 8; e += 2) {
+                                const uint4 t = te4[(c * 8 + e) >> 1];
+                                v[ci * 8 + e] = ldg_u16_if(xb + (int)t.x, t.y, M);
+                                v[ci * 8 + e + 1] = ldg_u16_if(xb + (int)t.z, t.w, M);
+                            }
                         }
                     }
-                } else {
+                    if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, a.status)) { ok = false; break; }
+                    uint8_t* tile = sA + (size_t)s * kATileBytes;
 #pragma unroll
                     for (int ci = 0; ci < kChunksPerThread; ++ci) {
-                        const int c = chunk0 + kGatherGroups * ci;
-#pragma unroll
-                        for (int e = 0; e < 8; e += 2) {
-                            const uint4 t = te4[(c * 8 + e) >> 1];
-                            v[ci * 8 + e] = ldg_u16_if(xb + (int)t.x, t.y, M);
-                            v[ci * 8 + e + 1] = ldg_u16_if(xb + (int)t.z, t.w, M);
-                        }
+                        const int c = chunk0 + kSetGroups * ci;
+                        const uint32_t* q = v + ci * 8;
+                        *reinterpret_cast<uint4*>(tile + sw128_offset((uint32_t)prow, (uint32_t)c)) =
+                            make_uint4(__byte_perm(q[0], q[1], 0x5410), __byte_perm(q[2], q[3], 0x5410),
+                                       __byte_perm(q[4], q[5], 0x5410), __byte_perm(q[6], q[7], 0x5410));
                     }
+                    fence_proxy_async_smem();
+                    mbar_arrive(&full_a[s]);
                 }
-                if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, a.status)) { ok = false; break; }
-                uint8_t* tile = sA + (size_t)s * kATileBytes;
-#pragma unroll
-                for (int ci = 0; ci < kChunksPerThread; ++ci) {
-                    const int c = chunk0 + kGatherGroups * ci;
-                    const uint32_t* q = v + ci * 8;
-                    *reinterpret_cast<uint4*>(tile + sw128_offset((uint32_t)prow, (uint32_t)c)) =
-                        make_uint4(__byte_perm(q[0], q[1], 0x5410), __byte_perm(q[2], q[3], 0x5410),
-                                   __byte_perm(q[4], q[5], 0x5410), __byte_perm(q[6], q[7], 0x5410));
-                }
-                fence_proxy_async_smem();
-                mbar_arrive(&full_a[s]);
                 if (++s == S) { s = 0; ph ^= 1u; }
+                if (++turn == kGatherSets) turn = 0;
             }
-            touched = min(kTouchAhead, a.nks);
         }
     }
 
@@ -565,7 +572,6 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     a.y = y;
     a.bias = bias;
     a.gather = reinterpret_cast<const uint2*>(base + plan->off_gather);
-    a.stage_chan = reinterpret_cast<const int2*>(a.gather + plan->k_pad);
     a.rowmap = reinterpret_cast<const int*>(base + plan->off_rowmap);
     a.zeromap = reinterpret_cast<const int*>(base + plan->off_zeromap);
     a.counts = reinterpret_cast<const int*>(base + plan->off_counts);
@@ -617,12 +623,23 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     a.stages = budget / stage_bytes;
     if (a.stages > kMaxStages) a.stages = kMaxStages;
     if (a.stages < 2) return SADMM_EUNSUPPORTED;
+    // Zero-plane offsets of a conv group (at most min(Fg, F - kept)) in shared
+    // memory, as far as the stages leave room; the rest are read from HBM.
+    {
+        long long zmax = g.f - plan->n_filt;
+        if (zmax > g.fg) zmax = g.fg;
+        if (zmax < 0) zmax = 0;
+        long long room = (budget - (long long)a.stages * stage_bytes) / 8;  // two buffers of 4-byte entries
+        if (room > 4096) room = 4096;
+        a.zcap = (int)(((zmax < room ? zmax : room) + 3) & ~3LL);
+        if ((long long)a.zcap > room) a.zcap = (int)(room & ~3LL);
+    }
     a.tmem_stride = (plan->bn + 31) & ~31;
     a.acc_bufs = (2 * a.nacc * a.tmem_stride <= 512) ? 2 : 1;
     int cols = 32;
     while (cols < a.acc_bufs * a.nacc * a.tmem_stride) cols <<= 1;
     a.tmem_cols = cols;
-    const size_t smem = 1024 + (size_t)a.stages * stage_bytes + table_bytes + kSmemTail;
+    const size_t smem = 1024 + (size_t)a.stages * stage_bytes + table_bytes + kSmemTail + (size_t)a.zcap * 8;
 
     long long grid = device_sm_count();
     if (grid > a.units) grid = a.units;
