@@ -393,6 +393,53 @@ def sweep_report(dev, out_dtype, reps=5):
     return out
 
 
+def admm_report(dev, peak_gbs, reps=5):
+    """sadmm_admm_update (the ADMM Z- and U-update, Sec. 4) on every AlexNet
+    CONV layer with fp32 W and U resident in HBM, L2 flushed before each
+    timed pass over the five layers.  Algorithmic bytes per layer: W and U read
+    once, Z and U written once (16 B per weight)."""
+    import torch
+    from paper_1807_11091_gb300 import sadmm
+    layers = wl.alexnet()
+    steps, bufs = [], []
+    for L in layers:
+        s = L.shape
+        st = wl.gen_admm_state(s, L.seed)
+        W, U = st["W"].to(dev), st["U"].to(dev)
+        bufs.append((W, U, torch.empty_like(W)))
+        steps.append(sadmm.AdmmStep(s.desc16(), L.k_filters, L.colkind, L.k_cols, dev))
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    for step, (W, U, Z) in zip(steps, bufs):
+        step(W, U, Z)
+    torch.cuda.synchronize()
+    per = [[] for _ in layers]
+    for _ in range(reps):
+        for i, (step, (W, U, Z)) in enumerate(zip(steps, bufs)):
+            flush.fill_(1)
+            torch.cuda._sleep(200_000)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+            step(W, U, Z)
+            e1.record()
+            torch.cuda.synchronize()
+            per[i].append(e0.elapsed_time(e1))
+    out = {"what": "sadmm_admm_update per AlexNet CONV layer, fp32 W/U/Z, L2 flushed", "layers": {}}
+    tot_ms = tot_bytes = 0.0
+    for L, ms in zip(layers, per):
+        t = statistics.median(ms)
+        nbytes = 16.0 * L.shape.f * L.shape.k
+        tot_ms += t
+        tot_bytes += nbytes
+        out["layers"][L.name] = {"us": t * 1e3, "gbs": nbytes / (t * 1e-3) / 1e9}
+    out["total_us"] = tot_ms * 1e3
+    out["gbs"] = tot_bytes / (tot_ms * 1e-3) / 1e9
+    out["hbm_frac"] = out["gbs"] / peak_gbs if peak_gbs else None
+    del bufs, steps, flush
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_gpu(args):
     import torch
     ws, rank, local = dist_env()
@@ -549,6 +596,8 @@ def run_gpu(args):
     }
     if rank == 0 and not args.no_sweep:
         line["sweep"] = sweep_report(dev, args.out_dtype)
+    if rank == 0 and not args.no_admm:
+        line["admm"] = admm_report(dev, peaks.get("hbm_gbs"))
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(layers, [wl.gen_tensors(L.shape.with_batch(16), seed=L.seed)
                                                      for L in layers])
@@ -569,6 +618,7 @@ def main():
     ap.add_argument("--out-dtype", default="fp32", choices=["fp32", "bf16"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--no-admm", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -140,6 +140,35 @@ sadmm_status sadmm_project_groups(const sadmm_conv_desc* d, const void* W, const
                                   int* filt_idx, int* col_idx, double* keys_out,
                                   void* workspace, size_t ws_bytes, void* stream);
 
+/* Device bytes of scratch sadmm_admm_update needs for this layer and column
+ * kind (the projection's keys plus row and column keep flags).  0 on a bad
+ * descriptor. */
+size_t sadmm_admm_workspace_size(const sadmm_conv_desc* d, int colkind);
+
+/*
+ * One ADMM Z- and U-update of a layer (Sec. 4): the Z-subproblem is solved by
+ * the Euclidean projection of V = W^{k+1} + U^k onto the structured-sparsity
+ * set, then the scaled dual becomes U^{k+1} = U^k + W^{k+1} - Z^{k+1}.
+ *
+ *   W       device [F][K] (OIDHW), dtype `wdt` (bf16 or fp32): W^{k+1}, read.
+ *   U       device [F][K], same dtype: U^k on entry, U^{k+1} on return.
+ *   Z       device [F][K], same dtype: Z^{k+1}, every element written.
+ *   k_filters, colkind, k_cols, filt_idx, col_idx, keys_out: as in
+ *           sadmm_project_groups, on V (the kept lists are returned too).
+ *   workspace  device scratch of at least sadmm_admm_workspace_size() bytes,
+ *           256-byte aligned.
+ *
+ * V is formed once in the tensors' precision (fp32 add, or bf16 inputs added
+ * in fp32 and rounded to nearest even); group keys use V widened exactly to
+ * fp64 as in sadmm_project_groups.  Z = V on every kept (filter, column) pair
+ * and 0 elsewhere; U^{k+1} = V - Z: 0 on the kept pairs and V elsewhere.
+ * W, U and Z must not overlap (SADMM_EINVAL).  F above 65535 gives
+ * SADMM_EUNSUPPORTED.
+ */
+sadmm_status sadmm_admm_update(const sadmm_conv_desc* d, const void* W, void* U, void* Z, int wdt,
+                               int k_filters, int colkind, int k_cols, int* filt_idx, int* col_idx,
+                               double* keys_out, void* workspace, size_t ws_bytes, void* stream);
+
 /*
  * Sizes a plan for `n_filt` kept filters and `n_colgroups` kept column groups
  * (columns or channels) of kind `colkind`.  Fills every size field of `plan`,

@@ -19,6 +19,8 @@ What it computes, with the passage each step follows:
 * ``masked_weights`` / ``masked_bias`` -- W with the pruned rows and columns
   of the GEMM matrix set to zero (Sec. 3, "Combination of structured
   sparsities"); the bias of a pruned filter is zero (a reading).
+* ``admm_update`` -- the ADMM Z-update (projection of W + U) and the dual
+  update U <- U + W - Z (Sec. 4), in the tensors' precision.
 * ``conv`` -- direct convolution over the full masked tensor (fp64).
 
 Parity pins: every function here is checked in ``tests/test_oracle_*.py``
@@ -222,6 +224,36 @@ def masked_bias(bias, F: int, filt_idx) -> np.ndarray:
     keep[np.asarray(filt_idx, dtype=np.int64)] = True
     b[~keep] = 0.0
     return b
+
+
+def admm_update(W, U, taps: int, k_filters: int, colkind: int, k_cols: int):
+    """One ADMM Z- and U-update (Sec. 4).
+
+    The Z-subproblem's optimum is the Euclidean projection of
+    V = W^{k+1} + U^k onto the structured-sparsity set (``project``), and the
+    scaled dual becomes U^{k+1} = U^k + W^{k+1} - Z^{k+1} = V - Z^{k+1}.
+    W and U are torch tensors of one dtype (bf16 or fp32).  V is formed
+    exactly in fp64 and rounded once to that dtype for Z and U^{k+1} (a
+    reading: the paper works in real arithmetic, the tensors keep their
+    precision), so Z is V on the kept (row, column) pairs and 0 elsewhere and
+    U^{k+1} is 0 on the kept pairs and V elsewhere.
+
+    Returns (filt_idx, col_idx, Z, U_next); Z and U_next have W's dtype and shape.
+    """
+    import torch
+    rows, cols, _, _ = project(W, taps, k_filters, colkind, k_cols, U=U)
+    V = as_matrix(W, U)
+    F, K = V.shape
+    rkeep = np.zeros(F, dtype=bool)
+    rkeep[np.asarray(rows, dtype=np.int64)] = True
+    ckeep = np.zeros(K, dtype=bool)
+    ckeep[expand_columns(colkind, cols, taps, K)] = True
+    keep = rkeep[:, None] & ckeep[None, :]
+    Z64 = np.where(keep, V, 0.0)
+    U64 = V - Z64
+    Z = torch.from_numpy(Z64).to(W.dtype).reshape(W.shape)
+    Un = torch.from_numpy(U64).to(W.dtype).reshape(W.shape)
+    return rows, cols, Z, Un
 
 
 # ---------------------------------------------------------------------------

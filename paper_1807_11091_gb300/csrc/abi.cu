@@ -143,6 +143,44 @@ sadmm_status sadmm_project_groups(const sadmm_conv_desc* d, const void* W, const
                           static_cast<cudaStream_t>(stream));
 }
 
+size_t sadmm_admm_workspace_size(const sadmm_conv_desc* d, int colkind)
+{
+    Geometry g;
+    if (check_desc(d, &g) != SADMM_OK) return 0;
+    return admm_workspace_bytes(g, colkind);
+}
+
+sadmm_status sadmm_admm_update(const sadmm_conv_desc* d, const void* W, void* U, void* Z, int wdt, int k_filters,
+                               int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out,
+                               void* workspace, size_t ws_bytes, void* stream)
+{
+    Geometry g;
+    sadmm_status st = check_desc(d, &g);
+    if (st != SADMM_OK) return st;
+    if (!W || !U || !Z || !filt_idx || !workspace) return SADMM_EINVAL;
+    if (wdt != SADMM_BF16 && wdt != SADMM_FP32) return SADMM_EINVAL;
+    if (colkind != SADMM_COL_NONE && colkind != SADMM_COL_SHAPE && colkind != SADMM_COL_CHANNEL)
+        return SADMM_EINVAL;
+    if (k_filters < 0 || k_filters > g.f) return SADMM_EINVAL;
+    if (colkind != SADMM_COL_NONE) {
+        const long long G = (colkind == SADMM_COL_SHAPE) ? g.k : g.cg;
+        if (k_cols < 0 || k_cols > G || !col_idx) return SADMM_EINVAL;
+    }
+    if (ws_bytes < admm_workspace_bytes(g, colkind)) return SADMM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0) return SADMM_EINVAL;
+    if (keys_out && (reinterpret_cast<uintptr_t>(keys_out) & 7) != 0) return SADMM_EINVAL;
+    const size_t esz = (wdt == SADMM_FP32) ? 4 : 2;
+    const uintptr_t bytes = (uintptr_t)(g.f * g.k) * esz;
+    const uintptr_t w = reinterpret_cast<uintptr_t>(W), u = reinterpret_cast<uintptr_t>(U),
+                    z = reinterpret_cast<uintptr_t>(Z);
+    if (((w | u | z) & (esz - 1)) != 0) return SADMM_EINVAL;
+    auto overlap = [bytes](uintptr_t p, uintptr_t q) { return p < q + bytes && q < p + bytes; };
+    if (overlap(w, u) || overlap(w, z) || overlap(u, z)) return SADMM_EINVAL;
+    if (g.f > 65535) return SADMM_EUNSUPPORTED;
+    return launch_admm_update(g, W, U, Z, wdt, k_filters, colkind, k_cols, filt_idx, col_idx, keys_out,
+                              workspace, static_cast<cudaStream_t>(stream));
+}
+
 sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d, int n_filt, int colkind,
                              int n_colgroups)
 {

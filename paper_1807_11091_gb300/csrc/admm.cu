@@ -1,0 +1,133 @@
+// admm.cu -- the ADMM Z- and U-update of one layer (Sec. 4).
+//
+// The Z-subproblem's optimum is the Euclidean projection of
+// V = W^{k+1} + U^k onto the structured-sparsity set S (Eq. 4 and the
+// filter-/channel-/shape-wise solutions of Sec. 4), and the scaled dual then
+// moves to U^{k+1} = U^k + W^{k+1} - Z^{k+1}.  With V formed once in the
+// tensors' precision, Z keeps V on the kept groups and is zero elsewhere, and
+// U^{k+1} = V - Z is zero on the kept groups and V elsewhere.
+//
+// Kernels (after the projection kernels of project.cu have produced the kept
+// filter and column lists from V):
+//   k_admm_masks  one block: byte flags of the kept rows [F] and kept GEMM
+//                 columns [K] from the index lists.
+//   k_admm_apply  one pass over the [F][K] matrix: read W and U, write Z and
+//                 U^{k+1}.  HBM bound: 2 reads + 2 writes per element.
+#include "common.cuh"
+#include "internal.h"
+
+namespace sadmm {
+namespace {
+
+constexpr int kApplyThreads = 256;
+constexpr int kApplyCols = 4;  // columns per thread
+
+__global__ void __launch_bounds__(1024) k_admm_masks(int F, int K, int taps, int colkind, int k_filters,
+                                                     const int* __restrict__ filt_idx, int k_cols,
+                                                     const int* __restrict__ col_idx, uint8_t* __restrict__ rkeep,
+                                                     uint8_t* __restrict__ ckeep)
+{
+    const int tid = threadIdx.x;
+    const bool all_rows = (k_filters >= F);
+    for (int a = tid; a < F; a += blockDim.x) rkeep[a] = all_rows ? 1 : 0;
+    for (int j = tid; j < K; j += blockDim.x) ckeep[j] = (colkind == SADMM_COL_NONE) ? 1 : 0;
+    __syncthreads();
+    if (!all_rows)
+        for (int i = tid; i < k_filters; i += blockDim.x) {
+            const int a = filt_idx[i];
+            if (a >= 0 && a < F) rkeep[a] = 1;
+        }
+    if (colkind == SADMM_COL_SHAPE) {
+        for (int i = tid; i < k_cols; i += blockDim.x) {
+            const int j = col_idx[i];
+            if (j >= 0 && j < K) ckeep[j] = 1;
+        }
+    } else if (colkind == SADMM_COL_CHANNEL) {
+        for (int i = tid; i < k_cols * taps; i += blockDim.x) {
+            const int b = col_idx[i / taps];
+            const int j = b * taps + i % taps;
+            if (b >= 0 && j < K) ckeep[j] = 1;
+        }
+    }
+}
+
+// V = W + U rounded once to the tensors' type (fp32 add; bf16 inputs add
+// exactly in fp32 unless their exponents differ by more than 16, and the
+// result is then rounded to nearest even).
+SADMM_DEV float vsum(float w, float u) { return w + u; }
+SADMM_DEV __nv_bfloat16 vsum(__nv_bfloat16 w, __nv_bfloat16 u)
+{
+    return __float2bfloat16_rn(__bfloat162float(w) + __bfloat162float(u));
+}
+template <typename T>
+SADMM_DEV T zero_of();
+template <>
+SADMM_DEV float zero_of<float>() { return 0.0f; }
+template <>
+SADMM_DEV __nv_bfloat16 zero_of<__nv_bfloat16>() { return __float2bfloat16_rn(0.0f); }
+
+// Block (bx, a): row a, columns bx*1024 .. bx*1024+1023, kApplyCols per thread
+// at a stride of kApplyThreads (coalesced).
+template <typename T>
+__global__ void __launch_bounds__(kApplyThreads) k_admm_apply(const T* __restrict__ W, T* __restrict__ U,
+                                                              T* __restrict__ Z, int K,
+                                                              const uint8_t* __restrict__ rkeep,
+                                                              const uint8_t* __restrict__ ckeep)
+{
+    const int a = blockIdx.y;
+    const bool rk = rkeep[a] != 0;
+    const long long base = (long long)a * K;
+    const int j0 = blockIdx.x * (kApplyThreads * kApplyCols) + threadIdx.x;
+    T w[kApplyCols], u[kApplyCols];
+#pragma unroll
+    for (int q = 0; q < kApplyCols; ++q) {
+        const int j = j0 + q * kApplyThreads;
+        if (j < K) {
+            w[q] = W[base + j];
+            u[q] = U[base + j];
+        }
+    }
+#pragma unroll
+    for (int q = 0; q < kApplyCols; ++q) {
+        const int j = j0 + q * kApplyThreads;
+        if (j < K) {
+            const T v = vsum(w[q], u[q]);
+            const bool keep = rk && ckeep[j] != 0;
+            Z[base + j] = keep ? v : zero_of<T>();
+            U[base + j] = keep ? zero_of<T>() : v;
+        }
+    }
+}
+
+size_t mask_bytes(const Geometry& g) { return (size_t)(round_up(g.f, 256) + round_up(g.k, 256)); }
+
+}  // namespace
+
+size_t admm_workspace_bytes(const Geometry& g, int colkind)
+{
+    return round_up((long long)project_workspace_bytes(g, colkind), 256) + mask_bytes(g);
+}
+
+sadmm_status launch_admm_update(const Geometry& g, const void* W, void* U, void* Z, int wdt, int k_filters,
+                                int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out, void* ws,
+                                cudaStream_t s)
+{
+    sadmm_status st = launch_project(g, W, U, wdt, k_filters, colkind, k_cols, filt_idx, col_idx, keys_out, ws, s);
+    if (st != SADMM_OK) return st;
+    uint8_t* rkeep = static_cast<uint8_t*>(ws) + round_up((long long)project_workspace_bytes(g, colkind), 256);
+    uint8_t* ckeep = rkeep + round_up(g.f, 256);
+    const int F = (int)g.f, K = (int)g.k;
+    k_admm_masks<<<1, 1024, 0, s>>>(F, K, (int)g.taps, colkind, k_filters, filt_idx, k_cols, col_idx, rkeep,
+                                    ckeep);
+    const dim3 grid((unsigned)((K + kApplyThreads * kApplyCols - 1) / (kApplyThreads * kApplyCols)), (unsigned)F);
+    if (wdt == SADMM_BF16)
+        k_admm_apply<__nv_bfloat16><<<grid, kApplyThreads, 0, s>>>(
+            static_cast<const __nv_bfloat16*>(W), static_cast<__nv_bfloat16*>(U), static_cast<__nv_bfloat16*>(Z),
+            K, rkeep, ckeep);
+    else
+        k_admm_apply<float><<<grid, kApplyThreads, 0, s>>>(static_cast<const float*>(W), static_cast<float*>(U),
+                                                           static_cast<float*>(Z), K, rkeep, ckeep);
+    return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
+}
+
+}  // namespace sadmm

@@ -37,6 +37,12 @@ sadmm_status launch_project(const Geometry& g, const void* W, const void* U, int
                             int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out,
                             void* ws, cudaStream_t s);
 
+// ---- ADMM Z/U update (admm.cu) ----
+size_t admm_workspace_bytes(const Geometry& g, int colkind);
+sadmm_status launch_admm_update(const Geometry& g, const void* W, void* U, void* Z, int wdt, int k_filters,
+                                int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out, void* ws,
+                                cudaStream_t s);
+
 // ---- pack (pack.cu) ----
 sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* filt_idx,
                          const int* col_idx, cudaStream_t s);

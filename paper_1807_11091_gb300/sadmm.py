@@ -90,6 +90,10 @@ def load():
     lib.sadmm_pack.argtypes = [P(Plan), vp, ci, vp, vp, vp, sz, vp]
     lib.sadmm_conv_fwd.restype = ci
     lib.sadmm_conv_fwd.argtypes = [P(Plan), vp, vp, ci, vp, ci, vp]
+    lib.sadmm_admm_workspace_size.restype = sz
+    lib.sadmm_admm_workspace_size.argtypes = [P(ConvDesc), ci]
+    lib.sadmm_admm_update.restype = ci
+    lib.sadmm_admm_update.argtypes = [P(ConvDesc), vp, vp, vp, ci, ci, ci, ci, vp, vp, vp, vp, sz, vp]
     lib.sadmm_last_device_status.restype = ci
     lib.sadmm_last_device_status.argtypes = [vp]
     lib.sadmm_project_groups_noalloc.restype = ci
@@ -152,6 +156,17 @@ def sadmm_project_groups_noalloc(desc: ConvDesc, W: int, U: Optional[int], wdt: 
     keys live in a fixed array inside the library (see include/sadmm.h)."""
     return load().sadmm_project_groups_noalloc(ctypes.byref(desc), W, U, int(wdt), int(k_filters),
                                                int(colkind), int(k_cols), filt_idx, col_idx, keys_out, stream)
+
+
+def sadmm_admm_workspace_size(desc: ConvDesc, colkind: int) -> int:
+    return load().sadmm_admm_workspace_size(ctypes.byref(desc), int(colkind))
+
+
+def sadmm_admm_update(desc: ConvDesc, W: int, U: int, Z: int, wdt: int, k_filters: int, colkind: int, k_cols: int,
+                      filt_idx: int, col_idx: Optional[int], keys_out: Optional[int], workspace: int,
+                      ws_bytes: int, stream: Optional[int]) -> int:
+    return load().sadmm_admm_update(ctypes.byref(desc), W, U, Z, int(wdt), int(k_filters), int(colkind),
+                                    int(k_cols), filt_idx, col_idx, keys_out, workspace, int(ws_bytes), stream)
 
 
 def sadmm_plan_init(desc: ConvDesc, n_filt: int, colkind: int, n_colgroups: int) -> Tuple[int, Plan]:
@@ -227,6 +242,39 @@ def project_groups(desc16: Sequence[int], W, k_filters: int, colkind: int, k_col
     fi = filt_idx[:k_filters]
     ci = col_idx[:k_cols] if col_idx is not None else None
     return fi, ci, keys
+
+
+class AdmmStep:
+    """Device buffers for repeated sadmm_admm_update calls on one layer: the
+    kept index lists, the optional keys and the workspace."""
+
+    def __init__(self, desc16: Sequence[int], k_filters: int, colkind: int, k_cols: int, device,
+                 with_keys: bool = False):
+        torch = _torch()
+        self.desc16 = [int(v) for v in desc16]
+        self.desc = make_desc(self.desc16)
+        self.k_filters, self.colkind, self.k_cols = int(k_filters), int(colkind), int(k_cols)
+        self.ws_bytes = sadmm_admm_workspace_size(self.desc, colkind)
+        if self.ws_bytes == 0:
+            raise SadmmError(SADMM_EINVAL, "sadmm_admm_workspace_size")
+        self.workspace = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device)
+        f = self.desc16[5]
+        cg = self.desc16[1] // self.desc16[6]
+        taps = self.desc16[7] * self.desc16[8] * self.desc16[9]
+        G = 0 if colkind == SADMM_COL_NONE else (cg * taps if colkind == SADMM_COL_SHAPE else cg)
+        self.filt_idx = torch.empty(max(k_filters, 1), dtype=torch.int32, device=device)
+        self.col_idx = (torch.empty(max(k_cols, 1), dtype=torch.int32, device=device)
+                        if colkind != SADMM_COL_NONE else None)
+        self.keys = torch.empty(f + G, dtype=torch.float64, device=device) if with_keys else None
+
+    def __call__(self, W, U, Z, stream=None):
+        """Z <- Proj_S(W + U); U <- (W + U) - Z.  Returns (filt_idx, col_idx)."""
+        st = sadmm_admm_update(self.desc, _ptr(W), _ptr(U), _ptr(Z), _wdt(W), self.k_filters, self.colkind,
+                               self.k_cols, _ptr(self.filt_idx), _ptr(self.col_idx), _ptr(self.keys),
+                               _ptr(self.workspace), self.ws_bytes, _stream(stream))
+        _check(st, "sadmm_admm_update")
+        ci = self.col_idx[:self.k_cols] if self.col_idx is not None else None
+        return self.filt_idx[:self.k_filters], ci
 
 
 class PrunedConv:

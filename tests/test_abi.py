@@ -94,3 +94,20 @@ def test_conv_rejects_unbound_plan_and_nulls():
     assert sadmm.sadmm_conv_fwd(p, fake, None, 1, fake, 7, None) == sadmm.SADMM_EINVAL
     assert sadmm.sadmm_pack(p, fake, 0, None, fake, fake, p.dev_bytes - 1, None) == sadmm.SADMM_EINVAL
     assert sadmm.sadmm_pack(p, fake, 0, None, fake, fake + 8, p.dev_bytes, None) == sadmm.SADMM_EINVAL
+
+
+def test_admm_update_rejects_bad_arguments_on_host():
+    s = wl.single2d()[0].shape
+    d = sadmm.make_desc(s.desc16())
+    ws = sadmm.sadmm_admm_workspace_size(d, wl.COL_SHAPE)
+    assert ws >= sadmm.sadmm_workspace_size(d, wl.COL_SHAPE) + s.f + s.k
+    nbytes = s.f * s.k * 4
+    W, U, Z, ws_ptr = 1 << 24, (1 << 24) + (1 << 22), (1 << 24) + (2 << 22), 1 << 30  # never dereferenced
+    args = dict(W=W, U=U, Z=Z, wdt=sadmm.SADMM_FP32, k_filters=1, colkind=wl.COL_SHAPE, k_cols=1, filt_idx=W,
+                col_idx=W, keys_out=None, workspace=ws_ptr, ws_bytes=ws, stream=None)
+    for bad in (dict(U=None), dict(Z=None), dict(W=None), dict(workspace=None), dict(ws_bytes=ws - 1),
+                dict(workspace=ws_ptr + 16), dict(k_filters=s.f + 1), dict(k_cols=s.k + 1), dict(wdt=4),
+                dict(colkind=5), dict(Z=U), dict(Z=U + nbytes - 4), dict(U=W + 4), dict(W=W + 2),
+                dict(keys_out=ws_ptr + 4)):
+        a = dict(args, **bad)
+        assert sadmm.sadmm_admm_update(d, **a) == sadmm.SADMM_EINVAL, bad

@@ -198,6 +198,18 @@ def gen_dual(shape: ConvShape, seed: int, scale: float = 0.01) -> torch.Tensor:
     return (torch.randn(shape.w_shape(), generator=g, dtype=torch.float32) * scale).to(torch.bfloat16)
 
 
+def gen_admm_state(shape: ConvShape, seed: int, dtype=torch.float32) -> Dict[str, torch.Tensor]:
+    """Seeded ADMM state of one layer in training precision: W ~ N(0, 2/fan_in)
+    and the scaled dual U ~ N(0, 0.1 * 2/fan_in), drawn in fp32 in that order
+    (then cast to `dtype`)."""
+    g = torch.Generator().manual_seed(int(seed) + 104729)
+    fan_in = shape.cg * shape.taps
+    sd = math.sqrt(2.0 / fan_in)
+    W = torch.randn(shape.w_shape(), generator=g, dtype=torch.float32) * sd
+    U = torch.randn(shape.w_shape(), generator=g, dtype=torch.float32) * (sd * math.sqrt(0.1))
+    return {"W": W.to(dtype), "U": U.to(dtype)}
+
+
 def gen_integer_weights(shape: ConvShape, seed: int, lo: int = -3, hi: int = 3) -> torch.Tensor:
     """Small-integer weights (exact in bf16; group sums exact in any order) for tie tests."""
     g = torch.Generator().manual_seed(int(seed))
