@@ -48,7 +48,9 @@ constexpr int kSetGroups = kSetThreads / kBM;       // threads of a set per pixe
 constexpr int kChunksPerThread = 8 / kSetGroups;    // 16-byte chunks of a stage row per thread
 static_assert(kSetThreads % kBM == 0 && 8 % kSetGroups == 0, "a gather set must split a 64-column row evenly");
 constexpr int kATileBytes = kBM * kBK * 2;  // 16 KB
-constexpr int kMaxStages = 4;
+constexpr int kMaxStages = 8;        // A stages (and B stages when B streams)
+constexpr int kStreamStages = 4;     // stages when B streams with A
+constexpr int kResidentStages = 6;   // A stages when the packed weights stay in shared memory
 constexpr int kMaxGroups = 64;
 constexpr int kEpiCols = 16;       // accumulator columns per epilogue TMEM load
 constexpr int kTabCap = 512;       // kept-row entries of an epilogue table buffer
@@ -61,6 +63,27 @@ constexpr int kTailBars = kTailCounts + 2 * kMaxGroups * 4;
 constexpr int kTailZero = kTailBars + 512;
 constexpr int kSmemTail = kTailZero;
 
+// Division of a non-negative int below 2^31 by an invariant divisor d >= 1:
+// q = (umulhi(n, mul) + n) >> shift with shift = ceil(log2 d) and
+// mul = floor(2^32 (2^shift - d) / d) + 1 (the round-up method of Granlund
+// and Montgomery); umulhi(n, mul) <= n, so the sum stays below 2^32.
+struct FastDiv {
+    uint32_t d, mul, shift;
+};
+
+inline FastDiv make_fastdiv(uint32_t d)
+{
+    FastDiv f;
+    f.d = d;
+    uint32_t s = 0;
+    while ((1ull << s) < d) ++s;
+    f.shift = s;
+    f.mul = (uint32_t)((((1ull << s) - d) << 32) / d + 1);
+    return f;
+}
+
+SADMM_DEV uint32_t fdiv(uint32_t n, const FastDiv& f) { return (__umulhi(n, f.mul) + n) >> f.shift; }
+
 struct ConvArgs {
     const __nv_bfloat16* x;
     void* y;
@@ -70,10 +93,11 @@ struct ConvArgs {
     const int* zeromap;
     const int* counts;
     int* status;
-    long long M;      // N * plane
+    int M;            // N * plane (below 2^31)
     long long x_chw;  // elements per input image
     long long thw;    // elements per input channel
-    long long units;  // m_tiles * groups * upairs
+    int units;        // m_tiles * groups * upairs (below 2^31)
+    FastDiv upairs_div, mtiles_div, plane_div, ohw_div, ow_div;
     int hw, W, H, T;
     int F, groups, Cg, Fg;
     int OW, OHW, plane;
@@ -84,6 +108,7 @@ struct ConvArgs {
     int nacc;      // filter tiles per unit (TMEM accumulators sharing one A tile)
     int upairs;    // units per (pixel tile, group): ceil(n_tiles / nacc)
     int acc_bufs;  // accumulator sets in TMEM (2: the epilogue overlaps the next unit's MMAs)
+    int b_res;     // 1: a conv group's packed weights stay in shared memory for all its units
     int stages;
     int k_pad;
     int n_cols;          // K' (columns past it are padding)
@@ -96,13 +121,15 @@ struct ConvArgs {
 };
 
 // Unit u covers filter tiles p*nacc .. p*nacc+nacc-1 of conv group g for pixel
-// tile mt.
-SADMM_DEV void decode_unit(const ConvArgs& a, long long u, int& p, int& g, long long& mt)
+// tile mt.  Groups are outermost, so a CTA (units u, u + grid, ...) stays in
+// one conv group for long runs and rarely reloads resident weights.
+SADMM_DEV void decode_unit(const ConvArgs& a, int u, int& p, int& g, int& mt)
 {
-    p = (int)(u % a.upairs);
-    const long long t = u / a.upairs;
-    g = (int)(t % a.groups);
-    mt = t / a.groups;
+    const uint32_t t = fdiv((uint32_t)u, a.upairs_div);
+    p = u - (int)(t * a.upairs_div.d);
+    const uint32_t gq = fdiv(t, a.mtiles_div);
+    mt = (int)(t - gq * a.mtiles_div.d);
+    g = (int)gq;
 }
 
 // Tap-validity mask of one output pixel: a bit is set where a tap reads inside
@@ -156,7 +183,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t bstage = b_bytes * (uint32_t)a.nacc;  // a B stage holds nacc boxes
     uint8_t* sA = smem;
     uint8_t* sB = smem + (size_t)S * kATileBytes;
-    uint2* s_table = reinterpret_cast<uint2*>(sB + (size_t)S * bstage);
+    // resident weights: the nks boxes of one conv group's filter tile
+    uint2* s_table = reinterpret_cast<uint2*>(sB + (a.b_res ? (size_t)a.nks * b_bytes : (size_t)S * bstage));
     uint8_t* tail = reinterpret_cast<uint8_t*>(s_table + a.k_pad);  // 512-byte aligned
     int* s_eoff = reinterpret_cast<int*>(tail + kTailOffBias);                   // [2][kTabCap] plane offsets
     float* s_ebias = reinterpret_cast<float*>(tail + kTailOffBias) + 2 * kTabCap;  // [2][kTabCap] biases
@@ -169,22 +197,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* acc_full = bars + 3 * S;
     uint64_t* acc_empty = acc_full + 2;
     uint64_t* drain = acc_empty + 2;
-    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+    uint64_t* b_full = drain + 1;   // resident weights landed
+    uint64_t* b_empty = drain + 2;  // every MMA on the resident weights completed
+    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 3);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
-            mbar_init(&full_a[s], kSetThreads);
+            mbar_init(&full_a[s], kSetThreads / 32);  // one arrival per gather warp of a set
             mbar_init(&full_b[s], 1);
             mbar_init(&empty[s], 1);
         }
         for (int b = 0; b < a.acc_bufs; ++b) {
             mbar_init(&acc_full[b], 1);
-            mbar_init(&acc_empty[b], kEpiWarps * 32);
+            mbar_init(&acc_empty[b], kEpiWarps);  // one arrival per epilogue warp
         }
         mbar_init(drain, 1);
+        mbar_init(b_full, 1);
+        mbar_init(b_empty, 1);
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -207,15 +239,44 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (warp == 0) {
         // ------------------------------------------------ TMA producer (Wp)
-        if (lane == 0) {
+        if (lane == 0 && a.b_res) {
+            // One load of the unit's filter tile (all nks boxes) per change of
+            // (group, filter tile), after the MMAs on the previous one retired.
+            long long cur = -1;
+            uint32_t e_ph = 0;
+            int loads = 0;
+            for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
+                int p, g;
+                int mt;
+                decode_unit(a, u, p, g, mt);
+                if (s_counts[2 * g] <= p * a.bn) continue;
+                const long long key = (long long)g * a.upairs + p;
+                if (key == cur) continue;
+                if (loads > 0) {
+                    if (!mbar_wait(b_empty, e_ph, abort_flag, a.status)) break;
+                    e_ph ^= 1u;
+                }
+                mbar_arrive_expect_tx(b_full, b_bytes * (uint32_t)a.nks);
+                const int row0 = g * a.n_pad + p * a.bn;
+                for (int ks = 0; ks < a.nks; ++ks)
+                    tma_load_2d(sB + (size_t)ks * b_bytes, &tmap, b_full, ks * kBK, row0);
+                cur = key;
+                ++loads;
+            }
+            // the last load has landed before the CTA retires
+            if (loads > 0) {
+                const unsigned long long t0 = globaltimer();
+                while (!mbar_try_wait(b_full, (uint32_t)((loads - 1) & 1)) && globaltimer() - t0 < kWaitLimitNs) {}
+            }
+        } else if (lane == 0) {
             int s = 0;
             uint32_t ph = 0;
             uint32_t issued_parity[kMaxStages];
             uint32_t issued_mask = 0;
             bool ok = true;
-            for (long long u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
+            for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
                 int p, g;
-                long long mt;
+                int mt;
                 decode_unit(a, u, p, g, mt);
                 const int nt0 = p * a.nacc;
                 if (s_counts[2 * g] <= nt0 * a.bn) continue;
@@ -250,12 +311,24 @@ __global__ void __launch_bounds__(kThreads, 1)
             int ab = 0;
             uint32_t acc_ph = 0;
             bool ok = true;
-            for (long long u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
+            long long cur = -1;    // (group, filter tile) of the resident weights
+            uint32_t bf_ph = 0;
+            const uint32_t sB0 = smem_u32(sB);
+            for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
                 int p, g;
-                long long mt;
+                int mt;
                 decode_unit(a, u, p, g, mt);
                 const int cnt = s_counts[2 * g] - p * a.nacc * a.bn;  // kept rows from the unit's first tile
                 if (cnt <= 0) continue;
+                if (a.b_res) {
+                    const long long key = (long long)g * a.upairs + p;
+                    if (key != cur) {
+                        if (cur >= 0) mma_commit(b_empty);  // the old weights are free once these MMAs finish
+                        if (!mbar_wait(b_full, bf_ph, abort_flag, a.status)) break;
+                        bf_ph ^= 1u;
+                        cur = key;
+                    }
+                }
                 // one accumulator per filter tile with kept rows, N rounded up to 16
                 const int rows1 = (a.nacc == 2 && p * 2 + 1 < a.n_tiles) ? min(a.bn, cnt - a.bn) : 0;
                 const uint32_t idesc0 = idesc_bf16_f32(kBM, min(a.bn, (cnt + 15) & ~15));
@@ -266,13 +339,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t d_tmem = tmem_base + (uint32_t)(ab * a.nacc * a.tmem_stride);
                 for (int ks = 0; ks < a.nks; ++ks) {
                     if (!mbar_wait(&full_a[s], ph, abort_flag, a.status) ||
-                        !mbar_wait(&full_b[s], ph, abort_flag, a.status)) {
+                        (!a.b_res && !mbar_wait(&full_b[s], ph, abort_flag, a.status))) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
                     const uint32_t a0 = smem_u32(sA + (size_t)s * kATileBytes);
-                    const uint32_t b0 = smem_u32(sB + (size_t)s * bstage);
+                    const uint32_t b0 = sB0 + (a.b_res ? (uint32_t)ks * b_bytes : (uint32_t)s * bstage);
                     // The issuing thread is on the critical path: straight-line
                     // code, descriptors in registers.
                     if (!two) {
@@ -323,9 +396,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         // After a failed wait (another role aborted) the warp keeps walking the
         // units, without TMEM or stores, so the named barrier stays balanced.
         bool alive = true;
-        for (long long u = blockIdx.x; u < a.units; u += gridDim.x) {
+        for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
             int p, g;
-            long long mt;
+            int mt;
             decode_unit(a, u, p, g, mt);
             const int nt0 = p * a.nacc;
             const int cnt = s_counts[2 * g] - nt0 * a.bn;  // kept rows from the unit's first tile
@@ -353,9 +426,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             const int* u_off = s_eoff + ub * kTabCap;
             const float* u_bias = s_ebias + ub * kTabCap;
-            const long long m = mt * kBM + row;
+            const int m = mt * kBM + row;
             const bool valid = m < a.M;
-            const long long n_img = valid ? m / a.plane : 0;
+            const long long n_img = valid ? (long long)fdiv((uint32_t)m, a.plane_div) : 0;
             const long long pix = valid ? m - n_img * a.plane : 0;
             float* yf = reinterpret_cast<float*>(a.y) + (n_img * (long long)a.F * a.plane + pix);
             __nv_bfloat16* yh = reinterpret_cast<__nv_bfloat16*>(a.y) + (n_img * (long long)a.F * a.plane + pix);
@@ -417,7 +490,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     chunks += nch;
                 }
                 tc_fence_before();
-                mbar_arrive(&acc_empty[ab]);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&acc_empty[ab]);
                 if (++ab == a.acc_bufs) { ab = 0; acc_ph ^= 1u; }
             }
             if (zc > 0 && valid && alive) {
@@ -464,20 +538,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t ph = 0;
         int turn = 0;  // running stage index modulo kGatherSets
         bool ok = true;
-        for (long long u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
+        for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
             int p, g;
-            long long mt;
+            int mt;
             decode_unit(a, u, p, g, mt);
             if (s_counts[2 * g] <= p * a.nacc * a.bn) continue;
-            const long long m = mt * kBM + prow;
+            const int m = mt * kBM + prow;
             uint32_t M = 0;
             const unsigned short* xb = xs;
             if (m < a.M) {
-                const long long n_img = m / a.plane;
+                const long long n_img = fdiv((uint32_t)m, a.plane_div);
                 const int p = (int)(m - n_img * a.plane);
-                const int ot = p / a.OHW;
+                const int ot = (int)fdiv((uint32_t)p, a.ohw_div);
                 const int r2 = p - ot * a.OHW;
-                const int oh = r2 / a.OW;
+                const int oh = (int)fdiv((uint32_t)r2, a.ow_div);
                 const int ow = r2 - oh * a.OW;
                 const int it0 = ot * a.st - a.pt, ih0 = oh * a.sh - a.ph, iw0 = ow * a.sw - a.pw;
                 M = pixel_mask(a, it0, ih0, iw0);
@@ -527,8 +601,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                             make_uint4(__byte_perm(q[0], q[1], 0x5410), __byte_perm(q[2], q[3], 0x5410),
                                        __byte_perm(q[4], q[5], 0x5410), __byte_perm(q[6], q[7], 0x5410));
                     }
+                    // every lane's stores are visible to the tensor core's async
+                    // proxy, then one arrival for the warp
                     fence_proxy_async_smem();
-                    mbar_arrive(&full_a[s]);
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&full_a[s]);
                 }
                 if (++s == S) { s = 0; ph ^= 1u; }
                 if (++turn == kGatherSets) turn = 0;
@@ -576,7 +653,8 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     a.zeromap = reinterpret_cast<const int*>(base + plan->off_zeromap);
     a.counts = reinterpret_cast<const int*>(base + plan->off_counts);
     a.status = device_status_ptr();
-    a.M = g.m;
+    if (g.m >= (1ll << 31) - 256) return SADMM_EUNSUPPORTED;  // pixel indices stay in int
+    a.M = (int)g.m;
     a.x_chw = g.c * g.t * g.h * g.w;
     a.thw = g.t * g.h * g.w;
     a.hw = (int)(g.h * g.w);
@@ -607,7 +685,14 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     a.n_pad = plan->n_pad;
     a.relu = relu ? 1 : 0;
     const long long m_tiles = (g.m + kBM - 1) / kBM;
-    a.units = m_tiles * g.groups * a.upairs;
+    const long long units = m_tiles * g.groups * a.upairs;
+    if (units >= (1ll << 31) - (1ll << 20)) return SADMM_EUNSUPPORTED;  // u + grid stays below 2^31
+    a.units = (int)units;
+    a.upairs_div = make_fastdiv((uint32_t)a.upairs);
+    a.mtiles_div = make_fastdiv((uint32_t)m_tiles);
+    a.plane_div = make_fastdiv((uint32_t)g.plane);
+    a.ohw_div = make_fastdiv((uint32_t)(g.oh * g.ow));
+    a.ow_div = make_fastdiv((uint32_t)g.ow);
 
     a.k_pad = plan->k_pad;
     a.n_cols = plan->n_cols;
@@ -616,20 +701,35 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
         a.full_mask = ((1u << (g.kt * g.kh)) - 1u) | (((1u << g.kw) - 1u) << 16);
     else
         a.full_mask = (uint32_t)((1ull << g.taps) - 1ull);
-    const int stage_bytes = kATileBytes + a.nacc * plan->bn * 128;
     const int table_bytes = plan->k_pad * 8;
     const int budget = 232448 - 1024 - kSmemTail - table_bytes;
-    // At most kMaxStages: what shared memory leaves over serves as L1 for x.
-    a.stages = budget / stage_bytes;
-    if (a.stages > kMaxStages) a.stages = kMaxStages;
-    if (a.stages < 2) return SADMM_EUNSUPPORTED;
+    // One filter tile per group: keep the group's packed weights (nks boxes)
+    // in shared memory when that leaves room for at least 3 A stages.
+    const long long res_bytes = (long long)plan->bn * 128 * a.nks;
+    int stage_bytes;
+    long long fixed_bytes;
+    if (plan->n_tiles == 1 && budget - res_bytes >= 3LL * kATileBytes) {
+        a.b_res = 1;
+        stage_bytes = kATileBytes;
+        fixed_bytes = res_bytes;
+        a.stages = (int)((budget - res_bytes) / kATileBytes);
+        if (a.stages > kResidentStages) a.stages = kResidentStages;
+    } else {
+        // At most kStreamStages: what shared memory leaves over serves as L1 for x.
+        a.b_res = 0;
+        stage_bytes = kATileBytes + a.nacc * plan->bn * 128;
+        fixed_bytes = 0;
+        a.stages = budget / stage_bytes;
+        if (a.stages > kStreamStages) a.stages = kStreamStages;
+        if (a.stages < 2) return SADMM_EUNSUPPORTED;
+    }
     // Zero-plane offsets of a conv group (at most min(Fg, F - kept)) in shared
     // memory, as far as the stages leave room; the rest are read from HBM.
     {
         long long zmax = g.f - plan->n_filt;
         if (zmax > g.fg) zmax = g.fg;
         if (zmax < 0) zmax = 0;
-        long long room = (budget - (long long)a.stages * stage_bytes) / 8;  // two buffers of 4-byte entries
+        long long room = (budget - fixed_bytes - (long long)a.stages * stage_bytes) / 8;  // two buffers of 4-byte entries
         if (room > 4096) room = 4096;
         a.zcap = (int)(((zmax < room ? zmax : room) + 3) & ~3LL);
         if ((long long)a.zcap > room) a.zcap = (int)(room & ~3LL);
@@ -639,7 +739,8 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     int cols = 32;
     while (cols < a.acc_bufs * a.nacc * a.tmem_stride) cols <<= 1;
     a.tmem_cols = cols;
-    const size_t smem = 1024 + (size_t)a.stages * stage_bytes + table_bytes + kSmemTail + (size_t)a.zcap * 8;
+    const size_t smem =
+        1024 + (size_t)fixed_bytes + (size_t)a.stages * stage_bytes + table_bytes + kSmemTail + (size_t)a.zcap * 8;
 
     long long grid = device_sm_count();
     if (grid > a.units) grid = a.units;

@@ -3,7 +3,8 @@
     python -m paper_1807_11091_gb300.run_layer --workload sweep --layer 0 --reps 3
 
 Projection and pack run once; sadmm_conv_fwd runs `reps` times, each timed with
-CUDA events on the launching stream.  Prints one line per run: time, TFLOP/s on
+CUDA events on the launching stream (after a device-side sleep, so the host's
+launch latency stays outside the timed interval).  Prints one line per run: time, TFLOP/s on
 retained MACs and the plan's tile sizes.  This is the program the per-kernel
 profiles run under ncu.
 """
@@ -48,6 +49,9 @@ def main(argv=None) -> int:
     for i in range(args.reps):
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
+        # a short device-side sleep first, so the host finishes enqueueing the
+        # forward call before the start event is reached on the GPU
+        torch.cuda._sleep(200_000)
         e0.record()
         pc.forward(t["x"], t["bias"], out=y)
         e1.record()
