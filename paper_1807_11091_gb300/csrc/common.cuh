@@ -78,6 +78,22 @@ SADMM_DEV bool mbar_try_wait(uint64_t* bar, uint32_t parity)
     return ok != 0;
 }
 
+// try_wait with a suspend-time hint: a thread whose phase is not complete is
+// suspended (it issues nothing) until the phase completes or about `hint_ns`
+// pass, instead of spinning on the barrier.
+constexpr uint32_t kSuspendHintNs = 1000000;  // 1 ms
+
+SADMM_DEV bool mbar_try_wait_suspend(uint64_t* bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(kSuspendHintNs)
+        : "memory");
+    return ok != 0;
+}
+
 // Waits until the phase with the given parity of `bar` has completed.
 // Returns false (and raises the abort flag and the status word) when the wait
 // runs past kWaitLimitNs, or false at once when another role aborted.
@@ -85,15 +101,13 @@ SADMM_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_fla
 {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = globaltimer();
-    for (uint32_t it = 1;; ++it) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if ((it & 63u) == 0) {
-            if (*abort_flag) return false;
-            if (globaltimer() - t0 > kWaitLimitNs) {
-                *abort_flag = 1;
-                raise_status(status, kDevTimeout);
-                return false;
-            }
+    for (;;) {
+        if (mbar_try_wait_suspend(bar, parity)) return true;
+        if (*abort_flag) return false;
+        if (globaltimer() - t0 > kWaitLimitNs) {
+            *abort_flag = 1;
+            raise_status(status, kDevTimeout);
+            return false;
         }
     }
 }

@@ -303,6 +303,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 while (!mbar_try_wait(&full_b[q], issued_parity[q]) && globaltimer() - t0 < kWaitLimitNs) {}
             }
         }
+        __syncwarp();  // the whole warp reaches the block barrier below together
     } else if (warp == 1) {
         // ------------------------------------------------------- MMA issuer
         if (lane == 0) {
