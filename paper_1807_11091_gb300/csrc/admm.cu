@@ -7,10 +7,8 @@
 // tensors' precision, Z keeps V on the kept groups and is zero elsewhere, and
 // U^{k+1} = V - Z is zero on the kept groups and V elsewhere.
 //
-// Kernels (after the projection kernels of project.cu have produced the kept
-// filter and column lists from V):
-//   k_admm_masks  one block: byte flags of the kept rows [F] and kept GEMM
-//                 columns [K] from the index lists.
+// After the projection kernels of project.cu have selected the kept filters
+// and column groups from V (and written a keep flag per group),
 //   k_admm_apply  one pass over the [F][K] matrix: read W and U, write Z and
 //                 U^{k+1}.  HBM bound: 2 reads + 2 writes per element.
 #include "common.cuh"
@@ -21,35 +19,6 @@ namespace {
 
 constexpr int kApplyThreads = 256;
 constexpr int kApplyCols = 4;  // columns per thread
-
-__global__ void __launch_bounds__(1024) k_admm_masks(int F, int K, int taps, int colkind, int k_filters,
-                                                     const int* __restrict__ filt_idx, int k_cols,
-                                                     const int* __restrict__ col_idx, uint8_t* __restrict__ rkeep,
-                                                     uint8_t* __restrict__ ckeep)
-{
-    const int tid = threadIdx.x;
-    const bool all_rows = (k_filters >= F);
-    for (int a = tid; a < F; a += blockDim.x) rkeep[a] = all_rows ? 1 : 0;
-    for (int j = tid; j < K; j += blockDim.x) ckeep[j] = (colkind == SADMM_COL_NONE) ? 1 : 0;
-    __syncthreads();
-    if (!all_rows)
-        for (int i = tid; i < k_filters; i += blockDim.x) {
-            const int a = filt_idx[i];
-            if (a >= 0 && a < F) rkeep[a] = 1;
-        }
-    if (colkind == SADMM_COL_SHAPE) {
-        for (int i = tid; i < k_cols; i += blockDim.x) {
-            const int j = col_idx[i];
-            if (j >= 0 && j < K) ckeep[j] = 1;
-        }
-    } else if (colkind == SADMM_COL_CHANNEL) {
-        for (int i = tid; i < k_cols * taps; i += blockDim.x) {
-            const int b = col_idx[i / taps];
-            const int j = b * taps + i % taps;
-            if (b >= 0 && j < K) ckeep[j] = 1;
-        }
-    }
-}
 
 // V = W + U rounded once to the tensors' type (fp32 add; bf16 inputs add
 // exactly in fp32 unless their exponents differ by more than 16, and the
@@ -68,11 +37,15 @@ SADMM_DEV __nv_bfloat16 zero_of<__nv_bfloat16>() { return __float2bfloat16_rn(0.
 
 // Block (bx, a): row a, columns bx*1024 .. bx*1024+1023, kApplyCols per thread
 // at a stride of kApplyThreads (coalesced).
+// Column j keeps when its group's flag is set: ckeep[j] (shape-wise),
+// ckeep[j / taps] (channel-wise), always (ckeep == NULL).  The division by
+// taps is q = (umulhi(j, tmul) + j) >> tshift (exact for j < 2^31).
 template <typename T>
 __global__ void __launch_bounds__(kApplyThreads) k_admm_apply(const T* __restrict__ W, T* __restrict__ U,
                                                               T* __restrict__ Z, int K,
                                                               const uint8_t* __restrict__ rkeep,
-                                                              const uint8_t* __restrict__ ckeep)
+                                                              const uint8_t* __restrict__ ckeep, uint32_t tmul,
+                                                              uint32_t tshift)
 {
     const int a = blockIdx.y;
     const bool rk = rkeep[a] != 0;
@@ -92,7 +65,8 @@ __global__ void __launch_bounds__(kApplyThreads) k_admm_apply(const T* __restric
         const int j = j0 + q * kApplyThreads;
         if (j < K) {
             const T v = vsum(w[q], u[q]);
-            const bool keep = rk && ckeep[j] != 0;
+            const uint32_t grp = (__umulhi((uint32_t)j, tmul) + (uint32_t)j) >> tshift;
+            const bool keep = rk && (!ckeep || ckeep[grp] != 0);
             Z[base + j] = keep ? v : zero_of<T>();
             U[base + j] = keep ? zero_of<T>() : v;
         }
@@ -112,21 +86,26 @@ sadmm_status launch_admm_update(const Geometry& g, const void* W, void* U, void*
                                 int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out, void* ws,
                                 cudaStream_t s)
 {
-    sadmm_status st = launch_project(g, W, U, wdt, k_filters, colkind, k_cols, filt_idx, col_idx, keys_out, ws, s);
-    if (st != SADMM_OK) return st;
     uint8_t* rkeep = static_cast<uint8_t*>(ws) + round_up((long long)project_workspace_bytes(g, colkind), 256);
     uint8_t* ckeep = rkeep + round_up(g.f, 256);
+    sadmm_status st = launch_project(g, W, U, wdt, k_filters, colkind, k_cols, filt_idx, col_idx, keys_out, ws, s,
+                                     rkeep, colkind == SADMM_COL_NONE ? nullptr : ckeep);
+    if (st != SADMM_OK) return st;
     const int F = (int)g.f, K = (int)g.k;
-    k_admm_masks<<<1, 1024, 0, s>>>(F, K, (int)g.taps, colkind, k_filters, filt_idx, k_cols, col_idx, rkeep,
-                                    ckeep);
+    // group of column j: j (shape), j / taps (channel); multiply-shift constants
+    const uint32_t d = (colkind == SADMM_COL_CHANNEL) ? (uint32_t)g.taps : 1u;
+    uint32_t sh = 0;
+    while ((1ull << sh) < d) ++sh;
+    const uint32_t mul = (uint32_t)((((1ull << sh) - d) << 32) / d + 1);
+    const uint8_t* ck = (colkind == SADMM_COL_NONE) ? nullptr : ckeep;
     const dim3 grid((unsigned)((K + kApplyThreads * kApplyCols - 1) / (kApplyThreads * kApplyCols)), (unsigned)F);
     if (wdt == SADMM_BF16)
         k_admm_apply<__nv_bfloat16><<<grid, kApplyThreads, 0, s>>>(
             static_cast<const __nv_bfloat16*>(W), static_cast<__nv_bfloat16*>(U), static_cast<__nv_bfloat16*>(Z),
-            K, rkeep, ckeep);
+            K, rkeep, ck, mul, sh);
     else
         k_admm_apply<float><<<grid, kApplyThreads, 0, s>>>(static_cast<const float*>(W), static_cast<float*>(U),
-                                                           static_cast<float*>(Z), K, rkeep, ckeep);
+                                                           static_cast<float*>(Z), K, rkeep, ck, mul, sh);
     return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
 }
 

@@ -33,9 +33,10 @@ inline long long round_up(long long x, long long a) { return (x + a - 1) / a * a
 
 // ---- projection (project.cu) ----
 size_t project_workspace_bytes(const Geometry& g, int colkind);
+// rkeep / ckeep (optional): a byte per filter / per column group, 1 when kept.
 sadmm_status launch_project(const Geometry& g, const void* W, const void* U, int wdt, int k_filters,
                             int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out,
-                            void* ws, cudaStream_t s);
+                            void* ws, cudaStream_t s, uint8_t* rkeep = nullptr, uint8_t* ckeep = nullptr);
 
 // ---- ADMM Z/U update (admm.cu) ----
 size_t admm_workspace_bytes(const Geometry& g, int colkind);

@@ -48,11 +48,25 @@ SADMM_DEV int lower_bound(const int* a, int n, int v)
     return lo;
 }
 
-__global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status)
+// Dynamic shared memory (when the host passes enough): the filter and column
+// lists, so the binary searches below read shared memory, not HBM.
+__global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status, int lists_in_smem)
 {
     __shared__ int s_start[65];
     __shared__ int s_bad;
+    extern __shared__ int s_lists[];
     const int tid = threadIdx.x;
+    if (lists_in_smem) {
+        int* fl = s_lists;
+        int* cl = s_lists + (a.all_kept ? 0 : a.n_filt);
+        if (!a.all_kept)
+            for (int i = tid; i < a.n_filt; i += blockDim.x) fl[i] = a.filt_idx[i];
+        if (a.col_idx && a.colkind != SADMM_COL_NONE)
+            for (int i = tid; i < a.n_colgroups; i += blockDim.x) cl[i] = a.col_idx[i];
+        __syncthreads();
+        if (!a.all_kept) a.filt_idx = fl;
+        if (a.col_idx && a.colkind != SADMM_COL_NONE) a.col_idx = cl;
+    }
     // Index lists must be strictly ascending and in range.  A list that is not
     // gives a plan with every filter pruned and every column dropped (an
     // all-zero output) and raises the device status word.
@@ -224,7 +238,10 @@ sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int
     a.rowmap = reinterpret_cast<int*>(base + plan->off_rowmap);
     a.zeromap = reinterpret_cast<int*>(base + plan->off_zeromap);
     a.counts = reinterpret_cast<int*>(base + plan->off_counts);
-    k_pack_meta<<<1, 1024, 0, s>>>(a, device_status_ptr());
+    const size_t list_bytes =
+        (size_t)((a.all_kept ? 0 : a.n_filt) + ((col_idx && a.colkind != SADMM_COL_NONE) ? a.n_colgroups : 0)) * 4;
+    const bool in_smem = list_bytes <= 40 * 1024;
+    k_pack_meta<<<1, 1024, in_smem ? list_bytes : 0, s>>>(a, device_status_ptr(), in_smem ? 1 : 0);
 
     __nv_bfloat16* wp = reinterpret_cast<__nv_bfloat16*>(base + plan->off_wp);
     const unsigned rows = (unsigned)(g.groups * plan->n_pad);

@@ -3,14 +3,16 @@
 // channel or shape groups of V = W (+U), then an exact top-k.
 //
 // Kernels:
-//   k_filter_keys   one warp per GEMM row (filter): fp64 sum of squares,
-//                   warp-shuffle reduction.
+//   k_filter_keys   one block per GEMM row (filter): fp64 sums of squares in
+//                   four independent partials per thread, warp-shuffle and
+//                   fixed-order block reduction.
 //   k_column_keys   32 columns per block, 8 warps over the (kept) rows, fixed
 //                   order shared-memory reduction: one key per GEMM column.
-//   k_select        one block: optional channel sums of column keys, an MSB-
-//                   first radix select over the fp64 key bit patterns (exact
-//                   k-th largest key), then an ordered compaction that keeps
-//                   every key above it and the lowest-index keys equal to it.
+//   k_select        one block: optional channel sums of column keys (the keys
+//                   stay in registers, eight per thread), an MSB-first radix
+//                   select over the fp64 key bit patterns (exact k-th largest
+//                   key), then an ordered compaction that keeps every key above
+//                   it and the lowest-index keys equal to it.
 //
 // Keys are non-negative fp64 values, so their IEEE bit patterns order like the
 // values; selection compares bit patterns (a NaN key would rank above +Inf).
@@ -48,11 +50,23 @@ __global__ void __launch_bounds__(256) k_filter_keys(const T* __restrict__ W, co
     const int a = blockIdx.x;
     const int lane = threadIdx.x & 31, wy = threadIdx.x >> 5;
     const long long base = (long long)a * K;
-    double s = 0.0;
-    for (int k = threadIdx.x; k < K; k += 256) {
-        const double v = v_elem(W, U, base + k);
-        s = fma(v, v, s);
+    // four independent partial sums per thread (loads and fp64 FMAs overlap),
+    // added in a fixed order
+    double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
+    int k = threadIdx.x;
+    for (; k + 768 < K; k += 1024) {
+        const double v0 = v_elem(W, U, base + k), v1 = v_elem(W, U, base + k + 256);
+        const double v2 = v_elem(W, U, base + k + 512), v3 = v_elem(W, U, base + k + 768);
+        s0 = fma(v0, v0, s0);
+        s1 = fma(v1, v1, s1);
+        s2 = fma(v2, v2, s2);
+        s3 = fma(v3, v3, s3);
     }
+    for (; k < K; k += 256) {
+        const double v = v_elem(W, U, base + k);
+        s0 = fma(v, v, s0);
+    }
+    double s = (s0 + s1) + (s2 + s3);
     for (int o = 16; o > 0; o >>= 1) s += __shfl_down_sync(0xffffffffu, s, o);
     if (lane == 0) part[wy] = s;
     __syncthreads();
@@ -122,40 +136,88 @@ SADMM_DEV int block_excl_count(bool pred, int* warp_tot, int* total)
     return r;
 }
 
+constexpr int kSelPer = 8;  // keys per thread held in registers (G <= 8192)
+
+// hist[d] += 1 for every lane with `active` set, one atomic per distinct digit
+// of the warp (keys share their high bits, so per-lane atomics would
+// serialise on a few bins).
+SADMM_DEV void hist_add(unsigned int* hist, unsigned d, bool active)
+{
+    const unsigned act = __ballot_sync(0xffffffffu, active);
+    if (!active) return;
+    const unsigned peers = __match_any_sync(act, d);
+    if ((threadIdx.x & 31) == (unsigned)(__ffs(peers) - 1)) atomicAdd(&hist[d], (unsigned)__popc(peers));
+}
+
 // Exact top-k of G fp64 keys (ties to the lower index), ascending index list.
 // When taps > 1 the keys are first formed as sums of `taps` consecutive source
-// keys (channel-wise groups from column keys).
+// keys (channel-wise groups from column keys).  keep_out (optional) gets a
+// byte per group: 1 when kept.  With G <= kSelThreads * kSelPer every thread
+// holds its keys (i = tid + q * kSelThreads) in registers, so the radix passes
+// and the compaction read no memory; larger G re-reads the keys from global
+// memory.
+template <bool REG>
 __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict__ src, int G, int taps, int k,
                                                         int nparts, long long part_stride,
                                                         double* __restrict__ keys, double* __restrict__ keys_out,
-                                                        int* __restrict__ out_idx)
+                                                        int* __restrict__ out_idx, uint8_t* __restrict__ keep_out)
 {
     __shared__ unsigned int hist[256];
     __shared__ unsigned long long s_prefix;
     __shared__ int s_kk;
     __shared__ int warp_tot[33];
     const int tid = threadIdx.x;
+    unsigned long long kr[REG ? kSelPer : 1];
 
     // 1. keys: the sum of the nparts partial sums of each source key, then of
     //    `taps` consecutive source keys (channel-wise groups); and the optional
     //    copy for the caller
-    for (int i = tid; i < G; i += kSelThreads) {
-        double v = 0.0;
-        for (int t = 0; t < taps; ++t) {
-            const long long si = (long long)i * taps + t;
-            double w = 0.0;
-            for (int q = 0; q < nparts; ++q) w += src[q * part_stride + si];
-            v += w;
+    const bool formed = (taps > 1 || nparts > 1);
+    // the taps * nparts source values of key i, in four independent partial
+    // sums (fixed order: entry e goes to partial e % 4)
+    auto form = [&](int i) -> double {
+        const int n = taps * nparts;
+        double v0 = 0.0, v1 = 0.0, v2 = 0.0, v3 = 0.0;
+        int e = 0;
+        for (; e + 3 < n; e += 4) {
+            const int t0 = e / nparts, t1 = (e + 1) / nparts, t2 = (e + 2) / nparts, t3 = (e + 3) / nparts;
+            v0 += src[(e - t0 * nparts) * part_stride + (long long)i * taps + t0];
+            v1 += src[(e + 1 - t1 * nparts) * part_stride + (long long)i * taps + t1];
+            v2 += src[(e + 2 - t2 * nparts) * part_stride + (long long)i * taps + t2];
+            v3 += src[(e + 3 - t3 * nparts) * part_stride + (long long)i * taps + t3];
         }
-        if (taps > 1 || nparts > 1) keys[i] = v;
+        for (; e < n; ++e) {
+            const int t = e / nparts;
+            v0 += src[(e - t * nparts) * part_stride + (long long)i * taps + t];
+        }
+        const double v = (v0 + v1) + (v2 + v3);
         if (keys_out) keys_out[i] = v;
+        return v;
+    };
+    if (REG) {
+#pragma unroll
+        for (int q = 0; q < kSelPer; ++q) {
+            const int i = tid + q * kSelThreads;
+            kr[q] = (i < G) ? (unsigned long long)__double_as_longlong(form(i)) : 0ull;
+        }
+    } else {
+        for (int i = tid; i < G; i += kSelThreads) {
+            const double v = form(i);
+            if (formed) keys[i] = v;
+        }
     }
-    const double* kv = (taps > 1 || nparts > 1) ? keys : src;
+    const double* kv = formed ? keys : src;
     __syncthreads();
+    auto key_at = [&](int q, int i) -> unsigned long long {
+        if (REG) return kr[q];
+        return (unsigned long long)__double_as_longlong(kv[i]);
+    };
 
-    if (k <= 0) return;
-    if (k >= G) {
-        for (int i = tid; i < G; i += kSelThreads) out_idx[i] = i;
+    if (k <= 0 || k >= G) {
+        for (int i = tid; i < G; i += kSelThreads) {
+            if (k >= G) out_idx[i] = i;
+            if (keep_out) keep_out[i] = (k >= G) ? 1 : 0;
+        }
         return;
     }
 
@@ -166,9 +228,18 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
         for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0u;
         __syncthreads();
         const unsigned long long prefix = s_prefix;
-        for (int i = tid; i < G; i += kSelThreads) {
-            const unsigned long long u = (unsigned long long)__double_as_longlong(kv[i]);
-            if ((u & mask) == prefix) atomicAdd(&hist[(u >> shift) & 255u], 1u);
+        if (REG) {
+#pragma unroll
+            for (int q = 0; q < kSelPer; ++q) {
+                const int i = tid + q * kSelThreads;
+                hist_add(hist, (unsigned)((kr[q] >> shift) & 255u), i < G && (kr[q] & mask) == prefix);
+            }
+        } else {
+            for (int base = 0; base < G; base += kSelThreads) {
+                const int i = base + tid;
+                const unsigned long long u = i < G ? key_at(0, i) : 0ull;
+                hist_add(hist, (unsigned)((u >> shift) & 255u), i < G && (u & mask) == prefix);
+            }
         }
         __syncthreads();
         if (tid < 32) {
@@ -203,10 +274,17 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
 
     // 3. ordered compaction
     int run_out = 0, run_eq = 0;
-    for (int base = 0; base < G; base += kSelThreads) {
+    for (int base = 0, q = 0; base < G; base += kSelThreads, ++q) {
         const int i = base + tid;
         const bool valid = i < G;
-        const unsigned long long u = valid ? (unsigned long long)__double_as_longlong(kv[i]) : 0ull;
+        unsigned long long u = 0ull;
+        if (REG) {
+#pragma unroll
+            for (int r = 0; r < kSelPer; ++r)
+                if (r == q) u = kr[r];
+        } else if (valid) {
+            u = key_at(0, i);
+        }
         const bool gt = valid && u > T;
         const bool eq = valid && u == T;
         int eq_tot, take_tot;
@@ -214,9 +292,21 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
         const bool take = gt || (eq && run_eq + eq_before < take_eq);
         const int pos = block_excl_count(take, warp_tot, &take_tot);
         if (take) out_idx[run_out + pos] = i;
+        if (keep_out && valid) keep_out[i] = take ? 1 : 0;
         run_eq += eq_tot;
         run_out += take_tot;
     }
+}
+
+void launch_select(const double* src, int G, int taps, int k, int nparts, long long part_stride, double* keys,
+                   double* keys_out, int* out_idx, uint8_t* keep_out, cudaStream_t s)
+{
+    if (G <= kSelThreads * kSelPer)
+        k_select<true><<<1, kSelThreads, 0, s>>>(src, G, taps, k, nparts, part_stride, keys, keys_out, out_idx,
+                                                 keep_out);
+    else
+        k_select<false><<<1, kSelThreads, 0, s>>>(src, G, taps, k, nparts, part_stride, keys, keys_out, out_idx,
+                                                  keep_out);
 }
 
 // Row chunks of the column-key pass: enough blocks to fill the GPU, with the
@@ -231,7 +321,8 @@ int column_parts(long long K, long long nrows)
 
 template <typename T>
 sadmm_status run_project(const Geometry& g, const T* W, const T* U, int k_filters, int colkind, int k_cols,
-                         int* filt_idx, int* col_idx, double* keys_out, void* ws, cudaStream_t s)
+                         int* filt_idx, int* col_idx, double* keys_out, void* ws, uint8_t* rkeep, uint8_t* ckeep,
+                         cudaStream_t s)
 {
     const int F = (int)g.f, K = (int)g.k;
     double* fkeys = reinterpret_cast<double*>(ws);
@@ -239,7 +330,7 @@ sadmm_status run_project(const Geometry& g, const T* W, const T* U, int k_filter
     double* parts = ckeys + round_up(K, 32);                   // [R][K] partial column keys
 
     k_filter_keys<T><<<F, 256, 0, s>>>(W, U, F, K, fkeys);
-    k_select<<<1, kSelThreads, 0, s>>>(fkeys, F, 1, k_filters, 1, 0, fkeys, keys_out, filt_idx);
+    launch_select(fkeys, F, 1, k_filters, 1, 0, fkeys, keys_out, filt_idx, rkeep, s);
     if (colkind != SADMM_COL_NONE) {
         const bool all_rows = (k_filters == F);
         const int nrows = all_rows ? F : k_filters;
@@ -248,8 +339,7 @@ sadmm_status run_project(const Geometry& g, const T* W, const T* U, int k_filter
                                                                 parts);
         const int taps = (colkind == SADMM_COL_CHANNEL) ? (int)g.taps : 1;
         const int G = (colkind == SADMM_COL_CHANNEL) ? (int)g.cg : K;
-        k_select<<<1, kSelThreads, 0, s>>>(parts, G, taps, k_cols, R, K, ckeys,
-                                           keys_out ? keys_out + F : nullptr, col_idx);
+        launch_select(parts, G, taps, k_cols, R, K, ckeys, keys_out ? keys_out + F : nullptr, col_idx, ckeep, s);
     }
     return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
 }
@@ -267,13 +357,13 @@ size_t project_workspace_bytes(const Geometry& g, int colkind)
 
 sadmm_status launch_project(const Geometry& g, const void* W, const void* U, int wdt, int k_filters,
                             int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out,
-                            void* ws, cudaStream_t s)
+                            void* ws, cudaStream_t s, uint8_t* rkeep, uint8_t* ckeep)
 {
     if (wdt == SADMM_BF16)
         return run_project<__nv_bfloat16>(g, (const __nv_bfloat16*)W, (const __nv_bfloat16*)U, k_filters,
-                                          colkind, k_cols, filt_idx, col_idx, keys_out, ws, s);
+                                          colkind, k_cols, filt_idx, col_idx, keys_out, ws, rkeep, ckeep, s);
     return run_project<float>(g, (const float*)W, (const float*)U, k_filters, colkind, k_cols, filt_idx,
-                              col_idx, keys_out, ws, s);
+                              col_idx, keys_out, ws, rkeep, ckeep, s);
 }
 
 // ---------------------------------------------------------------------------

@@ -32,7 +32,11 @@ def main(argv=None) -> int:
     ap.add_argument("--reps", type=int, default=3)
     ap.add_argument("--out-dtype", default="fp32", choices=["fp32", "bf16"])
     ap.add_argument("--dense", action="store_true", help="keep every filter and column")
+    ap.add_argument("--admm", action="store_true",
+                    help="time sadmm_admm_update on fp32 W/U of the layer instead of the forward call")
     args = ap.parse_args(argv)
+    if args.admm:
+        return run_admm(args)
 
     L = wl.get(args.workload)[args.layer]
     s = L.shape if args.batch == 0 else L.shape.with_batch(args.batch)
@@ -64,6 +68,33 @@ def main(argv=None) -> int:
         print(f"device status {st}")
         return 1
     return 0
+
+
+def run_admm(args) -> int:
+    """sadmm_admm_update `reps` times on the layer's seeded fp32 ADMM state."""
+    import torch
+
+    import workloads as wl
+    from paper_1807_11091_gb300 import sadmm
+
+    L = wl.get(args.workload)[args.layer]
+    s = L.shape
+    st = wl.gen_admm_state(s, L.seed)
+    W, U = st["W"].cuda(), st["U"].cuda()
+    Z = torch.empty_like(W)
+    step = sadmm.AdmmStep(s.desc16(), L.k_filters, L.colkind, L.k_cols, W.device)
+    nbytes = 16.0 * s.f * s.k
+    for i in range(args.reps):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        torch.cuda._sleep(200_000)
+        e0.record()
+        step(W, U, Z)
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        print(f"{L.name} admm run {i}: {ms * 1e3:.1f} us  {nbytes / ms / 1e6:.1f} GB/s (16 B per weight)")
+    return 1 if sadmm.device_status() != 0 else 0
 
 
 if __name__ == "__main__":
