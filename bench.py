@@ -186,7 +186,9 @@ class LayerRun:
         ytype = torch.bfloat16 if out_dtype == "bf16" else torch.float32
         self.y = torch.empty(s.y_shape(), dtype=ytype, device=dev)
         self.out_bytes = 2 if out_dtype == "bf16" else 4
-        self.launches = (2 + (2 if self.colkind != wl.COL_NONE else 0)) + 2 + 1
+        # projection (keys + select per kind), pack (meta + rows), conv (+ split-K finalize)
+        self.launches = ((2 + (2 if self.colkind != wl.COL_NONE else 0)) + 2
+                         + (2 if self.plan.splits > 1 else 1))
 
     def flops(self):
         s = self.s
@@ -389,6 +391,53 @@ def sweep_report(dev, out_dtype, reps=5):
                                 "speedup_vs_dense": times[0] / ms,
                                 "retained_fraction": r.flops() / runs[0].flops()})
     del runs, flush
+    torch.cuda.empty_cache()
+    return out
+
+
+def batch1_report(dev, out_dtype, reps=7):
+    """The paper's timing setting (Sec. 5): every AlexNet CONV layer at batch 1,
+    sadmm_conv_fwd alone (projection and pack done once), against the same
+    kernel at 0% sparsity.  Small layers split K' over several CTAs per output
+    tile (plan.splits)."""
+    import torch
+    out = {"what": "AlexNet CONV1-5 at batch 1, sadmm_conv_fwd alone, L2 flushed, median of "
+                   f"{reps}", "layers": {}}
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    sp = int(torch.cuda.current_stream().cuda_stream)
+    tot_p = tot_d = 0.0
+    for L in wl.alexnet():
+        L1 = wl.subset_layer(L, 1)
+        t = wl.gen_tensors(L1.shape, seed=L.seed)
+        runs = [LayerRun(L1, t, dev, out_dtype), LayerRun(L1, t, dev, out_dtype, dense=True)]
+        times = []
+        for r in runs:
+            r.project(sp)
+            r.pack(sp)
+            r.conv(sp)
+            torch.cuda.synchronize()
+            ms = []
+            for _ in range(reps):
+                flush.fill_(1)
+                torch.cuda._sleep(200_000)
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record()
+                r.conv(sp)
+                e1.record()
+                torch.cuda.synchronize()
+                ms.append(e0.elapsed_time(e1))
+            times.append(statistics.median(ms))
+        tot_p += times[0]
+        tot_d += times[1]
+        out["layers"][L.name] = {"pruned_us": times[0] * 1e3, "dense_us": times[1] * 1e3,
+                                 "speedup_vs_dense": times[1] / times[0],
+                                 "tflops_retained": runs[0].flops() / (times[0] * 1e-3) / 1e12,
+                                 "splits": int(runs[0].plan.splits)}
+    out["total_pruned_us"] = tot_p * 1e3
+    out["total_dense_us"] = tot_d * 1e3
+    out["speedup_vs_dense"] = tot_d / tot_p
+    del flush
     torch.cuda.empty_cache()
     return out
 
@@ -596,6 +645,8 @@ def run_gpu(args):
     }
     if rank == 0 and not args.no_sweep:
         line["sweep"] = sweep_report(dev, args.out_dtype)
+    if rank == 0 and not args.no_batch1:
+        line["batch1"] = batch1_report(dev, args.out_dtype)
     if rank == 0 and not args.no_admm:
         line["admm"] = admm_report(dev, peaks.get("hbm_gbs"))
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
@@ -619,6 +670,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-admm", action="store_true")
+    ap.add_argument("--no-batch1", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -42,7 +42,7 @@
 extern "C" {
 #endif
 
-#define SADMM_ABI_VERSION 1
+#define SADMM_ABI_VERSION 2
 
 /* Bytes of the fixed device array of sadmm_project_groups_noalloc. */
 #define SADMM_NOALLOC_SCRATCH_BYTES (256 * 1024)
@@ -92,6 +92,9 @@ typedef struct {
     size_t dev_bytes; /* device bytes the plan needs (see sadmm_plan_init)    */
     void* dev;        /* device buffer bound by sadmm_pack                    */
     size_t off_wp, off_gather, off_rowmap, off_zeromap, off_counts, off_colidx;
+    size_t off_partial; /* split-K partial sums (when splits > 1)              */
+    int splits;         /* K' split over this many CTAs per output tile (>= 1)  */
+    int stages_per_split; /* 64-column stages of K' per split                  */
     uint64_t tmap[16];/* 128-byte TMA tensor map of the packed matrix         */
 } sadmm_plan;
 
@@ -175,6 +178,13 @@ sadmm_status sadmm_admm_update(const sadmm_conv_desc* d, const void* W, void* U,
  * including plan->dev_bytes, the device buffer sadmm_pack needs.  Host only;
  * enqueues nothing.  SADMM_EUNSUPPORTED when the packed row count per conv
  * group would exceed 4096 or K' would exceed 8192.
+ *
+ * Small batches (the paper times batch 1, Sec. 5): when the layer has fewer
+ * output tiles (128 pixels x one filter tile of one conv group) than the
+ * current device has SMs, K' is split over plan->splits CTAs per tile; each
+ * writes fp32 partial sums to a region of the plan's device buffer and a
+ * second kernel adds them in split order, then applies bias and ReLU.  The
+ * split depends on the current device's SM count and is fixed in the plan.
  */
 sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d,
                              int n_filt, int colkind, int n_colgroups);

@@ -232,6 +232,29 @@ sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d, int n_f
     p.off_rowmap = take((size_t)g.groups * p.n_pad * 4);
     p.off_zeromap = take((size_t)g.f * 4);
     p.off_counts = take((size_t)g.groups * 2 * 4);
+    // split K' when the layer has fewer output tiles than the device has SMs
+    p.splits = 1;
+    p.stages_per_split = p.k_pad / 64;
+    {
+        const long long nks = p.k_pad / 64;
+        const long long m_tiles = (g.m + 127) / 128;
+        const long long upairs = (p.n_tiles + (p.n_tiles >= 2 ? 1 : 0)) / (p.n_tiles >= 2 ? 2 : 1);
+        const long long units = m_tiles * g.groups * upairs;
+        const long long sms = device_sm_count();
+        const long long rows = g.groups * p.n_pad + g.groups * g.fg;  // finalize rows
+        if (units < sms && nks >= 2 && rows <= 65535) {
+            long long want = (sms + units - 1) / units;
+            if (want > nks) want = nks;
+            const long long ksps = (nks + want - 1) / want;
+            const long long splits = (nks + ksps - 1) / ksps;
+            const long long bytes = splits * g.groups * p.n_pad * m_tiles * 128 * 4;
+            if (splits > 1 && bytes <= (256ll << 20)) {
+                p.splits = (int)splits;
+                p.stages_per_split = (int)ksps;
+                p.off_partial = take((size_t)bytes);
+            }
+        }
+    }
     p.dev_bytes = off;
     p.dev = nullptr;
     *plan = p;

@@ -96,8 +96,13 @@ struct ConvArgs {
     int M;            // N * plane (below 2^31)
     long long x_chw;  // elements per input image
     long long thw;    // elements per input channel
-    int units;        // m_tiles * groups * upairs (below 2^31)
-    FastDiv upairs_div, mtiles_div, plane_div, ohw_div, ow_div;
+    int units;        // work items: m_tiles * groups * upairs * splits (below 2^31)
+    FastDiv split_div, upairs_div, mtiles_div, plane_div, ohw_div, ow_div;
+    int splits;       // K' splits per output tile (1: no split)
+    int ksps;         // stages per split
+    float* partial;   // [splits][groups * n_pad][m_pad] fp32 partial sums (splits > 1)
+    int m_pad;        // m_tiles * 128
+    int ncols_all;    // groups * n_pad
     int hw, W, H, T;
     int F, groups, Cg, Fg;
     int OW, OHW, plane;
@@ -120,13 +125,18 @@ struct ConvArgs {
     int relu;
 };
 
-// Unit u covers filter tiles p*nacc .. p*nacc+nacc-1 of conv group g for pixel
-// tile mt.  Groups are outermost, so a CTA (units u, u + grid, ...) stays in
+// Work item w is split sp (stages ks0 .. ks1-1 of K') of unit w / splits; a
+// unit covers filter tiles p*nacc .. p*nacc+nacc-1 of conv group g for pixel
+// tile mt.  Groups are outermost, so a CTA (items w, w + grid, ...) stays in
 // one conv group for long runs and rarely reloads resident weights.
-SADMM_DEV void decode_unit(const ConvArgs& a, int u, int& p, int& g, int& mt)
+SADMM_DEV void decode_unit(const ConvArgs& a, int w, int& p, int& g, int& mt, int& sp, int& ks0, int& ks1)
 {
-    const uint32_t t = fdiv((uint32_t)u, a.upairs_div);
-    p = u - (int)(t * a.upairs_div.d);
+    const uint32_t u = fdiv((uint32_t)w, a.split_div);
+    sp = w - (int)(u * a.split_div.d);
+    ks0 = sp * a.ksps;
+    ks1 = min(a.nks, ks0 + a.ksps);
+    const uint32_t t = fdiv(u, a.upairs_div);
+    p = (int)(u - t * a.upairs_div.d);
     const uint32_t gq = fdiv(t, a.mtiles_div);
     mt = (int)(t - gq * a.mtiles_div.d);
     g = (int)gq;
@@ -246,9 +256,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t e_ph = 0;
             int loads = 0;
             for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
-                int p, g;
+                int p, g, sp, ks0, ks1;
                 int mt;
-                decode_unit(a, u, p, g, mt);
+                decode_unit(a, u, p, g, mt, sp, ks0, ks1);
                 if (s_counts[2 * g] <= p * a.bn) continue;
                 const long long key = (long long)g * a.upairs + p;
                 if (key == cur) continue;
@@ -275,16 +285,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t issued_mask = 0;
             bool ok = true;
             for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-                int p, g;
+                int p, g, sp, ks0, ks1;
                 int mt;
-                decode_unit(a, u, p, g, mt);
+                decode_unit(a, u, p, g, mt, sp, ks0, ks1);
                 const int nt0 = p * a.nacc;
                 if (s_counts[2 * g] <= nt0 * a.bn) continue;
                 int nbox = 0;  // filter tiles of this unit with kept rows
                 for (int i = 0; i < a.nacc; ++i)
                     if (nt0 + i < a.n_tiles && s_counts[2 * g] > (nt0 + i) * a.bn) nbox = i + 1;
                 const int row0 = g * a.n_pad + nt0 * a.bn;
-                for (int ks = 0; ks < a.nks; ++ks) {
+                for (int ks = ks0; ks < ks1; ++ks) {
                     if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, a.status)) { ok = false; break; }
                     mbar_arrive_expect_tx(&full_b[s], b_bytes * (uint32_t)nbox);
                     for (int i = 0; i < nbox; ++i)
@@ -316,9 +326,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t bf_ph = 0;
             const uint32_t sB0 = smem_u32(sB);
             for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-                int p, g;
+                int p, g, sp, ks0, ks1;
                 int mt;
-                decode_unit(a, u, p, g, mt);
+                decode_unit(a, u, p, g, mt, sp, ks0, ks1);
                 const int cnt = s_counts[2 * g] - p * a.nacc * a.bn;  // kept rows from the unit's first tile
                 if (cnt <= 0) continue;
                 if (a.b_res) {
@@ -338,7 +348,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!mbar_wait(&acc_empty[ab], acc_ph ^ 1u, abort_flag, a.status)) break;
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + (uint32_t)(ab * a.nacc * a.tmem_stride);
-                for (int ks = 0; ks < a.nks; ++ks) {
+                for (int ks = ks0; ks < ks1; ++ks) {
                     if (!mbar_wait(&full_a[s], ph, abort_flag, a.status) ||
                         (!a.b_res && !mbar_wait(&full_b[s], ph, abort_flag, a.status))) {
                         ok = false;
@@ -353,14 +363,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                         for (int kk = 0; kk < kBK / 16; ++kk)
                             mma_bf16_ss(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32), sdesc_kmajor_sw128(b0 + kk * 32),
-                                        idesc0, (ks | kk) != 0 ? 1u : 0u);
+                                        idesc0, (ks != ks0 || kk != 0) ? 1u : 0u);
                     } else {
                         const uint32_t d1 = d_tmem + (uint32_t)a.tmem_stride;
                         const uint32_t b1 = b0 + b_bytes;
 #pragma unroll
                         for (int kk = 0; kk < kBK / 16; ++kk) {
                             const uint64_t adesc = sdesc_kmajor_sw128(a0 + kk * 32);
-                            const uint32_t acc = (ks | kk) != 0 ? 1u : 0u;
+                            const uint32_t acc = (ks != ks0 || kk != 0) ? 1u : 0u;
                             mma_bf16_ss(d_tmem, adesc, sdesc_kmajor_sw128(b0 + kk * 32), idesc0, acc);
                             mma_bf16_ss(d1, adesc, sdesc_kmajor_sw128(b1 + kk * 32), idesc1, acc);
                         }
@@ -398,9 +408,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         // units, without TMEM or stores, so the named barrier stays balanced.
         bool alive = true;
         for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
-            int p, g;
+            int p, g, sp, ks0, ks1;
             int mt;
-            decode_unit(a, u, p, g, mt);
+            decode_unit(a, u, p, g, mt, sp, ks0, ks1);
             const int nt0 = p * a.nacc;
             const int cnt = s_counts[2 * g] - nt0 * a.bn;  // kept rows from the unit's first tile
             const int zc = (p == 0) ? s_counts[2 * g + 1] : 0;  // pruned filters whose planes this unit zeroes
@@ -453,7 +463,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                         uint32_t r[kEpiCols];
                         tmem_ld_32x32b_x16(taddr + (uint32_t)c0, r);
                         tmem_ld_wait();
-                        if (valid) {
+                        if (valid && a.splits > 1) {
+                            // split K': raw fp32 partial sums, [split][column][pixel]
+                            float* pp = a.partial +
+                                        ((size_t)sp * a.ncols_all + (size_t)g * a.n_pad + (size_t)(nt0 + ti) * a.bn + c0) *
+                                            a.m_pad +
+                                        m;
+#pragma unroll
+                            for (int j = 0; j < kEpiCols; ++j)
+                                if (c0 + j < nrows) __stcs(pp + (size_t)j * a.m_pad, __uint_as_float(r[j]));
+                        } else if (valid) {
                             if (c0 + kEpiCols <= nrows) {
 #pragma unroll
                                 for (int j = 0; j < kEpiCols; j += 4) {
@@ -495,7 +514,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (lane == 0) mbar_arrive(&acc_empty[ab]);
                 if (++ab == a.acc_bufs) { ab = 0; acc_ph ^= 1u; }
             }
-            if (zc > 0 && valid && alive) {
+            if (zc > 0 && valid && alive && a.splits == 1) {
                 // pruned filters of this conv group: their planes are zero.
                 // Chunks of 16 planes continue the unit's chunk sequence.
                 const int* zmap = a.zeromap + (long long)g * a.Fg;
@@ -540,9 +559,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         int turn = 0;  // running stage index modulo kGatherSets
         bool ok = true;
         for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-            int p, g;
+            int p, g, sp, ks0, ks1;
             int mt;
-            decode_unit(a, u, p, g, mt);
+            decode_unit(a, u, p, g, mt, sp, ks0, ks1);
             if (s_counts[2 * g] <= p * a.nacc * a.bn) continue;
             const int m = mt * kBM + prow;
             uint32_t M = 0;
@@ -561,7 +580,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             // Every lane's pixel sees every tap: no bounds test is needed.
             const bool interior = __all_sync(0xffffffffu, M == a.full_mask);
-            for (int ks = 0; ks < a.nks; ++ks) {
+            for (int ks = ks0; ks < ks1; ++ks) {
                 if (turn == set) {
                     // Issue every load of this thread's columns first (they
                     // read only x), then wait for the stage buffer and store.
@@ -621,6 +640,48 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
+// Split K': y = ReLU(bias + sum of the splits' partial sums, in split order)
+// for every kept row, zeros for the pruned filters' planes.  Block (bx, r):
+// row r of [kept rows of all groups | pruned-filter slots], pixels
+// bx*1024 .. bx*1024+1023.
+template <bool OUT_BF16>
+__global__ void __launch_bounds__(256) k_splitk_finalize(const ConvArgs a)
+{
+    const int r = blockIdx.y;
+    int f;
+    bool zero;
+    if (r < a.ncols_all) {
+        f = __ldg(a.rowmap + r);
+        zero = false;
+    } else {
+        const int z = r - a.ncols_all;
+        const int g = z / a.Fg, zi = z - g * a.Fg;
+        if (zi >= __ldg(a.counts + 2 * g + 1)) return;
+        f = __ldg(a.zeromap + g * a.Fg + zi);
+        zero = true;
+    }
+    if (f < 0) return;
+    const float b = (!zero && a.bias) ? __ldg(a.bias + f) : 0.0f;
+    for (int q = 0; q < 4; ++q) {
+        const int m = blockIdx.x * 1024 + q * 256 + threadIdx.x;
+        if (m >= a.M) break;
+        float v = 0.0f;
+        if (!zero) {
+            float acc = 0.0f;
+            for (int sp = 0; sp < a.splits; ++sp)
+                acc += __ldcs(a.partial + ((size_t)sp * a.ncols_all + r) * a.m_pad + m);
+            v = acc + b;
+            if (a.relu) v = fmaxf(v, 0.0f);
+        }
+        const int n_img = (int)fdiv((uint32_t)m, a.plane_div);
+        const size_t off = ((size_t)n_img * a.F + f) * a.plane + (m - n_img * a.plane);
+        if (OUT_BF16)
+            reinterpret_cast<__nv_bfloat16*>(a.y)[off] = __float2bfloat16_rn(v);
+        else
+            reinterpret_cast<float*>(a.y)[off] = v;
+    }
+}
+
 template <bool OUT_BF16>
 cudaError_t launch(const CUtensorMap& map, const ConvArgs& a, int grid, size_t smem, cudaStream_t s)
 {
@@ -634,6 +695,10 @@ cudaError_t launch(const CUtensorMap& map, const ConvArgs& a, int grid, size_t s
         configured_dev = dev;
     }
     kern<<<grid, kThreads, smem, s>>>(map, a);
+    if (a.splits > 1) {
+        const dim3 fgrid((unsigned)((a.M + 1023) / 1024), (unsigned)(a.ncols_all + a.groups * a.Fg));
+        k_splitk_finalize<OUT_BF16><<<fgrid, 256, 0, s>>>(a);
+    }
     return cudaGetLastError();
 }
 
@@ -686,7 +751,15 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     a.n_pad = plan->n_pad;
     a.relu = relu ? 1 : 0;
     const long long m_tiles = (g.m + kBM - 1) / kBM;
-    const long long units = m_tiles * g.groups * a.upairs;
+    a.splits = plan->splits > 1 ? plan->splits : 1;
+    a.ksps = a.splits > 1 ? plan->stages_per_split : a.nks;
+    if (a.splits > 1 && ((long long)a.ksps * (a.splits - 1) >= a.nks || (long long)a.ksps * a.splits < a.nks))
+        return SADMM_EINVAL;  // a plan whose split does not tile K'
+    a.partial = a.splits > 1 ? reinterpret_cast<float*>(const_cast<char*>(base) + plan->off_partial) : nullptr;
+    a.m_pad = (int)(m_tiles * kBM);
+    a.ncols_all = (int)(g.groups * plan->n_pad);
+    a.split_div = make_fastdiv((uint32_t)a.splits);
+    const long long units = m_tiles * g.groups * a.upairs * a.splits;
     if (units >= (1ll << 31) - (1ll << 20)) return SADMM_EUNSUPPORTED;  // u + grid stays below 2^31
     a.units = (int)units;
     a.upairs_div = make_fastdiv((uint32_t)a.upairs);
@@ -709,7 +782,8 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     const long long res_bytes = (long long)plan->bn * 128 * a.nks;
     int stage_bytes;
     long long fixed_bytes;
-    if (plan->n_tiles == 1 && budget - res_bytes >= 3LL * kATileBytes) {
+    // (not when K' is split: a work item then uses only a few of the boxes)
+    if (plan->n_tiles == 1 && plan->splits <= 1 && budget - res_bytes >= 3LL * kATileBytes) {
         a.b_res = 1;
         stage_bytes = kATileBytes;
         fixed_bytes = res_bytes;

@@ -54,6 +54,9 @@ class Plan(ctypes.Structure):
         ("off_zeromap", ctypes.c_size_t),
         ("off_counts", ctypes.c_size_t),
         ("off_colidx", ctypes.c_size_t),
+        ("off_partial", ctypes.c_size_t),
+        ("splits", ctypes.c_int),
+        ("stages_per_split", ctypes.c_int),
         ("tmap", ctypes.c_uint64 * 16),
     ]
 
