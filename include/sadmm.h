@@ -172,6 +172,37 @@ sadmm_status sadmm_admm_update(const sadmm_conv_desc* d, const void* W, void* U,
                                int k_filters, int colkind, int k_cols, int* filt_idx, int* col_idx,
                                double* keys_out, void* workspace, size_t ws_bytes, void* stream);
 
+/* Device bytes of scratch the non-structured projection needs for this
+ * layer (selection state, a 2048-bin histogram, one counter per 4096
+ * weights).  0 on a bad descriptor. */
+size_t sadmm_elements_workspace_size(const sadmm_conv_desc* d);
+
+/*
+ * Non-structured projection (Sec. 4, non-structured weight sparsity): keep the
+ * k_elems entries of V = W (+U) with the largest magnitudes |V|, zero the rest.
+ * |V| is compared exactly (V formed in fp64); equal magnitudes go to the lower
+ * flat index a*K + j (the reading used for every top-k in this library).
+ *
+ *   W, U      device [F][K], dtype `wdt`; U may be NULL.
+ *   k_elems   0 .. F*K.
+ *   keep_out  device uint8 [F*K]: 1 for a kept entry, 0 otherwise.
+ *   workspace sadmm_elements_workspace_size() bytes, 256-byte aligned.
+ * The paper finds this sparsity hard to speed up on a GPU (Sec. 5, cuSPARSE);
+ * the library offers the projection (for ADMM training), not a sparse conv.
+ */
+sadmm_status sadmm_project_elements(const sadmm_conv_desc* d, const void* W, const void* U, int wdt,
+                                    long long k_elems, unsigned char* keep_out, void* workspace,
+                                    size_t ws_bytes, void* stream);
+
+/*
+ * The ADMM Z- and U-update for non-structured sparsity (Sec. 4): Z = the
+ * k_elems largest-magnitude entries of V = W + U (V rounded once to the
+ * tensors' precision, as in sadmm_admm_update), U <- V - Z.  W, U, Z as in
+ * sadmm_admm_update (no overlap); workspace as for sadmm_project_elements.
+ */
+sadmm_status sadmm_admm_update_elements(const sadmm_conv_desc* d, const void* W, void* U, void* Z, int wdt,
+                                        long long k_elems, void* workspace, size_t ws_bytes, void* stream);
+
 /*
  * Sizes a plan for `n_filt` kept filters and `n_colgroups` kept column groups
  * (columns or channels) of kind `colkind`.  Fills every size field of `plan`,

@@ -21,6 +21,8 @@ What it computes, with the passage each step follows:
   sparsities"); the bias of a pruned filter is zero (a reading).
 * ``admm_update`` -- the ADMM Z-update (projection of W + U) and the dual
   update U <- U + W - Z (Sec. 4), in the tensors' precision.
+* ``project_elements`` / ``admm_update_elements`` -- the non-structured case
+  (Sec. 4): keep the largest |V| entries.
 * ``conv`` -- direct convolution over the full masked tensor (fp64).
 
 Parity pins: every function here is checked in ``tests/test_oracle_*.py``
@@ -254,6 +256,28 @@ def admm_update(W, U, taps: int, k_filters: int, colkind: int, k_cols: int):
     Z = torch.from_numpy(Z64).to(W.dtype).reshape(W.shape)
     Un = torch.from_numpy(U64).to(W.dtype).reshape(W.shape)
     return rows, cols, Z, Un
+
+
+def project_elements(W, k_elems: int, U=None) -> np.ndarray:
+    """Non-structured projection (Sec. 4): keep the k_elems entries of
+    V = W (+U) with the largest |V| (V exact in fp64), equal magnitudes to the
+    lower flat index.  Returns a bool mask of W's shape."""
+    V = as_matrix(W, U)
+    flat = np.abs(V).reshape(-1)
+    keep = np.zeros(flat.shape[0], dtype=bool)
+    keep[topk(flat, int(k_elems))] = True
+    return keep.reshape(_as_f64(W).shape)
+
+
+def admm_update_elements(W, U, k_elems: int):
+    """ADMM Z- and U-update for non-structured sparsity: Z = V on the kept
+    entries (V rounded once to the tensors' dtype), U_next = V - Z."""
+    import torch
+    keep = project_elements(W, k_elems, U=U)
+    V = _as_f64(W) + _as_f64(U)
+    Z64 = np.where(keep, V, 0.0)
+    U64 = V - Z64
+    return keep, torch.from_numpy(Z64).to(W.dtype), torch.from_numpy(U64).to(W.dtype)
 
 
 # ---------------------------------------------------------------------------

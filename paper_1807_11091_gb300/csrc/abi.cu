@@ -181,6 +181,52 @@ sadmm_status sadmm_admm_update(const sadmm_conv_desc* d, const void* W, void* U,
                               workspace, static_cast<cudaStream_t>(stream));
 }
 
+size_t sadmm_elements_workspace_size(const sadmm_conv_desc* d)
+{
+    Geometry g;
+    if (check_desc(d, &g) != SADMM_OK) return 0;
+    return elements_workspace_bytes(g);
+}
+
+sadmm_status sadmm_project_elements(const sadmm_conv_desc* d, const void* W, const void* U, int wdt,
+                                    long long k_elems, unsigned char* keep_out, void* workspace, size_t ws_bytes,
+                                    void* stream)
+{
+    Geometry g;
+    sadmm_status st = check_desc(d, &g);
+    if (st != SADMM_OK) return st;
+    if (!W || !keep_out || !workspace) return SADMM_EINVAL;
+    if (wdt != SADMM_BF16 && wdt != SADMM_FP32) return SADMM_EINVAL;
+    if (k_elems < 0 || k_elems > g.f * g.k) return SADMM_EINVAL;
+    if (ws_bytes < elements_workspace_bytes(g)) return SADMM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0) return SADMM_EINVAL;
+    const size_t esz = (wdt == SADMM_FP32) ? 4 : 2;
+    if (((reinterpret_cast<uintptr_t>(W) | reinterpret_cast<uintptr_t>(U)) & (esz - 1)) != 0) return SADMM_EINVAL;
+    return launch_elements(g, W, const_cast<void*>(U), nullptr, wdt, k_elems, keep_out, workspace,
+                           static_cast<cudaStream_t>(stream));
+}
+
+sadmm_status sadmm_admm_update_elements(const sadmm_conv_desc* d, const void* W, void* U, void* Z, int wdt,
+                                        long long k_elems, void* workspace, size_t ws_bytes, void* stream)
+{
+    Geometry g;
+    sadmm_status st = check_desc(d, &g);
+    if (st != SADMM_OK) return st;
+    if (!W || !U || !Z || !workspace) return SADMM_EINVAL;
+    if (wdt != SADMM_BF16 && wdt != SADMM_FP32) return SADMM_EINVAL;
+    if (k_elems < 0 || k_elems > g.f * g.k) return SADMM_EINVAL;
+    if (ws_bytes < elements_workspace_bytes(g)) return SADMM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0) return SADMM_EINVAL;
+    const size_t esz = (wdt == SADMM_FP32) ? 4 : 2;
+    const uintptr_t bytes = (uintptr_t)(g.f * g.k) * esz;
+    const uintptr_t w = reinterpret_cast<uintptr_t>(W), u = reinterpret_cast<uintptr_t>(U),
+                    z = reinterpret_cast<uintptr_t>(Z);
+    if (((w | u | z) & (esz - 1)) != 0) return SADMM_EINVAL;
+    auto overlap = [bytes](uintptr_t p, uintptr_t q) { return p < q + bytes && q < p + bytes; };
+    if (overlap(w, u) || overlap(w, z) || overlap(u, z)) return SADMM_EINVAL;
+    return launch_elements(g, W, U, Z, wdt, k_elems, nullptr, workspace, static_cast<cudaStream_t>(stream));
+}
+
 sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d, int n_filt, int colkind,
                              int n_colgroups)
 {

@@ -163,10 +163,6 @@ SADMM_DEV uint32_t pixel_mask(const ConvArgs& a, int it0, int ih0, int iw0)
     return m;
 }
 
-// Gather entry e = {offset in x, tap bits}: the column reads inside the input
-// for a pixel of mask M when every tap bit of the entry is set in M.
-SADMM_DEV bool tap_ok(uint32_t bits, uint32_t M) { return (M & bits) == bits; }
-
 // Branch-free conditional gather: the 16-bit element at p when every tap bit
 // of `bits` is set in the pixel mask M, else 0 (a predicated load).
 SADMM_DEV uint32_t ldg_u16_if(const unsigned short* p, uint32_t bits, uint32_t M)

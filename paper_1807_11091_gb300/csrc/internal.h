@@ -44,6 +44,12 @@ sadmm_status launch_admm_update(const Geometry& g, const void* W, void* U, void*
                                 int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out, void* ws,
                                 cudaStream_t s);
 
+// ---- non-structured projection (elements.cu) ----
+size_t elements_workspace_bytes(const Geometry& g);
+// keep_out (optional) and/or the ADMM update (Z and U non-null).
+sadmm_status launch_elements(const Geometry& g, const void* W, void* U, void* Z, int wdt, long long k,
+                             uint8_t* keep_out, void* ws, cudaStream_t s);
+
 // ---- pack (pack.cu) ----
 sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* filt_idx,
                          const int* col_idx, cudaStream_t s);

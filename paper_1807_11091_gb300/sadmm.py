@@ -97,6 +97,13 @@ def load():
     lib.sadmm_admm_workspace_size.argtypes = [P(ConvDesc), ci]
     lib.sadmm_admm_update.restype = ci
     lib.sadmm_admm_update.argtypes = [P(ConvDesc), vp, vp, vp, ci, ci, ci, ci, vp, vp, vp, vp, sz, vp]
+    ll = ctypes.c_longlong
+    lib.sadmm_elements_workspace_size.restype = sz
+    lib.sadmm_elements_workspace_size.argtypes = [P(ConvDesc)]
+    lib.sadmm_project_elements.restype = ci
+    lib.sadmm_project_elements.argtypes = [P(ConvDesc), vp, vp, ci, ll, vp, vp, sz, vp]
+    lib.sadmm_admm_update_elements.restype = ci
+    lib.sadmm_admm_update_elements.argtypes = [P(ConvDesc), vp, vp, vp, ci, ll, vp, sz, vp]
     lib.sadmm_last_device_status.restype = ci
     lib.sadmm_last_device_status.argtypes = [vp]
     lib.sadmm_project_groups_noalloc.restype = ci
@@ -172,6 +179,22 @@ def sadmm_admm_update(desc: ConvDesc, W: int, U: int, Z: int, wdt: int, k_filter
                                     int(k_cols), filt_idx, col_idx, keys_out, workspace, int(ws_bytes), stream)
 
 
+def sadmm_elements_workspace_size(desc: ConvDesc) -> int:
+    return load().sadmm_elements_workspace_size(ctypes.byref(desc))
+
+
+def sadmm_project_elements(desc: ConvDesc, W: int, U: Optional[int], wdt: int, k_elems: int, keep_out: int,
+                           workspace: int, ws_bytes: int, stream: Optional[int]) -> int:
+    return load().sadmm_project_elements(ctypes.byref(desc), W, U, int(wdt), int(k_elems), keep_out, workspace,
+                                         int(ws_bytes), stream)
+
+
+def sadmm_admm_update_elements(desc: ConvDesc, W: int, U: int, Z: int, wdt: int, k_elems: int, workspace: int,
+                               ws_bytes: int, stream: Optional[int]) -> int:
+    return load().sadmm_admm_update_elements(ctypes.byref(desc), W, U, Z, int(wdt), int(k_elems), workspace,
+                                             int(ws_bytes), stream)
+
+
 def sadmm_plan_init(desc: ConvDesc, n_filt: int, colkind: int, n_colgroups: int) -> Tuple[int, Plan]:
     plan = Plan()
     st = load().sadmm_plan_init(ctypes.byref(plan), ctypes.byref(desc), int(n_filt), int(colkind),
@@ -245,6 +268,31 @@ def project_groups(desc16: Sequence[int], W, k_filters: int, colkind: int, k_col
     fi = filt_idx[:k_filters]
     ci = col_idx[:k_cols] if col_idx is not None else None
     return fi, ci, keys
+
+
+def project_elements(desc16: Sequence[int], W, k_elems: int, U=None, stream=None):
+    """Runs sadmm_project_elements; returns the keep flags as a uint8 device tensor of W's shape."""
+    torch = _torch()
+    desc = make_desc(desc16)
+    ws_bytes = sadmm_elements_workspace_size(desc)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=W.device)
+    keep = torch.empty(W.shape, dtype=torch.uint8, device=W.device)
+    st = sadmm_project_elements(desc, _ptr(W), _ptr(U), _wdt(W), k_elems, _ptr(keep), _ptr(ws), ws_bytes,
+                                _stream(stream))
+    _check(st, "sadmm_project_elements")
+    return keep
+
+
+def admm_update_elements(desc16: Sequence[int], W, U, Z, k_elems: int, stream=None, workspace=None):
+    """Z <- the k_elems largest-magnitude entries of W + U; U <- (W + U) - Z."""
+    torch = _torch()
+    desc = make_desc(desc16)
+    ws_bytes = sadmm_elements_workspace_size(desc)
+    if workspace is None or workspace.numel() < ws_bytes:
+        workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=W.device)
+    st = sadmm_admm_update_elements(desc, _ptr(W), _ptr(U), _ptr(Z), _wdt(W), k_elems, _ptr(workspace), ws_bytes,
+                                    _stream(stream))
+    _check(st, "sadmm_admm_update_elements")
 
 
 class AdmmStep:

@@ -111,3 +111,20 @@ def test_admm_update_rejects_bad_arguments_on_host():
                 dict(keys_out=ws_ptr + 4)):
         a = dict(args, **bad)
         assert sadmm.sadmm_admm_update(d, **a) == sadmm.SADMM_EINVAL, bad
+
+
+def test_elements_reject_bad_arguments_on_host():
+    s = wl.single2d()[0].shape
+    d = sadmm.make_desc(s.desc16())
+    ws = sadmm.sadmm_elements_workspace_size(d)
+    assert ws >= 2048 * 4
+    fake, ws_ptr = 1 << 24, 1 << 30
+    N = s.f * s.k
+    args = dict(W=fake, U=None, wdt=sadmm.SADMM_BF16, k_elems=10, keep_out=fake, workspace=ws_ptr, ws_bytes=ws,
+                stream=None)
+    for bad in (dict(W=None), dict(keep_out=None), dict(k_elems=-1), dict(k_elems=N + 1), dict(wdt=3),
+                dict(ws_bytes=ws - 1), dict(workspace=ws_ptr + 8), dict(W=fake + 1)):
+        assert sadmm.sadmm_project_elements(d, **dict(args, **bad)) == sadmm.SADMM_EINVAL, bad
+    Z = fake + (1 << 22)
+    assert sadmm.sadmm_admm_update_elements(d, fake, fake, Z, sadmm.SADMM_FP32, 5, ws_ptr, ws, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_admm_update_elements(d, fake, None, Z, sadmm.SADMM_FP32, 5, ws_ptr, ws, None) == sadmm.SADMM_EINVAL
