@@ -442,6 +442,58 @@ def batch1_report(dev, out_dtype, reps=7):
     return out
 
 
+def backward_report(dev, out_dtype, reps=3):
+    """Masked-retraining backward (sadmm_conv_bwd: dW, db and dx over the kept
+    weights) of every AlexNet CONV layer at batch 128, L2 flushed, median of
+    `reps`; TFLOP/s counts the two retained contractions (weight and input
+    gradient), 4 * M * F' * K'."""
+    import torch
+    from paper_1807_11091_gb300 import sadmm
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    out = {"what": "sadmm_conv_bwd per AlexNet CONV layer at batch 128 (dW, db, dx), L2 flushed", "layers": {}}
+    tot_ms = tot_fl = 0.0
+    for L in wl.alexnet():
+        s = L.shape
+        t = wl.gen_tensors(s, seed=L.seed)
+        r = LayerRun(L, t, dev, "fp32")
+        sp = int(torch.cuda.current_stream().cuda_stream)
+        r.project(sp)
+        r.pack(sp)
+        r.conv(sp)
+        g = torch.Generator().manual_seed(L.seed + 1)
+        dy = torch.randn(s.y_shape(), generator=g).to(torch.bfloat16).to(dev)
+        dW = torch.empty((s.f, s.k), dtype=torch.float32, device=dev)
+        db = torch.empty(s.f, dtype=torch.float32, device=dev)
+        dx = torch.empty(r.x.shape, dtype=torch.float32, device=dev)
+        ws_bytes = sadmm.sadmm_conv_bwd_workspace_size(r.plan)
+        ws = torch.empty(ws_bytes + 1024, dtype=torch.uint8, device=dev)
+        wptr = (ws.data_ptr() + 1023) // 1024 * 1024
+        ms = []
+        for _ in range(reps + 1):
+            flush.fill_(1)
+            torch.cuda._sleep(200_000)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+            st = sadmm.sadmm_conv_bwd(r.plan, r.x.data_ptr(), dy.data_ptr(), r.y.data_ptr(), sadmm.SADMM_FP32, 1,
+                                      dW.data_ptr(), db.data_ptr(), dx.data_ptr(), wptr, ws_bytes, sp)
+            e1.record()
+            torch.cuda.synchronize()
+            assert st == 0, st
+            ms.append(e0.elapsed_time(e1))
+        t_ms = statistics.median(ms[1:])
+        fl = 2.0 * r.flops()
+        tot_ms += t_ms
+        tot_fl += fl
+        out["layers"][L.name] = {"us": t_ms * 1e3, "tflops_retained": fl / (t_ms * 1e-3) / 1e12}
+        del r, dy, dW, db, dx, ws
+    out["total_us"] = tot_ms * 1e3
+    out["tflops_retained"] = tot_fl / (tot_ms * 1e-3) / 1e12
+    del flush
+    torch.cuda.empty_cache()
+    return out
+
+
 def admm_report(dev, peak_gbs, reps=5):
     """sadmm_admm_update (the ADMM Z- and U-update, Sec. 4) on every AlexNet
     CONV layer with fp32 W and U resident in HBM, L2 flushed before each
@@ -647,6 +699,8 @@ def run_gpu(args):
         line["sweep"] = sweep_report(dev, args.out_dtype)
     if rank == 0 and not args.no_batch1:
         line["batch1"] = batch1_report(dev, args.out_dtype)
+    if rank == 0 and not args.no_backward:
+        line["backward"] = backward_report(dev, args.out_dtype)
     if rank == 0 and not args.no_admm:
         line["admm"] = admm_report(dev, peaks.get("hbm_gbs"))
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
@@ -671,6 +725,7 @@ def main():
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-admm", action="store_true")
     ap.add_argument("--no-batch1", action="store_true")
+    ap.add_argument("--no-backward", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

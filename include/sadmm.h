@@ -286,6 +286,42 @@ sadmm_status sadmm_project_groups_noalloc(const sadmm_conv_desc* d, const void* 
                                           int* filt_idx, int* col_idx, double* keys_out,
                                           void* stream);
 
+/* Device bytes of scratch sadmm_conv_bwd needs for this plan (gathered
+ * operands of one chunk of at most 32768 output pixels, fp32 products). */
+size_t sadmm_conv_bwd_workspace_size(const sadmm_plan* plan);
+
+/*
+ * Backward of the packed pruned layer for masked retraining (Sec. 4, "Masked
+ * mapping and retraining": the pruned weights stay zero and only the kept ones
+ * are trained).  With dZ = dY * [y > 0] when relu is set (else dZ = dY):
+ *   dW[f][col] = sum over images and output pixels of dZ * x at (f, col), for
+ *                every kept filter f and kept GEMM column col; 0 elsewhere;
+ *   db[f]      = sum of dZ over images and pixels for kept f; 0 for pruned f;
+ *   dx         = the input gradient through the kept weights only.
+ * The contractions run on the tensor cores (bf16 operands, fp32 accumulation);
+ * dx is summed with fp32 atomics (its last bits depend on timing).
+ *
+ *   plan   a packed plan (sadmm_pack) of the layer.
+ *   x      device bf16 [N][C][T][H][W] (needed for dW).
+ *   dy     device bf16 [N][F][OT][OH][OW].
+ *   y      device forward output of dtype ydt (bf16/fp32), read when relu != 0.
+ *   dW     device fp32 [F][K] (OIDHW) or NULL; db fp32 [F] or NULL;
+ *          dx fp32 [N][C][T][H][W] or NULL.  Every element of each is written.
+ *   workspace  sadmm_conv_bwd_workspace_size(plan) bytes, 1024-byte aligned.
+ */
+sadmm_status sadmm_conv_bwd(const sadmm_plan* plan, const void* x, const void* dy, const void* y, int ydt,
+                            int relu, float* dW, float* db, float* dx, void* workspace, size_t ws_bytes,
+                            void* stream);
+
+/*
+ * The tensor-core GEMM the backward uses, for direct use and testing:
+ * C[M][N] = (accumulate ? C : 0) + A[M][K] * B[N][K]^T with bf16 A and B
+ * (row-major, K contiguous), fp32 C (row stride ldc).  M % 128 == 0,
+ * K % 64 == 0, N a multiple of 16, ldc % 4 == 0, 16-byte aligned pointers.
+ */
+sadmm_status sadmm_gemm_bf16(const void* A, const void* B, float* C, long long M, long long N, long long K,
+                             long long ldc, int accumulate, void* stream);
+
 /*
  * Synchronises `stream`, then reports and clears the device status word that
  * the kernels set when a bounded wait expires (SADMM_ETIMEOUT) or a

@@ -24,6 +24,7 @@ What it computes, with the passage each step follows:
 * ``project_elements`` / ``admm_update_elements`` -- the non-structured case
   (Sec. 4): keep the largest |V| entries.
 * ``conv`` -- direct convolution over the full masked tensor (fp64).
+* ``pruned_conv_backward`` -- gradients for masked retraining (Sec. 4).
 
 Parity pins: every function here is checked in ``tests/test_oracle_*.py``
 against brute force, a library convolution, closed forms and invariants.
@@ -319,3 +320,46 @@ def pruned_conv(x, W, bias, desc16, taps: int, filt_idx, colkind: int, col_idx,
     Wm = masked_weights(W, filt_idx, colkind, col_idx, taps)
     bm = masked_bias(bias, int(desc16[5]), filt_idx)
     return conv(x, Wm, bm, desc16, relu=relu, n0=n0, n1=n1)
+
+
+# ---------------------------------------------------------------------------
+# Backward for masked retraining
+# ---------------------------------------------------------------------------
+
+def pruned_conv_backward(x, W, bias, desc16, taps: int, filt_idx, colkind: int, col_idx, dy, relu: bool = True,
+                         y=None):
+    """Gradients of the pruned layer for masked retraining (Sec. 4: the zero
+    weights stay masked, only kept weights learn), in fp64.
+
+    y = ReLU(conv(x, Wm) + bm) with Wm, bm the masked weights and bias.
+    Returns (dx, dW, db) for the upstream gradient dy: dW and db are the
+    gradients with respect to the kept entries (zero on masked entries), dx the
+    input gradient.  The derivative is taken by torch's autograd in fp64 (a
+    library routine serving as the differentiation step); the tests pin it to
+    finite differences of ``pruned_conv``.  When ``y`` (a given forward
+    output) is passed, the ReLU derivative is [y > 0] from it, so that a
+    comparison takes the ReLU decision on the same values.
+    """
+    import torch
+    d = [int(v) for v in desc16]
+    N, C, T, H, Wd, F, G, KT, KH, KW, ST, SH, SW, PT, PH, PW = d
+    Wm = torch.from_numpy(masked_weights(W, filt_idx, colkind, col_idx, taps)).requires_grad_(True)
+    bm = torch.from_numpy(masked_bias(bias, F, filt_idx)).requires_grad_(True)
+    xd = torch.from_numpy(_as_f64(x)).requires_grad_(True)
+    if T == 1 and KT == 1 and xd.dim() == 4:
+        z = torch.nn.functional.conv2d(xd, Wm.reshape(F, C // G, KH, KW), bm, stride=(SH, SW), padding=(PH, PW),
+                                       groups=G)
+    else:
+        z = torch.nn.functional.conv3d(xd.reshape(N, C, T, H, Wd), Wm.reshape(F, C // G, KT, KH, KW), bm,
+                                       stride=(ST, SH, SW), padding=(PT, PH, PW), groups=G)
+    g = torch.from_numpy(_as_f64(dy)).reshape(z.shape)
+    if relu:
+        on = (torch.from_numpy(_as_f64(y)).reshape(z.shape) > 0) if y is not None else (z.detach() > 0)
+        g = g * on.to(g.dtype)
+    z.backward(g)
+    keep = masked_weights(np.ones(_as_f64(W).shape), filt_idx, colkind, col_idx, taps) != 0
+    dW = Wm.grad.numpy() * keep
+    bkeep = np.zeros(F, dtype=bool)
+    bkeep[np.asarray(filt_idx, dtype=np.int64)] = True
+    db = bm.grad.numpy() * bkeep
+    return xd.grad.numpy().reshape(_as_f64(x).shape), dW, db

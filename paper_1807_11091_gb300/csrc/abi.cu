@@ -339,6 +339,46 @@ sadmm_status sadmm_conv_fwd(const sadmm_plan* plan, const void* x, const float* 
     return launch_conv_fwd(plan, g, x, bias, relu, y, ydt, static_cast<cudaStream_t>(stream));
 }
 
+size_t sadmm_conv_bwd_workspace_size(const sadmm_plan* plan)
+{
+    if (!plan) return 0;
+    Geometry g;
+    if (check_desc(&plan->desc, &g) != SADMM_OK) return 0;
+    return bwd_workspace_bytes(plan, g);
+}
+
+sadmm_status sadmm_conv_bwd(const sadmm_plan* plan, const void* x, const void* dy, const void* y, int ydt, int relu,
+                            float* dW, float* db, float* dx, void* workspace, size_t ws_bytes, void* stream)
+{
+    if (!plan || !plan->dev || !dy || !workspace) return SADMM_EINVAL;
+    Geometry g;
+    sadmm_status st = check_desc(&plan->desc, &g);
+    if (st != SADMM_OK) return st;
+    if (dW && !x) return SADMM_EINVAL;
+    if (relu && !y) return SADMM_EINVAL;
+    if (relu && ydt != SADMM_BF16 && ydt != SADMM_FP32) return SADMM_EINVAL;
+    if (ws_bytes < bwd_workspace_bytes(plan, g)) return SADMM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 1023) != 0) return SADMM_EINVAL;
+    if (((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(dy)) & 1) != 0) return SADMM_EINVAL;
+    if (((reinterpret_cast<uintptr_t>(dW) | reinterpret_cast<uintptr_t>(db) | reinterpret_cast<uintptr_t>(dx)) & 3) != 0)
+        return SADMM_EINVAL;
+    if (device_cc_major() < 10) return SADMM_EUNSUPPORTED;
+    return launch_conv_bwd(plan, g, x, dy, y, ydt, relu, dW, db, dx, workspace, static_cast<cudaStream_t>(stream));
+}
+
+sadmm_status sadmm_gemm_bf16(const void* A, const void* B, float* C, long long M, long long N, long long K,
+                             long long ldc, int accumulate, void* stream)
+{
+    if (!A || !B || !C) return SADMM_EINVAL;
+    if (((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(B) | reinterpret_cast<uintptr_t>(C)) & 15) != 0)
+        return SADMM_EINVAL;
+    int bn = 256;
+    while (bn >= 16 && N % bn != 0) bn -= 16;
+    if (bn < 16) return SADMM_EINVAL;
+    if (device_cc_major() < 10) return SADMM_EUNSUPPORTED;
+    return launch_gemm(A, B, C, M, N, K, ldc, bn, accumulate != 0, static_cast<cudaStream_t>(stream));
+}
+
 sadmm_status sadmm_last_device_status(void* stream)
 {
     if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return SADMM_ECUDA;

@@ -50,6 +50,19 @@ size_t elements_workspace_bytes(const Geometry& g);
 sadmm_status launch_elements(const Geometry& g, const void* W, void* U, void* Z, int wdt, long long k,
                              uint8_t* keep_out, void* ws, cudaStream_t s);
 
+// ---- generic bf16 GEMM on the tensor cores (gemm.cu) ----
+// C[M][N] (fp32, row stride ldc floats) = (accumulate ? C : 0) + A[M][K] * B[N][K]^T,
+// A and B bf16 row-major (K contiguous, row stride K).  M % 128 == 0,
+// N % bn == 0, bn a multiple of 16 in [16, 256], K % 64 == 0, ldc % 4 == 0,
+// A, B and C 16-byte aligned.
+sadmm_status launch_gemm(const void* A, const void* B, float* C, long long M, long long N, long long K,
+                         long long ldc, int bn, bool accumulate, cudaStream_t s);
+
+// ---- masked-retraining backward (bwd.cu) ----
+size_t bwd_workspace_bytes(const sadmm_plan* plan, const Geometry& g);
+sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const void* x, const void* dy, const void* y,
+                             int ydt, int relu, float* dW, float* db, float* dx, void* ws, cudaStream_t s);
+
 // ---- pack (pack.cu) ----
 sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* filt_idx,
                          const int* col_idx, cudaStream_t s);

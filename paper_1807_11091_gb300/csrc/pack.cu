@@ -189,6 +189,8 @@ __global__ void __launch_bounds__(128) k_pack_wp(const T* __restrict__ W, int K,
     }
 }
 
+}  // namespace
+
 PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn()
 {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -203,8 +205,6 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn()
     }
     return fn;
 }
-
-}  // namespace
 
 sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* filt_idx,
                          const int* col_idx, cudaStream_t s)

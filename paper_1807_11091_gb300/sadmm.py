@@ -104,6 +104,12 @@ def load():
     lib.sadmm_project_elements.argtypes = [P(ConvDesc), vp, vp, ci, ll, vp, vp, sz, vp]
     lib.sadmm_admm_update_elements.restype = ci
     lib.sadmm_admm_update_elements.argtypes = [P(ConvDesc), vp, vp, vp, ci, ll, vp, sz, vp]
+    lib.sadmm_conv_bwd_workspace_size.restype = sz
+    lib.sadmm_conv_bwd_workspace_size.argtypes = [P(Plan)]
+    lib.sadmm_conv_bwd.restype = ci
+    lib.sadmm_conv_bwd.argtypes = [P(Plan), vp, vp, vp, ci, ci, vp, vp, vp, vp, sz, vp]
+    lib.sadmm_gemm_bf16.restype = ci
+    lib.sadmm_gemm_bf16.argtypes = [vp, vp, vp, ll, ll, ll, ll, ci, vp]
     lib.sadmm_last_device_status.restype = ci
     lib.sadmm_last_device_status.argtypes = [vp]
     lib.sadmm_project_groups_noalloc.restype = ci
@@ -210,6 +216,21 @@ def sadmm_pack(plan: Plan, W: int, wdt: int, filt_idx: Optional[int], col_idx: O
 def sadmm_conv_fwd(plan: Plan, x: int, bias: Optional[int], relu: int, y: int, ydt: int,
                    stream: Optional[int]) -> int:
     return load().sadmm_conv_fwd(ctypes.byref(plan), x, bias, int(relu), y, int(ydt), stream)
+
+
+def sadmm_conv_bwd_workspace_size(plan: Plan) -> int:
+    return load().sadmm_conv_bwd_workspace_size(ctypes.byref(plan))
+
+
+def sadmm_conv_bwd(plan: Plan, x: Optional[int], dy: int, y: Optional[int], ydt: int, relu: int, dW: Optional[int],
+                   db: Optional[int], dx: Optional[int], workspace: int, ws_bytes: int, stream: Optional[int]) -> int:
+    return load().sadmm_conv_bwd(ctypes.byref(plan), x, dy, y, int(ydt), int(relu), dW, db, dx, workspace,
+                                 int(ws_bytes), stream)
+
+
+def sadmm_gemm_bf16(A: int, B: int, C: int, M: int, N: int, K: int, ldc: int, accumulate: int,
+                    stream: Optional[int]) -> int:
+    return load().sadmm_gemm_bf16(A, B, C, int(M), int(N), int(K), int(ldc), int(accumulate), stream)
 
 
 def sadmm_last_device_status(stream: Optional[int]) -> int:
@@ -347,6 +368,23 @@ class PrunedConv:
         st = sadmm_pack(self.plan, _ptr(W), _wdt(W), _ptr(filt_idx), _ptr(col_idx), _ptr(self.buf),
                         self.plan.dev_bytes, _stream(stream))
         _check(st, "sadmm_pack")
+
+    def backward(self, x, dy, y=None, relu=True, want_dw=True, want_db=True, want_dx=True, stream=None):
+        """Runs sadmm_conv_bwd; returns (dW, db, dx) fp32 device tensors (None where not requested)."""
+        torch = _torch()
+        n, c, t, h, w, f, g, kt, kh, kw = self.desc16[:10]
+        dev = dy.device
+        dW = torch.empty((f, (c // g) * kt * kh * kw), dtype=torch.float32, device=dev) if want_dw else None
+        db = torch.empty(f, dtype=torch.float32, device=dev) if want_db else None
+        dx = torch.empty(x.shape, dtype=torch.float32, device=dev) if want_dx else None
+        ws_bytes = sadmm_conv_bwd_workspace_size(self.plan)
+        ws = torch.empty(ws_bytes + 1024, dtype=torch.uint8, device=dev)
+        wptr = (_ptr(ws) + 1023) // 1024 * 1024
+        ydt = SADMM_BF16 if (y is not None and y.dtype == torch.bfloat16) else SADMM_FP32
+        st = sadmm_conv_bwd(self.plan, _ptr(x), _ptr(dy), _ptr(y), ydt, 1 if relu else 0, _ptr(dW), _ptr(db),
+                            _ptr(dx), wptr, ws_bytes, _stream(stream))
+        _check(st, "sadmm_conv_bwd")
+        return dW, db, dx
 
     def out_shape(self):
         n, c, t, h, w, f, g, kt, kh, kw, st_, sh, sw, pt, ph, pw = self.desc16

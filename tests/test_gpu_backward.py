@@ -1,0 +1,107 @@
+"""GPU parity of the masked-retraining backward (sadmm_conv_bwd) and of the
+tensor-core GEMM it uses.
+
+The GEMM is compared with a plain PyTorch fp64 product of the same bf16
+operands.  The backward is compared with the oracle's fp64 gradients: dW, db
+and dx within 2e-3 * max|reference| per tensor, masked weight entries and
+pruned filters' bias gradients exactly zero, every output element written.
+The ReLU derivative comes from the oracle's own forward output on both sides
+(passed in as y), so the two take the same ReLU decisions.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads as wl
+from workloads import ConvShape
+
+from _helpers import assert_close
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("shape", [(128, 256, 64), (384, 160, 640), (256, 48, 192)])
+@pytest.mark.parametrize("accumulate", [0, 1])
+def test_gemm_matches_torch(shape, accumulate):
+    from paper_1807_11091_gb300 import sadmm
+    M, N, K = shape
+    g = torch.Generator().manual_seed(M + N + K)
+    A = torch.randn(M, K, generator=g).to(torch.bfloat16)
+    B = torch.randn(N, K, generator=g).to(torch.bfloat16)
+    C0 = torch.randn(M, N, generator=g)
+    dev = torch.device("cuda", 0)
+    Ad, Bd, Cd = A.to(dev), B.to(dev), C0.to(dev).clone()
+    st = sadmm.sadmm_gemm_bf16(Ad.data_ptr(), Bd.data_ptr(), Cd.data_ptr(), M, N, K, N, accumulate,
+                               int(torch.cuda.current_stream().cuda_stream))
+    assert st == 0
+    ref = A.double() @ B.double().T + (C0.double() if accumulate else 0)
+    err = (Cd.cpu().double() - ref).abs().max().item()
+    assert err <= 1e-5 * ref.abs().max().item()
+
+
+CASES = [
+    ("ragged", ConvShape(n=3, c=5, h=11, w=13, f=37, kh=3, kw=3, ph=1, pw=1), 0.7, wl.COL_SHAPE, 0.4),
+    ("groups2_5x5", ConvShape(n=2, c=8, h=9, w=9, f=12, kh=5, kw=5, ph=2, pw=2, groups=2), 0.5, wl.COL_SHAPE, 0.5),
+    ("stride4_11x11", ConvShape(n=2, c=3, h=35, w=35, f=16, kh=11, kw=11, sh=4, sw=4), 1.0, wl.COL_SHAPE, 0.8),
+    ("c3d", ConvShape(n=2, c=4, t=5, h=6, w=7, f=20, kt=3, kh=3, kw=3, pt=1, ph=1, pw=1), 1.0, wl.COL_SHAPE, 0.3),
+    ("channel_3x3", ConvShape(n=2, c=24, h=9, w=9, f=40, kh=3, kw=3, ph=1, pw=1), 0.5, wl.COL_CHANNEL, 0.5),
+    ("two_filter_tiles", ConvShape(n=2, c=16, h=10, w=10, f=300, kh=3, kw=3, ph=1, pw=1), 1.0, wl.COL_SHAPE, 1.0),
+]
+
+
+def _backward(s, t, kf, ck, kc, relu=True, seed=0):
+    from paper_1807_11091_gb300 import sadmm
+    dev = torch.device("cuda", 0)
+    rows, cols, _, _ = oracle.project(t["W"], s.taps, kf, ck, kc)
+    # oracle forward output: the ReLU decision for both sides
+    y = torch.from_numpy(oracle.pruned_conv(t["x"], t["W"], t["bias"], s.desc16(), s.taps, rows, ck, cols,
+                                            relu=True)).float()
+    g = torch.Generator().manual_seed(seed)
+    dy = torch.randn(y.shape, generator=g).to(torch.bfloat16)
+    W, x = t["W"].to(dev), t["x"].to(dev)
+    fi = torch.as_tensor(rows, dtype=torch.int32, device=dev)
+    ci = torch.as_tensor(cols, dtype=torch.int32, device=dev) if ck != wl.COL_NONE else None
+    pc = sadmm.PrunedConv(s.desc16(), W, fi if kf < s.f else None, ck, ci, kf, kc if ck != wl.COL_NONE else s.k)
+    dW, db, dx = pc.backward(x, dy.to(dev), y=y.to(dev), relu=relu)
+    assert sadmm.device_status() == 0
+    rdx, rdW, rdb = oracle.pruned_conv_backward(t["x"], t["W"], t["bias"], s.desc16(), s.taps, rows, ck, cols, dy,
+                                                relu=relu, y=y)
+    return (dW.cpu().numpy(), db.cpu().numpy(), dx.cpu().numpy()), (rdW.reshape(s.f, -1), rdb, rdx), rows, cols
+
+
+@pytest.mark.parametrize("case", CASES, ids=lambda c: c[0])
+def test_backward_matches_oracle(case):
+    name, s, ff, ck, cf = case
+    G = s.cg if ck == wl.COL_CHANNEL else s.k
+    kf, kc = wl.retained(ff, s.f), (wl.retained(cf, G) if ck != wl.COL_NONE else 0)
+    t = wl.gen_tensors(s, seed=13)
+    (dW, db, dx), (rdW, rdb, rdx), rows, cols = _backward(s, t, kf, ck, kc)
+    assert np.all(np.isfinite(dW)) and np.all(np.isfinite(dx)) and np.all(np.isfinite(db))
+    assert_close(dW, rdW, what=f"{name} dW")
+    assert_close(db, rdb, what=f"{name} db")
+    assert_close(dx, rdx, what=f"{name} dx")
+    keep = oracle.masked_weights(np.ones(t["W"].shape), rows, ck, cols, s.taps).reshape(s.f, -1) != 0
+    assert np.all(dW[~keep] == 0.0)
+    pruned = np.setdiff1d(np.arange(s.f), rows)
+    assert np.all(db[pruned] == 0.0)
+
+
+@pytest.mark.parametrize("li", range(5))
+def test_backward_alexnet_layers_batch2(li):
+    L = wl.subset_layer(wl.alexnet()[li], 2)
+    s = L.shape
+    t = wl.gen_tensors(s, seed=L.seed)
+    (dW, db, dx), (rdW, rdb, rdx), _, _ = _backward(s, t, L.k_filters, L.colkind, L.k_cols, seed=li)
+    assert_close(dW, rdW, what=f"{L.name} dW")
+    assert_close(db, rdb, what=f"{L.name} db")
+    assert_close(dx, rdx, what=f"{L.name} dx")
+
+
+def test_backward_without_relu():
+    name, s, ff, ck, cf = CASES[0]
+    kf, kc = wl.retained(ff, s.f), wl.retained(cf, s.k)
+    t = wl.gen_tensors(s, seed=5)
+    (dW, db, dx), (rdW, rdb, rdx), _, _ = _backward(s, t, kf, ck, kc, relu=False)
+    assert_close(dW, rdW, what="no relu dW")
+    assert_close(dx, rdx, what="no relu dx")
