@@ -8,11 +8,10 @@
 //                   fixed-order block reduction.
 //   k_column_keys   32 columns per block, 8 warps over the (kept) rows, fixed
 //                   order shared-memory reduction: one key per GEMM column.
-//   k_select        one block: optional channel sums of column keys (the keys
-//                   stay in registers, eight per thread), an MSB-first radix
-//                   select over the fp64 key bit patterns (exact k-th largest
-//                   key), then an ordered compaction that keeps every key above
-//                   it and the lowest-index keys equal to it.
+//   k_select        one block: optional channel sums of column keys, an MSB-
+//                   first radix select over the fp64 key bit patterns (exact
+//                   k-th largest key), then an ordered compaction that keeps
+//                   every key above it and the lowest-index keys equal to it.
 //
 // Keys are non-negative fp64 values, so their IEEE bit patterns order like the
 // values; selection compares bit patterns (a NaN key would rank above +Inf).
@@ -136,27 +135,10 @@ SADMM_DEV int block_excl_count(bool pred, int* warp_tot, int* total)
     return r;
 }
 
-constexpr int kSelPer = 8;  // keys per thread held in registers (G <= 8192)
-
-// hist[d] += 1 for every lane with `active` set, one atomic per distinct digit
-// of the warp (keys share their high bits, so per-lane atomics would
-// serialise on a few bins).
-SADMM_DEV void hist_add(unsigned int* hist, unsigned d, bool active)
-{
-    const unsigned act = __ballot_sync(0xffffffffu, active);
-    if (!active) return;
-    const unsigned peers = __match_any_sync(act, d);
-    if ((threadIdx.x & 31) == (unsigned)(__ffs(peers) - 1)) atomicAdd(&hist[d], (unsigned)__popc(peers));
-}
-
 // Exact top-k of G fp64 keys (ties to the lower index), ascending index list.
 // When taps > 1 the keys are first formed as sums of `taps` consecutive source
 // keys (channel-wise groups from column keys).  keep_out (optional) gets a
-// byte per group: 1 when kept.  With G <= kSelThreads * kSelPer every thread
-// holds its keys (i = tid + q * kSelThreads) in registers, so the radix passes
-// and the compaction read no memory; larger G re-reads the keys from global
-// memory.
-template <bool REG>
+// byte per group: 1 when kept.
 __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict__ src, int G, int taps, int k,
                                                         int nparts, long long part_stride,
                                                         double* __restrict__ keys, double* __restrict__ keys_out,
@@ -167,15 +149,13 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
     __shared__ int s_kk;
     __shared__ int warp_tot[33];
     const int tid = threadIdx.x;
-    unsigned long long kr[REG ? kSelPer : 1];
 
     // 1. keys: the sum of the nparts partial sums of each source key, then of
     //    `taps` consecutive source keys (channel-wise groups); and the optional
     //    copy for the caller
-    const bool formed = (taps > 1 || nparts > 1);
     // the taps * nparts source values of key i, in four independent partial
     // sums (fixed order: entry e goes to partial e % 4)
-    auto form = [&](int i) -> double {
+    for (int i = tid; i < G; i += kSelThreads) {
         const int n = taps * nparts;
         double v0 = 0.0, v1 = 0.0, v2 = 0.0, v3 = 0.0;
         int e = 0;
@@ -191,27 +171,11 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
             v0 += src[(e - t * nparts) * part_stride + (long long)i * taps + t];
         }
         const double v = (v0 + v1) + (v2 + v3);
+        if (taps > 1 || nparts > 1) keys[i] = v;
         if (keys_out) keys_out[i] = v;
-        return v;
-    };
-    if (REG) {
-#pragma unroll
-        for (int q = 0; q < kSelPer; ++q) {
-            const int i = tid + q * kSelThreads;
-            kr[q] = (i < G) ? (unsigned long long)__double_as_longlong(form(i)) : 0ull;
-        }
-    } else {
-        for (int i = tid; i < G; i += kSelThreads) {
-            const double v = form(i);
-            if (formed) keys[i] = v;
-        }
     }
-    const double* kv = formed ? keys : src;
+    const double* kv = (taps > 1 || nparts > 1) ? keys : src;
     __syncthreads();
-    auto key_at = [&](int q, int i) -> unsigned long long {
-        if (REG) return kr[q];
-        return (unsigned long long)__double_as_longlong(kv[i]);
-    };
 
     if (k <= 0 || k >= G) {
         for (int i = tid; i < G; i += kSelThreads) {
@@ -228,18 +192,9 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
         for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0u;
         __syncthreads();
         const unsigned long long prefix = s_prefix;
-        if (REG) {
-#pragma unroll
-            for (int q = 0; q < kSelPer; ++q) {
-                const int i = tid + q * kSelThreads;
-                hist_add(hist, (unsigned)((kr[q] >> shift) & 255u), i < G && (kr[q] & mask) == prefix);
-            }
-        } else {
-            for (int base = 0; base < G; base += kSelThreads) {
-                const int i = base + tid;
-                const unsigned long long u = i < G ? key_at(0, i) : 0ull;
-                hist_add(hist, (unsigned)((u >> shift) & 255u), i < G && (u & mask) == prefix);
-            }
+        for (int i = tid; i < G; i += kSelThreads) {
+            const unsigned long long u = (unsigned long long)__double_as_longlong(kv[i]);
+            if ((u & mask) == prefix) atomicAdd(&hist[(u >> shift) & 255u], 1u);
         }
         __syncthreads();
         if (tid < 32) {
@@ -274,17 +229,10 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
 
     // 3. ordered compaction
     int run_out = 0, run_eq = 0;
-    for (int base = 0, q = 0; base < G; base += kSelThreads, ++q) {
+    for (int base = 0; base < G; base += kSelThreads) {
         const int i = base + tid;
         const bool valid = i < G;
-        unsigned long long u = 0ull;
-        if (REG) {
-#pragma unroll
-            for (int r = 0; r < kSelPer; ++r)
-                if (r == q) u = kr[r];
-        } else if (valid) {
-            u = key_at(0, i);
-        }
+        const unsigned long long u = valid ? (unsigned long long)__double_as_longlong(kv[i]) : 0ull;
         const bool gt = valid && u > T;
         const bool eq = valid && u == T;
         int eq_tot, take_tot;
@@ -301,12 +249,7 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
 void launch_select(const double* src, int G, int taps, int k, int nparts, long long part_stride, double* keys,
                    double* keys_out, int* out_idx, uint8_t* keep_out, cudaStream_t s)
 {
-    if (G <= kSelThreads * kSelPer)
-        k_select<true><<<1, kSelThreads, 0, s>>>(src, G, taps, k, nparts, part_stride, keys, keys_out, out_idx,
-                                                 keep_out);
-    else
-        k_select<false><<<1, kSelThreads, 0, s>>>(src, G, taps, k, nparts, part_stride, keys, keys_out, out_idx,
-                                                  keep_out);
+    k_select<<<1, kSelThreads, 0, s>>>(src, G, taps, k, nparts, part_stride, keys, keys_out, out_idx, keep_out);
 }
 
 // Row chunks of the column-key pass: enough blocks to fill the GPU, with the

@@ -34,9 +34,14 @@ def main(argv=None) -> int:
     ap.add_argument("--dense", action="store_true", help="keep every filter and column")
     ap.add_argument("--admm", action="store_true",
                     help="time sadmm_admm_update on fp32 W/U of the layer instead of the forward call")
+    ap.add_argument("--elements", type=float, default=0.0,
+                    help="time the non-structured ADMM update keeping this fraction of the weights")
+    ap.add_argument("--backward", action="store_true", help="time sadmm_conv_bwd (dW, db, dx) after one forward")
     args = ap.parse_args(argv)
     if args.admm:
         return run_admm(args)
+    if args.elements > 0:
+        return run_elements(args)
 
     L = wl.get(args.workload)[args.layer]
     s = L.shape if args.batch == 0 else L.shape.with_batch(args.batch)
@@ -50,6 +55,22 @@ def main(argv=None) -> int:
     ydt = torch.bfloat16 if args.out_dtype == "bf16" else torch.float32
     y = torch.empty(pc.out_shape(), dtype=ydt, device="cuda")
     flops = 2.0 * s.m * kf * pc.plan.n_cols
+    if args.backward:
+        pc.forward(t["x"], t["bias"], out=y)
+        g = torch.Generator().manual_seed(L.seed + 1)
+        dy = torch.randn(y.shape, generator=g).to(torch.bfloat16).cuda()
+        for i in range(args.reps):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            torch.cuda._sleep(200_000)
+            e0.record()
+            pc.backward(t["x"], dy, y=y)
+            e1.record()
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1)
+            print(f"{L.name} N={s.n} backward run {i}: {ms * 1e3:.1f} us  {2 * flops / ms / 1e9:.1f} TFLOP/s "
+                  "(dW and dx contractions)")
+        return 1 if sadmm.device_status() != 0 else 0
     for i in range(args.reps):
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
@@ -68,6 +89,36 @@ def main(argv=None) -> int:
         print(f"device status {st}")
         return 1
     return 0
+
+
+def run_elements(args) -> int:
+    """sadmm_admm_update_elements `reps` times on the layer's fp32 ADMM state."""
+    import torch
+
+    import workloads as wl
+    from paper_1807_11091_gb300 import sadmm
+
+    L = wl.get(args.workload)[args.layer]
+    s = L.shape
+    st = wl.gen_admm_state(s, L.seed)
+    W, U = st["W"].cuda(), st["U"].cuda()
+    Z = torch.empty_like(W)
+    k = int(args.elements * s.f * s.k)
+    ws = torch.empty(sadmm.sadmm_elements_workspace_size(sadmm.make_desc(s.desc16())), dtype=torch.uint8,
+                     device="cuda")
+    nbytes = 16.0 * s.f * s.k
+    for i in range(args.reps):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        torch.cuda._sleep(200_000)
+        e0.record()
+        sadmm.admm_update_elements(s.desc16(), W, U, Z, k, workspace=ws)
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        print(f"{L.name} elements {args.elements} run {i}: {ms * 1e3:.1f} us  {nbytes / ms / 1e6:.1f} GB/s "
+              "(16 B per weight)")
+    return 1 if sadmm.device_status() != 0 else 0
 
 
 def run_admm(args) -> int:
