@@ -9,8 +9,9 @@
 //   dA[m][j]  = sum_i dZ[m][f_i] * Wp[i][j]         (then col2im into dx)
 //   db[f_i]   = sum_m dZ[m][f_i]
 // Per conv group and per chunk of output pixels the two contractions run on
-// the tensor cores (gemm.cu) over bf16 operands gathered here; dWp
-// accumulates over chunks in fp32, dx receives the col2im sums with fp32
+// the tensor cores (gemm.cu) over bf16 operands gathered here; the weight
+// gradient's few output tiles split each chunk's pixels over many CTAs that
+// add into dWp with fp32 atomics, and dx receives the col2im sums with fp32
 // atomics.
 #include <algorithm>
 
@@ -37,17 +38,28 @@ struct BwdGeo {
     int fk;       // filter extent of the dgrad operand: n_pad rounded up to 64
     int kr;       // column rows of the dgrad product: k_pad rounded up to 128
     int mc;       // pixels per chunk (multiple of 256)
+    uint32_t plane_mul, plane_sh, ohw_mul, ohw_sh, ow_mul, ow_sh;  // multiply-shift divisors
 };
 
-// Output pixel m -> (n, ot, oh, ow).
+inline void divisor(uint32_t d, uint32_t& mul, uint32_t& sh)
+{
+    sh = 0;
+    while ((1ull << sh) < d) ++sh;
+    mul = (uint32_t)((((1ull << sh) - d) << 32) / d + 1);
+}
+
+// Output pixel m -> (n, ot, oh, ow), by multiply-shift division (m < 2^31).
+SADMM_DEV uint32_t udiv(uint32_t n, uint32_t mul, uint32_t sh) { return (__umulhi(n, mul) + n) >> sh; }
+
 SADMM_DEV void pixel_of(const BwdGeo& b, long long m, int& n, int& ot, int& oh, int& ow)
 {
-    n = (int)(m / b.plane);
-    int p = (int)(m - (long long)n * b.plane);
-    ot = p / (b.OH * b.OW);
-    p -= ot * b.OH * b.OW;
-    oh = p / b.OW;
-    ow = p - oh * b.OW;
+    const uint32_t mu = (uint32_t)m;
+    n = (int)udiv(mu, b.plane_mul, b.plane_sh);
+    const uint32_t p = mu - (uint32_t)n * (uint32_t)b.plane;
+    ot = (int)udiv(p, b.ohw_mul, b.ohw_sh);
+    const uint32_t r = p - (uint32_t)ot * (uint32_t)(b.OH * b.OW);
+    oh = (int)udiv(r, b.ow_mul, b.ow_sh);
+    ow = (int)(r - (uint32_t)oh * (uint32_t)b.OW);
 }
 
 // A_T[j][ml] = x at kept column j of output pixel m0 + ml (0 outside the input,
@@ -233,6 +245,9 @@ BwdGeo geometry(const sadmm_plan* plan, const Geometry& g)
     b.fk = (int)rup(plan->n_pad, 64);
     b.kr = (int)rup(plan->k_pad, 128);
     b.mc = (int)std::min<long long>(rup(g.m, 256), 32768);
+    divisor((uint32_t)b.plane, b.plane_mul, b.plane_sh);
+    divisor((uint32_t)(b.OH * b.OW), b.ohw_mul, b.ohw_sh);
+    divisor((uint32_t)b.OW, b.ow_mul, b.ow_sh);
     return b;
 }
 
@@ -253,6 +268,7 @@ size_t bwd_workspace_bytes(const sadmm_plan* plan, const Geometry& g)
 sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const void* x, const void* dy, const void* y,
                              int ydt, int relu, float* dW, float* db, float* dx, void* ws, cudaStream_t s)
 {
+    if (g.m >= (1ll << 31)) return SADMM_EUNSUPPORTED;  // pixel indices decode in 32 bits
     BwdGeo b = geometry(plan, g);
     const char* base = static_cast<const char*>(plan->dev);
     b.x = static_cast<const __nv_bfloat16*>(x);
@@ -275,7 +291,21 @@ sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const vo
     const unsigned xblocks = (unsigned)std::min<long long>((b.mc + 255) / 256, 64);
     const long long K = g.cg * g.taps;
 
-    if (dW) k_bwd_zero<<<1024, 256, 0, s>>>(dW, g.f * K);
+    if (dW) {
+        k_bwd_zero<<<1024, 256, 0, s>>>(dW, g.f * K);
+        k_bwd_zero<<<256, 256, 0, s>>>(dwp, (long long)b.groups * b.fr * b.k_pad);
+    }
+    // weight-gradient tiles are few (fr/128 x k_pad/bn): split the pixel
+    // dimension of each chunk over enough CTAs to fill the GPU
+    const int wbn = pick_bn(b.k_pad);
+    const long long wtiles = (long long)(b.fr / 128) * (b.k_pad / wbn);
+    int wsplit = 1;
+    {
+        const long long nk = b.mc / 64;
+        long long want = std::max<long long>(1, (2LL * device_sm_count()) / std::max<long long>(wtiles, 1));
+        for (long long d = std::min(want, nk); d >= 1; --d)
+            if (nk % d == 0) { wsplit = (int)d; break; }
+    }
     if (dx) k_bwd_zero<<<2048, 256, 0, s>>>(dx, g.n * g.c * g.t * g.h * g.w);
     if (db) k_bwd_db<<<(unsigned)g.f, 256, 0, s>>>(b, db);
     sadmm_status st = SADMM_OK;
@@ -287,8 +317,8 @@ sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const vo
             k_bwd_gather_dy<<<dim3(xblocks, dyrows), 256, 0, s>>>(b, grp, m0, gt, gm);
             if (dW) {
                 k_bwd_im2col<<<dim3(xblocks, (unsigned)b.k_pad), 256, 0, s>>>(b, grp, m0, at);
-                // dWp[i][j] (+)= sum_m gt[i][m] * at[j][m]
-                st = launch_gemm(gt, at, dwp_g, b.fr, b.k_pad, b.mc, b.k_pad, pick_bn(b.k_pad), m0 > 0, s);
+                // dWp[i][j] += sum_m gt[i][m] * at[j][m] (zeroed above; split over pixels)
+                st = launch_gemm(gt, at, dwp_g, b.fr, b.k_pad, b.mc, b.k_pad, wbn, true, s, wsplit);
             }
             if (dx && st == SADMM_OK) {
                 // dat[j][m] = sum_i wpt[j][i] * gm[m][i]

@@ -28,9 +28,9 @@ constexpr int kATile = 128 * 128;  // 128 rows x 64 bf16
 struct GemmArgs {
     float* C;
     long long ldc;
-    int nk;  // K / 64
+    int nk;  // K / 64 stages of this CTA (its split)
     int bn;
-    int accumulate;
+    int accumulate;  // 0: C = product; 1: C += product; 2: C += product with atomics (split K)
     int tmem_cols;
     int* status;
 };
@@ -52,6 +52,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int m0 = blockIdx.x * 128, n0 = blockIdx.y * a.bn;
+    const int k0 = blockIdx.z * a.nk * 64;  // first K column of this split
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kGemmStages; ++s) {
@@ -82,8 +83,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 const uint32_t ph = (uint32_t)(ks / kGemmStages) & 1u;
                 if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, a.status)) break;
                 mbar_arrive_expect_tx(&full[s], (uint32_t)kATile + b_bytes);
-                tma_load_2d(sA + (size_t)s * kATile, &ta, &full[s], ks * 64, m0);
-                tma_load_2d(sB + (size_t)s * b_bytes, &tb, &full[s], ks * 64, n0);
+                tma_load_2d(sA + (size_t)s * kATile, &ta, &full[s], k0 + ks * 64, m0);
+                tma_load_2d(sB + (size_t)s * b_bytes, &tb, &full[s], k0 + ks * 64, n0);
                 ++issued;
             }
             // the loads issued have landed before the CTA retires
@@ -129,6 +130,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 uint32_t r[16];
                 tmem_ld_32x32b_x16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, r);
                 tmem_ld_wait();
+                if (a.accumulate == 2) {
+                    // split K: several CTAs add into the same tile
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) atomicAdd(crow + c0 + j, __uint_as_float(r[j]));
+                    continue;
+                }
                 float4* dst = reinterpret_cast<float4*>(crow + c0);
 #pragma unroll
                 for (int j = 0; j < 4; ++j) {
@@ -168,19 +175,20 @@ bool encode_kmajor(CUtensorMap* map, const void* base, long long rows, long long
 }  // namespace
 
 sadmm_status launch_gemm(const void* A, const void* B, float* C, long long M, long long N, long long K,
-                         long long ldc, int bn, bool accumulate, cudaStream_t s)
+                         long long ldc, int bn, bool accumulate, cudaStream_t s, int splits)
 {
     if (M <= 0 || N <= 0 || K <= 0) return SADMM_OK;
     if (M % 128 || bn < 16 || bn > 256 || bn % 16 || N % bn || K % 64 || ldc % 4 || ldc < N) return SADMM_EINVAL;
+    if (splits < 1 || (K / 64) % splits != 0 || splits > 65535) return SADMM_EINVAL;
     if (M / 128 > 65535 * 1024ll || N / bn > 65535) return SADMM_EUNSUPPORTED;
     alignas(64) CUtensorMap ta, tb;
     if (!encode_kmajor(&ta, A, M, K, 128) || !encode_kmajor(&tb, B, N, K, bn)) return SADMM_ECUDA;
     GemmArgs a;
     a.C = C;
     a.ldc = ldc;
-    a.nk = (int)(K / 64);
+    a.nk = (int)(K / 64 / splits);
     a.bn = bn;
-    a.accumulate = accumulate ? 1 : 0;
+    a.accumulate = splits > 1 ? 2 : (accumulate ? 1 : 0);
     int cols = 32;
     while (cols < bn) cols <<= 1;
     a.tmem_cols = cols;
@@ -194,7 +202,7 @@ sadmm_status launch_gemm(const void* A, const void* B, float* C, long long M, lo
             return SADMM_ECUDA;
         configured_dev = dev;
     }
-    const dim3 grid((unsigned)(M / 128), (unsigned)(N / bn));
+    const dim3 grid((unsigned)(M / 128), (unsigned)(N / bn), (unsigned)splits);
     k_gemm<<<grid, kGemmThreads, smem, s>>>(ta, tb, a);
     return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
 }
