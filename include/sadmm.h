@@ -42,7 +42,7 @@
 extern "C" {
 #endif
 
-#define SADMM_ABI_VERSION 2
+#define SADMM_ABI_VERSION 3
 
 /* Bytes of the fixed device array of sadmm_project_groups_noalloc. */
 #define SADMM_NOALLOC_SCRATCH_BYTES (256 * 1024)
@@ -95,6 +95,9 @@ typedef struct {
     size_t off_partial; /* split-K partial sums (when splits > 1)              */
     int splits;         /* K' split over this many CTAs per output tile (>= 1)  */
     int stages_per_split; /* 64-column stages of K' per split                  */
+    size_t off_sk;      /* stream-K partial sums and arrival counters (sk_len > 0) */
+    int sk_len;         /* stream-K: 64-column stages per CTA (0: whole tiles)  */
+    int sk_grid;        /* stream-K: CTAs launched                              */
     uint64_t tmap[16];/* 128-byte TMA tensor map of the packed matrix         */
 } sadmm_plan;
 
@@ -216,6 +219,18 @@ sadmm_status sadmm_admm_update_elements(const sadmm_conv_desc* d, const void* W,
  * writes fp32 partial sums to a region of the plan's device buffer and a
  * second kernel adds them in split order, then applies bias and ReLU.  The
  * split depends on the current device's SM count and is fixed in the plan.
+ *
+ * Tail balance (stream-K): when the output tiles do not divide evenly over the
+ * SMs and an even share of the tiles' 64-column stages (plan->sk_len per CTA,
+ * plan->sk_grid CTAs) shortens the busiest CTA's work by at least 1/8, each
+ * CTA takes a contiguous run of stages instead of whole tiles (only when a
+ * tile's accumulator fits TMEM twice and K' is at least 4 * bn, where the cost
+ * of a cut tile measured below its gain).  A tile cut at
+ * a run boundary is finished by whichever of its two CTAs arrives last: both
+ * write fp32 partial sums to the plan's buffer, an arrival counter there
+ * (reset by the last arrival; zeroed by sadmm_pack) tells the second which
+ * it is, and it adds the two halves in K' order, then bias and ReLU.  After a
+ * device-side failure (sadmm_last_device_status) the plan must be packed again.
  */
 sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d,
                              int n_filt, int colkind, int n_colgroups);

@@ -300,6 +300,32 @@ sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d, int n_f
                 p.off_partial = take((size_t)bytes);
             }
         }
+        // stream-K when the tiles do not spread evenly: a run of L stages per
+        // CTA instead of ceil(units / sms) whole tiles, if that shortens the
+        // busiest CTA by at least 1/8 and no tile is cut more than once
+        // (L >= nks).  A cut tile costs a write and a read of 8 bytes per pixel
+        // and filter row; measured on GB300 that pays only with two TMEM
+        // accumulator sets (the finishing piece overlaps the next tile's MMAs)
+        // and a K' of at least four times the filter rows.
+        const long long total = units * nks;
+        const int nacc = p.n_tiles >= 2 ? 2 : 1;
+        const bool two_acc = 2 * nacc * round_up(p.bn, 32) <= 512;
+        if (p.splits == 1 && units >= sms && two_acc && p.k_pad >= 4ll * p.bn &&
+            total < (1ll << 31) - (1ll << 20)) {
+            const long long dp = (units + sms - 1) / sms * nks;
+            const long long L = (total + sms - 1) / sms;
+            if (L >= nks && (dp - L) * 8 >= dp) {
+                const long long grid = (total + L - 1) / L;
+                const long long cols = (long long)nacc * p.bn;
+                // arrival counters, then the partial sums [slot][2][cols][128 pixels]
+                const long long bytes = round_up(grid * 4, 1024) + grid * 2 * cols * 128 * 4;
+                if (bytes <= (256ll << 20)) {
+                    p.sk_len = (int)L;
+                    p.sk_grid = (int)grid;
+                    p.off_sk = take((size_t)bytes);
+                }
+            }
+        }
     }
     p.dev_bytes = off;
     p.dev = nullptr;
@@ -321,7 +347,14 @@ sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt, const int* fil
     if (plan->colkind != SADMM_COL_NONE && plan->n_colgroups > 0 && !col_idx) return SADMM_EINVAL;
     if (device_cc_major() < 10) return SADMM_EUNSUPPORTED;
     plan->dev = dev;
-    return launch_pack(plan, g, W, wdt, filt_idx, col_idx, static_cast<cudaStream_t>(stream));
+    st = launch_pack(plan, g, W, wdt, filt_idx, col_idx, static_cast<cudaStream_t>(stream));
+    if (st != SADMM_OK) return st;
+    // stream-K arrival counters start at zero (each launch leaves them so)
+    if (plan->sk_len > 0 &&
+        cudaMemsetAsync(static_cast<char*>(dev) + plan->off_sk, 0, (size_t)plan->sk_grid * 4,
+                        static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return SADMM_ECUDA;
+    return SADMM_OK;
 }
 
 sadmm_status sadmm_conv_fwd(const sadmm_plan* plan, const void* x, const float* bias, int relu, void* y,

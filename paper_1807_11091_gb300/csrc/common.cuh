@@ -36,6 +36,27 @@ SADMM_DEV unsigned long long globaltimer()
     return t;
 }
 
+// GPU-scope flag operations on global memory (PTX memory model): an acquire
+// load, a relaxed store, and an acquire-release fetch-add.
+SADMM_DEV int ld_acquire_gpu(const int* p)
+{
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+SADMM_DEV void st_relaxed_gpu(int* p, int v)
+{
+    asm volatile("st.relaxed.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+SADMM_DEV int atom_add_acq_rel_gpu(int* p, int v)
+{
+    int old;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+
 SADMM_DEV void raise_status(int* status, int code)
 {
     if (status) atomicCAS(status, 0, code);

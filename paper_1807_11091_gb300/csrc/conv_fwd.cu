@@ -61,6 +61,9 @@ constexpr int kTailOffBias = 0;
 constexpr int kTailCounts = kTailOffBias + 2 * 2 * kTabCap * 4;
 constexpr int kTailBars = kTailCounts + 2 * kMaxGroups * 4;
 constexpr int kTailZero = kTailBars + 512;
+constexpr int kTailCutFlag = kTailBars + 448;  // stream-K flags [piece 0 (run end), piece 1 (run start)][looked, arrived]
+static_assert((3 * kMaxStages + 7) * 8 + 8 <= 448, "barriers, TMEM address and abort flag end below the flags");
+static_assert(448 + 4 * 4 <= 512, "four stream-K flags fit the barrier area");
 constexpr int kSmemTail = kTailZero;
 
 // Division of a non-negative int below 2^31 by an invariant divisor d >= 1:
@@ -123,6 +126,13 @@ struct ConvArgs {
     int tmem_cols;
     int zcap;  // zero-plane offsets per table buffer kept in shared memory
     int relu;
+    // stream-K: CTA b takes stages [b*sk_len, (b+1)*sk_len) of the units'
+    // stages laid end to end; sk_len >= nks, so a unit is cut at most once
+    int sk_len;      // 0: work items are whole units (or K' splits)
+    FastDiv nks_div;
+    int* skcnt;      // arrival counter per cut: cut b-1 lies at the start of CTA b's run
+    float* skpart;   // partial sums [cut][piece 0 | 1][sk_cols][128 pixels]
+    int sk_cols;     // nacc * bn
 };
 
 // Work item w is split sp (stages ks0 .. ks1-1 of K') of unit w / splits; a
@@ -140,6 +150,71 @@ SADMM_DEV void decode_unit(const ConvArgs& a, int w, int& p, int& g, int& mt, in
     const uint32_t gq = fdiv(t, a.mtiles_div);
     mt = (int)(t - gq * a.mtiles_div.d);
     g = (int)gq;
+}
+
+// The work items of this CTA in order: whole units u = blockIdx.x, + grid, ...
+// (K' splits included); or, under stream-K, the pieces of its run of stages
+// [b*sk_len, (b+1)*sk_len): the piece of the unit cut at the run's start, then
+// the piece of the unit cut at its end, then the whole units between them.
+// Both pieces of every cut unit thus come early in their CTAs' runs, so the
+// second to arrive finishes the unit while later units are still being
+// computed, not at the end of the kernel.
+struct Work {
+    int it, end;  // whole units (stream-K: stage bounds of the middle, unit-aligned)
+    int phase;    // stream-K: 0 start piece next, 1 end piece next, 2 whole units
+};
+
+template <bool SK>
+SADMM_DEV Work work_begin(const ConvArgs& a)
+{
+    Work w;
+    if (SK) {
+        const int s0 = blockIdx.x * a.sk_len;
+        const int e0 = min(s0 + a.sk_len, a.units * a.nks);
+        // sk_len >= nks: a run that starts inside a unit goes past that unit's end
+        w.it = ((int)fdiv((uint32_t)(s0 + a.nks - 1), a.nks_div)) * a.nks;
+        const int t0 = (int)fdiv((uint32_t)e0, a.nks_div) * a.nks;
+        w.end = t0 >= w.it ? t0 : e0;
+        w.phase = 0;
+    } else {
+        w.it = blockIdx.x;
+        w.end = a.units;
+        w.phase = 2;
+    }
+    return w;
+}
+
+// Next work item: its unit and stage range ks0 .. ks1-1; false at the end.
+template <bool SK>
+SADMM_DEV bool work_next(const ConvArgs& a, Work& w, int& p, int& g, int& mt, int& sp, int& ks0, int& ks1)
+{
+    if (SK) {
+        int b = 0, e = 0;
+        while (w.phase < 2 && b == e) {
+            const int s0 = blockIdx.x * a.sk_len;
+            if (w.phase++ == 0) {
+                if (s0 < w.it) { b = s0; e = w.it; }  // the run starts inside a unit
+            } else {
+                const int e0 = min(s0 + a.sk_len, a.units * a.nks);
+                if (e0 > w.end) { b = w.end; e = e0; }  // the run ends inside a unit
+            }
+        }
+        if (b == e) {
+            if (w.it >= w.end) return false;
+            b = w.it;
+            e = w.it + a.nks;
+            w.it = e;
+        }
+        const int u = (int)fdiv((uint32_t)b, a.nks_div);
+        decode_unit(a, u, p, g, mt, sp, ks0, ks1);  // one split: sp = 0
+        ks0 = b - u * a.nks;
+        ks1 = ks0 + (e - b);
+        return true;
+    }
+    if (w.it >= w.end) return false;
+    decode_unit(a, w.it, p, g, mt, sp, ks0, ks1);
+    w.it += gridDim.x;
+    return true;
 }
 
 // Tap-validity mask of one output pixel: a bit is set where a tap reads inside
@@ -178,7 +253,49 @@ SADMM_DEV uint32_t ldg_u16_if(const unsigned short* p, uint32_t bits, uint32_t M
     return v;
 }
 
+// Bias, ReLU and the stores of accumulator columns c0 .. c0+kEpiCols-1 of one
+// pixel (columns at or past nrows are skipped): t_off / t_bias give each
+// column's output-plane offset and bias, yf / yh point at the pixel in plane 0.
 template <bool OUT_BF16>
+SADMM_DEV void store_cols(const float (&v)[kEpiCols], int c0, int nrows, const int* t_off, const float* t_bias,
+                          int relu, float* yf, __nv_bfloat16* yh)
+{
+    if (c0 + kEpiCols <= nrows) {
+#pragma unroll
+        for (int j = 0; j < kEpiCols; j += 4) {
+            const int4 o = *reinterpret_cast<const int4*>(t_off + c0 + j);
+            const float4 b = *reinterpret_cast<const float4*>(t_bias + c0 + j);
+            float v0 = v[j] + b.x, v1 = v[j + 1] + b.y, v2 = v[j + 2] + b.z, v3 = v[j + 3] + b.w;
+            if (relu) {
+                v0 = fmaxf(v0, 0.0f); v1 = fmaxf(v1, 0.0f);
+                v2 = fmaxf(v2, 0.0f); v3 = fmaxf(v3, 0.0f);
+            }
+            if (OUT_BF16) {
+                yh[o.x] = __float2bfloat16_rn(v0); yh[o.y] = __float2bfloat16_rn(v1);
+                yh[o.z] = __float2bfloat16_rn(v2); yh[o.w] = __float2bfloat16_rn(v3);
+            } else {
+                __stcs(yf + o.x, v0); __stcs(yf + o.y, v1);
+                __stcs(yf + o.z, v2); __stcs(yf + o.w, v3);
+            }
+        }
+    } else {
+#pragma unroll
+        for (int j = 0; j < kEpiCols; ++j) {
+            if (c0 + j < nrows) {
+                float x = v[j] + t_bias[c0 + j];
+                if (relu) x = fmaxf(x, 0.0f);
+                if (OUT_BF16)
+                    yh[t_off[c0 + j]] = __float2bfloat16_rn(x);
+                else
+                    __stcs(yf + t_off[c0 + j], x);
+            }
+        }
+    }
+}
+
+// SK: stream-K work items (a.sk_len > 0); a separate instantiation keeps the
+// whole-tile loops free of the extra state.
+template <bool OUT_BF16, bool SK>
 __global__ void __launch_bounds__(kThreads, 1)
     k_conv_fwd(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ ConvArgs a)
 {
@@ -196,6 +313,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     float* s_ebias = reinterpret_cast<float*>(tail + kTailOffBias) + 2 * kTabCap;  // [2][kTabCap] biases
     int* s_counts = reinterpret_cast<int*>(tail + kTailCounts);
     int* s_zoff = reinterpret_cast<int*>(tail + kTailZero);  // [2][zcap] zero-plane offsets
+    volatile int* s_cut = reinterpret_cast<volatile int*>(tail + kTailCutFlag);
     uint64_t* bars = reinterpret_cast<uint64_t*>(tail + kTailBars);
     uint64_t* full_a = bars;
     uint64_t* full_b = bars + S;
@@ -251,10 +369,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             long long cur = -1;
             uint32_t e_ph = 0;
             int loads = 0;
-            for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
-                int p, g, sp, ks0, ks1;
-                int mt;
-                decode_unit(a, u, p, g, mt, sp, ks0, ks1);
+            Work wk = work_begin<SK>(a);
+            int p, g, sp, ks0, ks1, mt;
+            while (work_next<SK>(a, wk, p, g, mt, sp, ks0, ks1)) {
                 if (s_counts[2 * g] <= p * a.bn) continue;
                 const long long key = (long long)g * a.upairs + p;
                 if (key == cur) continue;
@@ -280,10 +397,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t issued_parity[kMaxStages];
             uint32_t issued_mask = 0;
             bool ok = true;
-            for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-                int p, g, sp, ks0, ks1;
-                int mt;
-                decode_unit(a, u, p, g, mt, sp, ks0, ks1);
+            Work wk = work_begin<SK>(a);
+            int p, g, sp, ks0, ks1, mt;
+            while (ok && work_next<SK>(a, wk, p, g, mt, sp, ks0, ks1)) {
                 const int nt0 = p * a.nacc;
                 if (s_counts[2 * g] <= nt0 * a.bn) continue;
                 int nbox = 0;  // filter tiles of this unit with kept rows
@@ -321,10 +437,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             long long cur = -1;    // (group, filter tile) of the resident weights
             uint32_t bf_ph = 0;
             const uint32_t sB0 = smem_u32(sB);
-            for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-                int p, g, sp, ks0, ks1;
-                int mt;
-                decode_unit(a, u, p, g, mt, sp, ks0, ks1);
+            Work wk = work_begin<SK>(a);
+            int p, g, sp, ks0, ks1, mt;
+            while (ok && work_next<SK>(a, wk, p, g, mt, sp, ks0, ks1)) {
                 const int cnt = s_counts[2 * g] - p * a.nacc * a.bn;  // kept rows from the unit's first tile
                 if (cnt <= 0) continue;
                 if (a.b_res) {
@@ -403,10 +518,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         // After a failed wait (another role aborted) the warp keeps walking the
         // units, without TMEM or stores, so the named barrier stays balanced.
         bool alive = true;
-        for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
-            int p, g, sp, ks0, ks1;
-            int mt;
-            decode_unit(a, u, p, g, mt, sp, ks0, ks1);
+        Work wk = work_begin<SK>(a);
+        int p, g, sp, ks0, ks1, mt;
+        while (work_next<SK>(a, wk, p, g, mt, sp, ks0, ks1)) {
             const int nt0 = p * a.nacc;
             const int cnt = s_counts[2 * g] - nt0 * a.bn;  // kept rows from the unit's first tile
             const int zc = (p == 0) ? s_counts[2 * g + 1] : 0;  // pruned filters whose planes this unit zeroes
@@ -433,90 +547,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             const int* u_off = s_eoff + ub * kTabCap;
             const float* u_bias = s_ebias + ub * kTabCap;
+            // stream-K: a unit cut at the start of CTA b's run has piece 0 (its
+            // first stages) in CTA b-1 and piece 1 in CTA b, and cut index b-1
+            const bool cut = SK && (ks0 > 0 || ks1 < a.nks);
+            const int piece = ks0 > 0 ? 1 : 0;
+            const int cut_idx = (int)blockIdx.x - piece;
             const int m = mt * kBM + row;
             const bool valid = m < a.M;
             const long long n_img = valid ? (long long)fdiv((uint32_t)m, a.plane_div) : 0;
             const long long pix = valid ? m - n_img * a.plane : 0;
             float* yf = reinterpret_cast<float*>(a.y) + (n_img * (long long)a.F * a.plane + pix);
             __nv_bfloat16* yh = reinterpret_cast<__nv_bfloat16*>(a.y) + (n_img * (long long)a.F * a.plane + pix);
-            int chunks = 0;  // accumulator chunks of this unit, over all its tiles
-            // warp-uniform outcome: the TMEM loads below are .sync.aligned
-            if (cnt > 0 && alive && !__all_sync(0xffffffffu, mbar_wait(&acc_full[ab], acc_ph, abort_flag, a.status)))
-                alive = false;
-            if (cnt > 0 && alive) {
-                tc_fence_after();
-                for (int ti = 0; ti < a.nacc && nt0 + ti < a.n_tiles; ++ti) {
-                    const int nrows = min(a.bn, cnt - ti * a.bn);
-                    if (nrows <= 0) break;
-                    const int nch = (nrows + kEpiCols - 1) / kEpiCols;
-                    const uint32_t taddr = tmem_base + (uint32_t)((ab * a.nacc + ti) * a.tmem_stride) +
-                                           ((uint32_t)(q * 32) << 16);
-                    const int* t_off = u_off + ti * a.bn;
-                    const float* t_bias = u_bias + ti * a.bn;
-                    // chunk k of this tile is the unit's chunk chunks + k; warp h takes those = h mod kHalves
-                    for (int k = (h - chunks % kHalves + kHalves) % kHalves; k < nch; k += kHalves) {
-                        const int c0 = k * kEpiCols;
-                        uint32_t r[kEpiCols];
-                        tmem_ld_32x32b_x16(taddr + (uint32_t)c0, r);
-                        tmem_ld_wait();
-                        if (valid && a.splits > 1) {
-                            // split K': raw fp32 partial sums, [split][column][pixel]
-                            float* pp = a.partial +
-                                        ((size_t)sp * a.ncols_all + (size_t)g * a.n_pad + (size_t)(nt0 + ti) * a.bn + c0) *
-                                            a.m_pad +
-                                        m;
-#pragma unroll
-                            for (int j = 0; j < kEpiCols; ++j)
-                                if (c0 + j < nrows) __stcs(pp + (size_t)j * a.m_pad, __uint_as_float(r[j]));
-                        } else if (valid) {
-                            if (c0 + kEpiCols <= nrows) {
-#pragma unroll
-                                for (int j = 0; j < kEpiCols; j += 4) {
-                                    const int4 o = *reinterpret_cast<const int4*>(t_off + c0 + j);
-                                    const float4 b = *reinterpret_cast<const float4*>(t_bias + c0 + j);
-                                    float v0 = __uint_as_float(r[j]) + b.x, v1 = __uint_as_float(r[j + 1]) + b.y;
-                                    float v2 = __uint_as_float(r[j + 2]) + b.z, v3 = __uint_as_float(r[j + 3]) + b.w;
-                                    if (a.relu) {
-                                        v0 = fmaxf(v0, 0.0f); v1 = fmaxf(v1, 0.0f);
-                                        v2 = fmaxf(v2, 0.0f); v3 = fmaxf(v3, 0.0f);
-                                    }
-                                    if (OUT_BF16) {
-                                        yh[o.x] = __float2bfloat16_rn(v0); yh[o.y] = __float2bfloat16_rn(v1);
-                                        yh[o.z] = __float2bfloat16_rn(v2); yh[o.w] = __float2bfloat16_rn(v3);
-                                    } else {
-                                        __stcs(yf + o.x, v0); __stcs(yf + o.y, v1);
-                                        __stcs(yf + o.z, v2); __stcs(yf + o.w, v3);
-                                    }
-                                }
-                            } else {
-#pragma unroll
-                                for (int j = 0; j < kEpiCols; ++j) {
-                                    if (c0 + j < nrows) {
-                                        float v = __uint_as_float(r[j]) + t_bias[c0 + j];
-                                        if (a.relu) v = fmaxf(v, 0.0f);
-                                        if (OUT_BF16)
-                                            yh[t_off[c0 + j]] = __float2bfloat16_rn(v);
-                                        else
-                                            __stcs(yf + t_off[c0 + j], v);
-                                    }
-                                }
-                            }
-                        }
-                    }
-                    chunks += nch;
-                }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&acc_empty[ab]);
-                if (++ab == a.acc_bufs) { ab = 0; acc_ph ^= 1u; }
-            }
-            if (zc > 0 && valid && alive && a.splits == 1) {
-                // pruned filters of this conv group: their planes are zero.
-                // Chunks of 16 planes continue the unit's chunk sequence.
+            int chunks = 0;  // chunks of this unit so far (zero planes, then accumulator columns)
+            if (zc > 0 && alive && a.splits == 1 && ks0 == 0) {
+                // Pruned filters of this conv group: their planes are zero.  They
+                // need no accumulator, so they go out while the unit's MMAs run;
+                // these chunks of 16 planes start the unit's chunk sequence
+                // (warp-uniform: it decides which warp reads which TMEM chunk).
                 const int* zmap = a.zeromap + (long long)g * a.Fg;
                 const int* u_zero = s_zoff + ub * a.zcap;
                 const int nzc = (zc + kEpiCols - 1) / kEpiCols;
-                for (int k = (h - chunks % kHalves + kHalves) % kHalves; k < nzc; k += kHalves) {
+                for (int k = h; valid && k < nzc; k += kHalves) {
                     const int z0 = k * kEpiCols;
                     if (z0 + kEpiCols <= a.zcap && z0 + kEpiCols <= zc) {
 #pragma unroll
@@ -540,6 +591,121 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                     }
                 }
+                chunks = nzc;
+            }
+            // warp-uniform outcome: the TMEM loads below are .sync.aligned
+            if (cnt > 0 && alive && !__all_sync(0xffffffffu, mbar_wait(&acc_full[ab], acc_ph, abort_flag, a.status)))
+                alive = false;
+            // Stream-K piece of a cut unit.  If the unit's other piece has
+            // arrived already, this one finishes the unit: its accumulator plus
+            // the other's fp32 partial sums, then bias, ReLU, stores (mode 2).
+            // Otherwise it writes its own partial sums and arrives (mode 1);
+            // should the other piece have arrived meanwhile, it finishes after
+            // all.  The two-term fp32 sum is the same whichever piece adds it.
+            int cut_mode = 0;
+            volatile int* cf = s_cut + 2 * piece;  // [looked, arrived]: one pair per head / tail piece of the CTA
+            const float* other = nullptr;
+            if (cut && cnt > 0) {
+                if (et == 0) {
+                    const int seen = alive ? ld_acquire_gpu(a.skcnt + cut_idx) : 0;
+                    if (seen) st_relaxed_gpu(a.skcnt + cut_idx, 0);  // zero again for the next launch
+                    cf[0] = seen;
+                }
+                asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+                cut_mode = cf[0] ? 2 : 1;
+                other = a.skpart + (size_t)(cut_idx * 2 + 1 - piece) * a.sk_cols * kBM + row;
+            }
+            if (cnt > 0 && alive) {
+                tc_fence_after();
+                for (int ti = 0; ti < a.nacc && nt0 + ti < a.n_tiles; ++ti) {
+                    const int nrows = min(a.bn, cnt - ti * a.bn);
+                    if (nrows <= 0) break;
+                    const int nch = (nrows + kEpiCols - 1) / kEpiCols;
+                    const uint32_t taddr = tmem_base + (uint32_t)((ab * a.nacc + ti) * a.tmem_stride) +
+                                           ((uint32_t)(q * 32) << 16);
+                    const int* t_off = u_off + ti * a.bn;
+                    const float* t_bias = u_bias + ti * a.bn;
+                    // chunk k of this tile is the unit's chunk chunks + k; warp h takes those = h mod kHalves
+                    for (int k = (h - chunks % kHalves + kHalves) % kHalves; k < nch; k += kHalves) {
+                        const int c0 = k * kEpiCols;
+                        uint32_t r[kEpiCols];
+                        tmem_ld_32x32b_x16(taddr + (uint32_t)c0, r);
+                        tmem_ld_wait();
+                        const size_t col0 = ((size_t)ti * a.bn + c0) * kBM;  // partial-sum offset of the chunk
+                        if (cut_mode == 1) {
+                            // this piece's raw fp32 partial sums, every lane (pixel) of the tile
+                            float* pp = a.skpart + (size_t)(cut_idx * 2 + piece) * a.sk_cols * kBM + row + col0;
+#pragma unroll
+                            for (int j = 0; j < kEpiCols; ++j) __stcg(pp + (size_t)j * kBM, __uint_as_float(r[j]));
+                        } else if (cut_mode == 2) {
+                            float v[kEpiCols];
+#pragma unroll
+                            for (int j = 0; j < kEpiCols; ++j)
+                                v[j] = __uint_as_float(r[j]) + __ldcg(other + col0 + (size_t)j * kBM);
+                            if (valid) store_cols<OUT_BF16>(v, c0, nrows, t_off, t_bias, a.relu, yf, yh);
+                        } else if (valid && a.splits > 1) {
+                            // split K': raw fp32 partial sums, [split][column][pixel]
+                            float* pp = a.partial +
+                                        ((size_t)sp * a.ncols_all + (size_t)g * a.n_pad + (size_t)(nt0 + ti) * a.bn + c0) *
+                                            a.m_pad +
+                                        m;
+#pragma unroll
+                            for (int j = 0; j < kEpiCols; ++j)
+                                if (c0 + j < nrows) __stcs(pp + (size_t)j * a.m_pad, __uint_as_float(r[j]));
+                        } else if (valid) {
+                            float v[kEpiCols];
+#pragma unroll
+                            for (int j = 0; j < kEpiCols; ++j) v[j] = __uint_as_float(r[j]);
+                            store_cols<OUT_BF16>(v, c0, nrows, t_off, t_bias, a.relu, yf, yh);
+                        }
+                    }
+                    chunks += nch;
+                }
+            }
+            if (cut_mode == 1) {
+                // every partial store of this CTA's epilogue precedes the arrival
+                asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+                if (et == 0) {
+                    int last = 0;
+                    if (alive) {
+                        last = atom_add_acq_rel_gpu(a.skcnt + cut_idx, 1) == 1;
+                        if (last) st_relaxed_gpu(a.skcnt + cut_idx, 0);
+                    }
+                    cf[1] = last;
+                }
+                asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+                if (cf[1] && alive) {
+                    // the other piece arrived first after all: finish from TMEM
+                    int ch = 0;
+                    for (int ti = 0; ti < a.nacc && nt0 + ti < a.n_tiles; ++ti) {
+                        const int nrows = min(a.bn, cnt - ti * a.bn);
+                        if (nrows <= 0) break;
+                        const int nch = (nrows + kEpiCols - 1) / kEpiCols;
+                        const uint32_t taddr = tmem_base + (uint32_t)((ab * a.nacc + ti) * a.tmem_stride) +
+                                               ((uint32_t)(q * 32) << 16);
+                        const int* t_off = u_off + ti * a.bn;
+                        const float* t_bias = u_bias + ti * a.bn;
+                        for (int k = (h - ch % kHalves + kHalves) % kHalves; k < nch; k += kHalves) {
+                            const int c0 = k * kEpiCols;
+                            uint32_t r[kEpiCols];
+                            tmem_ld_32x32b_x16(taddr + (uint32_t)c0, r);
+                            tmem_ld_wait();
+                            const size_t col0 = ((size_t)ti * a.bn + c0) * kBM;
+                            float v[kEpiCols];
+#pragma unroll
+                            for (int j = 0; j < kEpiCols; ++j)
+                                v[j] = __uint_as_float(r[j]) + __ldcg(other + col0 + (size_t)j * kBM);
+                            if (valid) store_cols<OUT_BF16>(v, c0, nrows, t_off, t_bias, a.relu, yf, yh);
+                        }
+                        ch += nch;
+                    }
+                }
+            }
+            if (cnt > 0 && alive) {
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&acc_empty[ab]);
+                if (++ab == a.acc_bufs) { ab = 0; acc_ph ^= 1u; }
             }
         }
     } else if (warp >= 4 + kEpiWarps) {
@@ -554,19 +720,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t ph = 0;
         int turn = 0;  // running stage index modulo kGatherSets
         bool ok = true;
-        for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-            int p, g, sp, ks0, ks1;
-            int mt;
-            decode_unit(a, u, p, g, mt, sp, ks0, ks1);
+        Work wk = work_begin<SK>(a);
+        int p, g, sp, ks0, ks1, mt;
+        while (ok && work_next<SK>(a, wk, p, g, mt, sp, ks0, ks1)) {
             if (s_counts[2 * g] <= p * a.nacc * a.bn) continue;
             const int m = mt * kBM + prow;
             uint32_t M = 0;
             const unsigned short* xb = xs;
             if (m < a.M) {
                 const long long n_img = fdiv((uint32_t)m, a.plane_div);
-                const int p = (int)(m - n_img * a.plane);
-                const int ot = (int)fdiv((uint32_t)p, a.ohw_div);
-                const int r2 = p - ot * a.OHW;
+                const int pix = (int)(m - n_img * a.plane);
+                const int ot = (int)fdiv((uint32_t)pix, a.ohw_div);
+                const int r2 = pix - ot * a.OHW;
                 const int oh = (int)fdiv((uint32_t)r2, a.ow_div);
                 const int ow = r2 - oh * a.OW;
                 const int it0 = ot * a.st - a.pt, ih0 = oh * a.sh - a.ph, iw0 = ow * a.sw - a.pw;
@@ -678,10 +843,10 @@ __global__ void __launch_bounds__(256) k_splitk_finalize(const ConvArgs a)
     }
 }
 
-template <bool OUT_BF16>
+template <bool OUT_BF16, bool SK>
 cudaError_t launch(const CUtensorMap& map, const ConvArgs& a, int grid, size_t smem, cudaStream_t s)
 {
-    auto kern = k_conv_fwd<OUT_BF16>;
+    auto kern = k_conv_fwd<OUT_BF16, SK>;
     static int configured_dev = -1;
     int dev = 0;
     cudaGetDevice(&dev);
@@ -816,11 +981,32 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     long long grid = device_sm_count();
     if (grid > a.units) grid = a.units;
     if (grid < 1) grid = 1;
+    if (plan->sk_len > 0) {
+        // stream-K: the plan's run length and CTA count must tile the stages
+        // with every unit cut at most once
+        const long long total = units * a.nks;
+        const long long L = plan->sk_len;
+        if (a.splits > 1 || L < a.nks || total >= (1ll << 31) - (1ll << 20) || plan->sk_grid != (total + L - 1) / L ||
+            a.acc_bufs != 2)
+            return SADMM_EINVAL;
+        a.sk_len = (int)L;
+        a.nks_div = make_fastdiv((uint32_t)a.nks);
+        a.sk_cols = a.nacc * plan->bn;
+        a.skcnt = reinterpret_cast<int*>(const_cast<char*>(base) + plan->off_sk);
+        a.skpart = reinterpret_cast<float*>(const_cast<char*>(base) + plan->off_sk +
+                                            round_up((long long)plan->sk_grid * 4, 1024));
+        grid = plan->sk_grid;
+    }
 
     CUtensorMap map;
     memcpy(&map, plan->tmap, sizeof(map));
-    const cudaError_t e = (ydt == SADMM_BF16) ? launch<true>(map, a, (int)grid, smem, s)
-                                              : launch<false>(map, a, (int)grid, smem, s);
+    cudaError_t e;
+    if (a.sk_len > 0)
+        e = (ydt == SADMM_BF16) ? launch<true, true>(map, a, (int)grid, smem, s)
+                                : launch<false, true>(map, a, (int)grid, smem, s);
+    else
+        e = (ydt == SADMM_BF16) ? launch<true, false>(map, a, (int)grid, smem, s)
+                                : launch<false, false>(map, a, (int)grid, smem, s);
     return e == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
 }
 

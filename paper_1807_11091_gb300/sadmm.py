@@ -57,6 +57,9 @@ class Plan(ctypes.Structure):
         ("off_partial", ctypes.c_size_t),
         ("splits", ctypes.c_int),
         ("stages_per_split", ctypes.c_int),
+        ("off_sk", ctypes.c_size_t),
+        ("sk_len", ctypes.c_int),
+        ("sk_grid", ctypes.c_int),
         ("tmap", ctypes.c_uint64 * 16),
     ]
 
