@@ -42,7 +42,7 @@
 extern "C" {
 #endif
 
-#define SADMM_ABI_VERSION 3
+#define SADMM_ABI_VERSION 4
 
 /* Bytes of the fixed device array of sadmm_project_groups_noalloc. */
 #define SADMM_NOALLOC_SCRATCH_BYTES (256 * 1024)
@@ -98,6 +98,7 @@ typedef struct {
     size_t off_sk;      /* stream-K partial sums and arrival counters (sk_len > 0) */
     int sk_len;         /* stream-K: 64-column stages per CTA (0: whole tiles)  */
     int sk_grid;        /* stream-K: CTAs launched                              */
+    int ctas;           /* CTAs a forward launches at most (one per SM)         */
     uint64_t tmap[16];/* 128-byte TMA tensor map of the packed matrix         */
 } sadmm_plan;
 
@@ -139,7 +140,8 @@ size_t sadmm_workspace_size(const sadmm_conv_desc* d, int colkind);
  * the order of equal-key groups is resolved by index, so the index lists are
  * deterministic.  Grouped convs: a filter group is one filter among all F; a
  * column group spans all F filters (the same column set serves every conv
- * group).
+ * group).  A kind kept whole (k_filters = F, or k_cols = G) with keys_out
+ * NULL skips its keys: its list is 0..F-1 (0..G-1), exactly the top-k.
  */
 sadmm_status sadmm_project_groups(const sadmm_conv_desc* d, const void* W, const void* U,
                                   int wdt, int k_filters, int colkind, int k_cols,
@@ -236,6 +238,17 @@ sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d,
                              int n_filt, int colkind, int n_colgroups);
 
 /*
+ * sadmm_plan_init for a forward that may occupy at most `max_ctas` SMs
+ * (0 or above the SM count: all of them).  The conv kernel keeps one CTA per
+ * SM for its whole run, so nothing else runs beside it; a cap leaves
+ * SM count - max_ctas SMs to work on other streams (the next layers'
+ * projection and pack, say).  The split-K and stream-K choices, and so the
+ * plan's device bytes, follow the cap.  Results do not depend on it.
+ */
+sadmm_status sadmm_plan_init_ctas(sadmm_plan* plan, const sadmm_conv_desc* d,
+                                  int n_filt, int colkind, int n_colgroups, int max_ctas);
+
+/*
  * Compacts the kept weights (Sec. 3, row/column pruning of the GEMM matrix):
  *   Wp[g][i][j] = bf16(W[f_i][col_j]) for the i-th kept filter f_i of conv
  *   group g and the j-th kept column, zero beyond the kept counts;
@@ -269,7 +282,9 @@ sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt,
  *   y     device [N][F][OT][OH][OW] of dtype `ydt` (fp32 or bf16, rounded
  *         to nearest even); every element is written.
  * Requires sm_100-family tensor cores (SADMM_EUNSUPPORTED otherwise) and
- * N*C*T*H*W < 2^31.
+ * N*C*T*H*W < 2^31.  Launches that use one plan must not overlap on the GPU
+ * (stream-ordered is fine): split-K partial sums and stream-K arrival
+ * counters live in the plan's buffer.
  */
 sadmm_status sadmm_conv_fwd(const sadmm_plan* plan, const void* x, const float* bias,
                             int relu, void* y, int ydt, void* stream);

@@ -230,7 +230,13 @@ sadmm_status sadmm_admm_update_elements(const sadmm_conv_desc* d, const void* W,
 sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d, int n_filt, int colkind,
                              int n_colgroups)
 {
-    if (!plan) return SADMM_EINVAL;
+    return sadmm_plan_init_ctas(plan, d, n_filt, colkind, n_colgroups, 0);
+}
+
+sadmm_status sadmm_plan_init_ctas(sadmm_plan* plan, const sadmm_conv_desc* d, int n_filt, int colkind,
+                                  int n_colgroups, int max_ctas)
+{
+    if (!plan || max_ctas < 0) return SADMM_EINVAL;
     Geometry g;
     sadmm_status st = check_desc(d, &g);
     if (st != SADMM_OK) return st;
@@ -252,6 +258,8 @@ sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d, int n_f
     sadmm_plan p;
     memset(&p, 0, sizeof(p));
     p.desc = *d;
+    p.ctas = device_sm_count();  // CTAs a forward launches at most (one per SM)
+    if (max_ctas > 0 && max_ctas < p.ctas) p.ctas = max_ctas;
     p.n_filt = n_filt;
     p.colkind = colkind;
     p.n_colgroups = n_colgroups;
@@ -286,7 +294,7 @@ sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d, int n_f
         const long long m_tiles = (g.m + 127) / 128;
         const long long upairs = (p.n_tiles + (p.n_tiles >= 2 ? 1 : 0)) / (p.n_tiles >= 2 ? 2 : 1);
         const long long units = m_tiles * g.groups * upairs;
-        const long long sms = device_sm_count();
+        const long long sms = p.ctas;
         const long long rows = g.groups * p.n_pad + g.groups * g.fg;  // finalize rows
         if (units < sms && nks >= 2 && rows <= 65535) {
             long long want = (sms + units - 1) / units;

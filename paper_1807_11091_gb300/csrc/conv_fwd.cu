@@ -978,7 +978,7 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     const size_t smem =
         1024 + (size_t)fixed_bytes + (size_t)a.stages * stage_bytes + table_bytes + kSmemTail + (size_t)a.zcap * 8;
 
-    long long grid = device_sm_count();
+    long long grid = plan->ctas > 0 ? plan->ctas : device_sm_count();
     if (grid > a.units) grid = a.units;
     if (grid < 1) grid = 1;
     if (plan->sk_len > 0) {

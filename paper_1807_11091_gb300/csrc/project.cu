@@ -262,6 +262,22 @@ int column_parts(long long K, long long nrows)
     return (int)std::max(r, 1ll);
 }
 
+// Index lists 0..n-1 and keep flags of one for the kinds kept whole (a null
+// list is skipped).
+__global__ void __launch_bounds__(256) k_keep_all(int* idx_a, int na, uint8_t* keep_a, int* idx_b, int nb,
+                                                  uint8_t* keep_b)
+{
+    const int i = blockIdx.x * 256 + threadIdx.x;
+    if (idx_a && i < na) {
+        idx_a[i] = i;
+        if (keep_a) keep_a[i] = 1;
+    }
+    if (idx_b && i < nb) {
+        idx_b[i] = i;
+        if (keep_b) keep_b[i] = 1;
+    }
+}
+
 template <typename T>
 sadmm_status run_project(const Geometry& g, const T* W, const T* U, int k_filters, int colkind, int k_cols,
                          int* filt_idx, int* col_idx, double* keys_out, void* ws, uint8_t* rkeep, uint8_t* ckeep,
@@ -272,16 +288,28 @@ sadmm_status run_project(const Geometry& g, const T* W, const T* U, int k_filter
     double* ckeys = fkeys + round_up(F, 32);                   // column keys
     double* parts = ckeys + round_up(K, 32);                   // [R][K] partial column keys
 
-    k_filter_keys<T><<<F, 256, 0, s>>>(W, U, F, K, fkeys);
-    launch_select(fkeys, F, 1, k_filters, 1, 0, fkeys, keys_out, filt_idx, rkeep, s);
-    if (colkind != SADMM_COL_NONE) {
+    // Keeping every group of a kind needs no keys: the top-G of G keys is the
+    // whole ascending index list.  Unless the caller asked for the keys, such
+    // lists (and keep flags) are written directly, in one launch for both kinds.
+    const int taps = (colkind == SADMM_COL_CHANNEL) ? (int)g.taps : 1;
+    const int G = (colkind == SADMM_COL_CHANNEL) ? (int)g.cg : K;
+    const bool rows_all = (k_filters == F) && !keys_out;
+    const bool cols_all = (colkind != SADMM_COL_NONE) && (k_cols == G) && !keys_out;
+    if (rows_all || cols_all) {
+        const int n = (rows_all ? F : 0) > (cols_all ? G : 0) ? F : (cols_all ? G : 0);
+        k_keep_all<<<(n + 255) / 256, 256, 0, s>>>(rows_all ? filt_idx : nullptr, F, rows_all ? rkeep : nullptr,
+                                                   cols_all ? col_idx : nullptr, G, cols_all ? ckeep : nullptr);
+    }
+    if (!rows_all) {
+        k_filter_keys<T><<<F, 256, 0, s>>>(W, U, F, K, fkeys);
+        launch_select(fkeys, F, 1, k_filters, 1, 0, fkeys, keys_out, filt_idx, rkeep, s);
+    }
+    if (colkind != SADMM_COL_NONE && !cols_all) {
         const bool all_rows = (k_filters == F);
         const int nrows = all_rows ? F : k_filters;
         const int R = column_parts(K, nrows);
         k_column_keys<T><<<dim3((K + 31) / 32, R), 256, 0, s>>>(W, U, K, all_rows ? nullptr : filt_idx, nrows,
                                                                 parts);
-        const int taps = (colkind == SADMM_COL_CHANNEL) ? (int)g.taps : 1;
-        const int G = (colkind == SADMM_COL_CHANNEL) ? (int)g.cg : K;
         launch_select(parts, G, taps, k_cols, R, K, ckeys, keys_out ? keys_out + F : nullptr, col_idx, ckeep, s);
     }
     return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;

@@ -60,6 +60,7 @@ class Plan(ctypes.Structure):
         ("off_sk", ctypes.c_size_t),
         ("sk_len", ctypes.c_int),
         ("sk_grid", ctypes.c_int),
+        ("ctas", ctypes.c_int),
         ("tmap", ctypes.c_uint64 * 16),
     ]
 
@@ -92,6 +93,8 @@ def load():
     lib.sadmm_project_groups.argtypes = [P(ConvDesc), vp, vp, ci, ci, ci, ci, vp, vp, vp, vp, sz, vp]
     lib.sadmm_plan_init.restype = ci
     lib.sadmm_plan_init.argtypes = [P(Plan), P(ConvDesc), ci, ci, ci]
+    lib.sadmm_plan_init_ctas.restype = ci
+    lib.sadmm_plan_init_ctas.argtypes = [P(Plan), P(ConvDesc), ci, ci, ci, ci]
     lib.sadmm_pack.restype = ci
     lib.sadmm_pack.argtypes = [P(Plan), vp, ci, vp, vp, vp, sz, vp]
     lib.sadmm_conv_fwd.restype = ci
@@ -208,6 +211,14 @@ def sadmm_plan_init(desc: ConvDesc, n_filt: int, colkind: int, n_colgroups: int)
     plan = Plan()
     st = load().sadmm_plan_init(ctypes.byref(plan), ctypes.byref(desc), int(n_filt), int(colkind),
                                 int(n_colgroups))
+    return st, plan
+
+
+def sadmm_plan_init_ctas(desc: ConvDesc, n_filt: int, colkind: int, n_colgroups: int,
+                         max_ctas: int) -> Tuple[int, Plan]:
+    plan = Plan()
+    st = load().sadmm_plan_init_ctas(ctypes.byref(plan), ctypes.byref(desc), int(n_filt), int(colkind),
+                                     int(n_colgroups), int(max_ctas))
     return st, plan
 
 
@@ -356,12 +367,12 @@ class PrunedConv:
     """A packed pruned layer: plan plus its device buffer (sadmm_plan_init + sadmm_pack)."""
 
     def __init__(self, desc16: Sequence[int], W, filt_idx, colkind: int, col_idx, n_filt: int,
-                 n_colgroups: int, stream=None):
+                 n_colgroups: int, stream=None, max_ctas: int = 0):
         torch = _torch()
         self.desc16 = [int(v) for v in desc16]
         desc = make_desc(self.desc16)
-        st, plan = sadmm_plan_init(desc, n_filt, colkind, n_colgroups)
-        _check(st, "sadmm_plan_init")
+        st, plan = sadmm_plan_init_ctas(desc, n_filt, colkind, n_colgroups, max_ctas)
+        _check(st, "sadmm_plan_init_ctas")
         self.plan = plan
         self.buf = torch.empty(plan.dev_bytes, dtype=torch.uint8, device=W.device)
         self.W = W

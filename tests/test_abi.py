@@ -33,7 +33,7 @@ def test_library_exports_every_declared_entry_point():
 
 
 def test_struct_layout_and_version():
-    assert sadmm.sadmm_abi_version() == 3
+    assert sadmm.sadmm_abi_version() == 4
     assert sadmm.sadmm_plan_struct_size() == ctypes.sizeof(sadmm.Plan)
     assert sadmm.sadmm_status_string(-1) == "invalid argument"
 
@@ -128,3 +128,20 @@ def test_elements_reject_bad_arguments_on_host():
     Z = fake + (1 << 22)
     assert sadmm.sadmm_admm_update_elements(d, fake, fake, Z, sadmm.SADMM_FP32, 5, ws_ptr, ws, None) == sadmm.SADMM_EINVAL
     assert sadmm.sadmm_admm_update_elements(d, fake, None, Z, sadmm.SADMM_FP32, 5, ws_ptr, ws, None) == sadmm.SADMM_EINVAL
+
+
+def test_plan_cta_cap_on_host():
+    """sadmm_plan_init_ctas records the cap, ignores 0 and caps above the SM
+    count, rejects a negative cap, and sizes split-K for the capped count."""
+    L = wl.alexnet()[2]
+    d = sadmm.make_desc(L.shape.with_batch(1).desc16())
+    st, full = sadmm.sadmm_plan_init(d, L.k_filters, L.colkind, L.k_cols)
+    assert st == 0 and full.ctas >= 1
+    st, same = sadmm.sadmm_plan_init_ctas(d, L.k_filters, L.colkind, L.k_cols, 0)
+    assert st == 0 and same.ctas == full.ctas and same.dev_bytes == full.dev_bytes
+    st, big = sadmm.sadmm_plan_init_ctas(d, L.k_filters, L.colkind, L.k_cols, 1 << 20)
+    assert st == 0 and big.ctas == full.ctas
+    st, capped = sadmm.sadmm_plan_init_ctas(d, L.k_filters, L.colkind, L.k_cols, 1)
+    assert st == 0 and capped.ctas == 1 and capped.splits == 1 and capped.sk_len == 0
+    st, _ = sadmm.sadmm_plan_init_ctas(d, L.k_filters, L.colkind, L.k_cols, -1)
+    assert st == sadmm.SADMM_EINVAL

@@ -43,6 +43,25 @@ def test_tiny_all_k(si, ck):
             _check(s, t["W"], kf, ck, kc if ck != wl.COL_NONE else 0)
 
 
+@pytest.mark.parametrize("si", range(len(TINY)))
+@pytest.mark.parametrize("ck", [wl.COL_NONE, wl.COL_SHAPE, wl.COL_CHANNEL])
+def test_tiny_all_k_without_keys(si, ck):
+    """No keys requested: a kind kept whole skips its keys and select (its list
+    is 0..G-1); the lists must equal the oracle's for every mix of kept counts."""
+    s = TINY[si]
+    t = wl.gen_tensors(s, seed=60 + si)
+    G = s.k if ck == wl.COL_SHAPE else s.cg
+    for kf in sorted({0, 1, s.f // 2, s.f}):
+        for kc in sorted({0, 1, G // 3, G}):
+            kc = kc if ck != wl.COL_NONE else 0
+            fi, ci, keys = gpu_project(s, t["W"].cuda(), kf, ck, kc, with_keys=False)
+            rows, cols, _, _ = oracle.project(t["W"], s.taps, kf, ck, kc)
+            assert keys is None
+            assert np.array_equal(fi, rows), (kf, kc)
+            if ck != wl.COL_NONE:
+                assert np.array_equal(ci, cols), (kf, kc)
+
+
 def test_dual_and_fp32_weights():
     s = TINY[3]
     t = wl.gen_tensors(s, seed=3)
