@@ -47,6 +47,7 @@ __global__ void __launch_bounds__(kApplyThreads) k_admm_apply(const T* __restric
                                                               const uint8_t* __restrict__ ckeep, uint32_t tmul,
                                                               uint32_t tshift)
 {
+    pdl_wait();  // after the kernel before it in the stream
     const int a = blockIdx.y;
     const bool rk = rkeep[a] != 0;
     const long long base = (long long)a * K;
@@ -100,12 +101,13 @@ sadmm_status launch_admm_update(const Geometry& g, const void* W, void* U, void*
     const uint8_t* ck = (colkind == SADMM_COL_NONE) ? nullptr : ckeep;
     const dim3 grid((unsigned)((K + kApplyThreads * kApplyCols - 1) / (kApplyThreads * kApplyCols)), (unsigned)F);
     if (wdt == SADMM_BF16)
-        k_admm_apply<__nv_bfloat16><<<grid, kApplyThreads, 0, s>>>(
-            static_cast<const __nv_bfloat16*>(W), static_cast<__nv_bfloat16*>(U), static_cast<__nv_bfloat16*>(Z),
-            K, rkeep, ck, mul, sh);
+        launch_pdl(k_admm_apply<__nv_bfloat16>, grid, dim3(kApplyThreads), 0, s,
+                   static_cast<const __nv_bfloat16*>(W), static_cast<__nv_bfloat16*>(U),
+                   static_cast<__nv_bfloat16*>(Z), K, static_cast<const uint8_t*>(rkeep), ck, mul, sh);
     else
-        k_admm_apply<float><<<grid, kApplyThreads, 0, s>>>(static_cast<const float*>(W), static_cast<float*>(U),
-                                                           static_cast<float*>(Z), K, rkeep, ck, mul, sh);
+        launch_pdl(k_admm_apply<float>, grid, dim3(kApplyThreads), 0, s, static_cast<const float*>(W),
+                   static_cast<float*>(U), static_cast<float*>(Z), K, static_cast<const uint8_t*>(rkeep), ck, mul,
+                   sh);
     return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
 }
 

@@ -57,6 +57,34 @@ SADMM_DEV int atom_add_acq_rel_gpu(int* p, int v)
     return old;
 }
 
+// Programmatic dependent launch (kernels launched with the programmatic stream
+// serialization attribute): a kernel may start while the previous kernel of
+// its stream is still running; pdl_wait() blocks until that kernel has
+// completed and its memory is visible, so it comes before the first read of
+// anything an earlier kernel wrote.  pdl_trigger() lets the next kernel of the
+// stream be scheduled once every CTA of this one has issued it (or exited).
+SADMM_DEV void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+SADMM_DEV void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// Host: launch `kern` with programmatic stream serialization (the kernel calls
+// pdl_wait() before its first global-memory read).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              Args... args)
+{
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 SADMM_DEV void raise_status(int* status, int code)
 {
     if (status) atomicCAS(status, 0, code);

@@ -344,6 +344,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         *abort_flag = 0;
         fence_mbar_init();
     }
+    if (warp == 1) {
+        tmem_alloc(tmem_holder, (uint32_t)a.tmem_cols);
+        tmem_relinquish();
+    }
+    // Nothing above reads global memory: it overlaps the previous kernel's tail.
+    pdl_wait();
+    pdl_trigger();
     for (int i = threadIdx.x; i < 2 * a.groups; i += blockDim.x) s_counts[i] = a.counts[i];
     {
         // the gather table is the same for every tile: keep it in shared memory
@@ -352,10 +359,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = threadIdx.x; i < a.k_pad / 2; i += blockDim.x) dst[i] = __ldg(src + i);
     }
     if (warp == 0 && lane == 0) tma_prefetch_desc(&tmap);
-    if (warp == 1) {
-        tmem_alloc(tmem_holder, (uint32_t)a.tmem_cols);
-        tmem_relinquish();
-    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -808,6 +811,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 template <bool OUT_BF16>
 __global__ void __launch_bounds__(256) k_splitk_finalize(const ConvArgs a)
 {
+    pdl_wait();  // the partial sums of the conv kernel before it
     const int r = blockIdx.y;
     int f;
     bool zero;
@@ -855,10 +859,26 @@ cudaError_t launch(const CUtensorMap& map, const ConvArgs& a, int grid, size_t s
         if (e != cudaSuccess) return e;
         configured_dev = dev;
     }
-    kern<<<grid, kThreads, smem, s>>>(map, a);
+    // Both kernels may be scheduled while the kernel before them finishes
+    // (programmatic dependent launch); each waits for it before reading memory.
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, kern, map, a);
+    if (e != cudaSuccess) return e;
     if (a.splits > 1) {
-        const dim3 fgrid((unsigned)((a.M + 1023) / 1024), (unsigned)(a.ncols_all + a.groups * a.Fg));
-        k_splitk_finalize<OUT_BF16><<<fgrid, 256, 0, s>>>(a);
+        cfg.gridDim = dim3((unsigned)((a.M + 1023) / 1024), (unsigned)(a.ncols_all + a.groups * a.Fg));
+        cfg.blockDim = dim3(256);
+        cfg.dynamicSmemBytes = 0;
+        e = cudaLaunchKernelEx(&cfg, k_splitk_finalize<OUT_BF16>, a);
+        if (e != cudaSuccess) return e;
     }
     return cudaGetLastError();
 }

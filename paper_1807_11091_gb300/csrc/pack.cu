@@ -52,6 +52,7 @@ SADMM_DEV int lower_bound(const int* a, int n, int v)
 // lists, so the binary searches below read shared memory, not HBM.
 __global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status, int lists_in_smem)
 {
+    pdl_wait();  // after the kernel before it in the stream
     __shared__ int s_start[65];
     __shared__ int s_bad;
     extern __shared__ int s_lists[];
@@ -171,6 +172,7 @@ __global__ void __launch_bounds__(128) k_pack_wp(const T* __restrict__ W, int K,
                                                  const int* __restrict__ colidx, int k_pad,
                                                  __nv_bfloat16* __restrict__ wp)
 {
+    pdl_wait();  // after the kernel before it in the stream
     const long long r = blockIdx.x;
     const int f = rowmap[r];
     uint4* dst = reinterpret_cast<uint4*>(wp + r * k_pad);
@@ -241,15 +243,17 @@ sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int
     const size_t list_bytes =
         (size_t)((a.all_kept ? 0 : a.n_filt) + ((col_idx && a.colkind != SADMM_COL_NONE) ? a.n_colgroups : 0)) * 4;
     const bool in_smem = list_bytes <= 40 * 1024;
-    k_pack_meta<<<1, 1024, in_smem ? list_bytes : 0, s>>>(a, device_status_ptr(), in_smem ? 1 : 0);
+    launch_pdl(k_pack_meta, dim3(1), dim3(1024), in_smem ? list_bytes : 0, s, a, device_status_ptr(),
+               in_smem ? 1 : 0);
 
     __nv_bfloat16* wp = reinterpret_cast<__nv_bfloat16*>(base + plan->off_wp);
     const unsigned rows = (unsigned)(g.groups * plan->n_pad);
     if (wdt == SADMM_BF16)
-        k_pack_wp<__nv_bfloat16><<<rows, 128, 0, s>>>((const __nv_bfloat16*)W, (int)g.k, a.rowmap, a.colidx,
-                                                       plan->k_pad, wp);
+        launch_pdl(k_pack_wp<__nv_bfloat16>, dim3(rows), dim3(128), 0, s, (const __nv_bfloat16*)W, (int)g.k,
+                   a.rowmap, a.colidx, plan->k_pad, wp);
     else
-        k_pack_wp<float><<<rows, 128, 0, s>>>((const float*)W, (int)g.k, a.rowmap, a.colidx, plan->k_pad, wp);
+        launch_pdl(k_pack_wp<float>, dim3(rows), dim3(128), 0, s, (const float*)W, (int)g.k, a.rowmap, a.colidx,
+                   plan->k_pad, wp);
     if (cudaGetLastError() != cudaSuccess) return SADMM_ECUDA;
 
     // TMA descriptor of Wp: [groups*n_pad rows][k_pad bf16], boxes of 64 x bn,

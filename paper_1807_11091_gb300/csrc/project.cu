@@ -45,6 +45,7 @@ template <typename T>
 __global__ void __launch_bounds__(256) k_filter_keys(const T* __restrict__ W, const T* __restrict__ U, int F,
                                                      int K, double* __restrict__ keys)
 {
+    pdl_wait();  // after the kernel before it in the stream
     __shared__ double part[8];
     const int a = blockIdx.x;
     const int lane = threadIdx.x & 31, wy = threadIdx.x >> 5;
@@ -85,6 +86,7 @@ __global__ void __launch_bounds__(256) k_column_keys(const T* __restrict__ W, co
                                                      const int* __restrict__ rows, int nrows,
                                                      double* __restrict__ part_out)
 {
+    pdl_wait();  // after the kernel before it in the stream
     __shared__ double part[8][33];
     const int lane = threadIdx.x & 31;
     const int wy = threadIdx.x >> 5;
@@ -144,6 +146,7 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
                                                         double* __restrict__ keys, double* __restrict__ keys_out,
                                                         int* __restrict__ out_idx, uint8_t* __restrict__ keep_out)
 {
+    pdl_wait();  // after the kernel before it in the stream
     __shared__ unsigned int hist[256];
     __shared__ unsigned long long s_prefix;
     __shared__ int s_kk;
@@ -249,7 +252,8 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
 void launch_select(const double* src, int G, int taps, int k, int nparts, long long part_stride, double* keys,
                    double* keys_out, int* out_idx, uint8_t* keep_out, cudaStream_t s)
 {
-    k_select<<<1, kSelThreads, 0, s>>>(src, G, taps, k, nparts, part_stride, keys, keys_out, out_idx, keep_out);
+    launch_pdl(k_select, dim3(1), dim3(kSelThreads), 0, s, src, G, taps, k, nparts, part_stride, keys, keys_out,
+               out_idx, keep_out);
 }
 
 // Row chunks of the column-key pass: enough blocks to fill the GPU, with the
@@ -267,6 +271,7 @@ int column_parts(long long K, long long nrows)
 __global__ void __launch_bounds__(256) k_keep_all(int* idx_a, int na, uint8_t* keep_a, int* idx_b, int nb,
                                                   uint8_t* keep_b)
 {
+    pdl_wait();  // after the kernel before it in the stream
     const int i = blockIdx.x * 256 + threadIdx.x;
     if (idx_a && i < na) {
         idx_a[i] = i;
@@ -297,19 +302,19 @@ sadmm_status run_project(const Geometry& g, const T* W, const T* U, int k_filter
     const bool cols_all = (colkind != SADMM_COL_NONE) && (k_cols == G) && !keys_out;
     if (rows_all || cols_all) {
         const int n = (rows_all ? F : 0) > (cols_all ? G : 0) ? F : (cols_all ? G : 0);
-        k_keep_all<<<(n + 255) / 256, 256, 0, s>>>(rows_all ? filt_idx : nullptr, F, rows_all ? rkeep : nullptr,
-                                                   cols_all ? col_idx : nullptr, G, cols_all ? ckeep : nullptr);
+        launch_pdl(k_keep_all, dim3((n + 255) / 256), dim3(256), 0, s, rows_all ? filt_idx : nullptr, F,
+                   rows_all ? rkeep : nullptr, cols_all ? col_idx : nullptr, G, cols_all ? ckeep : nullptr);
     }
     if (!rows_all) {
-        k_filter_keys<T><<<F, 256, 0, s>>>(W, U, F, K, fkeys);
+        launch_pdl(k_filter_keys<T>, dim3(F), dim3(256), 0, s, W, U, F, K, fkeys);
         launch_select(fkeys, F, 1, k_filters, 1, 0, fkeys, keys_out, filt_idx, rkeep, s);
     }
     if (colkind != SADMM_COL_NONE && !cols_all) {
         const bool all_rows = (k_filters == F);
         const int nrows = all_rows ? F : k_filters;
         const int R = column_parts(K, nrows);
-        k_column_keys<T><<<dim3((K + 31) / 32, R), 256, 0, s>>>(W, U, K, all_rows ? nullptr : filt_idx, nrows,
-                                                                parts);
+        launch_pdl(k_column_keys<T>, dim3((K + 31) / 32, R), dim3(256), 0, s, W, U, K,
+                   all_rows ? nullptr : filt_idx, nrows, parts);
         launch_select(parts, G, taps, k_cols, R, K, ckeys, keys_out ? keys_out + F : nullptr, col_idx, ckeep, s);
     }
     return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
