@@ -150,6 +150,7 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
     __shared__ unsigned int hist[256];
     __shared__ unsigned long long s_prefix;
     __shared__ int s_kk;
+    __shared__ int s_done;
     __shared__ int warp_tot[33];
     const int tid = threadIdx.x;
 
@@ -188,8 +189,11 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
         return;
     }
 
-    // 2. radix select, 8 bits per pass from the most significant digit
-    if (tid == 0) { s_prefix = 0ull; s_kk = k; }
+    // 2. radix select, 8 bits per pass from the most significant digit.  Once
+    //    the digit's bucket holds exactly the keys still needed, all of them are
+    //    kept and the lower digits cannot change the selection: stop there and
+    //    compare keys on the digits examined so far.
+    if (tid == 0) { s_prefix = 0ull; s_kk = k; s_done = 0; }
     unsigned long long mask = 0ull;
     for (int shift = 56; shift >= 0; shift -= 8) {
         for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0u;
@@ -218,6 +222,7 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
                         const unsigned d = 255u - 8u * tid - j;
                         s_prefix = prefix | ((unsigned long long)d << shift);
                         s_kk = (int)(kk - cum);
+                        if (c[j] == kk - cum) s_done = 1;
                         break;
                     }
                     cum += c[j];
@@ -226,16 +231,19 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
         }
         mask |= 0xFFull << shift;
         __syncthreads();
+        if (s_done) break;
     }
-    const unsigned long long T = s_prefix;  // exact k-th largest key
-    const int take_eq = s_kk;               // how many keys equal to T are kept
+    // T: the k-th largest key on the examined digits (`mask`); take_eq: how
+    // many keys equal to T there are kept (all of them after an early stop)
+    const unsigned long long T = s_prefix;
+    const int take_eq = s_kk;
 
     // 3. ordered compaction
     int run_out = 0, run_eq = 0;
     for (int base = 0; base < G; base += kSelThreads) {
         const int i = base + tid;
         const bool valid = i < G;
-        const unsigned long long u = valid ? (unsigned long long)__double_as_longlong(kv[i]) : 0ull;
+        const unsigned long long u = valid ? (unsigned long long)__double_as_longlong(kv[i]) & mask : 0ull;
         const bool gt = valid && u > T;
         const bool eq = valid && u == T;
         int eq_tot, take_tot;
