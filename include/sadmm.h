@@ -329,7 +329,8 @@ size_t sadmm_conv_bwd_workspace_size(const sadmm_plan* plan);
  *   db[f]      = sum of dZ over images and pixels for kept f; 0 for pruned f;
  *   dx         = the input gradient through the kept weights only.
  * The contractions run on the tensor cores (bf16 operands, fp32 accumulation);
- * dW and dx are summed with fp32 atomics (their last bits depend on timing).
+ * dW and db are summed in a fixed order (deterministic); dx is summed with
+ * fp32 atomics (its last bits depend on timing).
  *
  *   plan   a packed plan (sadmm_pack) of the layer.
  *   x      device bf16 [N][C][T][H][W] (needed for dW).

@@ -39,6 +39,10 @@ struct BwdGeo {
     int kr;       // column rows of the dgrad product: k_pad rounded up to 128
     int mc;       // pixels per chunk (multiple of 256)
     uint32_t plane_mul, plane_sh, ohw_mul, ohw_sh, ow_mul, ow_sh;  // multiply-shift divisors
+    long long x_chw, thw;  // elements per input image, per input channel
+    int hw;
+    int split_mask;        // tap-mask encoding of the gather table (see tap_mask)
+    const uint2* table;    // the plan's gather table: [k_pad] {x offset from the window origin, tap bits}
 };
 
 inline void divisor(uint32_t d, uint32_t& mul, uint32_t& sh)
@@ -62,32 +66,42 @@ SADMM_DEV void pixel_of(const BwdGeo& b, long long m, int& n, int& ot, int& oh, 
     ow = (int)(r - (uint32_t)oh * (uint32_t)b.OW);
 }
 
-// A_T[j][ml] = x at kept column j of output pixel m0 + ml (0 outside the input,
-// for padding columns and past the last pixel).
+// Packed columns per block of k_bwd_im2col / k_bwd_col2im: their gather-table
+// entries sit in shared memory, and each thread decodes its pixel once for all.
+constexpr int kTableCols = 32;
+
+// A_T[j][ml] = x at packed column j of output pixel m0 + ml, through the plan's
+// gather table (the column's x offset from the pixel's window origin, its tap
+// bits tested against the pixel's tap mask); 0 outside the input, for padding
+// columns and past the last pixel.  Block (bx, by): columns by*32 .. by*32+31.
 __global__ void __launch_bounds__(256) k_bwd_im2col(const BwdGeo b, int g, long long m0, __nv_bfloat16* at)
 {
-    const int j = blockIdx.y;
-    const int col = j < b.n_cols ? __ldg(b.colidx + j) : -1;
-    int c = 0, kt = 0, kh = 0, kw = 0;
-    if (col >= 0) {
-        c = col / b.taps;
-        const int r = col - c * b.taps;
-        kt = r / (b.KH * b.KW);
-        kh = (r / b.KW) % b.KH;
-        kw = r % b.KW;
+    __shared__ uint2 s_t[kTableCols];
+    const int j0 = blockIdx.y * kTableCols;
+    if (threadIdx.x < kTableCols) {
+        const int j = j0 + threadIdx.x;
+        s_t[threadIdx.x] = j < b.k_pad ? __ldg(b.table + j) : make_uint2(0u, 1u << 31);
     }
+    __syncthreads();
+    const int nj = min(kTableCols, b.k_pad - j0);
+    const unsigned short* xs = reinterpret_cast<const unsigned short*>(b.x);
+    unsigned short* as = reinterpret_cast<unsigned short*>(at);
     for (int ml = blockIdx.x * 256 + threadIdx.x; ml < b.mc; ml += gridDim.x * 256) {
         const long long m = m0 + ml;
-        float v = 0.0f;
-        if (col >= 0 && m < b.M) {
+        uint32_t M = 0;  // no tap is valid past the last pixel (tap bits are never 0)
+        long long base = 0;
+        if (m < b.M) {
             int n, ot, oh, ow;
             pixel_of(b, m, n, ot, oh, ow);
-            const int it = ot * b.st - b.pt + kt, ih = oh * b.sh - b.ph + kh, iw = ow * b.sw - b.pw + kw;
-            if ((unsigned)it < (unsigned)b.T && (unsigned)ih < (unsigned)b.H && (unsigned)iw < (unsigned)b.W)
-                v = __bfloat162float(b.x[((((long long)n * b.C + (long long)g * b.Cg + c) * b.T + it) * b.H + ih) *
-                                             b.W + iw]);
+            const int it0 = ot * b.st - b.pt, ih0 = oh * b.sh - b.ph, iw0 = ow * b.sw - b.pw;
+            M = tap_mask(it0, ih0, iw0, b.KT, b.KH, b.KW, b.T, b.H, b.W, b.split_mask);
+            base = (long long)n * b.x_chw + (long long)g * b.Cg * b.thw + (long long)it0 * b.hw +
+                   (long long)ih0 * b.W + iw0;
         }
-        at[(size_t)j * b.mc + ml] = __float2bfloat16_rn(v);
+        for (int jj = 0; jj < nj; ++jj) {
+            const uint2 t = s_t[jj];
+            as[(size_t)(j0 + jj) * b.mc + ml] = ((M & t.y) == t.y) ? __ldg(xs + base + (int)t.x) : (unsigned short)0;
+        }
     }
 }
 
@@ -101,22 +115,48 @@ SADMM_DEV float relu_grad(const BwdGeo& b, size_t off)
 
 // dZ for the kept filters of group g and pixels m0 .. m0+mc-1, in two layouts:
 // gt[i][ml] (filter-major, rows up to fr) and gm[ml][i] (pixel-major, i < fk).
+// Block (bx, by): pixels bx*64 .. +63 of the chunk, packed rows by*32 .. +31;
+// the pixel-major copy goes out through a shared-memory transpose, 8 rows of a
+// pixel per 16-byte store.
+constexpr int kDyPix = 64, kDyRows = 32;
+
 __global__ void __launch_bounds__(256) k_bwd_gather_dy(const BwdGeo b, int g, long long m0, __nv_bfloat16* gt,
                                                        __nv_bfloat16* gm)
 {
-    const int i = blockIdx.y;  // 0 .. max(fr, fk)-1
-    const int f = i < b.n_pad ? __ldg(b.rowmap + (long long)g * b.n_pad + i) : -1;
-    for (int ml = blockIdx.x * 256 + threadIdx.x; ml < b.mc; ml += gridDim.x * 256) {
-        const long long m = m0 + ml;
+    __shared__ __nv_bfloat16 tile[kDyRows][kDyPix + 2];
+    const int i0 = blockIdx.y * kDyRows, p0 = blockIdx.x * kDyPix;
+    const int pl = threadIdx.x & (kDyPix - 1), r0 = threadIdx.x / kDyPix;  // 64 pixels x 4 rows
+    const int ml = p0 + pl;
+    const long long m = m0 + ml;
+    const bool valid = ml < b.mc && m < b.M;
+    size_t pbase = 0;  // offset of the pixel in plane 0 of its image
+    if (valid) {
+        const uint32_t n = udiv((uint32_t)m, b.plane_mul, b.plane_sh);
+        pbase = (size_t)n * b.F * b.plane + ((uint32_t)m - n * (uint32_t)b.plane);
+    }
+    for (int k = 0; k < kDyRows / 4; ++k) {
+        const int r = r0 + 4 * k, i = i0 + r;
         float v = 0.0f;
-        if (f >= 0 && m < b.M) {
-            const int n = (int)(m / b.plane);
-            const size_t off = ((size_t)n * b.F + f) * b.plane + (size_t)(m - (long long)n * b.plane);
-            v = __bfloat162float(b.dy[off]) * relu_grad(b, off);
+        if (valid && i < b.n_pad) {
+            const int f = __ldg(b.rowmap + (long long)g * b.n_pad + i);
+            if (f >= 0) {
+                const size_t off = pbase + (size_t)f * b.plane;
+                v = __bfloat162float(b.dy[off]) * relu_grad(b, off);
+            }
         }
         const __nv_bfloat16 h = __float2bfloat16_rn(v);
-        if (i < b.fr) gt[(size_t)i * b.mc + ml] = h;
-        if (i < b.fk) gm[(size_t)ml * b.fk + i] = h;
+        tile[r][pl] = h;
+        if (i < b.fr && ml < b.mc) gt[(size_t)i * b.mc + ml] = h;
+    }
+    __syncthreads();
+    const int pl2 = threadIdx.x >> 2, rq = (threadIdx.x & 3) * 8;  // pixel, first of its 8 rows
+    const int ml2 = p0 + pl2;
+    if (ml2 < b.mc && i0 + rq < b.fk) {  // fk is a multiple of 64: all 8 rows are inside
+        uint32_t w[4];
+        for (int e = 0; e < 4; ++e)
+            w[e] = (uint32_t)__bfloat16_as_ushort(tile[rq + 2 * e][pl2]) |
+                   ((uint32_t)__bfloat16_as_ushort(tile[rq + 2 * e + 1][pl2]) << 16);
+        *reinterpret_cast<uint4*>(gm + (size_t)ml2 * b.fk + i0 + rq) = make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
 
@@ -132,47 +172,63 @@ __global__ void __launch_bounds__(256) k_bwd_transpose_wp(const BwdGeo b, int g,
     }
 }
 
-// dx += col2im(dA): dat[j][ml] for kept column j of pixel m0 + ml.
+// dx += dA at every valid (packed column, output pixel) position, through the
+// gather table as in k_bwd_im2col; fp32 atomics (several pixels' windows
+// overlap), zeros skipped.
 __global__ void __launch_bounds__(256) k_bwd_col2im(const BwdGeo b, int g, long long m0, const float* dat, float* dx)
 {
-    const int j = blockIdx.y;
-    const int col = j < b.n_cols ? __ldg(b.colidx + j) : -1;
-    if (col < 0) return;
-    const int c = col / b.taps;
-    const int r = col - c * b.taps;
-    const int kt = r / (b.KH * b.KW), kh = (r / b.KW) % b.KH, kw = r % b.KW;
+    __shared__ uint2 s_t[kTableCols];
+    const int j0 = blockIdx.y * kTableCols;
+    if (threadIdx.x < kTableCols) {
+        const int j = j0 + threadIdx.x;
+        s_t[threadIdx.x] = j < b.k_pad ? __ldg(b.table + j) : make_uint2(0u, 1u << 31);
+    }
+    __syncthreads();
+    const int nj = min(kTableCols, b.k_pad - j0);
     for (int ml = blockIdx.x * 256 + threadIdx.x; ml < b.mc; ml += gridDim.x * 256) {
         const long long m = m0 + ml;
         if (m >= b.M) break;
         int n, ot, oh, ow;
         pixel_of(b, m, n, ot, oh, ow);
-        const int it = ot * b.st - b.pt + kt, ih = oh * b.sh - b.ph + kh, iw = ow * b.sw - b.pw + kw;
-        if ((unsigned)it < (unsigned)b.T && (unsigned)ih < (unsigned)b.H && (unsigned)iw < (unsigned)b.W) {
-            const float v = dat[(size_t)j * b.mc + ml];
-            if (v != 0.0f)
-                atomicAdd(dx + ((((long long)n * b.C + (long long)g * b.Cg + c) * b.T + it) * b.H + ih) * b.W + iw,
-                          v);
+        const int it0 = ot * b.st - b.pt, ih0 = oh * b.sh - b.ph, iw0 = ow * b.sw - b.pw;
+        const uint32_t M = tap_mask(it0, ih0, iw0, b.KT, b.KH, b.KW, b.T, b.H, b.W, b.split_mask);
+        const long long base = (long long)n * b.x_chw + (long long)g * b.Cg * b.thw + (long long)it0 * b.hw +
+                               (long long)ih0 * b.W + iw0;
+        for (int jj = 0; jj < nj; ++jj) {
+            const uint2 t = s_t[jj];
+            if ((M & t.y) == t.y) {
+                const float v = dat[(size_t)(j0 + jj) * b.mc + ml];
+                if (v != 0.0f) atomicAdd(dx + base + (int)t.x, v);
+            }
         }
     }
 }
 
-// dW[f_i][col_j] = dWp[g][i][j] for kept pairs (dW zeroed before).
-__global__ void __launch_bounds__(256) k_bwd_scatter_dw(const BwdGeo b, int g, const float* dwp, float* dW)
+// dW[f_i][col_j] = sum over the pixel splits z, in order, of dws[z][i][j] for
+// the kept pairs of conv group g (dW zeroed before): deterministic.
+__global__ void __launch_bounds__(256) k_bwd_reduce_dw(const BwdGeo b, int g, const float* dws, int nsplit, float* dW)
 {
     const int i = blockIdx.y;
     const int f = __ldg(b.rowmap + (long long)g * b.n_pad + i);
     if (f < 0) return;
     const long long K = (long long)b.Cg * b.taps;
+    const size_t slice = (size_t)b.fr * b.k_pad;
     for (int j = blockIdx.x * 256 + threadIdx.x; j < b.n_cols; j += gridDim.x * 256) {
         const int col = __ldg(b.colidx + j);
-        if (col >= 0) dW[(long long)f * K + col] = dwp[(size_t)i * b.k_pad + j];
+        if (col < 0) continue;
+        float acc = 0.0f;
+        for (int z = 0; z < nsplit; ++z) acc += dws[z * slice + (size_t)i * b.k_pad + j];
+        dW[(long long)f * K + col] = acc;
     }
 }
 
-// db[f] = sum over images and pixels of dZ (fixed order), 0 for pruned filters.
-__global__ void __launch_bounds__(256) k_bwd_db(const BwdGeo b, float* db)
+// Bias gradient in two fixed-order stages.  Block (f, sl): the sum of dZ over
+// every pixel of images sl, sl + S, ... (S = gridDim.y), 0 for a pruned filter.
+constexpr int kDbSlices = 64;
+
+__global__ void __launch_bounds__(256) k_bwd_db_part(const BwdGeo b, float* part)
 {
-    __shared__ float part[256];
+    __shared__ float red[256];
     const int f = blockIdx.x;
     const int g = f / b.Fg;
     // kept?  rowmap of group g lists the kept filters
@@ -183,19 +239,29 @@ __global__ void __launch_bounds__(256) k_bwd_db(const BwdGeo b, float* db)
     kept = __syncthreads_or(kept);
     float s = 0.0f;
     if (kept) {
-        for (long long m = threadIdx.x; m < b.M; m += 256) {
-            const int n = (int)(m / b.plane);
-            const size_t off = ((size_t)n * b.F + f) * b.plane + (size_t)(m - (long long)n * b.plane);
-            s += __bfloat162float(b.dy[off]) * relu_grad(b, off);
+        for (int n = blockIdx.y; n < b.N; n += gridDim.y) {
+            const size_t base = ((size_t)n * b.F + f) * b.plane;  // the plane is contiguous
+            for (int p = threadIdx.x; p < b.plane; p += 256)
+                s += __bfloat162float(b.dy[base + p]) * relu_grad(b, base + p);
         }
     }
-    part[threadIdx.x] = s;
+    red[threadIdx.x] = s;
     __syncthreads();
     for (int o = 128; o > 0; o >>= 1) {
-        if (threadIdx.x < o) part[threadIdx.x] += part[threadIdx.x + o];
+        if (threadIdx.x < o) red[threadIdx.x] += red[threadIdx.x + o];
         __syncthreads();
     }
-    if (threadIdx.x == 0) db[f] = part[0];
+    if (threadIdx.x == 0) part[(size_t)f * gridDim.y + blockIdx.y] = red[0];
+}
+
+// db[f] = sum over the S slices, in order, of the partial sums.
+__global__ void __launch_bounds__(256) k_bwd_db_final(const float* part, int F, int S, float* db)
+{
+    const int f = blockIdx.x * 256 + threadIdx.x;
+    if (f >= F) return;
+    float acc = 0.0f;
+    for (int sl = 0; sl < S; ++sl) acc += part[(size_t)f * S + sl];
+    db[f] = acc;
 }
 
 __global__ void __launch_bounds__(256) k_bwd_zero(float* p, long long n)
@@ -206,8 +272,26 @@ __global__ void __launch_bounds__(256) k_bwd_zero(float* p, long long n)
 inline long long rup(long long x, long long a) { return (x + a - 1) / a * a; }
 
 struct Layout {
-    size_t at, gt, gm, wpt, dat, dwp, total;
+    size_t at, gt, gm, wpt, dat, dws, dbp, total;
 };
+
+int pick_bn(long long n);
+
+// The weight gradient has only fr/128 x k_pad/bn output tiles, so each chunk's
+// pixels (the GEMM's K) are split over enough CTAs to fill the GPU: about
+// kWgradCtas CTAs in all, the split count a divisor of the chunk's 64-pixel
+// stages.  Fixed (not the device's SM count) so that the workspace size is.
+constexpr long long kWgradCtas = 256;
+
+int wgrad_splits(const BwdGeo& b)
+{
+    const long long wtiles = (long long)(b.fr / 128) * (b.k_pad / pick_bn(b.k_pad));
+    const long long nk = b.mc / 64;
+    const long long want = std::max<long long>(1, kWgradCtas / std::max<long long>(wtiles, 1));
+    for (long long d = std::min(want, nk); d >= 1; --d)
+        if (nk % d == 0) return (int)d;
+    return 1;
+}
 
 Layout layout(const BwdGeo& b)
 {
@@ -223,7 +307,8 @@ Layout layout(const BwdGeo& b)
     l.gm = take((size_t)b.mc * b.fk * 2);
     l.wpt = take((size_t)b.kr * b.fk * 2);
     l.dat = take((size_t)b.kr * b.mc * 4);
-    l.dwp = take((size_t)b.groups * b.fr * b.k_pad * 4);
+    l.dws = take((size_t)wgrad_splits(b) * b.fr * b.k_pad * 4);  // [split][fr][k_pad]
+    l.dbp = take((size_t)b.F * kDbSlices * 4);                    // [F][slices] bias-gradient partials
     l.total = off;
     return l;
 }
@@ -248,6 +333,10 @@ BwdGeo geometry(const sadmm_plan* plan, const Geometry& g)
     divisor((uint32_t)b.plane, b.plane_mul, b.plane_sh);
     divisor((uint32_t)(b.OH * b.OW), b.ohw_mul, b.ohw_sh);
     divisor((uint32_t)b.OW, b.ow_mul, b.ow_sh);
+    b.x_chw = g.c * g.t * g.h * g.w;
+    b.thw = g.t * g.h * g.w;
+    b.hw = (int)(g.h * g.w);
+    b.split_mask = tap_mask_mode(g);
     return b;
 }
 
@@ -279,6 +368,7 @@ sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const vo
     b.rowmap = reinterpret_cast<const int*>(base + plan->off_rowmap);
     b.colidx = reinterpret_cast<const int*>(base + plan->off_colidx);
     b.counts = reinterpret_cast<const int*>(base + plan->off_counts);
+    b.table = reinterpret_cast<const uint2*>(base + plan->off_gather);
     const __nv_bfloat16* wp = reinterpret_cast<const __nv_bfloat16*>(base + plan->off_wp);
     const Layout l = layout(b);
     char* w = static_cast<char*>(ws);
@@ -287,49 +377,45 @@ sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const vo
     __nv_bfloat16* gm = reinterpret_cast<__nv_bfloat16*>(w + l.gm);
     __nv_bfloat16* wpt = reinterpret_cast<__nv_bfloat16*>(w + l.wpt);
     float* dat = reinterpret_cast<float*>(w + l.dat);
-    float* dwp = reinterpret_cast<float*>(w + l.dwp);
-    const unsigned xblocks = (unsigned)std::min<long long>((b.mc + 255) / 256, 64);
+    float* dws = reinterpret_cast<float*>(w + l.dws);
+    float* dbp = reinterpret_cast<float*>(w + l.dbp);
+    // table-driven im2col / col2im: one pixel per thread, 32 packed columns per block
+    const unsigned tblocks = (unsigned)((b.mc + 255) / 256);
+    const unsigned tcols = (unsigned)((b.k_pad + kTableCols - 1) / kTableCols);
     const long long K = g.cg * g.taps;
 
-    if (dW) {
-        k_bwd_zero<<<1024, 256, 0, s>>>(dW, g.f * K);
-        k_bwd_zero<<<256, 256, 0, s>>>(dwp, (long long)b.groups * b.fr * b.k_pad);
-    }
-    // weight-gradient tiles are few (fr/128 x k_pad/bn): split the pixel
-    // dimension of each chunk over enough CTAs to fill the GPU
+    if (dW) k_bwd_zero<<<1024, 256, 0, s>>>(dW, g.f * K);
     const int wbn = pick_bn(b.k_pad);
-    const long long wtiles = (long long)(b.fr / 128) * (b.k_pad / wbn);
-    int wsplit = 1;
-    {
-        const long long nk = b.mc / 64;
-        long long want = std::max<long long>(1, (2LL * device_sm_count()) / std::max<long long>(wtiles, 1));
-        for (long long d = std::min(want, nk); d >= 1; --d)
-            if (nk % d == 0) { wsplit = (int)d; break; }
-    }
+    const int wsplit = wgrad_splits(b);
     if (dx) k_bwd_zero<<<2048, 256, 0, s>>>(dx, g.n * g.c * g.t * g.h * g.w);
-    if (db) k_bwd_db<<<(unsigned)g.f, 256, 0, s>>>(b, db);
+    if (db) {
+        const int slices = (int)std::min<long long>(g.n, kDbSlices);
+        k_bwd_db_part<<<dim3((unsigned)g.f, (unsigned)slices), 256, 0, s>>>(b, dbp);
+        k_bwd_db_final<<<(unsigned)((g.f + 255) / 256), 256, 0, s>>>(dbp, (int)g.f, slices, db);
+    }
     sadmm_status st = SADMM_OK;
     for (int grp = 0; grp < b.groups && st == SADMM_OK; ++grp) {
-        float* dwp_g = dwp + (size_t)grp * b.fr * b.k_pad;
         if (dx) k_bwd_transpose_wp<<<dim3((unsigned)((b.fk + 255) / 256), (unsigned)b.kr), 256, 0, s>>>(b, grp, wp, wpt);
         for (long long m0 = 0; m0 < g.m && st == SADMM_OK; m0 += b.mc) {
             const unsigned dyrows = (unsigned)std::max(b.fr, b.fk);
-            k_bwd_gather_dy<<<dim3(xblocks, dyrows), 256, 0, s>>>(b, grp, m0, gt, gm);
+            k_bwd_gather_dy<<<dim3((unsigned)((b.mc + kDyPix - 1) / kDyPix), (dyrows + kDyRows - 1) / kDyRows), 256, 0,
+                              s>>>(b, grp, m0, gt, gm);
             if (dW) {
-                k_bwd_im2col<<<dim3(xblocks, (unsigned)b.k_pad), 256, 0, s>>>(b, grp, m0, at);
-                // dWp[i][j] += sum_m gt[i][m] * at[j][m] (zeroed above; split over pixels)
-                st = launch_gemm(gt, at, dwp_g, b.fr, b.k_pad, b.mc, b.k_pad, wbn, true, s, wsplit);
+                k_bwd_im2col<<<dim3(tblocks, tcols), 256, 0, s>>>(b, grp, m0, at);
+                // split z: dws[z][i][j] (+)= sum over its pixels m of gt[i][m] * at[j][m]
+                st = launch_gemm(gt, at, dws, b.fr, b.k_pad, b.mc, b.k_pad, wbn, m0 > 0, s, wsplit,
+                                 (long long)b.fr * b.k_pad);
             }
             if (dx && st == SADMM_OK) {
                 // dat[j][m] = sum_i wpt[j][i] * gm[m][i]
                 st = launch_gemm(wpt, gm, dat, b.kr, b.mc, b.fk, b.mc, pick_bn(b.mc), false, s);
                 if (st == SADMM_OK)
-                    k_bwd_col2im<<<dim3(xblocks, (unsigned)b.k_pad), 256, 0, s>>>(b, grp, m0, dat, dx);
+                    k_bwd_col2im<<<dim3(tblocks, tcols), 256, 0, s>>>(b, grp, m0, dat, dx);
             }
         }
         if (dW && st == SADMM_OK)
-            k_bwd_scatter_dw<<<dim3((unsigned)((b.k_pad + 255) / 256), (unsigned)b.n_pad), 256, 0, s>>>(b, grp, dwp_g,
-                                                                                                     dW);
+            k_bwd_reduce_dw<<<dim3((unsigned)((b.k_pad + 255) / 256), (unsigned)b.n_pad), 256, 0, s>>>(b, grp, dws,
+                                                                                                    wsplit, dW);
     }
     if (st != SADMM_OK) return st;
     return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;

@@ -85,6 +85,29 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
     return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
 
+// Tap-validity mask of one output pixel whose receptive window starts at
+// (it0, ih0, iw0) of a T x H x W input: a bit is set where a tap reads inside
+// the input.  One bit per tap t = (kt*KH + kh)*KW + kw when the kernel has at
+// most 31 taps (split = 0); otherwise (split = 1) bits 0..15 mark valid rows
+// kt*KH + kh and bits 16..30 valid kw.  Bit 31 is never set (the gather
+// tables mark padding columns with it).
+SADMM_DEV uint32_t tap_mask(int it0, int ih0, int iw0, int KT, int KH, int KW, int T, int H, int W, int split)
+{
+    uint32_t rm = 0, cm = 0;
+    for (int kt = 0; kt < KT; ++kt) {
+        const bool vt = (unsigned)(it0 + kt) < (unsigned)T;
+        for (int kh = 0; kh < KH; ++kh)
+            if (vt && (unsigned)(ih0 + kh) < (unsigned)H) rm |= 1u << (kt * KH + kh);
+    }
+    for (int kw = 0; kw < KW; ++kw)
+        if ((unsigned)(iw0 + kw) < (unsigned)W) cm |= 1u << kw;
+    if (split) return rm | (cm << 16);
+    uint32_t m = 0;
+    for (int r = 0; r < KT * KH; ++r)
+        if (rm & (1u << r)) m |= cm << (r * KW);
+    return m;
+}
+
 SADMM_DEV void raise_status(int* status, int code)
 {
     if (status) atomicCAS(status, 0, code);

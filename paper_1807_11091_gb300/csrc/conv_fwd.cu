@@ -217,10 +217,9 @@ SADMM_DEV bool work_next(const ConvArgs& a, Work& w, int& p, int& g, int& mt, in
     return true;
 }
 
-// Tap-validity mask of one output pixel: a bit is set where a tap reads inside
-// the input.  One bit per tap t = (kt*KH + kh)*KW + kw when the kernel has at
-// most 31 taps; otherwise bits 0..15 mark valid rows kt*KH + kh and bits
-// 16..30 valid kw.  Bit 31 is never set (it marks padding columns).
+// Tap-validity mask of one output pixel: the rule of tap_mask (common.cuh),
+// written against the kernel arguments directly (a call through tap_mask costs
+// this 72-register kernel a spill).
 SADMM_DEV uint32_t pixel_mask(const ConvArgs& a, int it0, int ih0, int iw0)
 {
     uint32_t rm = 0, cm = 0;

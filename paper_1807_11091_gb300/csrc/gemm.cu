@@ -31,6 +31,7 @@ struct GemmArgs {
     int nk;  // K / 64 stages of this CTA (its split)
     int bn;
     int accumulate;  // 0: C = product; 1: C += product; 2: C += product with atomics (split K)
+    long long slice;  // > 0: split z owns C + z * slice (its own slice, no atomics)
     int tmem_cols;
     int* status;
 };
@@ -124,7 +125,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         const int row = m0 + q * 32 + lane;
         if (__all_sync(0xffffffffu, mbar_wait(acc_full, 0, abort_flag, a.status))) {
             tc_fence_after();
-            float* crow = a.C + (size_t)row * a.ldc + n0;
+            float* crow = a.C + (size_t)blockIdx.z * (size_t)a.slice + (size_t)row * a.ldc + n0;
             // 16-column chunks: bn is a multiple of 16, so no chunk passes the tile
             for (int c0 = 0; c0 < a.bn; c0 += 16) {
                 uint32_t r[16];
@@ -175,7 +176,7 @@ bool encode_kmajor(CUtensorMap* map, const void* base, long long rows, long long
 }  // namespace
 
 sadmm_status launch_gemm(const void* A, const void* B, float* C, long long M, long long N, long long K,
-                         long long ldc, int bn, bool accumulate, cudaStream_t s, int splits)
+                         long long ldc, int bn, bool accumulate, cudaStream_t s, int splits, long long slice)
 {
     if (M <= 0 || N <= 0 || K <= 0) return SADMM_OK;
     if (M % 128 || bn < 16 || bn > 256 || bn % 16 || N % bn || K % 64 || ldc % 4 || ldc < N) return SADMM_EINVAL;
@@ -188,7 +189,9 @@ sadmm_status launch_gemm(const void* A, const void* B, float* C, long long M, lo
     a.ldc = ldc;
     a.nk = (int)(K / 64 / splits);
     a.bn = bn;
-    a.accumulate = splits > 1 ? 2 : (accumulate ? 1 : 0);
+    if (slice < 0 || (slice > 0 && slice < M * ldc)) return SADMM_EINVAL;
+    a.slice = splits > 1 ? slice : 0;
+    a.accumulate = (splits > 1 && slice == 0) ? 2 : (accumulate ? 1 : 0);
     int cols = 32;
     while (cols < bn) cols <<= 1;
     a.tmem_cols = cols;

@@ -56,10 +56,13 @@ sadmm_status launch_elements(const Geometry& g, const void* W, void* U, void* Z,
 // N % bn == 0, bn a multiple of 16 in [16, 256], K % 64 == 0, ldc % 4 == 0,
 // A, B and C 16-byte aligned.
 // splits > 1: K is cut into `splits` equal ranges (K/64 divisible by splits),
-// one CTA per (tile, range), each adding its product into C with fp32 atomics
-// (C must hold the starting value; `accumulate` is then implied).
+// one CTA per (tile, range).  slice == 0: each adds its product into C with
+// fp32 atomics (C must hold the starting value; `accumulate` is then implied).
+// slice > 0 (at least M * ldc): range z writes (accumulate: adds) its product
+// into its own slice C + z * slice, without atomics; the caller sums them.
 sadmm_status launch_gemm(const void* A, const void* B, float* C, long long M, long long N, long long K,
-                         long long ldc, int bn, bool accumulate, cudaStream_t s, int splits = 1);
+                         long long ldc, int bn, bool accumulate, cudaStream_t s, int splits = 1,
+                         long long slice = 0);
 
 // ---- masked-retraining backward (bwd.cu) ----
 size_t bwd_workspace_bytes(const sadmm_plan* plan, const Geometry& g);
