@@ -13,6 +13,9 @@
 //   k_elem_pick   one block: the digit at which the running count from the top
 //                 reaches the remaining rank; extends the prefix, clears the
 //                 histogram for the next pass.
+// The passes stop early once the digit's bucket holds exactly the keys still
+// needed: all of them are kept, the lower digits cannot change the choice, and
+// keys are compared on the digits examined so far (T below is then the prefix).
 // Entries with key > T are kept, and of the entries with key == T the ones
 // with the lowest flat index e = a*K + j (ties to the lower index):
 //   k_elem_eq     per chunk of kChunk consecutive entries: how many equal T.
@@ -38,6 +41,7 @@ struct SelState {
     unsigned long long prefix;  // key bits fixed so far
     unsigned long long mask;    // which bits the prefix fixes
     long long kk;               // rank still to find among keys matching the prefix
+    int done;                   // 1: the choice is made (no further passes)
 };
 
 template <typename T>
@@ -61,10 +65,11 @@ SADMM_DEV __nv_bfloat16 zero_of<__nv_bfloat16>() { return __float2bfloat16_rn(0.
 __global__ void __launch_bounds__(256) k_elem_init(SelState* st, unsigned int* hist, unsigned int* eq_count,
                                                    long long nchunks, long long k, long long N)
 {
+    pdl_wait();  // after the kernel before it in the stream
     if (threadIdx.x == 0 && blockIdx.x == 0) {
-        if (k <= 0) *st = SelState{~0ull, ~0ull, 0};
-        else if (k >= N) *st = SelState{0ull, ~0ull, N};
-        else *st = SelState{0ull, 0ull, k};
+        if (k <= 0) *st = SelState{~0ull, ~0ull, 0, 1};
+        else if (k >= N) *st = SelState{0ull, ~0ull, N, 1};
+        else *st = SelState{0ull, 0ull, k, 0};
     }
     for (int i = blockIdx.x * 256 + threadIdx.x; i < kHistBins; i += gridDim.x * 256) hist[i] = 0u;
     if (k <= 0 || k >= N)
@@ -85,7 +90,9 @@ __global__ void __launch_bounds__(kHistThreads) k_elem_hist(const T* __restrict_
                                                             long long N, int pass, const SelState* __restrict__ st,
                                                             unsigned int* __restrict__ hist)
 {
+    pdl_wait();  // after the kernel before it in the stream
     __shared__ unsigned int h[kHistBins];
+    if (st->done) return;
     for (int i = threadIdx.x; i < kHistBins; i += kHistThreads) h[i] = 0u;
     __syncthreads();
     const unsigned long long prefix = st->prefix, mask = st->mask;
@@ -104,7 +111,9 @@ __global__ void __launch_bounds__(kHistThreads) k_elem_hist(const T* __restrict_
 // One block of 1024 threads, two bins per thread.
 __global__ void __launch_bounds__(1024) k_elem_pick(int pass, SelState* st, unsigned int* hist)
 {
+    pdl_wait();  // after the kernel before it in the stream
     __shared__ unsigned long long s_tot[1024];
+    if (st->done) return;
     const int tid = threadIdx.x;
     const int nb = 1 << pass_bits(pass);
     // bins in descending digit order: position q holds digit nb-1-q
@@ -127,11 +136,13 @@ __global__ void __launch_bounds__(1024) k_elem_pick(int pass, SelState* st, unsi
         const int shift = pass_shift(pass);
         int q = q0;
         unsigned long long cum = before;
-        if (cum + c0 < (unsigned long long)kk) { cum += c0; q = q1; }
+        unsigned c = c0;
+        if (cum + c0 < (unsigned long long)kk) { cum += c0; q = q1; c = c1; }
         const unsigned long long d = (unsigned long long)(nb - 1 - q);
         st->prefix |= d << shift;
         st->mask |= (unsigned long long)(nb - 1) << shift;
         st->kk = kk - (long long)cum;
+        if ((unsigned long long)c == (unsigned long long)kk - cum) st->done = 1;  // the whole bucket is kept
     }
     // clear for the next pass (every block of this pass has finished)
     for (int i = tid; i < kHistBins; i += 1024) hist[i] = 0u;
@@ -142,15 +153,16 @@ __global__ void __launch_bounds__(kChunkThreads) k_elem_eq(const T* __restrict__
                                                            long long N, const SelState* __restrict__ st,
                                                            unsigned int* __restrict__ eq_count)
 {
+    pdl_wait();  // after the kernel before it in the stream
     __shared__ unsigned int s_n;
     if (threadIdx.x == 0) s_n = 0u;
     __syncthreads();
-    const unsigned long long thr = st->prefix;
+    const unsigned long long thr = st->prefix, mask = st->mask;
     const long long c0 = (long long)blockIdx.x * kChunk;
     unsigned n = 0;
     for (int i = threadIdx.x; i < kChunk; i += kChunkThreads) {
         const long long e = c0 + i;
-        if (e < N && elem_key(W, U, e) == thr) ++n;
+        if (e < N && (elem_key(W, U, e) & mask) == thr) ++n;
     }
     if (n) atomicAdd(&s_n, n);
     __syncthreads();
@@ -160,6 +172,7 @@ __global__ void __launch_bounds__(kChunkThreads) k_elem_eq(const T* __restrict__
 // Exclusive prefix of eq_count[0..nchunks) in place (one block, fixed order).
 __global__ void __launch_bounds__(1024) k_elem_scan(unsigned int* eq_count, int nchunks)
 {
+    pdl_wait();  // after the kernel before it in the stream
     __shared__ unsigned int s[1024];
     __shared__ unsigned int carry;
     if (threadIdx.x == 0) carry = 0u;
@@ -191,11 +204,12 @@ __global__ void __launch_bounds__(kChunkThreads) k_elem_apply(const T* __restric
                                                               const unsigned int* __restrict__ eq_off,
                                                               uint8_t* __restrict__ keep_out)
 {
+    pdl_wait();  // after the kernel before it in the stream
     const long long take_eq = st->kk;  // how many keys equal to the threshold are kept
     __shared__ unsigned int warp_n[kChunkThreads / 32];
     __shared__ unsigned int run;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const unsigned long long Tk = st->prefix;
+    const unsigned long long Tk = st->prefix, kmask = st->mask;
     if (threadIdx.x == 0) run = eq_off[blockIdx.x];
     __syncthreads();
     const long long c0 = (long long)blockIdx.x * kChunk;
@@ -209,7 +223,7 @@ __global__ void __launch_bounds__(kChunkThreads) k_elem_apply(const T* __restric
             if (U) u = U[e];
             double v = to_f64<T>(w);
             if (U) v += to_f64<T>(u);
-            key = (unsigned long long)__double_as_longlong(fabs(v));
+            key = (unsigned long long)__double_as_longlong(fabs(v)) & kmask;
         }
         const bool eq = valid && key == Tk;
         const unsigned b = __ballot_sync(0xffffffffu, eq);
@@ -255,17 +269,20 @@ sadmm_status run_elements(const Geometry& g, const T* W, T* U, T* Z, long long k
     unsigned int* eq_count = hist + kHistBins;
     const long long nchunks = (N + kChunk - 1) / kChunk;
     const unsigned init_blocks = (unsigned)std::min<long long>((nchunks + 255) / 256 + 1, 1024);
-    k_elem_init<<<init_blocks, 256, 0, s>>>(st, hist, eq_count, nchunks, k, N);
+    launch_pdl(k_elem_init, dim3(init_blocks), dim3(256), 0, s, st, hist, eq_count, nchunks, k, N);
     if (k > 0 && k < N) {
         const int blocks = (int)std::min<long long>((N + kHistThreads - 1) / kHistThreads, 4LL * device_sm_count());
         for (int pass = 0; pass < 6; ++pass) {
-            k_elem_hist<T><<<blocks, kHistThreads, 0, s>>>(W, U, N, pass, st, hist);
-            k_elem_pick<<<1, 1024, 0, s>>>(pass, st, hist);
+            launch_pdl(k_elem_hist<T>, dim3(blocks), dim3(kHistThreads), 0, s, W, U, N, pass,
+                       static_cast<const SelState*>(st), hist);
+            launch_pdl(k_elem_pick, dim3(1), dim3(1024), 0, s, pass, st, hist);
         }
-        k_elem_eq<T><<<(unsigned)nchunks, kChunkThreads, 0, s>>>(W, U, N, st, eq_count);
-        k_elem_scan<<<1, 1024, 0, s>>>(eq_count, (int)nchunks);
+        launch_pdl(k_elem_eq<T>, dim3((unsigned)nchunks), dim3(kChunkThreads), 0, s, W, U, N,
+                   static_cast<const SelState*>(st), eq_count);
+        launch_pdl(k_elem_scan, dim3(1), dim3(1024), 0, s, eq_count, (int)nchunks);
     }
-    k_elem_apply<T><<<(unsigned)nchunks, kChunkThreads, 0, s>>>(W, U, Z, N, st, eq_count, keep_out);
+    launch_pdl(k_elem_apply<T>, dim3((unsigned)nchunks), dim3(kChunkThreads), 0, s, W, U, Z, N,
+               static_cast<const SelState*>(st), static_cast<const unsigned int*>(eq_count), keep_out);
     return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
 }
 
