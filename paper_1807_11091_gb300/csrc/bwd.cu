@@ -76,6 +76,7 @@ constexpr int kTableCols = 32;
 // columns and past the last pixel.  Block (bx, by): columns by*32 .. by*32+31.
 __global__ void __launch_bounds__(256) k_bwd_im2col(const BwdGeo b, int g, long long m0, __nv_bfloat16* at)
 {
+    pdl_wait();  // after the kernel before it in the stream
     __shared__ uint2 s_t[kTableCols];
     const int j0 = blockIdx.y * kTableCols;
     if (threadIdx.x < kTableCols) {
@@ -123,6 +124,7 @@ constexpr int kDyPix = 64, kDyRows = 32;
 __global__ void __launch_bounds__(256) k_bwd_gather_dy(const BwdGeo b, int g, long long m0, __nv_bfloat16* gt,
                                                        __nv_bfloat16* gm)
 {
+    pdl_wait();  // after the kernel before it in the stream
     __shared__ __nv_bfloat16 tile[kDyRows][kDyPix + 2];
     const int i0 = blockIdx.y * kDyRows, p0 = blockIdx.x * kDyPix;
     const int pl = threadIdx.x & (kDyPix - 1), r0 = threadIdx.x / kDyPix;  // 64 pixels x 4 rows
@@ -164,6 +166,7 @@ __global__ void __launch_bounds__(256) k_bwd_gather_dy(const BwdGeo b, int g, lo
 __global__ void __launch_bounds__(256) k_bwd_transpose_wp(const BwdGeo b, int g, const __nv_bfloat16* wp,
                                                           __nv_bfloat16* wpt)
 {
+    pdl_wait();  // after the kernel before it in the stream
     const int j = blockIdx.y;
     for (int i = blockIdx.x * 256 + threadIdx.x; i < b.fk; i += gridDim.x * 256) {
         __nv_bfloat16 v = __float2bfloat16_rn(0.0f);
@@ -177,6 +180,7 @@ __global__ void __launch_bounds__(256) k_bwd_transpose_wp(const BwdGeo b, int g,
 // overlap), zeros skipped.
 __global__ void __launch_bounds__(256) k_bwd_col2im(const BwdGeo b, int g, long long m0, const float* dat, float* dx)
 {
+    pdl_wait();  // after the kernel before it in the stream
     __shared__ uint2 s_t[kTableCols];
     const int j0 = blockIdx.y * kTableCols;
     if (threadIdx.x < kTableCols) {
@@ -208,6 +212,7 @@ __global__ void __launch_bounds__(256) k_bwd_col2im(const BwdGeo b, int g, long 
 // the kept pairs of conv group g (dW zeroed before): deterministic.
 __global__ void __launch_bounds__(256) k_bwd_reduce_dw(const BwdGeo b, int g, const float* dws, int nsplit, float* dW)
 {
+    pdl_wait();  // after the kernel before it in the stream
     const int i = blockIdx.y;
     const int f = __ldg(b.rowmap + (long long)g * b.n_pad + i);
     if (f < 0) return;
@@ -228,6 +233,7 @@ constexpr int kDbSlices = 64;
 
 __global__ void __launch_bounds__(256) k_bwd_db_part(const BwdGeo b, float* part)
 {
+    pdl_wait();  // after the kernel before it in the stream
     __shared__ float red[256];
     const int f = blockIdx.x;
     const int g = f / b.Fg;
@@ -257,6 +263,7 @@ __global__ void __launch_bounds__(256) k_bwd_db_part(const BwdGeo b, float* part
 // db[f] = sum over the S slices, in order, of the partial sums.
 __global__ void __launch_bounds__(256) k_bwd_db_final(const float* part, int F, int S, float* db)
 {
+    pdl_wait();  // after the kernel before it in the stream
     const int f = blockIdx.x * 256 + threadIdx.x;
     if (f >= F) return;
     float acc = 0.0f;
@@ -266,6 +273,7 @@ __global__ void __launch_bounds__(256) k_bwd_db_final(const float* part, int F, 
 
 __global__ void __launch_bounds__(256) k_bwd_zero(float* p, long long n)
 {
+    pdl_wait();  // after the kernel before it in the stream
     for (long long i = (long long)blockIdx.x * 256 + threadIdx.x; i < n; i += (long long)gridDim.x * 256) p[i] = 0.0f;
 }
 
@@ -384,24 +392,27 @@ sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const vo
     const unsigned tcols = (unsigned)((b.k_pad + kTableCols - 1) / kTableCols);
     const long long K = g.cg * g.taps;
 
-    if (dW) k_bwd_zero<<<1024, 256, 0, s>>>(dW, g.f * K);
+    if (dW) launch_pdl(k_bwd_zero, dim3(1024), dim3(256), 0, s, dW, g.f * K);
     const int wbn = pick_bn(b.k_pad);
     const int wsplit = wgrad_splits(b);
-    if (dx) k_bwd_zero<<<2048, 256, 0, s>>>(dx, g.n * g.c * g.t * g.h * g.w);
+    if (dx) launch_pdl(k_bwd_zero, dim3(2048), dim3(256), 0, s, dx, g.n * g.c * g.t * g.h * g.w);
     if (db) {
         const int slices = (int)std::min<long long>(g.n, kDbSlices);
-        k_bwd_db_part<<<dim3((unsigned)g.f, (unsigned)slices), 256, 0, s>>>(b, dbp);
-        k_bwd_db_final<<<(unsigned)((g.f + 255) / 256), 256, 0, s>>>(dbp, (int)g.f, slices, db);
+        launch_pdl(k_bwd_db_part, dim3((unsigned)g.f, (unsigned)slices), dim3(256), 0, s, b, dbp);
+        launch_pdl(k_bwd_db_final, dim3((unsigned)((g.f + 255) / 256)), dim3(256), 0, s,
+                   static_cast<const float*>(dbp), (int)g.f, slices, db);
     }
     sadmm_status st = SADMM_OK;
     for (int grp = 0; grp < b.groups && st == SADMM_OK; ++grp) {
-        if (dx) k_bwd_transpose_wp<<<dim3((unsigned)((b.fk + 255) / 256), (unsigned)b.kr), 256, 0, s>>>(b, grp, wp, wpt);
+        if (dx)
+            launch_pdl(k_bwd_transpose_wp, dim3((unsigned)((b.fk + 255) / 256), (unsigned)b.kr), dim3(256), 0, s, b,
+                       grp, wp, wpt);
         for (long long m0 = 0; m0 < g.m && st == SADMM_OK; m0 += b.mc) {
             const unsigned dyrows = (unsigned)std::max(b.fr, b.fk);
-            k_bwd_gather_dy<<<dim3((unsigned)((b.mc + kDyPix - 1) / kDyPix), (dyrows + kDyRows - 1) / kDyRows), 256, 0,
-                              s>>>(b, grp, m0, gt, gm);
+            launch_pdl(k_bwd_gather_dy, dim3((unsigned)((b.mc + kDyPix - 1) / kDyPix), (dyrows + kDyRows - 1) / kDyRows),
+                       dim3(256), 0, s, b, grp, m0, gt, gm);
             if (dW) {
-                k_bwd_im2col<<<dim3(tblocks, tcols), 256, 0, s>>>(b, grp, m0, at);
+                launch_pdl(k_bwd_im2col, dim3(tblocks, tcols), dim3(256), 0, s, b, grp, m0, at);
                 // split z: dws[z][i][j] (+)= sum over its pixels m of gt[i][m] * at[j][m]
                 st = launch_gemm(gt, at, dws, b.fr, b.k_pad, b.mc, b.k_pad, wbn, m0 > 0, s, wsplit,
                                  (long long)b.fr * b.k_pad);
@@ -410,12 +421,13 @@ sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const vo
                 // dat[j][m] = sum_i wpt[j][i] * gm[m][i]
                 st = launch_gemm(wpt, gm, dat, b.kr, b.mc, b.fk, b.mc, pick_bn(b.mc), false, s);
                 if (st == SADMM_OK)
-                    k_bwd_col2im<<<dim3(tblocks, tcols), 256, 0, s>>>(b, grp, m0, dat, dx);
+                    launch_pdl(k_bwd_col2im, dim3(tblocks, tcols), dim3(256), 0, s, b, grp, m0,
+                               static_cast<const float*>(dat), dx);
             }
         }
         if (dW && st == SADMM_OK)
-            k_bwd_reduce_dw<<<dim3((unsigned)((b.k_pad + 255) / 256), (unsigned)b.n_pad), 256, 0, s>>>(b, grp, dws,
-                                                                                                    wsplit, dW);
+            launch_pdl(k_bwd_reduce_dw, dim3((unsigned)((b.k_pad + 255) / 256), (unsigned)b.n_pad), dim3(256), 0, s, b,
+                       grp, static_cast<const float*>(dws), wsplit, dW);
     }
     if (st != SADMM_OK) return st;
     return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;

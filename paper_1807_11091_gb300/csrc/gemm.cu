@@ -69,6 +69,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         tmem_alloc(tmem_holder, (uint32_t)a.tmem_cols);
         tmem_relinquish();
     }
+    pdl_wait();  // nothing above reads global memory
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -206,7 +207,7 @@ sadmm_status launch_gemm(const void* A, const void* B, float* C, long long M, lo
         configured_dev = dev;
     }
     const dim3 grid((unsigned)(M / 128), (unsigned)(N / bn), (unsigned)splits);
-    k_gemm<<<grid, kGemmThreads, smem, s>>>(ta, tb, a);
+    if (launch_pdl(k_gemm, grid, dim3(kGemmThreads), smem, s, ta, tb, a) != cudaSuccess) return SADMM_ECUDA;
     return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
 }
 
