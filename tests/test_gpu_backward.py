@@ -105,3 +105,61 @@ def test_backward_without_relu():
     (dW, db, dx), (rdW, rdb, rdx), _, _ = _backward(s, t, kf, ck, kc, relu=False)
     assert_close(dW, rdW, what="no relu dW")
     assert_close(dx, rdx, what="no relu dx")
+
+
+def test_backward_several_pixel_chunks():
+    """41772 output pixels: two chunks of the backward (32768 + a ragged 9004),
+    so the weight gradient accumulates per pixel split across chunks."""
+    s = ConvShape(n=3, c=6, h=120, w=120, f=24, kh=3, kw=3)
+    kf, kc = wl.retained(0.75, s.f), wl.retained(0.6, s.k)
+    assert s.n * s.oh * s.ow > 32768
+    t = wl.gen_tensors(s, seed=21)
+    (dW, db, dx), (rdW, rdb, rdx), rows, cols = _backward(s, t, kf, wl.COL_SHAPE, kc)
+    assert_close(dW, rdW, what="two chunks dW")
+    assert_close(db, rdb, what="two chunks db")
+    assert_close(dx, rdx, what="two chunks dx")
+
+
+def _raw_backward(pc, x, dy, y, want_dw, want_dx):
+    from paper_1807_11091_gb300 import sadmm
+    dev = x.device
+    s_f, K = pc.plan.desc.f, (pc.plan.desc.c // pc.plan.desc.groups) * pc.plan.desc.kt * pc.plan.desc.kh * pc.plan.desc.kw
+    dW = torch.full((s_f, K), float("nan"), device=dev) if want_dw else None
+    db = torch.full((s_f,), float("nan"), device=dev) if want_dw else None
+    dx = torch.full(x.shape, float("nan"), device=dev) if want_dx else None
+    ws_bytes = sadmm.sadmm_conv_bwd_workspace_size(pc.plan)
+    ws = torch.empty(ws_bytes + 1024, dtype=torch.uint8, device=dev)
+    wptr = (ws.data_ptr() + 1023) // 1024 * 1024
+    st = sadmm.sadmm_conv_bwd(pc.plan, x.data_ptr(), dy.data_ptr(), y.data_ptr(), sadmm.SADMM_FP32, 1,
+                              dW.data_ptr() if dW is not None else None, db.data_ptr() if db is not None else None,
+                              dx.data_ptr() if dx is not None else None, wptr, ws_bytes,
+                              int(torch.cuda.current_stream().cuda_stream))
+    assert st == 0 and sadmm.device_status() == 0
+    return dW, db, dx
+
+
+def test_backward_weight_gradient_deterministic_and_partial_calls():
+    """dW and db come out bit-identical on every call (fixed-order sums); a call
+    that asks for the weight gradient only, or the input gradient only, gives
+    what the full call gives (dx up to its atomic summation order)."""
+    from paper_1807_11091_gb300 import sadmm
+    name, s, ff, ck, cf = CASES[1]
+    kf, kc = wl.retained(ff, s.f), wl.retained(cf, s.k)
+    t = wl.gen_tensors(s, seed=31)
+    dev = torch.device("cuda", 0)
+    rows, cols, _, _ = oracle.project(t["W"], s.taps, kf, ck, kc)
+    W, x = t["W"].to(dev), t["x"].to(dev)
+    fi = torch.as_tensor(rows, dtype=torch.int32, device=dev)
+    ci = torch.as_tensor(cols, dtype=torch.int32, device=dev)
+    pc = sadmm.PrunedConv(s.desc16(), W, fi, ck, ci, kf, kc)
+    y = pc.forward(x, t["bias"].to(dev))
+    g = torch.Generator().manual_seed(7)
+    dy = torch.randn(y.shape, generator=g).to(torch.bfloat16).to(dev)
+    dW1, db1, dx1 = _raw_backward(pc, x, dy, y, True, True)
+    dW2, db2, dx2 = _raw_backward(pc, x, dy, y, True, True)
+    assert torch.equal(dW1, dW2) and torch.equal(db1, db2)
+    dW3, db3, none = _raw_backward(pc, x, dy, y, True, False)
+    assert none is None and torch.equal(dW1, dW3) and torch.equal(db1, db3)
+    none, _, dx4 = _raw_backward(pc, x, dy, y, False, True)
+    assert torch.isfinite(dx4).all()
+    assert_close(dx4.cpu().numpy(), dx1.cpu().double().numpy(), tol=1e-6, what="dx alone")
