@@ -217,7 +217,8 @@ sadmm_status sadmm_admm_update_elements(const sadmm_conv_desc* d, const void* W,
  *
  * Small batches (the paper times batch 1, Sec. 5): when the layer has fewer
  * output tiles (128 pixels x one filter tile of one conv group) than the
- * current device has SMs, K' is split over plan->splits CTAs per tile; each
+ * current device has SMs, K' is split over plan->splits CTAs per tile (at
+ * least two 64-column stages per split when K' has at most eight); each
  * writes fp32 partial sums to a region of the plan's device buffer and a
  * second kernel adds them in split order, then applies bias and ReLU.  The
  * split depends on the current device's SM count and is fixed in the plan.

@@ -299,7 +299,11 @@ sadmm_status sadmm_plan_init_ctas(sadmm_plan* plan, const sadmm_conv_desc* d, in
         if (units < sms && nks >= 2 && rows <= 65535) {
             long long want = (sms + units - 1) / units;
             if (want > nks) want = nks;
-            const long long ksps = (nks + want - 1) / want;
+            long long ksps = (nks + want - 1) / want;
+            // a split of a short K' (at most 8 stages) carries at least two
+            // stages: a one-stage split pays a whole prologue and a partial-sum
+            // round trip for one stage of work (measured slower on GB300)
+            if (nks <= 8 && ksps < 2) ksps = 2;
             const long long splits = (nks + ksps - 1) / ksps;
             const long long bytes = splits * g.groups * p.n_pad * m_tiles * 128 * 4;
             if (splits > 1 && bytes <= (256ll << 20)) {
