@@ -23,7 +23,10 @@
  *    never allocates device memory and never synchronises the stream, except
  *    sadmm_last_device_status, which synchronises to read the device flag.
  *  - `stream` is a cudaStream_t (NULL = legacy default stream).  All work is
- *    enqueued on it, in order, asynchronously.
+ *    enqueued on it, in order, asynchronously.  The kernels are launched with
+ *    programmatic stream serialization: one may be scheduled while the kernel
+ *    before it on the stream finishes, and it waits for that kernel to complete
+ *    before it reads or writes global memory, so stream order is kept.
  *  - Arguments are validated on the host before any launch; a bad argument
  *    returns SADMM_EINVAL and enqueues nothing.  A failed launch returns
  *    SADMM_ECUDA.  Shapes the kernels do not support (see each call) return
