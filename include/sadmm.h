@@ -45,7 +45,7 @@
 extern "C" {
 #endif
 
-#define SADMM_ABI_VERSION 4
+#define SADMM_ABI_VERSION 5
 
 /* Bytes of the fixed device array of sadmm_project_groups_noalloc. */
 #define SADMM_NOALLOC_SCRATCH_BYTES (256 * 1024)
@@ -102,7 +102,22 @@ typedef struct {
     int sk_len;         /* stream-K: 64-column stages per CTA (0: whole tiles)  */
     int sk_grid;        /* stream-K: CTAs launched                              */
     int ctas;           /* CTAs a forward launches at most (one per SM)         */
-    uint64_t tmap[16];/* 128-byte TMA tensor map of the packed matrix         */
+    /* Input-slab forward (xs_mode = 1, see sadmm_plan_init): geometry of the
+     * space-to-depth input and of the slab one 128-row tile reads. */
+    int xs_mode;        /* 1: the forward runs the slab path                    */
+    int xs_r, xs_q;     /* block taps: ceil(KH / sh), ceil(KW / sw)             */
+    int xs_cs;          /* slab channels: kept channels * sh * sw, to 16        */
+    int xs_hb, xs_wb;   /* block rows / columns: OH + xs_r - 1, OW + xs_q - 1   */
+    int xs_pimg;        /* block pixels per image and chunk: xs_hb*xs_wb, to 8  */
+    int xs_sp;          /* slab pixels of a tile: 128 + (xs_r-1)*xs_wb + xs_q-1, to 8 */
+    int xs_kpad;        /* slab GEMM columns xs_r*xs_q*xs_cs, rounded up to 64  */
+    size_t off_xs;      /* space-to-depth input [N][xs_cs/8][xs_pimg][8] bf16   */
+    size_t off_wps;     /* slab-ordered packed weights [bn][xs_kpad] bf16       */
+    size_t off_scol;    /* slab column -> GEMM column (-1: zero) [xs_kpad] int32,
+                           then the kept input channels [xs_cs] int32          */
+    uint64_t tmap[16];    /* 128-byte TMA tensor map of the packed matrix       */
+    uint64_t tmap_ws[16]; /* TMA map of the slab-ordered weights (xs_mode)      */
+    uint64_t tmap_xs[16]; /* TMA map of the space-to-depth input (xs_mode)      */
 } sadmm_plan;
 
 /* ------------------------------------------------------------------------ */
@@ -238,6 +253,26 @@ sadmm_status sadmm_admm_update_elements(const sadmm_conv_desc* d, const void* W,
  * it is, and it adds the two halves in K' order, then bias and ReLU.  After a
  * device-side failure (sadmm_last_device_status) the plan must be packed again.
  */
+/*
+ * Input-slab path (plan->xs_mode = 1): a 2-D layer with one conv group, at
+ * most 256 kept filters and every column of its kept channels kept (no
+ * column pruning, or whole channels pruned), whose kept channels times
+ * sh * sw come to at most 64, and whose slab GEMM is at most twice as wide
+ * as K' -- the first layer of a network, typically (the paper keeps AlexNet's
+ * CONV1 whole).  The forward then first rewrites x as a space-to-depth copy
+ * in the plan's buffer: block pixel (hb, wb) holds, for each kept channel c
+ * and phase (a, b) < (sh, sw), the input x[c][hb*sh + a - ph][wb*sw + b - pw]
+ * (zero outside), which turns the strided KH x KW conv into a stride-1
+ * xs_r x xs_q conv over xs_cs channels.  A tile of 128 consecutive block
+ * pixels of one image (output rows of xs_wb pixels, the last xs_q - 1 of
+ * each discarded) reads one contiguous slab of block pixels, loaded once into
+ * shared memory; each block tap (r, q) is the slab shifted by r * xs_wb + q
+ * pixels, fed to the tensor cores directly (the pixels on the MMA's M side,
+ * the kept filters on its N side), so no im2col copy is built.  The
+ * slab GEMM has xs_r * xs_q * xs_cs columns (the taps and channels past the
+ * kernel or the kept channels hold zero weights): the same sums as the
+ * gathered path, in another order.  No K' split or stream-K in this path.
+ */
 sadmm_status sadmm_plan_init(sadmm_plan* plan, const sadmm_conv_desc* d,
                              int n_filt, int colkind, int n_colgroups);
 
@@ -265,8 +300,10 @@ sadmm_status sadmm_plan_init_ctas(sadmm_plan* plan, const sadmm_conv_desc* d,
  *             (shape) or channels in [0,Cg) (channel); NULL for COL_NONE.
  *   dev       device buffer of >= plan->dev_bytes bytes, 256-byte aligned;
  *             becomes plan->dev.
- * Writes the TMA descriptor of Wp into plan->tmap.  Index lists that are not
- * ascending or out of range give undefined (but in-bounds) plans.
+ * Writes the TMA descriptor of Wp into plan->tmap.  For a slab plan it also
+ * packs the weights in slab column order (plan->off_wps, plan->tmap_ws) and
+ * writes the TMA map of the space-to-depth input (plan->tmap_xs).  Index lists
+ * that are not ascending or out of range give undefined (but in-bounds) plans.
  */
 sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt,
                         const int* filt_idx, const int* col_idx,
@@ -287,8 +324,9 @@ sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt,
  *         to nearest even); every element is written.
  * Requires sm_100-family tensor cores (SADMM_EUNSUPPORTED otherwise) and
  * N*C*T*H*W < 2^31.  Launches that use one plan must not overlap on the GPU
- * (stream-ordered is fine): split-K partial sums and stream-K arrival
- * counters live in the plan's buffer.
+ * (stream-ordered is fine): split-K partial sums, stream-K arrival
+ * counters and the slab path's space-to-depth input live in the plan's
+ * buffer.
  */
 sadmm_status sadmm_conv_fwd(const sadmm_plan* plan, const void* x, const float* bias,
                             int relu, void* y, int ydt, void* stream);

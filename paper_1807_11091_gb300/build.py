@@ -21,7 +21,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libsadmm.so")
 
-SOURCES = ["abi.cu", "project.cu", "pack.cu", "conv_fwd.cu", "admm.cu", "elements.cu", "gemm.cu", "bwd.cu"]
+SOURCES = ["abi.cu", "project.cu", "pack.cu", "conv_fwd.cu", "conv_slab.cu", "admm.cu", "elements.cu", "gemm.cu",
+           "bwd.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

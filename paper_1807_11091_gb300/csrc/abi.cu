@@ -286,10 +286,39 @@ sadmm_status sadmm_plan_init_ctas(sadmm_plan* plan, const sadmm_conv_desc* d, in
     p.off_rowmap = take((size_t)g.groups * p.n_pad * 4);
     p.off_zeromap = take((size_t)g.f * 4);
     p.off_counts = take((size_t)g.groups * 2 * 4);
-    // split K' when the layer has fewer output tiles than the device has SMs
     p.splits = 1;
     p.stages_per_split = p.k_pad / 64;
-    {
+    // input-slab path: one conv group, every column of the kept channels kept,
+    // few slab channels, one filter tile, and a slab GEMM at most twice as wide
+    const bool cols_whole = colkind == SADMM_COL_NONE || colkind == SADMM_COL_CHANNEL ||
+                            (colkind == SADMM_COL_SHAPE && n_cols == g.k);
+    if (g.t == 1 && g.kt == 1 && g.groups == 1 && p.n_tiles == 1 && cols_whole && n_cols > 0) {
+        const long long nck = colkind == SADMM_COL_CHANNEL ? n_colgroups : g.c;
+        const long long R = (g.kh + g.sh - 1) / g.sh, Q = (g.kw + g.sw - 1) / g.sw;
+        const long long cs = round_up(nck * g.sh * g.sw, 16);
+        const long long hb = g.oh + R - 1, wb = g.ow + Q - 1;
+        const long long pimg = round_up(hb * wb, 8);
+        const long long sp = round_up(128 + (R - 1) * wb + (Q - 1), 8);
+        const long long kpad_s = round_up(R * Q * cs, 64);
+        const long long xs_bytes = g.n * cs * pimg * 2;
+        if (cs <= 64 && sp / 8 <= 256 && kpad_s <= 2 * p.k_pad && pimg < (1ll << 28) && hb <= 65535 && g.n <= 65535 &&
+            xs_bytes <= (4ll << 30) && slab_stages(p.bn, (int)kpad_s, (int)cs, (int)sp) >= 2) {
+            p.xs_mode = 1;
+            p.xs_r = (int)R;
+            p.xs_q = (int)Q;
+            p.xs_cs = (int)cs;
+            p.xs_hb = (int)hb;
+            p.xs_wb = (int)wb;
+            p.xs_pimg = (int)pimg;
+            p.xs_sp = (int)sp;
+            p.xs_kpad = (int)kpad_s;
+            p.off_xs = take((size_t)xs_bytes);
+            p.off_wps = take((size_t)p.bn * kpad_s * 2);
+            p.off_scol = take((size_t)(kpad_s + cs) * 4);
+        }
+    }
+    // split K' when the layer has fewer output tiles than the device has SMs
+    if (!p.xs_mode) {
         const long long nks = p.k_pad / 64;
         const long long m_tiles = (g.m + 127) / 128;
         const long long upairs = (p.n_tiles + (p.n_tiles >= 2 ? 1 : 0)) / (p.n_tiles >= 2 ? 2 : 1);

@@ -197,6 +197,17 @@ SADMM_DEV void tma_load_2d(void* dst, const void* tmap, uint64_t* bar, int c0, i
         : "memory");
 }
 
+// 4-D tiled TMA load (coordinates innermost first); completion as for
+// tma_load_2d.
+SADMM_DEV void tma_load_4d(void* dst, const void* tmap, uint64_t* bar, int c0, int c1, int c2, int c3)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(smem_u32(dst)),
+        "l"(tmap), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+        : "memory");
+}
+
 SADMM_DEV void tma_prefetch_desc(const void* tmap)
 {
     asm volatile("prefetch.tensormap [%0];" ::"l"(tmap) : "memory");
@@ -305,6 +316,20 @@ SADMM_DEV uint64_t sdesc_kmajor_sw128(uint32_t saddr)
     d |= (uint64_t)1 << 46;                     // descriptor version for tcgen05
     d |= (uint64_t)2 << 61;                     // layout: 128-byte swizzle
     return d;
+}
+
+// Shared-memory descriptor of a K-major operand without swizzle: core
+// matrices of 8 rows x 16 bytes (rows 16 bytes apart), `lbo` bytes between
+// core matrices adjacent along K and `sbo` bytes between adjacent groups of 8
+// rows.  The start address needs 16-byte alignment only.
+SADMM_DEV uint64_t sdesc_kmajor_none(uint32_t saddr, uint32_t lbo, uint32_t sbo)
+{
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);       // start address, bits [0,14)
+    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;    // leading byte offset, bits [16,30)
+    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;    // stride byte offset, bits [32,46)
+    d |= (uint64_t)1 << 46;                         // descriptor version for tcgen05
+    return d;                                       // layout 0: no swizzle
 }
 
 // Instruction descriptor of tcgen05.mma kind::f16: bf16 A and B, both

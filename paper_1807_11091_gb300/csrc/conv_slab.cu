@@ -1,0 +1,404 @@
+// conv_slab.cu -- the input-slab forward of a pruned CONV layer whose kept
+// channels keep every column (Sec. 3: the pruned layer is a smaller full GEMM;
+// here the layers with no column pruning, or whole channels pruned, and few
+// input channels -- a network's first layer, which the paper keeps whole).
+//
+// k_slab_input rewrites x as a space-to-depth copy xs[n][chunk][pixel][8]:
+// block pixel (hb, wb) of image n holds, for kept channel ci and phase
+// (a, b) < (sh, sw), slab channel cc = (ci*sh + a)*sw + b (8 per chunk) =
+// x[n][chan[ci]][hb*sh + a - ph][wb*sw + b - pw], zero outside.  Output pixel
+// (oh, ow) and kernel tap (kh, kw) = (r*sh + a, q*sw + b) read block pixel
+// (oh + r, ow + q), phase (a, b): the layer becomes a stride-1 R x Q conv over
+// cs slab channels (R = ceil(KH/sh), Q = ceil(KW/sw)).
+//
+// k_conv_slab: GEMM row i of tile t of image n is block pixel p = 128t + i of
+// that image's output grid laid out in rows of Wb = OW + Q - 1 block pixels
+// (row oh = p / Wb, column ow = p % Wb; columns past OW and rows past OH are
+// computed and dropped).  Block tap (r, q) of row i reads block pixel
+// p + r*Wb + q, so a tile needs the sp = 128 + (R-1)*Wb + Q-1 consecutive
+// block pixels from 128t on -- its slab, one TMA box of every chunk,
+// [chunk][pixel][8 channels] in shared memory.  The A operand of tap (r, q)
+// is that slab shifted by r*Wb + q pixels: K-major core matrices of 8 pixels
+// x 8 channels (16-byte rows), no swizzle, so any pixel offset is a valid
+// start.  B (the kept filters' weights in slab column order, tap-major) stays
+// resident in shared memory, 128-byte swizzled.
+//   warp 0      TMA: the weights once, then one slab per tile
+//   warp 1      TMEM allocator and MMA issuer (R*Q*cs/16 MMAs of
+//               128 x bn x 16 per tile, fp32 accumulator in TMEM, two sets)
+//   warps 2-9   epilogue: tcgen05.ld (lane = GEMM row), bias, ReLU, stores
+//               to the NCHW output, zero planes of the pruned filters
+#include <cuda.h>
+#include <string.h>
+
+#include "common.cuh"
+#include "conv_common.cuh"
+#include "internal.h"
+
+namespace sadmm {
+namespace {
+
+constexpr int kSlabWarps = 10;
+constexpr int kSlabThreads = kSlabWarps * 32;
+constexpr int kSlabEpiWarps = 8;        // warps 2..9: two per TMEM lane quadrant (warp % 4)
+constexpr int kMaxSlabStages = 4;
+constexpr int kSlabTables = 2 * 256 * 4;  // plane offset and bias of each kept row
+constexpr int kSlabBars = 256;            // barriers, TMEM address, abort flag
+constexpr int kSlabSmemLimit = 232448;
+
+struct SlabArgs {
+    void* y;
+    const float* bias;
+    const int* rowmap;   // packed row -> filter (-1: padding)
+    const int* zeromap;  // pruned filters, ascending
+    const int* counts;   // [kept, pruned]
+    int* status;
+    int F, OH, OW, plane;
+    int Wb, MT, units;     // block-pixel row width, tiles per image, tiles in all
+    FastDiv mt_div, wb_div;
+    int sp, R, Q, ksteps;  // slab pixels, block taps, MMAs of 16 columns per tap
+    int bn, nbox;          // MMA N, 64-column weight boxes
+    int stages, stage_bytes, stage_stride;
+    int tmem_stride, tmem_cols;
+    int relu;
+};
+
+struct XsArgs {
+    int C, H, W, sh, sw, ph, pw;
+    int nck, cs, Wb, pimg;
+};
+
+// Thread (tx, ty) of block (bw, hb, n) writes the 16-byte vectors (8 slab
+// channels) of chunks ty, ty + 4, ... of block pixel wb = 64*bw + tx in block
+// row hb of image n.  Its 8 input loads are independent (all in flight); the
+// channel and phase of each slab channel come from a table decoded once per
+// block in shared memory.
+constexpr int kXsPix = 64;     // block pixels per block (threadIdx.x)
+constexpr int kXsChunkRows = 4;  // chunks in flight per block (threadIdx.y)
+__global__ void __launch_bounds__(kXsPix * kXsChunkRows) k_slab_input(const __nv_bfloat16* __restrict__ x,
+                                                                      const int* __restrict__ chan, const XsArgs b,
+                                                                      __nv_bfloat16* __restrict__ xs)
+{
+    __shared__ int4 s_dec[64];  // per slab channel: {channel plane offset (-1: zero), a - ph, b - pw, 0}
+    pdl_wait();  // after the kernel before it in the stream
+    const int hb = blockIdx.y, n = blockIdx.z;
+    const int tid = threadIdx.y * kXsPix + threadIdx.x;
+    if (tid < b.cs) {
+        const int cc = tid;
+        const int ci = cc / (b.sh * b.sw);
+        const int ch = ci < b.nck ? __ldg(chan + ci) : -1;
+        s_dec[cc] = make_int4(ch >= 0 ? ch * b.H * b.W : -1, (cc / b.sw) % b.sh - b.ph, cc % b.sw - b.pw, 0);
+    }
+    __syncthreads();
+    const int wb = blockIdx.x * kXsPix + threadIdx.x;
+    if (wb >= b.Wb) return;
+    const unsigned short* xi = reinterpret_cast<const unsigned short*>(x) + (long long)n * b.C * b.H * b.W;
+    const int ih0 = hb * b.sh, iw0 = wb * b.sw;
+    const int chunks = b.cs / 8;
+    for (int k = threadIdx.y; k < chunks; k += kXsChunkRows) {
+        uint32_t h[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int4 d = s_dec[8 * k + e];
+            const int ih = ih0 + d.y, iw = iw0 + d.z;
+            h[e] = (d.x >= 0 && (unsigned)ih < (unsigned)b.H && (unsigned)iw < (unsigned)b.W)
+                       ? (uint32_t)__ldg(xi + d.x + ih * b.W + iw)
+                       : 0u;
+        }
+        uint4* dst = reinterpret_cast<uint4*>(xs + (((long long)n * chunks + k) * b.pimg + (long long)hb * b.Wb + wb) * 8);
+        *dst = make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16), h[6] | (h[7] << 16));
+    }
+}
+
+template <bool OUT_BF16>
+__global__ void __launch_bounds__(kSlabThreads, 1)
+    k_conv_slab(const __grid_constant__ CUtensorMap tw, const __grid_constant__ CUtensorMap tx,
+                const __grid_constant__ SlabArgs a)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const uint32_t bbox = (uint32_t)a.bn * 128u;  // one 64-column box of the weights
+    uint8_t* sB = smem;
+    uint8_t* sA = sB + (size_t)a.nbox * bbox;  // 1024-aligned: bbox is a multiple of 2048
+    int* t_off = reinterpret_cast<int*>(sA + (size_t)a.stages * a.stage_stride);
+    float* t_bias = reinterpret_cast<float*>(t_off + 256);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(t_bias + 256);
+    uint64_t* full = bars;
+    uint64_t* empty = bars + kMaxSlabStages;
+    uint64_t* acc_full = bars + 2 * kMaxSlabStages;
+    uint64_t* acc_empty = acc_full + 2;
+    uint64_t* b_full = acc_empty + 2;
+    uint64_t* drain = b_full + 1;
+    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kMaxSlabStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], kSlabEpiWarps);
+        }
+        mbar_init(b_full, 1);
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_holder, (uint32_t)a.tmem_cols);
+        tmem_relinquish();
+    }
+    // Nothing above reads global memory: it overlaps the previous kernel's tail.
+    pdl_wait();
+    pdl_trigger();
+    for (int i = threadIdx.x; i < a.bn; i += blockDim.x) {
+        const int f = __ldg(a.rowmap + i);
+        t_off[i] = f >= 0 ? f * a.plane : 0;
+        t_bias[i] = (f >= 0 && a.bias) ? __ldg(a.bias + f) : 0.0f;
+    }
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(&tw);
+        tma_prefetch_desc(&tx);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_holder;
+
+    if (warp == 0) {
+        // ------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            mbar_arrive_expect_tx(b_full, bbox * (uint32_t)a.nbox);
+            for (int i = 0; i < a.nbox; ++i) tma_load_2d(sB + (size_t)i * bbox, &tw, b_full, i * 64, 0);
+            int s = 0;
+            uint32_t ph = 0;
+            uint32_t issued_parity[kMaxSlabStages];
+            uint32_t issued_mask = 0;
+            for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
+                const int n = (int)fdiv((uint32_t)u, a.mt_div);
+                const int t = u - n * a.MT;
+                if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, a.status)) break;
+                mbar_arrive_expect_tx(&full[s], (uint32_t)a.stage_bytes);
+                // the tile's slab: block pixels 128t .. 128t+sp-1 (octets 16t ..), every chunk
+                tma_load_4d(sA + (size_t)s * a.stage_stride, &tx, &full[s], 0, t * 16, 0, n);
+                issued_parity[s] = ph;
+                issued_mask |= 1u << s;
+                if (++s == a.stages) { s = 0; ph ^= 1u; }
+            }
+            // every copy this thread issued has landed before the CTA retires
+            for (int q = 0; q < a.stages; ++q) {
+                if (!(issued_mask & (1u << q))) continue;
+                const unsigned long long t0 = globaltimer();
+                while (!mbar_try_wait(&full[q], issued_parity[q]) && globaltimer() - t0 < kWaitLimitNs) {}
+            }
+            const unsigned long long t0 = globaltimer();
+            while (!mbar_try_wait(b_full, 0) && globaltimer() - t0 < kWaitLimitNs) {}
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ------------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            bool ok = mbar_wait(b_full, 0, abort_flag, a.status);
+            const uint32_t idesc = idesc_bf16_f32(128, a.bn);
+            const uint32_t lbo = (uint32_t)a.sp * 16u;  // next chunk (8 channels further along K)
+            const uint32_t sB0 = smem_u32(sB);
+            int s = 0, ab = 0;
+            uint32_t ph = 0, acc_ph = 0;
+            for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
+                if (!mbar_wait(&acc_empty[ab], acc_ph ^ 1u, abort_flag, a.status)) break;
+                tc_fence_after();
+                if (!mbar_wait(&full[s], ph, abort_flag, a.status)) break;
+                tc_fence_after();
+                const uint32_t d = tmem_base + (uint32_t)(ab * a.tmem_stride);
+                const uint32_t a0 = smem_u32(sA + (size_t)s * a.stage_stride);
+                int step = 0;
+                for (int r = 0; r < a.R; ++r) {
+                    for (int q = 0; q < a.Q; ++q) {
+                        const uint32_t at = a0 + (uint32_t)(r * a.Wb + q) * 16u;
+                        for (int j = 0; j < a.ksteps; ++j, ++step) {
+                            const uint64_t adesc = sdesc_kmajor_none(at + 2u * (uint32_t)j * lbo, lbo, 128u);
+                            const uint64_t bdesc =
+                                sdesc_kmajor_sw128(sB0 + (uint32_t)(step >> 2) * bbox + (uint32_t)(step & 3) * 32u);
+                            mma_bf16_ss(d, adesc, bdesc, idesc, step > 0 ? 1u : 0u);
+                        }
+                    }
+                }
+                mma_commit(&empty[s]);
+                mma_commit(&acc_full[ab]);
+                if (++s == a.stages) { s = 0; ph ^= 1u; }
+                if (++ab == 2) { ab = 0; acc_ph ^= 1u; }
+            }
+            // Every MMA this thread issued has completed before TMEM is freed.
+            mma_commit(drain);
+            const unsigned long long t0 = globaltimer();
+            while (!mbar_try_wait(drain, 0) && globaltimer() - t0 < kWaitLimitNs) {}
+        }
+        __syncwarp();
+    } else {
+        // --------------------------------------------------------- epilogue
+        const int q = warp & 3;          // TMEM lane quadrant this warp may access
+        const int h = (warp - 2) >> 2;   // which of the quadrant's two warps
+        const int row = q * 32 + lane;
+        const int kept = __ldg(a.counts), pruned = __ldg(a.counts + 1);
+        const int nch = (kept + kEpiCols - 1) / kEpiCols;
+        int ab = 0;
+        uint32_t acc_ph = 0;
+        bool alive = true;
+        for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
+            const int n = (int)fdiv((uint32_t)u, a.mt_div);
+            const int t = u - n * a.MT;
+            const int p = t * 128 + row;
+            const int oh = (int)fdiv((uint32_t)p, a.wb_div);
+            const int ow = p - oh * a.Wb;
+            const bool valid = oh < a.OH && ow < a.OW;
+            const long long pix = (long long)n * a.F * a.plane + (long long)oh * a.OW + ow;
+            float* yf = reinterpret_cast<float*>(a.y) + pix;
+            __nv_bfloat16* yh = reinterpret_cast<__nv_bfloat16*>(a.y) + pix;
+            // pruned filters' planes: zero, while the tile's MMAs run
+            if (alive && valid) {
+                for (int z = h; z < pruned; z += 2) {
+                    const long long off = (long long)__ldg(a.zeromap + z) * a.plane;
+                    if (OUT_BF16)
+                        yh[off] = __float2bfloat16_rn(0.0f);
+                    else
+                        __stcs(yf + off, 0.0f);
+                }
+            }
+            // warp-uniform outcome: the TMEM loads below are .sync.aligned
+            if (alive && !__all_sync(0xffffffffu, mbar_wait(&acc_full[ab], acc_ph, abort_flag, a.status)))
+                alive = false;
+            if (alive) {
+                tc_fence_after();
+                const uint32_t taddr = tmem_base + (uint32_t)(ab * a.tmem_stride) + ((uint32_t)(q * 32) << 16);
+                for (int k = h; k < nch; k += 2) {
+                    const int c0 = k * kEpiCols;
+                    uint32_t r[kEpiCols];
+                    tmem_ld_32x32b_x16(taddr + (uint32_t)c0, r);
+                    tmem_ld_wait();
+                    float v[kEpiCols];
+#pragma unroll
+                    for (int j = 0; j < kEpiCols; ++j) v[j] = __uint_as_float(r[j]);
+                    if (valid) store_cols<OUT_BF16>(v, c0, kept, t_off, t_bias, a.relu, yf, yh);
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&acc_empty[ab]);
+            }
+            if (++ab == 2) { ab = 0; acc_ph ^= 1u; }
+        }
+    }
+
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, (uint32_t)a.tmem_cols);
+    }
+}
+
+int slab_fixed_bytes(int bn, int kpad_s) { return 1024 + (kpad_s / 64) * bn * 128 + kSlabTables + kSlabBars; }
+int slab_stage_stride(int cs, int sp) { return (int)round_up((long long)cs * sp * 2, 1024); }
+
+template <bool OUT_BF16>
+cudaError_t launch_slab(const CUtensorMap& tw, const CUtensorMap& tx, const SlabArgs& a, int grid, size_t smem,
+                        cudaStream_t s)
+{
+    auto kern = k_conv_slab<OUT_BF16>;
+    static int configured_dev = -1;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (configured_dev != dev) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSlabSmemLimit);
+        if (e != cudaSuccess) return e;
+        configured_dev = dev;
+    }
+    return launch_pdl(kern, dim3((unsigned)grid), dim3(kSlabThreads), smem, s, tw, tx, a);
+}
+
+}  // namespace
+
+int slab_stages(int bn, int kpad_s, int cs, int sp)
+{
+    if (bn < 16 || bn > 256 || bn % 16 || kpad_s % 64 || cs % 16 || sp % 8) return 0;
+    const long long room = (long long)kSlabSmemLimit - slab_fixed_bytes(bn, kpad_s);
+    if (room <= 0) return 0;
+    const long long st = room / slab_stage_stride(cs, sp);
+    return (int)(st > kMaxSlabStages ? kMaxSlabStages : st);
+}
+
+sadmm_status launch_conv_slab(const sadmm_plan* plan, const Geometry& g, const void* x, const float* bias, int relu,
+                              void* y, int ydt, cudaStream_t s)
+{
+    const int stages = slab_stages(plan->bn, plan->xs_kpad, plan->xs_cs, plan->xs_sp);
+    if (stages < 2 || plan->n_tiles != 1 || g.groups != 1 || plan->xs_cs > 64 || plan->xs_cs % 16 ||
+        (long long)(plan->colkind == SADMM_COL_CHANNEL ? plan->n_colgroups : g.c) * g.sh * g.sw > plan->xs_cs)
+        return SADMM_EINVAL;  // not a slab plan
+    const char* base = static_cast<const char*>(plan->dev);
+    const long long mt = ((long long)g.oh * plan->xs_wb + 127) / 128;
+    const long long units = g.n * mt;
+    if (units >= (1ll << 31) - (1ll << 20) || (long long)plan->xs_hb * plan->xs_wb >= (1ll << 31) - 256)
+        return SADMM_EUNSUPPORTED;
+    XsArgs b;
+    b.C = (int)g.c;
+    b.H = (int)g.h;
+    b.W = (int)g.w;
+    b.sh = (int)g.sh;
+    b.sw = (int)g.sw;
+    b.ph = (int)g.ph;
+    b.pw = (int)g.pw;
+    b.nck = plan->colkind == SADMM_COL_CHANNEL ? plan->n_colgroups : (int)g.c;
+    b.cs = plan->xs_cs;
+    b.Wb = plan->xs_wb;
+    b.pimg = plan->xs_pimg;
+    const int* chan = reinterpret_cast<const int*>(base + plan->off_scol) + plan->xs_kpad;
+    __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(const_cast<char*>(base) + plan->off_xs);
+    if (launch_pdl(k_slab_input,
+                   dim3((unsigned)((plan->xs_wb + kXsPix - 1) / kXsPix), (unsigned)plan->xs_hb, (unsigned)g.n),
+                   dim3(kXsPix, kXsChunkRows), 0, s, static_cast<const __nv_bfloat16*>(x), chan, b, xs) != cudaSuccess)
+        return SADMM_ECUDA;
+
+    SlabArgs a;
+    memset(&a, 0, sizeof(a));
+    a.y = y;
+    a.bias = bias;
+    a.rowmap = reinterpret_cast<const int*>(base + plan->off_rowmap);
+    a.zeromap = reinterpret_cast<const int*>(base + plan->off_zeromap);
+    a.counts = reinterpret_cast<const int*>(base + plan->off_counts);
+    a.status = device_status_ptr();
+    a.F = (int)g.f;
+    a.OH = (int)g.oh;
+    a.OW = (int)g.ow;
+    a.plane = (int)g.plane;
+    a.Wb = plan->xs_wb;
+    a.MT = (int)mt;
+    a.units = (int)units;
+    a.mt_div = make_fastdiv((uint32_t)mt);
+    a.wb_div = make_fastdiv((uint32_t)plan->xs_wb);
+    a.sp = plan->xs_sp;
+    a.R = plan->xs_r;
+    a.Q = plan->xs_q;
+    a.ksteps = plan->xs_cs / 16;
+    a.bn = plan->bn;
+    a.nbox = plan->xs_kpad / 64;
+    a.stages = stages;
+    a.stage_bytes = plan->xs_cs * plan->xs_sp * 2;
+    a.stage_stride = slab_stage_stride(plan->xs_cs, plan->xs_sp);
+    a.tmem_stride = (int)round_up(plan->bn, 32);
+    int cols = 32;
+    while (cols < 2 * a.tmem_stride) cols <<= 1;
+    a.tmem_cols = cols;
+    a.relu = relu ? 1 : 0;
+    const size_t smem = (size_t)slab_fixed_bytes(a.bn, plan->xs_kpad) + (size_t)stages * a.stage_stride;
+    long long grid = plan->ctas > 0 ? plan->ctas : device_sm_count();
+    if (grid > units) grid = units;
+    if (grid < 1) grid = 1;
+    CUtensorMap tw, tx;
+    memcpy(&tw, plan->tmap_ws, sizeof(tw));
+    memcpy(&tx, plan->tmap_xs, sizeof(tx));
+    const cudaError_t e = (ydt == SADMM_BF16) ? launch_slab<true>(tw, tx, a, (int)grid, smem, s)
+                                              : launch_slab<false>(tw, tx, a, (int)grid, smem, s);
+    return e == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
+}
+
+}  // namespace sadmm

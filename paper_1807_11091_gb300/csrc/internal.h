@@ -73,6 +73,16 @@ sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const vo
 sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* filt_idx,
                          const int* col_idx, cudaStream_t s);
 
+sadmm_status launch_pack_slab(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* col_idx,
+                              cudaStream_t s);
+
+// ---- input-slab forward (conv_slab.cu) ----
+// Shared-memory stages (one tile's slab each) the slab kernel can hold with
+// the weights resident; below 2 the slab path is not available.
+int slab_stages(int bn, int kpad_s, int cs, int sp);
+sadmm_status launch_conv_slab(const sadmm_plan* plan, const Geometry& g, const void* x, const float* bias, int relu,
+                              void* y, int ydt, cudaStream_t s);
+
 // ---- forward (conv_fwd.cu) ----
 sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const void* x, const float* bias,
                              int relu, void* y, int ydt, cudaStream_t s);

@@ -191,6 +191,39 @@ __global__ void __launch_bounds__(128) k_pack_wp(const T* __restrict__ W, int K,
     }
 }
 
+// Slab column order of the input-slab path: column j is block tap
+// (r, q) = (j / cs / Q, j / cs % Q), slab channel cc = j % cs = (ci, a, b) with
+// cc = (ci * sh + a) * sw + b, i.e. kept channel ci at phase (a, b); it holds
+// GEMM column chan[ci] * taps + (r*sh + a) * KW + q*sw + b, or nothing (-1)
+// past the kernel, the kept channels or the slab width.  chan[ci] is the ci-th
+// kept input channel (-1 past them, or for an entry of a bad list).
+__global__ void __launch_bounds__(256) k_pack_slab_meta(const int* col_idx, int nck, int C, int cs, int kpad_s,
+                                                       int nsteps_cols, int Q, int sh, int sw, int KH, int KW,
+                                                       int taps, int* scol, int* chan)
+{
+    pdl_wait();  // after the kernel before it in the stream
+    for (int ci = threadIdx.x; ci < cs; ci += blockDim.x) {
+        int ch = -1;
+        if (ci < nck) {
+            ch = col_idx ? col_idx[ci] : ci;
+            if (ch < 0 || ch >= C) ch = -1;
+        }
+        chan[ci] = ch;
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < kpad_s; j += blockDim.x) {
+        int col = -1;
+        if (j < nsteps_cols) {
+            const int tap = j / cs, cc = j - tap * cs;
+            const int r = tap / Q, q = tap - r * Q;
+            const int ci = cc / (sh * sw), a = (cc / sw) % sh, b = cc % sw;
+            const int kh = r * sh + a, kw = q * sw + b;
+            if (ci < nck && kh < KH && kw < KW && chan[ci] >= 0) col = chan[ci] * taps + kh * KW + kw;
+        }
+        scol[j] = col;
+    }
+}
+
 }  // namespace
 
 PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn()
@@ -272,6 +305,62 @@ sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int
     if (r != CUDA_SUCCESS) return SADMM_ECUDA;
     static_assert(sizeof(CUtensorMap) == sizeof(plan->tmap), "tensor map size");
     memcpy(plan->tmap, &map, sizeof(map));
+    if (plan->xs_mode) return launch_pack_slab(plan, g, W, wdt, col_idx, s);
+    return SADMM_OK;
+}
+
+sadmm_status launch_pack_slab(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* col_idx,
+                              cudaStream_t s)
+{
+    char* base = static_cast<char*>(plan->dev);
+    int* scol = reinterpret_cast<int*>(base + plan->off_scol);
+    int* chan = scol + plan->xs_kpad;
+    const int nck = plan->colkind == SADMM_COL_CHANNEL ? plan->n_colgroups : (int)g.c;
+    launch_pdl(k_pack_slab_meta, dim3(1), dim3(256), 0, s, plan->colkind == SADMM_COL_CHANNEL ? col_idx : nullptr,
+               nck, (int)g.c, plan->xs_cs, plan->xs_kpad, plan->xs_r * plan->xs_q * plan->xs_cs, plan->xs_q,
+               (int)g.sh, (int)g.sw, (int)g.kh, (int)g.kw, (int)g.taps, scol, chan);
+    const int* rowmap = reinterpret_cast<const int*>(base + plan->off_rowmap);
+    __nv_bfloat16* wps = reinterpret_cast<__nv_bfloat16*>(base + plan->off_wps);
+    if (wdt == SADMM_BF16)
+        launch_pdl(k_pack_wp<__nv_bfloat16>, dim3((unsigned)plan->bn), dim3(128), 0, s, (const __nv_bfloat16*)W,
+                   (int)g.k, rowmap, (const int*)scol, plan->xs_kpad, wps);
+    else
+        launch_pdl(k_pack_wp<float>, dim3((unsigned)plan->bn), dim3(128), 0, s, (const float*)W, (int)g.k, rowmap,
+                   (const int*)scol, plan->xs_kpad, wps);
+    if (cudaGetLastError() != cudaSuccess) return SADMM_ECUDA;
+    PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
+    if (!enc) return SADMM_ECUDA;
+    {
+        // slab-ordered weights: [bn][xs_kpad], boxes of 64 columns x bn rows, 128-byte swizzle
+        alignas(64) CUtensorMap map;
+        memset(&map, 0, sizeof(map));
+        const cuuint64_t gdim[2] = {(cuuint64_t)plan->xs_kpad, (cuuint64_t)plan->bn};
+        const cuuint64_t gstride[1] = {(cuuint64_t)plan->xs_kpad * 2};
+        const cuuint32_t box[2] = {64u, (cuuint32_t)plan->bn};
+        const cuuint32_t estride[2] = {1u, 1u};
+        if (enc(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, wps, gdim, gstride, box, estride,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return SADMM_ECUDA;
+        memcpy(plan->tmap_ws, &map, sizeof(map));
+    }
+    {
+        // space-to-depth input [N][cs/8][pimg][8] viewed as [N][cs/8][pimg/8][64]:
+        // a box is one tile's slab, every chunk, as [chunk][sp pixels][8]
+        // (no swizzle: the operand descriptors address 16-byte rows directly)
+        alignas(64) CUtensorMap map;
+        memset(&map, 0, sizeof(map));
+        const long long oct = plan->xs_pimg / 8, chunks = plan->xs_cs / 8;
+        const cuuint64_t gdim[4] = {64u, (cuuint64_t)oct, (cuuint64_t)chunks, (cuuint64_t)g.n};
+        const cuuint64_t gstride[3] = {128u, (cuuint64_t)oct * 128u, (cuuint64_t)(chunks * oct * 128)};
+        const cuuint32_t box[4] = {64u, (cuuint32_t)(plan->xs_sp / 8), (cuuint32_t)chunks, 1u};
+        const cuuint32_t estride[4] = {1u, 1u, 1u, 1u};
+        if (enc(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, base + plan->off_xs, gdim, gstride, box, estride,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return SADMM_ECUDA;
+        memcpy(plan->tmap_xs, &map, sizeof(map));
+    }
     return SADMM_OK;
 }
 

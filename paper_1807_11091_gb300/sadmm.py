@@ -61,7 +61,21 @@ class Plan(ctypes.Structure):
         ("sk_len", ctypes.c_int),
         ("sk_grid", ctypes.c_int),
         ("ctas", ctypes.c_int),
+        ("xs_mode", ctypes.c_int),
+        ("xs_r", ctypes.c_int),
+        ("xs_q", ctypes.c_int),
+        ("xs_cs", ctypes.c_int),
+        ("xs_hb", ctypes.c_int),
+        ("xs_wb", ctypes.c_int),
+        ("xs_pimg", ctypes.c_int),
+        ("xs_sp", ctypes.c_int),
+        ("xs_kpad", ctypes.c_int),
+        ("off_xs", ctypes.c_size_t),
+        ("off_wps", ctypes.c_size_t),
+        ("off_scol", ctypes.c_size_t),
         ("tmap", ctypes.c_uint64 * 16),
+        ("tmap_ws", ctypes.c_uint64 * 16),
+        ("tmap_xs", ctypes.c_uint64 * 16),
     ]
 
 

@@ -33,7 +33,7 @@ def test_library_exports_every_declared_entry_point():
 
 
 def test_struct_layout_and_version():
-    assert sadmm.sadmm_abi_version() == 4
+    assert sadmm.sadmm_abi_version() == 5
     assert sadmm.sadmm_plan_struct_size() == ctypes.sizeof(sadmm.Plan)
     assert sadmm.sadmm_status_string(-1) == "invalid argument"
 
@@ -145,3 +145,29 @@ def test_plan_cta_cap_on_host():
     assert st == 0 and capped.ctas == 1 and capped.splits == 1 and capped.sk_len == 0
     st, _ = sadmm.sadmm_plan_init_ctas(d, L.k_filters, L.colkind, L.k_cols, -1)
     assert st == sadmm.SADMM_EINVAL
+
+
+def test_slab_plan_rule_host():
+    """The plan takes the input-slab path for AlexNet CONV1 (kept whole) with the
+    space-to-depth geometry of a stride-4 11x11 kernel over 3 channels, and
+    declines it for shape-wise pruned columns, two conv groups, more than 64
+    slab channels and a slab GEMM over twice as wide as K'."""
+    from workloads import ConvShape
+    L = wl.alexnet()[0]
+    st, p = sadmm.sadmm_plan_init(sadmm.make_desc(L.shape.desc16()), L.k_filters, wl.COL_SHAPE, L.k_cols)
+    assert st == 0 and p.xs_mode == 1
+    # 3 channels x 4 x 4 phases = 48 slab channels; ceil(11/4) = 3 block taps;
+    # 55 + 3 - 1 = 57 block rows and columns; 128 + 2*57 + 2 = 244 -> 248 slab pixels
+    assert (p.xs_cs, p.xs_r, p.xs_q, p.xs_hb, p.xs_wb, p.xs_sp) == (48, 3, 3, 57, 57, 248)
+    assert p.xs_pimg == 3256 and p.xs_kpad == 448 and p.splits == 1 and p.sk_len == 0
+    assert p.off_xs + 128 * 6 * 3256 * 16 <= p.dev_bytes
+    declined = [
+        (ConvShape(n=1, c=3, h=35, w=35, f=16, kh=11, kw=11, sh=4, sw=4), wl.COL_SHAPE, 300),
+        (ConvShape(n=1, c=8, h=9, w=9, f=16, kh=3, kw=3, ph=1, pw=1, groups=2), wl.COL_NONE, 0),
+        (ConvShape(n=1, c=5, h=35, w=35, f=16, kh=11, kw=11, sh=4, sw=4), wl.COL_NONE, 0),
+        (ConvShape(n=1, c=3, h=9, w=9, f=16, kh=3, kw=3, ph=1, pw=1), wl.COL_NONE, 0),
+        (ConvShape(n=1, c=3, h=9, w=9, f=300, kh=3, kw=3, sh=2, sw=2), wl.COL_NONE, 0),
+    ]
+    for s, ck, kc in declined:
+        st, p = sadmm.sadmm_plan_init(sadmm.make_desc(s.desc16()), s.f, ck, s.k if ck == wl.COL_NONE else kc)
+        assert st == 0 and p.xs_mode == 0, s

@@ -1,0 +1,113 @@
+"""GPU parity of the input-slab forward (plan.xs_mode = 1): layers with one conv
+group whose kept channels keep every column and whose space-to-depth input has
+at most 64 channels -- strided first layers (AlexNet CONV1, a 7x7 stride-2
+stem), stride-1 layers with few channels, channel-wise pruned layers.
+
+Every output is pre-filled with NaN; fp32 output within 2e-3 * max|oracle|,
+bf16 output within one bf16 ulp of the oracle rounded to bf16.  Each case
+asserts that the plan took the slab path."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads as wl
+from workloads import ConvShape
+
+from _helpers import assert_close, gpu_layer, oracle_layer, pruned_filters
+
+pytestmark = pytest.mark.gpu
+
+# (name, shape, filter fraction, column kind, column fraction)
+CASES = [
+    ("stride4_11x11", ConvShape(n=2, c=3, h=35, w=35, f=16, kh=11, kw=11, sh=4, sw=4), 1.0, wl.COL_NONE, 1.0),
+    ("stride4_pruned_filters", ConvShape(n=3, c=3, h=51, w=47, f=40, kh=11, kw=11, sh=4, sw=4), 0.6, wl.COL_NONE,
+     1.0),
+    ("stem_7x7_s2_p3", ConvShape(n=2, c=3, h=37, w=33, f=24, kh=7, kw=7, sh=2, sw=2, ph=3, pw=3), 1.0, wl.COL_NONE,
+     1.0),
+    ("stride1_3x3_c16", ConvShape(n=2, c=16, h=21, w=19, f=48, kh=3, kw=3, ph=1, pw=1), 0.75, wl.COL_NONE, 1.0),
+    ("channel_3x3", ConvShape(n=2, c=24, h=9, w=9, f=40, kh=3, kw=3, ph=1, pw=1), 0.5, wl.COL_CHANNEL, 0.5),
+    ("channel_1x1", ConvShape(n=2, c=32, h=8, w=8, f=48, kh=1, kw=1), 0.5, wl.COL_CHANNEL, 0.5),
+    ("shape_all_kept", ConvShape(n=2, c=4, h=15, w=16, f=20, kh=5, kw=5, sh=2, sw=2, ph=2, pw=2), 1.0, wl.COL_SHAPE,
+     1.0),
+    ("rect_stride_kernel", ConvShape(n=2, c=6, h=13, w=10, f=24, kh=3, kw=2, sh=2, sw=1, ph=1, pw=0), 0.75,
+     wl.COL_NONE, 1.0),
+    ("one_image_many_tiles", ConvShape(n=1, c=3, h=131, w=97, f=64, kh=5, kw=5, sh=2, sw=2, ph=1, pw=2), 1.0,
+     wl.COL_NONE, 1.0),
+    ("wide_256_filters", ConvShape(n=2, c=3, h=40, w=41, f=256, kh=3, kw=3, sh=2, sw=2, ph=1, pw=1), 1.0,
+     wl.COL_NONE, 1.0),
+]
+
+
+def _k(s, ff, ck, cf):
+    G = s.cg if ck == wl.COL_CHANNEL else s.k
+    return wl.retained(ff, s.f), (wl.retained(cf, G) if ck != wl.COL_NONE else 0)
+
+
+def _run(case, seed, **kw):
+    name, s, ff, ck, cf = case
+    kf, kc = _k(s, ff, ck, cf)
+    t = wl.gen_tensors(s, seed=seed)
+    fi, ci, y, pc = gpu_layer(s, t, kf, ck, kc, **kw)
+    assert pc.plan.xs_mode == 1, f"{name}: the plan did not take the slab path"
+    rows, cols, _, _ = oracle.project(t["W"], s.taps, kf, ck, kc)
+    assert np.array_equal(fi, rows)
+    if ck != wl.COL_NONE:
+        assert np.array_equal(ci, cols)
+    return s, t, rows, ck, cols, y, pc
+
+
+@pytest.mark.parametrize("case", CASES, ids=lambda c: c[0])
+def test_slab_layers_fp32(case):
+    s, t, rows, ck, cols, y, _ = _run(case, seed=301)
+    ref = oracle_layer(s, t, rows, ck, cols)
+    assert_close(y, ref, what=case[0])
+    assert np.all(y[:, pruned_filters(s.f, rows)] == 0.0)
+
+
+@pytest.mark.parametrize("case", [CASES[1], CASES[2], CASES[4]], ids=lambda c: c[0])
+def test_slab_bf16_output_no_relu_no_bias(case):
+    s, t, rows, ck, cols, y, _ = _run(case, seed=302, relu=False, use_bias=False, out_dtype=torch.bfloat16)
+    ref = oracle_layer(s, t, rows, ck, cols, relu=False, use_bias=False)
+    ref_b = torch.from_numpy(ref).to(torch.bfloat16).float().numpy()
+    scale = np.abs(ref).max()
+    assert np.all(np.abs(y - ref_b) <= np.abs(ref_b) * 2.0 ** -7 + 2e-3 * scale), case[0]
+    assert np.all(y[:, pruned_filters(s.f, rows)] == 0.0)
+
+
+def test_slab_all_filters_pruned_gives_zeros():
+    case = ("all_pruned", ConvShape(n=2, c=3, h=23, w=23, f=16, kh=5, kw=5, sh=2, sw=2), 0.0, wl.COL_NONE, 1.0)
+    s, t, rows, ck, cols, y, _ = _run(case, seed=303)
+    assert len(rows) == 0 and np.all(y == 0.0)
+
+
+def test_slab_repeated_launches_identical():
+    """The plan's space-to-depth buffer is rewritten by every launch: results
+    are bit-identical across launches and across a launch on other input."""
+    from paper_1807_11091_gb300 import sadmm
+    case = CASES[1]
+    s, t, rows, ck, cols, y, pc = _run(case, seed=304)
+    dev = torch.device("cuda", 0)
+    x = t["x"].to(dev)
+    bias = t["bias"].to(dev)
+    other = torch.randn_like(x.float()).to(torch.bfloat16)
+    y2 = torch.full(pc.out_shape(), float("nan"), device=dev)
+    pc.forward(other, bias, out=y2)
+    pc.forward(x, bias, out=y2)
+    assert sadmm.device_status() == 0
+    assert np.array_equal(y2.cpu().numpy(), y)
+
+
+def test_alexnet_conv1_batch128_sampled_images():
+    """AlexNet CONV1 at batch 128 (the layer kept whole): indices exact, and
+    images 0, 1, 63 and 127 against the oracle element by element."""
+    L = wl.alexnet()[0]
+    s = L.shape
+    t = wl.gen_tensors(s, seed=L.seed)
+    fi, ci, y, pc = gpu_layer(s, t, L.k_filters, L.colkind, L.k_cols)
+    assert pc.plan.xs_mode == 1 and pc.plan.xs_cs == 48 and pc.plan.xs_r == 3 and pc.plan.xs_wb == 57
+    rows, cols, _, _ = oracle.project(t["W"], s.taps, L.k_filters, L.colkind, L.k_cols)
+    assert np.array_equal(fi, rows) and np.array_equal(ci, cols)
+    for n in (0, 1, 63, 127):
+        ref = oracle_layer(s, t, rows, L.colkind, cols, n0=n, n1=n + 1)
+        assert_close(y[n:n + 1], ref, what=f"conv1 image {n}")
