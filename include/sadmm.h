@@ -257,8 +257,9 @@ sadmm_status sadmm_admm_update_elements(const sadmm_conv_desc* d, const void* W,
  * Input-slab path (plan->xs_mode = 1): a 2-D layer with one conv group, at
  * most 256 kept filters and every column of its kept channels kept (no
  * column pruning, or whole channels pruned), whose kept channels times
- * sh * sw come to at most 64, and whose slab GEMM is at most twice as wide
- * as K' -- the first layer of a network, typically (the paper keeps AlexNet's
+ * sh * sw come to at most 64, with more than one block tap (xs_r * xs_q >= 2)
+ * and a slab GEMM at most twice as wide as K' -- the first layer of a
+ * network, typically (the paper keeps AlexNet's
  * CONV1 whole).  The forward then first rewrites x as a space-to-depth copy
  * in the plan's buffer: block pixel (hb, wb) holds, for each kept channel c
  * and phase (a, b) < (sh, sw), the input x[c][hb*sh + a - ph][wb*sw + b - pw]

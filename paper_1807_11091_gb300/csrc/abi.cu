@@ -289,7 +289,10 @@ sadmm_status sadmm_plan_init_ctas(sadmm_plan* plan, const sadmm_conv_desc* d, in
     p.splits = 1;
     p.stages_per_split = p.k_pad / 64;
     // input-slab path: one conv group, every column of the kept channels kept,
-    // few slab channels, one filter tile, and a slab GEMM at most twice as wide
+    // few slab channels, one filter tile, more than one block tap (a 1 x 1
+    // block kernel reads contiguous input rows, which the gathered path does
+    // as fast without the space-to-depth pass), and a slab GEMM at most twice
+    // as wide
     const bool cols_whole = colkind == SADMM_COL_NONE || colkind == SADMM_COL_CHANNEL ||
                             (colkind == SADMM_COL_SHAPE && n_cols == g.k);
     if (g.t == 1 && g.kt == 1 && g.groups == 1 && p.n_tiles == 1 && cols_whole && n_cols > 0) {
@@ -301,7 +304,7 @@ sadmm_status sadmm_plan_init_ctas(sadmm_plan* plan, const sadmm_conv_desc* d, in
         const long long sp = round_up(128 + (R - 1) * wb + (Q - 1), 8);
         const long long kpad_s = round_up(R * Q * cs, 64);
         const long long xs_bytes = g.n * cs * pimg * 2;
-        if (cs <= 64 && sp / 8 <= 256 && kpad_s <= 2 * p.k_pad && pimg < (1ll << 28) && hb <= 65535 && g.n <= 65535 &&
+        if (R * Q >= 2 && cs <= 64 && sp / 8 <= 256 && kpad_s <= 2 * p.k_pad && pimg < (1ll << 28) && hb <= 65535 && g.n <= 65535 &&
             xs_bytes <= (4ll << 30) && slab_stages(p.bn, (int)kpad_s, (int)cs, (int)sp) >= 2) {
             p.xs_mode = 1;
             p.xs_r = (int)R;

@@ -42,6 +42,7 @@ constexpr int kSlabThreads = kSlabWarps * 32;
 constexpr int kSlabEpiWarps = 8;        // warps 2..9: two per TMEM lane quadrant (warp % 4)
 constexpr int kMaxSlabStages = 4;
 constexpr int kSlabTables = 2 * 256 * 4;  // plane offset and bias of each kept row
+constexpr int kSlabZcap = 1024;           // pruned filters whose plane offsets sit in shared memory
 constexpr int kSlabBars = 256;            // barriers, TMEM address, abort flag
 constexpr int kSlabSmemLimit = 232448;
 
@@ -64,23 +65,23 @@ struct SlabArgs {
 
 struct XsArgs {
     int C, H, W, sh, sw, ph, pw;
-    int nck, cs, Wb, pimg;
+    int nck, cs, Hb, Wb, pimg;
 };
 
-// Thread (tx, ty) of block (bw, hb, n) writes the 16-byte vectors (8 slab
-// channels) of chunks ty, ty + 4, ... of block pixel wb = 64*bw + tx in block
-// row hb of image n.  Its 8 input loads are independent (all in flight); the
-// channel and phase of each slab channel come from a table decoded once per
-// block in shared memory.
-constexpr int kXsPix = 64;     // block pixels per block (threadIdx.x)
-constexpr int kXsChunkRows = 4;  // chunks in flight per block (threadIdx.y)
-__global__ void __launch_bounds__(kXsPix * kXsChunkRows) k_slab_input(const __nv_bfloat16* __restrict__ x,
-                                                                      const int* __restrict__ chan, const XsArgs b,
-                                                                      __nv_bfloat16* __restrict__ xs)
+// Thread (tx, ty) of block (bw, bh, n) writes every chunk's 16-byte vector
+// (8 slab channels) of block pixel (hb, wb) = (4*bh + ty, 64*bw + tx) of image
+// n; the loads of two chunks (16) are in flight together.  The channel and
+// phase of each slab channel come from a table decoded once per block in
+// shared memory.
+constexpr int kXsPix = 64;   // block pixels of a block row per block (threadIdx.x)
+constexpr int kXsRows = 4;   // block rows per block (threadIdx.y)
+__global__ void __launch_bounds__(kXsPix * kXsRows) k_slab_input(const __nv_bfloat16* __restrict__ x,
+                                                                 const int* __restrict__ chan, const XsArgs b,
+                                                                 __nv_bfloat16* __restrict__ xs)
 {
     __shared__ int4 s_dec[64];  // per slab channel: {channel plane offset (-1: zero), a - ph, b - pw, 0}
     pdl_wait();  // after the kernel before it in the stream
-    const int hb = blockIdx.y, n = blockIdx.z;
+    const int n = blockIdx.z;
     const int tid = threadIdx.y * kXsPix + threadIdx.x;
     if (tid < b.cs) {
         const int cc = tid;
@@ -90,11 +91,14 @@ __global__ void __launch_bounds__(kXsPix * kXsChunkRows) k_slab_input(const __nv
     }
     __syncthreads();
     const int wb = blockIdx.x * kXsPix + threadIdx.x;
-    if (wb >= b.Wb) return;
+    const int hb = blockIdx.y * kXsRows + threadIdx.y;
+    if (wb >= b.Wb || hb >= b.Hb) return;
     const unsigned short* xi = reinterpret_cast<const unsigned short*>(x) + (long long)n * b.C * b.H * b.W;
     const int ih0 = hb * b.sh, iw0 = wb * b.sw;
     const int chunks = b.cs / 8;
-    for (int k = threadIdx.y; k < chunks; k += kXsChunkRows) {
+    __nv_bfloat16* dst0 = xs + ((long long)n * chunks * b.pimg + (long long)hb * b.Wb + wb) * 8;
+#pragma unroll 2
+    for (int k = 0; k < chunks; ++k) {
         uint32_t h[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
@@ -104,8 +108,8 @@ __global__ void __launch_bounds__(kXsPix * kXsChunkRows) k_slab_input(const __nv
                        ? (uint32_t)__ldg(xi + d.x + ih * b.W + iw)
                        : 0u;
         }
-        uint4* dst = reinterpret_cast<uint4*>(xs + (((long long)n * chunks + k) * b.pimg + (long long)hb * b.Wb + wb) * 8);
-        *dst = make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16), h[6] | (h[7] << 16));
+        *reinterpret_cast<uint4*>(dst0 + (long long)k * b.pimg * 8) =
+            make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16), h[6] | (h[7] << 16));
     }
 }
 
@@ -121,7 +125,8 @@ __global__ void __launch_bounds__(kSlabThreads, 1)
     uint8_t* sA = sB + (size_t)a.nbox * bbox;  // 1024-aligned: bbox is a multiple of 2048
     int* t_off = reinterpret_cast<int*>(sA + (size_t)a.stages * a.stage_stride);
     float* t_bias = reinterpret_cast<float*>(t_off + 256);
-    uint64_t* bars = reinterpret_cast<uint64_t*>(t_bias + 256);
+    int* z_off = reinterpret_cast<int*>(t_bias + 256);  // [kSlabZcap] plane offsets of pruned filters
+    uint64_t* bars = reinterpret_cast<uint64_t*>(z_off + kSlabZcap);
     uint64_t* full = bars;
     uint64_t* empty = bars + kMaxSlabStages;
     uint64_t* acc_full = bars + 2 * kMaxSlabStages;
@@ -158,6 +163,8 @@ __global__ void __launch_bounds__(kSlabThreads, 1)
         t_off[i] = f >= 0 ? f * a.plane : 0;
         t_bias[i] = (f >= 0 && a.bias) ? __ldg(a.bias + f) : 0.0f;
     }
+    const int zc = min(__ldg(a.counts + 1), kSlabZcap);
+    for (int z = threadIdx.x; z < zc; z += blockDim.x) z_off[z] = __ldg(a.zeromap + z) * a.plane;
     if (warp == 0 && lane == 0) {
         tma_prefetch_desc(&tw);
         tma_prefetch_desc(&tx);
@@ -259,7 +266,7 @@ __global__ void __launch_bounds__(kSlabThreads, 1)
             // pruned filters' planes: zero, while the tile's MMAs run
             if (alive && valid) {
                 for (int z = h; z < pruned; z += 2) {
-                    const long long off = (long long)__ldg(a.zeromap + z) * a.plane;
+                    const long long off = z < kSlabZcap ? z_off[z] : (long long)__ldg(a.zeromap + z) * a.plane;
                     if (OUT_BF16)
                         yh[off] = __float2bfloat16_rn(0.0f);
                     else
@@ -297,7 +304,10 @@ __global__ void __launch_bounds__(kSlabThreads, 1)
     }
 }
 
-int slab_fixed_bytes(int bn, int kpad_s) { return 1024 + (kpad_s / 64) * bn * 128 + kSlabTables + kSlabBars; }
+int slab_fixed_bytes(int bn, int kpad_s)
+{
+    return 1024 + (kpad_s / 64) * bn * 128 + kSlabTables + kSlabZcap * 4 + kSlabBars;
+}
 int slab_stage_stride(int cs, int sp) { return (int)round_up((long long)cs * sp * 2, 1024); }
 
 template <bool OUT_BF16>
@@ -349,13 +359,15 @@ sadmm_status launch_conv_slab(const sadmm_plan* plan, const Geometry& g, const v
     b.pw = (int)g.pw;
     b.nck = plan->colkind == SADMM_COL_CHANNEL ? plan->n_colgroups : (int)g.c;
     b.cs = plan->xs_cs;
+    b.Hb = plan->xs_hb;
     b.Wb = plan->xs_wb;
     b.pimg = plan->xs_pimg;
     const int* chan = reinterpret_cast<const int*>(base + plan->off_scol) + plan->xs_kpad;
     __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(const_cast<char*>(base) + plan->off_xs);
     if (launch_pdl(k_slab_input,
-                   dim3((unsigned)((plan->xs_wb + kXsPix - 1) / kXsPix), (unsigned)plan->xs_hb, (unsigned)g.n),
-                   dim3(kXsPix, kXsChunkRows), 0, s, static_cast<const __nv_bfloat16*>(x), chan, b, xs) != cudaSuccess)
+                   dim3((unsigned)((plan->xs_wb + kXsPix - 1) / kXsPix), (unsigned)((plan->xs_hb + kXsRows - 1) / kXsRows),
+                        (unsigned)g.n),
+                   dim3(kXsPix, kXsRows), 0, s, static_cast<const __nv_bfloat16*>(x), chan, b, xs) != cudaSuccess)
         return SADMM_ECUDA;
 
     SlabArgs a;

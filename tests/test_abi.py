@@ -151,7 +151,8 @@ def test_slab_plan_rule_host():
     """The plan takes the input-slab path for AlexNet CONV1 (kept whole) with the
     space-to-depth geometry of a stride-4 11x11 kernel over 3 channels, and
     declines it for shape-wise pruned columns, two conv groups, more than 64
-    slab channels and a slab GEMM over twice as wide as K'."""
+    slab channels, a slab GEMM over twice as wide as K', more than 256 kept
+    filters and a single block tap (1 x 1, or 2 x 2 at stride 2)."""
     from workloads import ConvShape
     L = wl.alexnet()[0]
     st, p = sadmm.sadmm_plan_init(sadmm.make_desc(L.shape.desc16()), L.k_filters, wl.COL_SHAPE, L.k_cols)
@@ -167,6 +168,8 @@ def test_slab_plan_rule_host():
         (ConvShape(n=1, c=5, h=35, w=35, f=16, kh=11, kw=11, sh=4, sw=4), wl.COL_NONE, 0),
         (ConvShape(n=1, c=3, h=9, w=9, f=16, kh=3, kw=3, ph=1, pw=1), wl.COL_NONE, 0),
         (ConvShape(n=1, c=3, h=9, w=9, f=300, kh=3, kw=3, sh=2, sw=2), wl.COL_NONE, 0),
+        (ConvShape(n=1, c=32, h=8, w=8, f=48, kh=1, kw=1), wl.COL_CHANNEL, 16),
+        (ConvShape(n=1, c=4, h=8, w=8, f=48, kh=2, kw=2, sh=2, sw=2), wl.COL_NONE, 0),
     ]
     for s, ck, kc in declined:
         st, p = sadmm.sadmm_plan_init(sadmm.make_desc(s.desc16()), s.f, ck, s.k if ck == wl.COL_NONE else kc)

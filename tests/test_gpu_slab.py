@@ -27,7 +27,8 @@ CASES = [
      1.0),
     ("stride1_3x3_c16", ConvShape(n=2, c=16, h=21, w=19, f=48, kh=3, kw=3, ph=1, pw=1), 0.75, wl.COL_NONE, 1.0),
     ("channel_3x3", ConvShape(n=2, c=24, h=9, w=9, f=40, kh=3, kw=3, ph=1, pw=1), 0.5, wl.COL_CHANNEL, 0.5),
-    ("channel_1x1", ConvShape(n=2, c=32, h=8, w=8, f=48, kh=1, kw=1), 0.5, wl.COL_CHANNEL, 0.5),
+    ("channel_5x5_stride2", ConvShape(n=2, c=32, h=17, w=16, f=48, kh=5, kw=5, sh=2, sw=2, ph=2, pw=2), 0.5,
+     wl.COL_CHANNEL, 0.125),
     ("shape_all_kept", ConvShape(n=2, c=4, h=15, w=16, f=20, kh=5, kw=5, sh=2, sw=2, ph=2, pw=2), 1.0, wl.COL_SHAPE,
      1.0),
     ("rect_stride_kernel", ConvShape(n=2, c=6, h=13, w=10, f=24, kh=3, kw=2, sh=2, sw=1, ph=1, pw=0), 0.75,
@@ -111,3 +112,15 @@ def test_alexnet_conv1_batch128_sampled_images():
     for n in (0, 1, 63, 127):
         ref = oracle_layer(s, t, rows, L.colkind, cols, n0=n, n1=n + 1)
         assert_close(y[n:n + 1], ref, what=f"conv1 image {n}")
+
+
+def test_slab_more_pruned_planes_than_the_shared_table():
+    """1060 pruned filters: the first 1024 plane offsets come from shared memory,
+    the rest from the plan's list; every pruned plane is zero."""
+    case = ("many_pruned", ConvShape(n=2, c=3, h=9, w=11, f=1100, kh=3, kw=3, sh=2, sw=2, pw=1), 40 / 1100,
+            wl.COL_NONE, 1.0)
+    s, t, rows, ck, cols, y, _ = _run(case, seed=305)
+    assert len(rows) == 40
+    ref = oracle_layer(s, t, rows, ck, cols)
+    assert_close(y, ref, what="many_pruned")
+    assert np.all(y[:, pruned_filters(s.f, rows)] == 0.0)
