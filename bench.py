@@ -364,14 +364,26 @@ class ClockSampler:
 
 
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "conv_fwd_alexnet_b128_dram.txt")
-CONV_SRC = os.path.join(ROOT, "paper_1807_11091_gb300", "csrc", "conv_fwd.cu")
+# the forward kernels' sources: the gathered kernel, the input-slab kernels and what they share
+CONV_SRCS = [os.path.join(ROOT, "paper_1807_11091_gb300", "csrc", f)
+             for f in ("conv_fwd.cu", "conv_slab.cu", "conv_common.cuh")]
+
+
+def conv_source_sha1():
+    """sha1 over the forward kernels' source files, in CONV_SRCS order."""
+    import hashlib
+    h = hashlib.sha1()
+    for f in CONV_SRCS:
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
 
 
 def conv_traffic(workload, out_dtype):
-    """DRAM bytes per sadmm_conv_fwd launch (read + write, averaged over the
-    step's launches) from the committed ncu summary, or None when that summary
-    is for another workload or the kernel source changed since it was taken."""
-    import hashlib
+    """DRAM bytes per sadmm_conv_fwd call (read + write of every kernel it
+    launches, averaged over the step's calls) from the committed ncu summary, or
+    None when that summary is for another workload or the kernel sources changed
+    since it was taken."""
     if workload != "alexnet" or out_dtype != "fp32":
         return None
     try:
@@ -381,11 +393,9 @@ def conv_traffic(workload, out_dtype):
                 if ":" in ln and not ln.startswith("#"):
                     k, v = ln.split(":", 1)
                     fields[k.strip()] = v.strip()
-        with open(CONV_SRC, "rb") as fh:
-            sha = hashlib.sha1(fh.read()).hexdigest()
-        if fields.get("kernel_source_sha1") != sha:
+        if fields.get("kernel_source_sha1") != conv_source_sha1():
             return None
-        return float(fields["dram_bytes_per_launch_avg"])
+        return float(fields["dram_bytes_per_call_avg"])
     except Exception:
         return None
 
@@ -695,7 +705,7 @@ def run_gpu(args):
     conv_avg = [statistics.mean(c) for c in conv_ms]
     dense_conv_avg = [statistics.mean(c) for c in dense_conv_ms]
 
-    # roofline of the dominant kernel (sadmm_conv_fwd over the step's launches)
+    # roofline of the dominant call (sadmm_conv_fwd over the step's five calls)
     conv_bytes = [r.conv_bytes() for r in runs]
     conv_flops = [r.flops() for r in runs]
     t_conv = sum(conv_avg) * 1e-3
@@ -711,7 +721,8 @@ def run_gpu(args):
                 "frac": achieved / peaks["bf16_tflops"]}
     roof["traffic"] = conv_traffic(args.workload, args.out_dtype)
     roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
-    roof["kernel"] = "k_conv_fwd (sadmm_conv_fwd), averaged over the step's launches"
+    roof["kernel"] = ("sadmm_conv_fwd (k_conv_fwd; CONV1: k_slab_input + k_conv_slab), "
+                      "averaged over the step's five calls")
     roof["combined_roofline_frac"] = max(t_mem, t_cmp) / t_conv
 
     e2e_med = ranks.max_over_ranks(statistics.median(e2e_ms), device=dev)
