@@ -493,17 +493,20 @@ def batch1_report(dev, out_dtype, reps=7):
 
 
 def backward_report(dev, out_dtype, reps=3):
-    """Masked-retraining backward (sadmm_conv_bwd: dW, db and dx over the kept
-    weights) of every AlexNet CONV layer at batch 128, L2 flushed, median of
-    `reps`; TFLOP/s counts the two retained contractions (weight and input
-    gradient), 4 * M * F' * K'."""
+    """Masked-retraining backward (sadmm_conv_bwd over the kept weights) of every
+    AlexNet CONV layer at batch 128, L2 flushed, median of `reps`: dW and db of
+    every layer, dx of conv2-5 (conv1's input is the image, whose gradient
+    training never uses).  TFLOP/s counts the retained contractions run: weight
+    and input gradient (4 * M * F' * K'), the weight gradient alone on conv1."""
     import torch
     from paper_1807_11091_gb300 import sadmm
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
-    out = {"what": "sadmm_conv_bwd per AlexNet CONV layer at batch 128 (dW, db, dx), L2 flushed", "layers": {}}
+    out = {"what": "sadmm_conv_bwd per AlexNet CONV layer at batch 128 (dW and db; dx for conv2-5: conv1's input "
+                   "is the image), L2 flushed", "layers": {}}
     tot_ms = tot_fl = 0.0
-    for L in wl.alexnet():
+    for li, L in enumerate(wl.alexnet()):
         s = L.shape
+        want_dx = li > 0
         t = wl.gen_tensors(s, seed=L.seed)
         r = LayerRun(L, t, dev, "fp32")
         sp = int(torch.cuda.current_stream().cuda_stream)
@@ -514,7 +517,7 @@ def backward_report(dev, out_dtype, reps=3):
         dy = torch.randn(s.y_shape(), generator=g).to(torch.bfloat16).to(dev)
         dW = torch.empty((s.f, s.k), dtype=torch.float32, device=dev)
         db = torch.empty(s.f, dtype=torch.float32, device=dev)
-        dx = torch.empty(r.x.shape, dtype=torch.float32, device=dev)
+        dx = torch.empty(r.x.shape, dtype=torch.float32, device=dev) if want_dx else None
         ws_bytes = sadmm.sadmm_conv_bwd_workspace_size(r.plan)
         ws = torch.empty(ws_bytes + 1024, dtype=torch.uint8, device=dev)
         wptr = (ws.data_ptr() + 1023) // 1024 * 1024
@@ -526,16 +529,17 @@ def backward_report(dev, out_dtype, reps=3):
             e1 = torch.cuda.Event(enable_timing=True)
             e0.record()
             st = sadmm.sadmm_conv_bwd(r.plan, r.x.data_ptr(), dy.data_ptr(), r.y.data_ptr(), sadmm.SADMM_FP32, 1,
-                                      dW.data_ptr(), db.data_ptr(), dx.data_ptr(), wptr, ws_bytes, sp)
+                                      dW.data_ptr(), db.data_ptr(), dx.data_ptr() if want_dx else None, wptr,
+                                      ws_bytes, sp)
             e1.record()
             torch.cuda.synchronize()
             assert st == 0, st
             ms.append(e0.elapsed_time(e1))
         t_ms = statistics.median(ms[1:])
-        fl = 2.0 * r.flops()
+        fl = (2.0 if want_dx else 1.0) * r.flops()
         tot_ms += t_ms
         tot_fl += fl
-        out["layers"][L.name] = {"us": t_ms * 1e3, "tflops_retained": fl / (t_ms * 1e-3) / 1e12}
+        out["layers"][L.name] = {"us": t_ms * 1e3, "tflops_retained": fl / (t_ms * 1e-3) / 1e12, "dx": want_dx}
         del r, dy, dW, db, dx, ws
     out["total_us"] = tot_ms * 1e3
     out["tflops_retained"] = tot_fl / (tot_ms * 1e-3) / 1e12

@@ -359,9 +359,18 @@ sadmm_status sadmm_project_groups_noalloc(const sadmm_conv_desc* d, const void* 
                                           int* filt_idx, int* col_idx, double* keys_out,
                                           void* stream);
 
-/* Device bytes of scratch sadmm_conv_bwd needs for this plan (gathered
- * operands of one chunk of at most 32768 output pixels, fp32 products). */
+/* Device bytes of scratch for sadmm_conv_bwd to take the layer's output
+ * pixels in chunks of at most 32768 (sized so a chunk's gathered bf16
+ * operands and fp32 products stay in L2): the default.  0 on a bad plan. */
 size_t sadmm_conv_bwd_workspace_size(const sadmm_plan* plan);
+
+/* Device bytes of scratch for chunks of `chunk_pixels` output pixels (rounded
+ * up to a multiple of 256, at least 256, at most 32768).  sadmm_conv_bwd
+ * accepts any workspace at least the size for 256 pixels and takes the pixels
+ * in the largest chunks (up to 32768) the workspace holds: a smaller workspace
+ * costs more launches and partial-sum passes, not results (the dW and db
+ * reductions keep a fixed order for a given chunk size). */
+size_t sadmm_conv_bwd_workspace_size_chunk(const sadmm_plan* plan, long long chunk_pixels);
 
 /*
  * Backward of the packed pruned layer for masked retraining (Sec. 4, "Masked

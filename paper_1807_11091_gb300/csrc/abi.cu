@@ -424,6 +424,14 @@ size_t sadmm_conv_bwd_workspace_size(const sadmm_plan* plan)
     return bwd_workspace_bytes(plan, g);
 }
 
+size_t sadmm_conv_bwd_workspace_size_chunk(const sadmm_plan* plan, long long chunk_pixels)
+{
+    if (!plan || chunk_pixels < 1) return 0;
+    Geometry g;
+    if (check_desc(&plan->desc, &g) != SADMM_OK) return 0;
+    return bwd_workspace_bytes(plan, g, chunk_pixels);
+}
+
 sadmm_status sadmm_conv_bwd(const sadmm_plan* plan, const void* x, const void* dy, const void* y, int ydt, int relu,
                             float* dW, float* db, float* dx, void* workspace, size_t ws_bytes, void* stream)
 {
@@ -434,13 +442,14 @@ sadmm_status sadmm_conv_bwd(const sadmm_plan* plan, const void* x, const void* d
     if (dW && !x) return SADMM_EINVAL;
     if (relu && !y) return SADMM_EINVAL;
     if (relu && ydt != SADMM_BF16 && ydt != SADMM_FP32) return SADMM_EINVAL;
-    if (ws_bytes < bwd_workspace_bytes(plan, g)) return SADMM_EINVAL;
+    if (ws_bytes < bwd_workspace_bytes(plan, g, 256)) return SADMM_EINVAL;
     if ((reinterpret_cast<uintptr_t>(workspace) & 1023) != 0) return SADMM_EINVAL;
     if (((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(dy)) & 1) != 0) return SADMM_EINVAL;
     if (((reinterpret_cast<uintptr_t>(dW) | reinterpret_cast<uintptr_t>(db) | reinterpret_cast<uintptr_t>(dx)) & 3) != 0)
         return SADMM_EINVAL;
     if (device_cc_major() < 10) return SADMM_EUNSUPPORTED;
-    return launch_conv_bwd(plan, g, x, dy, y, ydt, relu, dW, db, dx, workspace, static_cast<cudaStream_t>(stream));
+    return launch_conv_bwd(plan, g, x, dy, y, ydt, relu, dW, db, dx, workspace, ws_bytes,
+                           static_cast<cudaStream_t>(stream));
 }
 
 sadmm_status sadmm_gemm_bf16(const void* A, const void* B, float* C, long long M, long long N, long long K,

@@ -115,7 +115,9 @@ SADMM_DEV float relu_grad(const BwdGeo& b, size_t off)
 }
 
 // dZ for the kept filters of group g and pixels m0 .. m0+mc-1, in two layouts:
-// gt[i][ml] (filter-major, rows up to fr) and gm[ml][i] (pixel-major, i < fk).
+// gt[i][ml] (filter-major, rows up to fr; for the weight gradient) and
+// gm[ml][i] (pixel-major, i < fk; for the input gradient).  A null pointer
+// skips that layout.
 // Block (bx, by): pixels bx*64 .. +63 of the chunk, packed rows by*32 .. +31;
 // the pixel-major copy goes out through a shared-memory transpose, 8 rows of a
 // pixel per 16-byte store.
@@ -148,12 +150,12 @@ __global__ void __launch_bounds__(256) k_bwd_gather_dy(const BwdGeo b, int g, lo
         }
         const __nv_bfloat16 h = __float2bfloat16_rn(v);
         tile[r][pl] = h;
-        if (i < b.fr && ml < b.mc) gt[(size_t)i * b.mc + ml] = h;
+        if (gt && i < b.fr && ml < b.mc) gt[(size_t)i * b.mc + ml] = h;
     }
     __syncthreads();
     const int pl2 = threadIdx.x >> 2, rq = (threadIdx.x & 3) * 8;  // pixel, first of its 8 rows
     const int ml2 = p0 + pl2;
-    if (ml2 < b.mc && i0 + rq < b.fk) {  // fk is a multiple of 64: all 8 rows are inside
+    if (gm && ml2 < b.mc && i0 + rq < b.fk) {  // fk is a multiple of 64: all 8 rows are inside
         uint32_t w[4];
         for (int e = 0; e < 4; ++e)
             w[e] = (uint32_t)__bfloat16_as_ushort(tile[rq + 2 * e][pl2]) |
@@ -321,7 +323,15 @@ Layout layout(const BwdGeo& b)
     return l;
 }
 
-BwdGeo geometry(const sadmm_plan* plan, const Geometry& g)
+// Output pixels per chunk: the whole layer up to kBwdMaxChunk (the default
+// workspace), or what a smaller workspace holds (at least 256).  A chunk's
+// gathered operands and fp32 products (about 50 MB at 32768 pixels on AlexNet
+// CONV1) stay in L2 from the kernel that writes them to the one that reads
+// them; whole-layer chunks measured slower on GB300 (CONV1 1.60 -> 1.84 ms,
+// CONV2 0.86 -> 1.54 ms at batch 128).
+constexpr long long kBwdMaxChunk = 32768;
+
+BwdGeo geometry(const sadmm_plan* plan, const Geometry& g, long long chunk)
 {
     BwdGeo b;
     memset(&b, 0, sizeof(b));
@@ -337,7 +347,7 @@ BwdGeo geometry(const sadmm_plan* plan, const Geometry& g)
     b.fr = (int)rup(plan->n_pad, 128);
     b.fk = (int)rup(plan->n_pad, 64);
     b.kr = (int)rup(plan->k_pad, 128);
-    b.mc = (int)std::min<long long>(rup(g.m, 256), 32768);
+    b.mc = (int)std::min<long long>(rup(g.m, 256), std::max<long long>(256, std::min(rup(chunk, 256), kBwdMaxChunk)));
     divisor((uint32_t)b.plane, b.plane_mul, b.plane_sh);
     divisor((uint32_t)(b.OH * b.OW), b.ohw_mul, b.ohw_sh);
     divisor((uint32_t)b.OW, b.ow_mul, b.ow_sh);
@@ -357,16 +367,32 @@ int pick_bn(long long n)
 
 }  // namespace
 
-size_t bwd_workspace_bytes(const sadmm_plan* plan, const Geometry& g)
+size_t bwd_workspace_bytes(const sadmm_plan* plan, const Geometry& g, long long chunk)
 {
-    return layout(geometry(plan, g)).total;
+    return layout(geometry(plan, g, chunk > 0 ? chunk : kBwdMaxChunk)).total;
+}
+
+// The largest chunk (a multiple of 256 pixels, at most the layer or
+// kBwdMaxChunk) whose workspace fits ws_bytes; 0 when not even 256 pixels fit.
+long long bwd_chunk_for(const sadmm_plan* plan, const Geometry& g, size_t ws_bytes)
+{
+    // The layout is not monotonic in the chunk (the weight-gradient split
+    // count, and so its partial-sum slices, follows the chunk's divisors), so
+    // every candidate from the largest down is checked: at most 128 of them.
+    for (long long c = std::min<long long>(rup(g.m, 256), kBwdMaxChunk) / 256; c >= 1; --c)
+        if (layout(geometry(plan, g, c * 256)).total <= ws_bytes) return c * 256;
+    return 0;
 }
 
 sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const void* x, const void* dy, const void* y,
-                             int ydt, int relu, float* dW, float* db, float* dx, void* ws, cudaStream_t s)
+                             int ydt, int relu, float* dW, float* db, float* dx, void* ws, size_t ws_bytes,
+                             cudaStream_t s)
 {
     if (g.m >= (1ll << 31)) return SADMM_EUNSUPPORTED;  // pixel indices decode in 32 bits
-    BwdGeo b = geometry(plan, g);
+    const long long chunk = bwd_chunk_for(plan, g, ws_bytes);
+    if (chunk <= 0) return SADMM_EINVAL;
+    BwdGeo b = geometry(plan, g, chunk);
+    if (layout(b).total > ws_bytes) return SADMM_EINVAL;
     const char* base = static_cast<const char*>(plan->dev);
     b.x = static_cast<const __nv_bfloat16*>(x);
     b.dy = static_cast<const __nv_bfloat16*>(dy);
@@ -407,10 +433,10 @@ sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const vo
         if (dx)
             launch_pdl(k_bwd_transpose_wp, dim3((unsigned)((b.fk + 255) / 256), (unsigned)b.kr), dim3(256), 0, s, b,
                        grp, wp, wpt);
-        for (long long m0 = 0; m0 < g.m && st == SADMM_OK; m0 += b.mc) {
-            const unsigned dyrows = (unsigned)std::max(b.fr, b.fk);
+        for (long long m0 = 0; (dW || dx) && m0 < g.m && st == SADMM_OK; m0 += b.mc) {
+            const unsigned dyrows = (unsigned)std::max(dW ? b.fr : 0, dx ? b.fk : 0);
             launch_pdl(k_bwd_gather_dy, dim3((unsigned)((b.mc + kDyPix - 1) / kDyPix), (dyrows + kDyRows - 1) / kDyRows),
-                       dim3(256), 0, s, b, grp, m0, gt, gm);
+                       dim3(256), 0, s, b, grp, m0, dW ? gt : nullptr, dx ? gm : nullptr);
             if (dW) {
                 launch_pdl(k_bwd_im2col, dim3(tblocks, tcols), dim3(256), 0, s, b, grp, m0, at);
                 // split z: dws[z][i][j] (+)= sum over its pixels m of gt[i][m] * at[j][m]

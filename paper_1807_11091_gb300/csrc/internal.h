@@ -65,9 +65,12 @@ sadmm_status launch_gemm(const void* A, const void* B, float* C, long long M, lo
                          long long slice = 0);
 
 // ---- masked-retraining backward (bwd.cu) ----
-size_t bwd_workspace_bytes(const sadmm_plan* plan, const Geometry& g);
+// Workspace of chunks of `chunk` output pixels (0: the default, the whole
+// layer up to 32768 pixels); the smallest chunk is 256 pixels.
+size_t bwd_workspace_bytes(const sadmm_plan* plan, const Geometry& g, long long chunk = 0);
 sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const void* x, const void* dy, const void* y,
-                             int ydt, int relu, float* dW, float* db, float* dx, void* ws, cudaStream_t s);
+                             int ydt, int relu, float* dW, float* db, float* dx, void* ws, size_t ws_bytes,
+                             cudaStream_t s);
 
 // ---- pack (pack.cu) ----
 sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* filt_idx,

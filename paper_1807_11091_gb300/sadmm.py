@@ -126,6 +126,8 @@ def load():
     lib.sadmm_admm_update_elements.argtypes = [P(ConvDesc), vp, vp, vp, ci, ll, vp, sz, vp]
     lib.sadmm_conv_bwd_workspace_size.restype = sz
     lib.sadmm_conv_bwd_workspace_size.argtypes = [P(Plan)]
+    lib.sadmm_conv_bwd_workspace_size_chunk.restype = sz
+    lib.sadmm_conv_bwd_workspace_size_chunk.argtypes = [P(Plan), ll]
     lib.sadmm_conv_bwd.restype = ci
     lib.sadmm_conv_bwd.argtypes = [P(Plan), vp, vp, vp, ci, ci, vp, vp, vp, vp, sz, vp]
     lib.sadmm_gemm_bf16.restype = ci
@@ -248,6 +250,10 @@ def sadmm_conv_fwd(plan: Plan, x: int, bias: Optional[int], relu: int, y: int, y
 
 def sadmm_conv_bwd_workspace_size(plan: Plan) -> int:
     return load().sadmm_conv_bwd_workspace_size(ctypes.byref(plan))
+
+
+def sadmm_conv_bwd_workspace_size_chunk(plan: Plan, chunk_pixels: int) -> int:
+    return load().sadmm_conv_bwd_workspace_size_chunk(ctypes.byref(plan), int(chunk_pixels))
 
 
 def sadmm_conv_bwd(plan: Plan, x: Optional[int], dy: int, y: Optional[int], ydt: int, relu: int, dW: Optional[int],
@@ -397,15 +403,19 @@ class PrunedConv:
                         self.plan.dev_bytes, _stream(stream))
         _check(st, "sadmm_pack")
 
-    def backward(self, x, dy, y=None, relu=True, want_dw=True, want_db=True, want_dx=True, stream=None):
-        """Runs sadmm_conv_bwd; returns (dW, db, dx) fp32 device tensors (None where not requested)."""
+    def backward(self, x, dy, y=None, relu=True, want_dw=True, want_db=True, want_dx=True, stream=None,
+                 chunk_pixels=0):
+        """Runs sadmm_conv_bwd; returns (dW, db, dx) fp32 device tensors (None where not requested).
+        chunk_pixels > 0 sizes the workspace for chunks of that many output pixels
+        (default: chunks of up to 32768 pixels)."""
         torch = _torch()
         n, c, t, h, w, f, g, kt, kh, kw = self.desc16[:10]
         dev = dy.device
         dW = torch.empty((f, (c // g) * kt * kh * kw), dtype=torch.float32, device=dev) if want_dw else None
         db = torch.empty(f, dtype=torch.float32, device=dev) if want_db else None
         dx = torch.empty(x.shape, dtype=torch.float32, device=dev) if want_dx else None
-        ws_bytes = sadmm_conv_bwd_workspace_size(self.plan)
+        ws_bytes = (sadmm_conv_bwd_workspace_size_chunk(self.plan, chunk_pixels) if chunk_pixels > 0
+                    else sadmm_conv_bwd_workspace_size(self.plan))
         ws = torch.empty(ws_bytes + 1024, dtype=torch.uint8, device=dev)
         wptr = (_ptr(ws) + 1023) // 1024 * 1024
         ydt = SADMM_BF16 if (y is not None and y.dtype == torch.bfloat16) else SADMM_FP32

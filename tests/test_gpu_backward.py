@@ -50,7 +50,7 @@ CASES = [
 ]
 
 
-def _backward(s, t, kf, ck, kc, relu=True, seed=0):
+def _backward(s, t, kf, ck, kc, relu=True, seed=0, chunk_pixels=0):
     from paper_1807_11091_gb300 import sadmm
     dev = torch.device("cuda", 0)
     rows, cols, _, _ = oracle.project(t["W"], s.taps, kf, ck, kc)
@@ -63,7 +63,7 @@ def _backward(s, t, kf, ck, kc, relu=True, seed=0):
     fi = torch.as_tensor(rows, dtype=torch.int32, device=dev)
     ci = torch.as_tensor(cols, dtype=torch.int32, device=dev) if ck != wl.COL_NONE else None
     pc = sadmm.PrunedConv(s.desc16(), W, fi if kf < s.f else None, ck, ci, kf, kc if ck != wl.COL_NONE else s.k)
-    dW, db, dx = pc.backward(x, dy.to(dev), y=y.to(dev), relu=relu)
+    dW, db, dx = pc.backward(x, dy.to(dev), y=y.to(dev), relu=relu, chunk_pixels=chunk_pixels)
     assert sadmm.device_status() == 0
     rdx, rdW, rdb = oracle.pruned_conv_backward(t["x"], t["W"], t["bias"], s.desc16(), s.taps, rows, ck, cols, dy,
                                                 relu=relu, y=y)
@@ -107,17 +107,36 @@ def test_backward_without_relu():
     assert_close(dx, rdx, what="no relu dx")
 
 
-def test_backward_several_pixel_chunks():
-    """41772 output pixels: two chunks of the backward (32768 + a ragged 9004),
-    so the weight gradient accumulates per pixel split across chunks."""
+@pytest.mark.parametrize("chunk", [32768, 9984, 256])
+def test_backward_several_pixel_chunks(chunk):
+    """41772 output pixels in chunks as large as a smaller workspace holds:
+    32768 + a ragged 9004, five chunks, or 164 chunks of 256, so the weight
+    gradient accumulates per pixel split across chunks."""
     s = ConvShape(n=3, c=6, h=120, w=120, f=24, kh=3, kw=3)
     kf, kc = wl.retained(0.75, s.f), wl.retained(0.6, s.k)
     assert s.n * s.oh * s.ow > 32768
     t = wl.gen_tensors(s, seed=21)
-    (dW, db, dx), (rdW, rdb, rdx), rows, cols = _backward(s, t, kf, wl.COL_SHAPE, kc)
-    assert_close(dW, rdW, what="two chunks dW")
-    assert_close(db, rdb, what="two chunks db")
-    assert_close(dx, rdx, what="two chunks dx")
+    (dW, db, dx), (rdW, rdb, rdx), rows, cols = _backward(s, t, kf, wl.COL_SHAPE, kc, chunk_pixels=chunk)
+    assert_close(dW, rdW, what=f"chunks of {chunk}: dW")
+    assert_close(db, rdb, what=f"chunks of {chunk}: db")
+    assert_close(dx, rdx, what=f"chunks of {chunk}: dx")
+
+
+def test_backward_workspace_below_one_chunk_is_rejected():
+    from paper_1807_11091_gb300 import sadmm
+    s = ConvShape(n=1, c=4, h=9, w=9, f=8, kh=3, kw=3)
+    t = wl.gen_tensors(s, seed=2)
+    dev = torch.device("cuda", 0)
+    pc = sadmm.PrunedConv(s.desc16(), t["W"].to(dev), None, wl.COL_NONE, None, s.f, s.k)
+    small = sadmm.sadmm_conv_bwd_workspace_size_chunk(pc.plan, 256)
+    assert 0 < small <= sadmm.sadmm_conv_bwd_workspace_size(pc.plan)
+    ws = torch.empty(small + 2048, dtype=torch.uint8, device=dev)
+    wptr = (ws.data_ptr() + 1023) // 1024 * 1024
+    x, dy = t["x"].to(dev), torch.zeros((1, 8, 7, 7), dtype=torch.bfloat16, device=dev)
+    dx = torch.empty(x.shape, device=dev)
+    st = sadmm.sadmm_conv_bwd(pc.plan, x.data_ptr(), dy.data_ptr(), None, sadmm.SADMM_FP32, 0, None, None,
+                              dx.data_ptr(), wptr, small - 1024, int(torch.cuda.current_stream().cuda_stream))
+    assert st == sadmm.SADMM_EINVAL
 
 
 def _raw_backward(pc, x, dy, y, want_dw, want_dx):
@@ -140,8 +159,9 @@ def _raw_backward(pc, x, dy, y, want_dw, want_dx):
 
 def test_backward_weight_gradient_deterministic_and_partial_calls():
     """dW and db come out bit-identical on every call (fixed-order sums); a call
-    that asks for the weight gradient only, or the input gradient only, gives
-    what the full call gives (dx up to its atomic summation order)."""
+    that asks for the weight gradient only, the input gradient only, or the bias
+    gradient only gives what the full call gives (dx up to its atomic
+    summation order)."""
     from paper_1807_11091_gb300 import sadmm
     name, s, ff, ck, cf = CASES[1]
     kf, kc = wl.retained(ff, s.f), wl.retained(cf, s.k)
@@ -163,3 +183,12 @@ def test_backward_weight_gradient_deterministic_and_partial_calls():
     none, _, dx4 = _raw_backward(pc, x, dy, y, False, True)
     assert torch.isfinite(dx4).all()
     assert_close(dx4.cpu().numpy(), dx1.cpu().double().numpy(), tol=1e-6, what="dx alone")
+    # the bias gradient alone (no pixel chunk is gathered)
+    db5 = torch.full_like(db1, float("nan"))
+    ws_bytes = sadmm.sadmm_conv_bwd_workspace_size(pc.plan)
+    ws = torch.empty(ws_bytes + 1024, dtype=torch.uint8, device=dev)
+    wptr = (ws.data_ptr() + 1023) // 1024 * 1024
+    st = sadmm.sadmm_conv_bwd(pc.plan, x.data_ptr(), dy.data_ptr(), y.data_ptr(), sadmm.SADMM_FP32, 1, None,
+                              db5.data_ptr(), None, wptr, ws_bytes, int(torch.cuda.current_stream().cuda_stream))
+    assert st == 0 and sadmm.device_status() == 0
+    assert torch.equal(db1, db5)
