@@ -76,8 +76,8 @@ sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const vo
 sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* filt_idx,
                          const int* col_idx, cudaStream_t s);
 
-sadmm_status launch_pack_slab(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* col_idx,
-                              cudaStream_t s);
+// TMA descriptors of a slab plan's weights and space-to-depth input (host only).
+sadmm_status launch_pack_slab(sadmm_plan* plan, const Geometry& g);
 
 // ---- input-slab forward (conv_slab.cu) ----
 // Shared-memory stages (one tile's slab each) the slab kernel can hold with

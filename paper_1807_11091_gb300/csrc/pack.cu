@@ -34,6 +34,10 @@ struct PackArgs {
     int* rowmap;
     int* zeromap;
     int* counts;
+    // input-slab plans (scol != NULL): slab column map and kept channel list
+    int* scol;   // [xs_kpad] slab column -> GEMM column (-1: zero)
+    int* chan;   // [xs_cs] kept input channels (-1 past them)
+    int C, xs_cs, xs_kpad, xs_r, xs_q, sh, sw;
 };
 
 // First position p in the ascending list a[0..n) with a[p] >= v.
@@ -100,6 +104,10 @@ __global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status, int
             a.gather[j] = make_uint2(0u, 1u << 31);
         }
         for (int st = tid; st < a.k_pad / 64; st += blockDim.x) a.stage_chan[st] = make_int2(0, -1);
+        if (a.scol) {
+            for (int j = tid; j < a.xs_kpad; j += blockDim.x) a.scol[j] = -1;
+            for (int ci = tid; ci < a.xs_cs; ci += blockDim.x) a.chan[ci] = -1;
+        }
         return;
     }
     // kept-filter range of each conv group in the ascending filter list
@@ -158,6 +166,29 @@ __global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status, int
         const int j0 = st * 64, j1 = min(j0 + 63, a.n_cols - 1);
         a.stage_chan[st] = (j1 < j0) ? make_int2(0, -1) : make_int2(a.colidx[j0] / a.taps, a.colidx[j1] / a.taps);
     }
+    if (a.scol) {
+        // Slab column order of the input-slab path: column j is block tap
+        // (r, q) = (j / cs / Q, j / cs % Q) and slab channel cc = j % cs =
+        // (ci * sh + a) * sw + b, i.e. kept channel ci at phase (a, b); it holds
+        // GEMM column chan[ci] * taps + (r*sh + a) * KW + q*sw + b, or nothing
+        // (-1) past the kernel, the kept channels or the slab width.
+        const int nck = a.colkind == SADMM_COL_CHANNEL ? a.n_colgroups : a.C;
+        for (int ci = tid; ci < a.xs_cs; ci += blockDim.x)
+            a.chan[ci] = ci < nck ? (a.colkind == SADMM_COL_CHANNEL ? a.col_idx[ci] : ci) : -1;
+        const int rq_cols = a.xs_r * a.xs_q * a.xs_cs;
+        for (int j = tid; j < a.xs_kpad; j += blockDim.x) {
+            int col = -1;
+            const int tap = j / a.xs_cs, cc = j - tap * a.xs_cs;
+            const int r = tap / a.xs_q, q = tap - r * a.xs_q;
+            const int ci = cc / (a.sh * a.sw), pa = (cc / a.sw) % a.sh, pb = cc % a.sw;
+            const int kh = r * a.sh + pa, kw = q * a.sw + pb;
+            if (j < rq_cols && ci < nck && kh < a.KH && kw < a.KW) {
+                const int ch = a.colkind == SADMM_COL_CHANNEL ? a.col_idx[ci] : ci;
+                col = ch * a.taps + kh * a.KW + kw;
+            }
+            a.scol[j] = col;
+        }
+    }
 }
 
 template <typename T>
@@ -167,13 +198,22 @@ SADMM_DEV float load_f32<__nv_bfloat16>(const __nv_bfloat16* p) { return __bfloa
 template <>
 SADMM_DEV float load_f32<float>(const float* p) { return *p; }
 
+// Blocks past `rows` pack the input-slab plan's weights: row r - rows of
+// conv group 0 through the slab column map scol, into wps [bn][kpad_s].
 template <typename T>
 __global__ void __launch_bounds__(128) k_pack_wp(const T* __restrict__ W, int K, const int* __restrict__ rowmap,
                                                  const int* __restrict__ colidx, int k_pad,
-                                                 __nv_bfloat16* __restrict__ wp)
+                                                 __nv_bfloat16* __restrict__ wp, long long rows,
+                                                 const int* __restrict__ scol, int kpad_s, __nv_bfloat16* wps)
 {
     pdl_wait();  // after the kernel before it in the stream
-    const long long r = blockIdx.x;
+    long long r = blockIdx.x;
+    if (r >= rows) {
+        r -= rows;
+        colidx = scol;
+        k_pad = kpad_s;
+        wp = wps;
+    }
     const int f = rowmap[r];
     uint4* dst = reinterpret_cast<uint4*>(wp + r * k_pad);
     for (int j8 = threadIdx.x; j8 < k_pad / 8; j8 += blockDim.x) {
@@ -188,39 +228,6 @@ __global__ void __launch_bounds__(128) k_pack_wp(const T* __restrict__ W, int K,
             w[e] = *reinterpret_cast<const uint32_t*>(&p);
         }
         dst[j8] = make_uint4(w[0], w[1], w[2], w[3]);
-    }
-}
-
-// Slab column order of the input-slab path: column j is block tap
-// (r, q) = (j / cs / Q, j / cs % Q), slab channel cc = j % cs = (ci, a, b) with
-// cc = (ci * sh + a) * sw + b, i.e. kept channel ci at phase (a, b); it holds
-// GEMM column chan[ci] * taps + (r*sh + a) * KW + q*sw + b, or nothing (-1)
-// past the kernel, the kept channels or the slab width.  chan[ci] is the ci-th
-// kept input channel (-1 past them, or for an entry of a bad list).
-__global__ void __launch_bounds__(256) k_pack_slab_meta(const int* col_idx, int nck, int C, int cs, int kpad_s,
-                                                       int nsteps_cols, int Q, int sh, int sw, int KH, int KW,
-                                                       int taps, int* scol, int* chan)
-{
-    pdl_wait();  // after the kernel before it in the stream
-    for (int ci = threadIdx.x; ci < cs; ci += blockDim.x) {
-        int ch = -1;
-        if (ci < nck) {
-            ch = col_idx ? col_idx[ci] : ci;
-            if (ch < 0 || ch >= C) ch = -1;
-        }
-        chan[ci] = ch;
-    }
-    __syncthreads();
-    for (int j = threadIdx.x; j < kpad_s; j += blockDim.x) {
-        int col = -1;
-        if (j < nsteps_cols) {
-            const int tap = j / cs, cc = j - tap * cs;
-            const int r = tap / Q, q = tap - r * Q;
-            const int ci = cc / (sh * sw), a = (cc / sw) % sh, b = cc % sw;
-            const int kh = r * sh + a, kw = q * sw + b;
-            if (ci < nck && kh < KH && kw < KW && chan[ci] >= 0) col = chan[ci] * taps + kh * KW + kw;
-        }
-        scol[j] = col;
     }
 }
 
@@ -273,6 +280,19 @@ sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int
     a.rowmap = reinterpret_cast<int*>(base + plan->off_rowmap);
     a.zeromap = reinterpret_cast<int*>(base + plan->off_zeromap);
     a.counts = reinterpret_cast<int*>(base + plan->off_counts);
+    a.scol = nullptr;
+    a.chan = nullptr;
+    a.C = (int)g.c;
+    if (plan->xs_mode) {
+        a.scol = reinterpret_cast<int*>(base + plan->off_scol);
+        a.chan = a.scol + plan->xs_kpad;
+        a.xs_cs = plan->xs_cs;
+        a.xs_kpad = plan->xs_kpad;
+        a.xs_r = plan->xs_r;
+        a.xs_q = plan->xs_q;
+        a.sh = (int)g.sh;
+        a.sw = (int)g.sw;
+    }
     const size_t list_bytes =
         (size_t)((a.all_kept ? 0 : a.n_filt) + ((col_idx && a.colkind != SADMM_COL_NONE) ? a.n_colgroups : 0)) * 4;
     const bool in_smem = list_bytes <= 40 * 1024;
@@ -281,12 +301,15 @@ sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int
 
     __nv_bfloat16* wp = reinterpret_cast<__nv_bfloat16*>(base + plan->off_wp);
     const unsigned rows = (unsigned)(g.groups * plan->n_pad);
+    // a slab plan also packs its weights in slab column order, in the same launch
+    __nv_bfloat16* wps = plan->xs_mode ? reinterpret_cast<__nv_bfloat16*>(base + plan->off_wps) : nullptr;
+    const unsigned srows = plan->xs_mode ? (unsigned)plan->bn : 0u;
     if (wdt == SADMM_BF16)
-        launch_pdl(k_pack_wp<__nv_bfloat16>, dim3(rows), dim3(128), 0, s, (const __nv_bfloat16*)W, (int)g.k,
-                   a.rowmap, a.colidx, plan->k_pad, wp);
+        launch_pdl(k_pack_wp<__nv_bfloat16>, dim3(rows + srows), dim3(128), 0, s, (const __nv_bfloat16*)W, (int)g.k,
+                   a.rowmap, a.colidx, plan->k_pad, wp, (long long)rows, (const int*)a.scol, plan->xs_kpad, wps);
     else
-        launch_pdl(k_pack_wp<float>, dim3(rows), dim3(128), 0, s, (const float*)W, (int)g.k, a.rowmap, a.colidx,
-                   plan->k_pad, wp);
+        launch_pdl(k_pack_wp<float>, dim3(rows + srows), dim3(128), 0, s, (const float*)W, (int)g.k, a.rowmap,
+                   a.colidx, plan->k_pad, wp, (long long)rows, (const int*)a.scol, plan->xs_kpad, wps);
     if (cudaGetLastError() != cudaSuccess) return SADMM_ECUDA;
 
     // TMA descriptor of Wp: [groups*n_pad rows][k_pad bf16], boxes of 64 x bn,
@@ -305,29 +328,16 @@ sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int
     if (r != CUDA_SUCCESS) return SADMM_ECUDA;
     static_assert(sizeof(CUtensorMap) == sizeof(plan->tmap), "tensor map size");
     memcpy(plan->tmap, &map, sizeof(map));
-    if (plan->xs_mode) return launch_pack_slab(plan, g, W, wdt, col_idx, s);
+    if (plan->xs_mode) return launch_pack_slab(plan, g);
     return SADMM_OK;
 }
 
-sadmm_status launch_pack_slab(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* col_idx,
-                              cudaStream_t s)
+sadmm_status launch_pack_slab(sadmm_plan* plan, const Geometry& g)
 {
+    // the slab column map, kept channels and slab-ordered weights were written
+    // by k_pack_meta and k_pack_wp; here only their TMA descriptors
     char* base = static_cast<char*>(plan->dev);
-    int* scol = reinterpret_cast<int*>(base + plan->off_scol);
-    int* chan = scol + plan->xs_kpad;
-    const int nck = plan->colkind == SADMM_COL_CHANNEL ? plan->n_colgroups : (int)g.c;
-    launch_pdl(k_pack_slab_meta, dim3(1), dim3(256), 0, s, plan->colkind == SADMM_COL_CHANNEL ? col_idx : nullptr,
-               nck, (int)g.c, plan->xs_cs, plan->xs_kpad, plan->xs_r * plan->xs_q * plan->xs_cs, plan->xs_q,
-               (int)g.sh, (int)g.sw, (int)g.kh, (int)g.kw, (int)g.taps, scol, chan);
-    const int* rowmap = reinterpret_cast<const int*>(base + plan->off_rowmap);
     __nv_bfloat16* wps = reinterpret_cast<__nv_bfloat16*>(base + plan->off_wps);
-    if (wdt == SADMM_BF16)
-        launch_pdl(k_pack_wp<__nv_bfloat16>, dim3((unsigned)plan->bn), dim3(128), 0, s, (const __nv_bfloat16*)W,
-                   (int)g.k, rowmap, (const int*)scol, plan->xs_kpad, wps);
-    else
-        launch_pdl(k_pack_wp<float>, dim3((unsigned)plan->bn), dim3(128), 0, s, (const float*)W, (int)g.k, rowmap,
-                   (const int*)scol, plan->xs_kpad, wps);
-    if (cudaGetLastError() != cudaSuccess) return SADMM_ECUDA;
     PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
     if (!enc) return SADMM_ECUDA;
     {
