@@ -225,11 +225,17 @@ class LayerRun:
                               self.buf.data_ptr(), self.plan.dev_bytes, stream)
         assert st == 0, st
 
-    def conv(self, stream):
+    def conv(self, stream, phase=0):
+        """sadmm_conv_fwd, or one phase of it (sadmm_conv_fwd_phase)."""
         from paper_1807_11091_gb300 import sadmm
-        st = sadmm.sadmm_conv_fwd(self.plan, self.x.data_ptr(), self.bias.data_ptr(), 1, self.y.data_ptr(),
-                                  self.ydt, stream)
+        st = sadmm.sadmm_conv_fwd_phase(self.plan, self.x.data_ptr(), self.bias.data_ptr(), 1, self.y.data_ptr(),
+                                        self.ydt, phase, stream)
         assert st == 0, st
+
+    @property
+    def early_input(self):
+        """The forward's input pass reads only x: it can run before the pack."""
+        return bool(self.plan.xs_mode) and self.colkind != wl.COL_CHANNEL
 
 
 class StepStreams:
@@ -249,7 +255,12 @@ class StepStreams:
 
 
 def enqueue_step(runs, ss, conv_events=None):
+    """One step.  An input-slab layer without channel pruning (the first
+    layer) runs its forward's input pass on the main stream at once, beside its
+    projection and pack, then the rest after them.  With conv_events (the
+    per-layer breakdown) every forward runs as one call between its events."""
     import torch
+    from paper_1807_11091_gb300 import sadmm
     ss.fork.record(ss.main)
     for r, side, done in zip(runs, ss.side, ss.done):
         side.wait_event(ss.fork)
@@ -258,11 +269,15 @@ def enqueue_step(runs, ss, conv_events=None):
         r.pack(sp)
         done.record(side)
     mp = int(ss.main.cuda_stream)
+    split = conv_events is None
+    for r in runs:
+        if split and r.early_input:
+            r.conv(mp, sadmm.SADMM_FWD_INPUT)
     for i, (r, done) in enumerate(zip(runs, ss.done)):
         ss.main.wait_event(done)
         if conv_events is not None:
             conv_events[i][0].record(ss.main)
-        r.conv(mp)
+        r.conv(mp, sadmm.SADMM_FWD_REST if split and r.early_input else sadmm.SADMM_FWD_ALL)
         if conv_events is not None:
             conv_events[i][1].record(ss.main)
 
@@ -274,21 +289,30 @@ def enqueue_step_e2e(runs, ss, copy_stream, h_x, h_w, h_b, h_y):
     conv has run, under the later layers' convs.  The main stream joins the copy
     stream at the end, so an event recorded after this call covers every copy."""
     import torch
+    from paper_1807_11091_gb300 import sadmm
     ss.fork.record(ss.main)
+    x_ready = []
     for r, side, done, a, b, c in zip(runs, ss.side, ss.done, h_x, h_w, h_b):
         side.wait_event(ss.fork)
         with torch.cuda.stream(side):
+            r.x.copy_(a, non_blocking=True)
+            ev = torch.cuda.Event()
+            ev.record(side)
+            x_ready.append(ev)
             r.W.copy_(b, non_blocking=True)
             r.bias.copy_(c, non_blocking=True)
-            r.x.copy_(a, non_blocking=True)
         sp = int(side.cuda_stream)
         r.project(sp)
         r.pack(sp)
         done.record(side)
     mp = int(ss.main.cuda_stream)
+    for r, ev in zip(runs, x_ready):
+        if r.early_input:
+            ss.main.wait_event(ev)
+            r.conv(mp, sadmm.SADMM_FWD_INPUT)
     for r, done, hy in zip(runs, ss.done, h_y):
         ss.main.wait_event(done)
-        r.conv(mp)
+        r.conv(mp, sadmm.SADMM_FWD_REST if r.early_input else sadmm.SADMM_FWD_ALL)
         ev = torch.cuda.Event()
         ev.record(ss.main)
         copy_stream.wait_event(ev)
@@ -742,8 +766,9 @@ def run_gpu(args):
                    "out_dtype": args.out_dtype,
                    "l2": "flushed before every timed step (256 MiB write, outside the timed window)",
                    "schedule": f"projection+pack of each layer on its own stream; convs back to back on the "
-                               f"main stream; first conv on {first_ctas or n_sm} of {n_sm} SMs",
-                   "breakdown": "per-conv times from separate steps with CUDA events around each conv",
+                               f"main stream; first conv on {first_ctas or n_sm} of {n_sm} SMs, its input-slab "
+                               f"space-to-depth pass issued at the step's start beside the projections and packs",
+                   "breakdown": "per-conv times from separate steps with CUDA events around each whole forward call",
                    "parallelism": "one replica per GPU, batch per GPU fixed, no collective"},
         "pct_bf16_peak": value / peaks["bf16_tflops"],
         "speedup_vs_dense": dense_step / pruned_step_med,

@@ -333,6 +333,29 @@ sadmm_status sadmm_conv_fwd(const sadmm_plan* plan, const void* x, const float* 
                             int relu, void* y, int ydt, void* stream);
 
 /*
+ * sadmm_conv_fwd in two calls, so that a caller can overlap an input-slab
+ * plan's space-to-depth pass with other work (the layer's projection and
+ * pack, for the first layer of a network, whose input is ready before its
+ * weights are):
+ *   SADMM_FWD_INPUT  the space-to-depth pass alone (x read, the plan's copy
+ *                    written; nothing for a gathered plan).  Without channel
+ *                    pruning it reads nothing sadmm_pack writes, so it may
+ *                    run while the plan is being packed again (the plan must
+ *                    have been packed once: its buffer is bound); with channel
+ *                    pruning it reads the kept-channel list and must follow
+ *                    sadmm_pack.
+ *   SADMM_FWD_REST   the rest: for a slab plan the conv kernel on the copy
+ *                    the last INPUT call wrote (x unused, may be NULL); a
+ *                    gathered plan runs whole.
+ *   SADMM_FWD_ALL    both (= sadmm_conv_fwd).
+ * The caller orders INPUT before REST (same stream, or an event).  Results
+ * equal those of sadmm_conv_fwd bit for bit.
+ */
+typedef enum { SADMM_FWD_ALL = 0, SADMM_FWD_INPUT = 1, SADMM_FWD_REST = 2 } sadmm_fwd_phase;
+sadmm_status sadmm_conv_fwd_phase(const sadmm_plan* plan, const void* x, const float* bias,
+                                  int relu, void* y, int ydt, int phase, void* stream);
+
+/*
  * sadmm_project_groups without a caller-provided workspace.  The paper has no
  * counterpart: this exists for callers that cannot hand the library device
  * scratch memory -- a plugin or host framework that passes only its input and

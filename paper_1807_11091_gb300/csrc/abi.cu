@@ -401,19 +401,29 @@ sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt, const int* fil
     return SADMM_OK;
 }
 
-sadmm_status sadmm_conv_fwd(const sadmm_plan* plan, const void* x, const float* bias, int relu, void* y,
-                            int ydt, void* stream)
+sadmm_status sadmm_conv_fwd_phase(const sadmm_plan* plan, const void* x, const float* bias, int relu, void* y,
+                                  int ydt, int phase, void* stream)
 {
-    if (!plan || !x || !y || !plan->dev) return SADMM_EINVAL;
+    if (!plan || !plan->dev) return SADMM_EINVAL;
+    if (phase != SADMM_FWD_ALL && phase != SADMM_FWD_INPUT && phase != SADMM_FWD_REST) return SADMM_EINVAL;
+    const bool needs_x = phase != SADMM_FWD_REST || !plan->xs_mode;  // the rest of a slab plan reads its copy
+    const bool needs_y = phase != SADMM_FWD_INPUT;
+    if ((needs_x && !x) || (needs_y && !y)) return SADMM_EINVAL;
     Geometry g;
     sadmm_status st = check_desc(&plan->desc, &g);
     if (st != SADMM_OK) return st;
-    if (ydt != SADMM_BF16 && ydt != SADMM_FP32) return SADMM_EINVAL;
+    if (needs_y && ydt != SADMM_BF16 && ydt != SADMM_FP32) return SADMM_EINVAL;
     if ((reinterpret_cast<uintptr_t>(x) & 1) != 0) return SADMM_EINVAL;
-    if ((reinterpret_cast<uintptr_t>(y) & (ydt == SADMM_FP32 ? 3 : 1)) != 0) return SADMM_EINVAL;
+    if (needs_y && (reinterpret_cast<uintptr_t>(y) & (ydt == SADMM_FP32 ? 3 : 1)) != 0) return SADMM_EINVAL;
     if (bias && (reinterpret_cast<uintptr_t>(bias) & 3) != 0) return SADMM_EINVAL;
     if (device_cc_major() < 10) return SADMM_EUNSUPPORTED;
-    return launch_conv_fwd(plan, g, x, bias, relu, y, ydt, static_cast<cudaStream_t>(stream));
+    return launch_conv_fwd(plan, g, x, bias, relu, y, ydt, phase, static_cast<cudaStream_t>(stream));
+}
+
+sadmm_status sadmm_conv_fwd(const sadmm_plan* plan, const void* x, const float* bias, int relu, void* y,
+                            int ydt, void* stream)
+{
+    return sadmm_conv_fwd_phase(plan, x, bias, relu, y, ydt, SADMM_FWD_ALL, stream);
 }
 
 size_t sadmm_conv_bwd_workspace_size(const sadmm_plan* plan)

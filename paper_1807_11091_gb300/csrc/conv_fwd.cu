@@ -825,9 +825,10 @@ cudaError_t launch(const CUtensorMap& map, const ConvArgs& a, int grid, size_t s
 }  // namespace
 
 sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const void* x, const float* bias,
-                             int relu, void* y, int ydt, cudaStream_t s)
+                             int relu, void* y, int ydt, int phase, cudaStream_t s)
 {
-    if (plan->xs_mode) return launch_conv_slab(plan, g, x, bias, relu, y, ydt, s);
+    if (plan->xs_mode) return launch_conv_slab(plan, g, x, bias, relu, y, ydt, phase, s);
+    if (phase == SADMM_FWD_INPUT) return SADMM_OK;  // the gathered path reads x in its own kernel
     if (g.groups > kMaxGroups) return SADMM_EUNSUPPORTED;
     const char* base = static_cast<const char*>(plan->dev);
     ConvArgs a;

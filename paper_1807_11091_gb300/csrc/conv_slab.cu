@@ -86,7 +86,7 @@ __global__ void __launch_bounds__(kXsPix * kXsRows) k_slab_input(const __nv_bflo
     if (tid < b.cs) {
         const int cc = tid;
         const int ci = cc / (b.sh * b.sw);
-        const int ch = ci < b.nck ? __ldg(chan + ci) : -1;
+        const int ch = ci < b.nck ? (chan ? __ldg(chan + ci) : ci) : -1;
         s_dec[cc] = make_int4(ch >= 0 ? ch * b.H * b.W : -1, (cc / b.sw) % b.sh - b.ph, cc % b.sw - b.pw, 0);
     }
     __syncthreads();
@@ -338,7 +338,7 @@ int slab_stages(int bn, int kpad_s, int cs, int sp)
 }
 
 sadmm_status launch_conv_slab(const sadmm_plan* plan, const Geometry& g, const void* x, const float* bias, int relu,
-                              void* y, int ydt, cudaStream_t s)
+                              void* y, int ydt, int phase, cudaStream_t s)
 {
     const int stages = slab_stages(plan->bn, plan->xs_kpad, plan->xs_cs, plan->xs_sp);
     if (stages < 2 || plan->n_tiles != 1 || g.groups != 1 || plan->xs_cs > 64 || plan->xs_cs % 16 ||
@@ -362,14 +362,20 @@ sadmm_status launch_conv_slab(const sadmm_plan* plan, const Geometry& g, const v
     b.Hb = plan->xs_hb;
     b.Wb = plan->xs_wb;
     b.pimg = plan->xs_pimg;
-    const int* chan = reinterpret_cast<const int*>(base + plan->off_scol) + plan->xs_kpad;
+    // without channel pruning the kept channels are 0 .. C-1: the pass then
+    // reads nothing sadmm_pack writes (it may overlap the layer's pack)
+    const int* chan = plan->colkind == SADMM_COL_CHANNEL
+                          ? reinterpret_cast<const int*>(base + plan->off_scol) + plan->xs_kpad
+                          : nullptr;
     __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(const_cast<char*>(base) + plan->off_xs);
-    if (launch_pdl(k_slab_input,
+    if (phase != SADMM_FWD_REST &&
+        launch_pdl(k_slab_input,
                    dim3((unsigned)((plan->xs_wb + kXsPix - 1) / kXsPix), (unsigned)((plan->xs_hb + kXsRows - 1) / kXsRows),
                         (unsigned)g.n),
                    dim3(kXsPix, kXsRows), 0, s, static_cast<const __nv_bfloat16*>(x), chan, b, xs) != cudaSuccess)
         return SADMM_ECUDA;
 
+    if (phase == SADMM_FWD_INPUT) return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
     SlabArgs a;
     memset(&a, 0, sizeof(a));
     a.y = y;

@@ -83,12 +83,14 @@ sadmm_status launch_pack_slab(sadmm_plan* plan, const Geometry& g);
 // Shared-memory stages (one tile's slab each) the slab kernel can hold with
 // the weights resident; below 2 the slab path is not available.
 int slab_stages(int bn, int kpad_s, int cs, int sp);
+// phase: SADMM_FWD_ALL, SADMM_FWD_INPUT (the space-to-depth pass) or
+// SADMM_FWD_REST (the conv kernel on the copy the last input pass wrote).
 sadmm_status launch_conv_slab(const sadmm_plan* plan, const Geometry& g, const void* x, const float* bias, int relu,
-                              void* y, int ydt, cudaStream_t s);
+                              void* y, int ydt, int phase, cudaStream_t s);
 
 // ---- forward (conv_fwd.cu) ----
 sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const void* x, const float* bias,
-                             int relu, void* y, int ydt, cudaStream_t s);
+                             int relu, void* y, int ydt, int phase, cudaStream_t s);
 
 // Tap-mask encoding of the gather table: 0 = one bit per tap (at most 31
 // taps), 1 = (kt,kh) row bits 0..15 and kw bits 16..30.  Bit 31 marks padding

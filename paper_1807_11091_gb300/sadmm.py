@@ -19,6 +19,7 @@ from . import build as _build
 SADMM_OK, SADMM_EINVAL, SADMM_ECUDA, SADMM_ETIMEOUT, SADMM_EUNSUPPORTED = 0, -1, -2, -3, -4
 SADMM_BF16, SADMM_FP32 = 0, 1
 SADMM_COL_NONE, SADMM_COL_SHAPE, SADMM_COL_CHANNEL = 0, 1, 2
+SADMM_FWD_ALL, SADMM_FWD_INPUT, SADMM_FWD_REST = 0, 1, 2
 
 SADMM_NOALLOC_SCRATCH_BYTES = 256 * 1024  # include/sadmm.h
 
@@ -111,6 +112,8 @@ def load():
     lib.sadmm_plan_init_ctas.argtypes = [P(Plan), P(ConvDesc), ci, ci, ci, ci]
     lib.sadmm_pack.restype = ci
     lib.sadmm_pack.argtypes = [P(Plan), vp, ci, vp, vp, vp, sz, vp]
+    lib.sadmm_conv_fwd_phase.restype = ci
+    lib.sadmm_conv_fwd_phase.argtypes = [P(Plan), vp, vp, ci, vp, ci, ci, vp]
     lib.sadmm_conv_fwd.restype = ci
     lib.sadmm_conv_fwd.argtypes = [P(Plan), vp, vp, ci, vp, ci, vp]
     lib.sadmm_admm_workspace_size.restype = sz
@@ -246,6 +249,11 @@ def sadmm_pack(plan: Plan, W: int, wdt: int, filt_idx: Optional[int], col_idx: O
 def sadmm_conv_fwd(plan: Plan, x: int, bias: Optional[int], relu: int, y: int, ydt: int,
                    stream: Optional[int]) -> int:
     return load().sadmm_conv_fwd(ctypes.byref(plan), x, bias, int(relu), y, int(ydt), stream)
+
+
+def sadmm_conv_fwd_phase(plan: Plan, x: Optional[int], bias: Optional[int], relu: int, y: Optional[int], ydt: int,
+                         phase: int, stream: Optional[int]) -> int:
+    return load().sadmm_conv_fwd_phase(ctypes.byref(plan), x, bias, int(relu), y, int(ydt), int(phase), stream)
 
 
 def sadmm_conv_bwd_workspace_size(plan: Plan) -> int:

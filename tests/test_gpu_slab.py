@@ -124,3 +124,53 @@ def test_slab_more_pruned_planes_than_the_shared_table():
     ref = oracle_layer(s, t, rows, ck, cols)
     assert_close(y, ref, what="many_pruned")
     assert np.all(y[:, pruned_filters(s.f, rows)] == 0.0)
+
+
+@pytest.mark.parametrize("case", [CASES[1], CASES[4]], ids=lambda c: c[0])
+def test_slab_forward_in_two_phases(case):
+    """sadmm_conv_fwd_phase: the space-to-depth pass (INPUT) then the conv on
+    its copy (REST, x not passed) equals the single call bit for bit; with no
+    channel pruning the INPUT pass does not read the packed kept-channel list
+    (the list is overwritten here before the pass and the result is the same)."""
+    from paper_1807_11091_gb300 import sadmm
+    s, t, rows, ck, cols, y, pc = _run(case, seed=306)
+    dev = torch.device("cuda", 0)
+    x, bias = t["x"].to(dev), t["bias"].to(dev)
+    sp = int(torch.cuda.current_stream().cuda_stream)
+    y2 = torch.full(pc.out_shape(), float("nan"), device=dev)
+    if ck != wl.COL_CHANNEL:
+        assert pc.plan.dev == pc.buf.data_ptr()
+        off = pc.plan.off_scol + 4 * pc.plan.xs_kpad
+        chan = pc.buf[off:off + 4 * pc.plan.xs_cs].view(torch.int32)
+        saved = chan.clone()
+        chan.fill_(-7)
+    assert sadmm.sadmm_conv_fwd_phase(pc.plan, x.data_ptr(), None, 0, None, sadmm.SADMM_FP32,
+                                      sadmm.SADMM_FWD_INPUT, sp) == 0
+    if ck != wl.COL_CHANNEL:
+        chan.copy_(saved)
+    assert sadmm.sadmm_conv_fwd_phase(pc.plan, None, bias.data_ptr(), 1, y2.data_ptr(), sadmm.SADMM_FP32,
+                                      sadmm.SADMM_FWD_REST, sp) == 0
+    assert sadmm.device_status() == 0
+    assert np.array_equal(y2.cpu().numpy(), y)
+
+
+def test_gathered_plan_in_two_phases():
+    """For a gathered plan INPUT does nothing and REST runs the whole forward."""
+    from paper_1807_11091_gb300 import sadmm
+    s = ConvShape(n=2, c=8, h=11, w=12, f=24, kh=3, kw=3, ph=1, pw=1)
+    kf, kc = wl.retained(0.75, s.f), wl.retained(0.5, s.k)
+    t = wl.gen_tensors(s, seed=307)
+    fi, ci, y, pc = gpu_layer(s, t, kf, wl.COL_SHAPE, kc)
+    assert pc.plan.xs_mode == 0
+    dev = torch.device("cuda", 0)
+    x, bias = t["x"].to(dev), t["bias"].to(dev)
+    sp = int(torch.cuda.current_stream().cuda_stream)
+    y2 = torch.full(pc.out_shape(), float("nan"), device=dev)
+    assert sadmm.sadmm_conv_fwd_phase(pc.plan, x.data_ptr(), None, 0, None, sadmm.SADMM_FP32,
+                                      sadmm.SADMM_FWD_INPUT, sp) == 0
+    assert sadmm.sadmm_conv_fwd_phase(pc.plan, None, bias.data_ptr(), 1, y2.data_ptr(), sadmm.SADMM_FP32,
+                                      sadmm.SADMM_FWD_REST, sp) == sadmm.SADMM_EINVAL  # needs x
+    assert sadmm.sadmm_conv_fwd_phase(pc.plan, x.data_ptr(), bias.data_ptr(), 1, y2.data_ptr(), sadmm.SADMM_FP32,
+                                      sadmm.SADMM_FWD_REST, sp) == 0
+    assert sadmm.device_status() == 0
+    assert np.array_equal(y2.cpu().numpy(), y)
