@@ -174,3 +174,16 @@ def test_gathered_plan_in_two_phases():
                                       sadmm.SADMM_FWD_REST, sp) == 0
     assert sadmm.device_status() == 0
     assert np.array_equal(y2.cpu().numpy(), y)
+
+
+@pytest.mark.parametrize("case", [
+    # 4 channels x 4 x 4 phases: exactly 64 slab channels (eight chunks)
+    ("cs_64", ConvShape(n=2, c=4, h=43, w=39, f=32, kh=11, kw=11, sh=4, sw=4), 1.0, wl.COL_NONE, 1.0),
+    # a 900-wide input: 450 block pixels per row, a slab of 584 block pixels (73 octets)
+    ("wide_rows", ConvShape(n=1, c=3, h=9, w=900, f=16, kh=3, kw=3, sh=2, sw=2, ph=1, pw=1), 1.0, wl.COL_NONE,
+     1.0),
+], ids=lambda c: c[0])
+def test_slab_extreme_geometry(case):
+    s, t, rows, ck, cols, y, pc = _run(case, seed=308)
+    ref = oracle_layer(s, t, rows, ck, cols)
+    assert_close(y, ref, what=case[0])
