@@ -405,7 +405,11 @@ size_t sadmm_conv_bwd_workspace_size_chunk(const sadmm_plan* plan, long long chu
  *   dx         = the input gradient through the kept weights only.
  * The contractions run on the tensor cores (bf16 operands, fp32 accumulation);
  * dW and db are summed in a fixed order (deterministic); dx is summed with
- * fp32 atomics (its last bits depend on timing).
+ * fp32 atomics (its last bits depend on timing).  For an input-slab plan
+ * (plan->xs_mode) with at most 128 kept filters, dW is contracted on the
+ * plan's space-to-depth copy of x (rewritten by this call) instead of an
+ * im2col copy; its workspace then also holds dZ in the output's block-pixel
+ * grid and one fp32 partial dW per CTA.
  *
  *   plan   a packed plan (sadmm_pack) of the layer.
  *   x      device bf16 [N][C][T][H][W] (needed for dW).

@@ -43,6 +43,7 @@ struct BwdGeo {
     int hw;
     int split_mask;        // tap-mask encoding of the gather table (see tap_mask)
     const uint2* table;    // the plan's gather table: [k_pad] {x offset from the window origin, tap bits}
+    size_t slab_wg_bytes;  // workspace of the slab weight gradient (0: gathered weight gradient)
 };
 
 inline void divisor(uint32_t d, uint32_t& mul, uint32_t& sh)
@@ -282,7 +283,7 @@ __global__ void __launch_bounds__(256) k_bwd_zero(float* p, long long n)
 inline long long rup(long long x, long long a) { return (x + a - 1) / a * a; }
 
 struct Layout {
-    size_t at, gt, gm, wpt, dat, dws, dbp, total;
+    size_t at, gt, gm, wpt, dat, dws, dbp, wsl, total;
 };
 
 int pick_bn(long long n);
@@ -319,6 +320,7 @@ Layout layout(const BwdGeo& b)
     l.dat = take((size_t)b.kr * b.mc * 4);
     l.dws = take((size_t)wgrad_splits(b) * b.fr * b.k_pad * 4);  // [split][fr][k_pad]
     l.dbp = take((size_t)b.F * kDbSlices * 4);                    // [F][slices] bias-gradient partials
+    l.wsl = take(b.slab_wg_bytes);                                // slab weight gradient (bwd_slab.cu)
     l.total = off;
     return l;
 }
@@ -355,6 +357,7 @@ BwdGeo geometry(const sadmm_plan* plan, const Geometry& g, long long chunk)
     b.thw = g.t * g.h * g.w;
     b.hw = (int)(g.h * g.w);
     b.split_mask = tap_mask_mode(g);
+    b.slab_wg_bytes = wgrad_slab_bytes(plan, g);
     return b;
 }
 
@@ -419,6 +422,13 @@ sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const vo
     const long long K = g.cg * g.taps;
 
     if (dW) launch_pdl(k_bwd_zero, dim3(1024), dim3(256), 0, s, dW, g.f * K);
+    // an input-slab plan's weight gradient runs on its slab, not through im2col
+    const bool slab_dw = dW && b.slab_wg_bytes > 0;
+    float* gdW = slab_dw ? nullptr : dW;  // the gathered weight gradient's output
+    if (slab_dw) {
+        const sadmm_status sst = launch_wgrad_slab(plan, g, x, dy, y, ydt, relu, dW, w + l.wsl, s);
+        if (sst != SADMM_OK) return sst;
+    }
     const int wbn = pick_bn(b.k_pad);
     const int wsplit = wgrad_splits(b);
     if (dx) launch_pdl(k_bwd_zero, dim3(2048), dim3(256), 0, s, dx, g.n * g.c * g.t * g.h * g.w);
@@ -433,11 +443,11 @@ sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const vo
         if (dx)
             launch_pdl(k_bwd_transpose_wp, dim3((unsigned)((b.fk + 255) / 256), (unsigned)b.kr), dim3(256), 0, s, b,
                        grp, wp, wpt);
-        for (long long m0 = 0; (dW || dx) && m0 < g.m && st == SADMM_OK; m0 += b.mc) {
-            const unsigned dyrows = (unsigned)std::max(dW ? b.fr : 0, dx ? b.fk : 0);
+        for (long long m0 = 0; (gdW || dx) && m0 < g.m && st == SADMM_OK; m0 += b.mc) {
+            const unsigned dyrows = (unsigned)std::max(gdW ? b.fr : 0, dx ? b.fk : 0);
             launch_pdl(k_bwd_gather_dy, dim3((unsigned)((b.mc + kDyPix - 1) / kDyPix), (dyrows + kDyRows - 1) / kDyRows),
-                       dim3(256), 0, s, b, grp, m0, dW ? gt : nullptr, dx ? gm : nullptr);
-            if (dW) {
+                       dim3(256), 0, s, b, grp, m0, gdW ? gt : nullptr, dx ? gm : nullptr);
+            if (gdW) {
                 launch_pdl(k_bwd_im2col, dim3(tblocks, tcols), dim3(256), 0, s, b, grp, m0, at);
                 // split z: dws[z][i][j] (+)= sum over its pixels m of gt[i][m] * at[j][m]
                 st = launch_gemm(gt, at, dws, b.fr, b.k_pad, b.mc, b.k_pad, wbn, m0 > 0, s, wsplit,
@@ -451,7 +461,7 @@ sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const vo
                                static_cast<const float*>(dat), dx);
             }
         }
-        if (dW && st == SADMM_OK)
+        if (gdW && st == SADMM_OK)
             launch_pdl(k_bwd_reduce_dw, dim3((unsigned)((b.k_pad + 255) / 256), (unsigned)b.n_pad), dim3(256), 0, s, b,
                        grp, static_cast<const float*>(dws), wsplit, dW);
     }

@@ -90,12 +90,23 @@ __global__ void __launch_bounds__(kXsPix * kXsRows) k_slab_input(const __nv_bflo
         s_dec[cc] = make_int4(ch >= 0 ? ch * b.H * b.W : -1, (cc / b.sw) % b.sh - b.ph, cc % b.sw - b.pw, 0);
     }
     __syncthreads();
+    const int chunks = b.cs / 8;
+    if (blockIdx.x == 0 && blockIdx.y == 0) {
+        // the pixels past Hb*Wb up to pimg (fewer than 8 per chunk row) are zero:
+        // they are read by the GEMM rows past the output, and the weight gradient
+        // multiplies them by those rows' zero dZ
+        const int pad = b.pimg - b.Hb * b.Wb;
+        for (int v = tid; v < chunks * pad; v += kXsPix * kXsRows) {
+            const int k = v / pad, j = v - k * pad;
+            *reinterpret_cast<uint4*>(xs + (((long long)n * chunks + k) * b.pimg + (long long)b.Hb * b.Wb + j) * 8) =
+                make_uint4(0u, 0u, 0u, 0u);
+        }
+    }
     const int wb = blockIdx.x * kXsPix + threadIdx.x;
     const int hb = blockIdx.y * kXsRows + threadIdx.y;
     if (wb >= b.Wb || hb >= b.Hb) return;
     const unsigned short* xi = reinterpret_cast<const unsigned short*>(x) + (long long)n * b.C * b.H * b.W;
     const int ih0 = hb * b.sh, iw0 = wb * b.sw;
-    const int chunks = b.cs / 8;
     __nv_bfloat16* dst0 = xs + ((long long)n * chunks * b.pimg + (long long)hb * b.Wb + wb) * 8;
 #pragma unroll 2
     for (int k = 0; k < chunks; ++k) {

@@ -72,6 +72,17 @@ sadmm_status launch_conv_bwd(const sadmm_plan* plan, const Geometry& g, const vo
                              int ydt, int relu, float* dW, float* db, float* dx, void* ws, size_t ws_bytes,
                              cudaStream_t s);
 
+// ---- weight gradient of an input-slab plan (bwd_slab.cu) ----
+// Whether the plan's weight gradient runs on the slab (one conv group, at most
+// 128 kept filters, at most 512 slab columns); the workspace it needs (0 when
+// it does not apply); and the run: the space-to-depth pass of x into the
+// plan's copy, dZ in the output's block-pixel grid, the GEMM into per-CTA
+// slices and their ordered sum into dW (which the caller has zeroed).
+bool wgrad_slab_ok(const sadmm_plan* plan, const Geometry& g);
+size_t wgrad_slab_bytes(const sadmm_plan* plan, const Geometry& g);
+sadmm_status launch_wgrad_slab(const sadmm_plan* plan, const Geometry& g, const void* x, const void* dy,
+                               const void* y, int ydt, int relu, float* dW, void* ws, cudaStream_t s);
+
 // ---- pack (pack.cu) ----
 sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* filt_idx,
                          const int* col_idx, cudaStream_t s);

@@ -192,3 +192,30 @@ def test_backward_weight_gradient_deterministic_and_partial_calls():
                               db5.data_ptr(), None, wptr, ws_bytes, int(torch.cuda.current_stream().cuda_stream))
     assert st == 0 and sadmm.device_status() == 0
     assert torch.equal(db1, db5)
+
+
+@pytest.mark.parametrize("case", [
+    ("slab_stride4_pruned_filters", ConvShape(n=3, c=3, h=51, w=47, f=40, kh=11, kw=11, sh=4, sw=4), 0.6,
+     wl.COL_NONE, 1.0),
+    ("slab_stem_7x7_s2_p3", ConvShape(n=2, c=3, h=37, w=33, f=24, kh=7, kw=7, sh=2, sw=2, ph=3, pw=3), 1.0,
+     wl.COL_SHAPE, 1.0),
+    ("slab_channel_5x5_s2", ConvShape(n=2, c=32, h=17, w=16, f=48, kh=5, kw=5, sh=2, sw=2, ph=2, pw=2), 0.5,
+     wl.COL_CHANNEL, 0.125),
+], ids=lambda c: c[0])
+def test_backward_weight_gradient_on_the_slab(case):
+    """Input-slab plans take the weight gradient on the space-to-depth slab (dZ
+    tiles against shifted slab operands, accumulated per CTA in TMEM, slices
+    summed in order): dW, db and dx against the oracle, the pruned entries of dW
+    exactly zero, and dW bit-identical across calls."""
+    from paper_1807_11091_gb300 import sadmm
+    name, s, ff, ck, cf = case
+    G = s.cg if ck == wl.COL_CHANNEL else s.k
+    kf, kc = wl.retained(ff, s.f), (wl.retained(cf, G) if ck != wl.COL_NONE else 0)
+    t = wl.gen_tensors(s, seed=17)
+    (dW, db, dx), (rdW, rdb, rdx), rows, cols = _backward(s, t, kf, ck, kc)
+    assert_close(dW, rdW, what=f"{name} dW")
+    assert_close(db, rdb, what=f"{name} db")
+    assert_close(dx, rdx, what=f"{name} dx")
+    assert np.all(dW[rdW == 0.0] == 0.0)
+    (dW2, _, _), _, _, _ = _backward(s, t, kf, ck, kc)
+    assert np.array_equal(dW, dW2)
