@@ -36,7 +36,6 @@ namespace {
 
 constexpr int kWgWarps = 10;
 constexpr int kWgThreads = kWgWarps * 32;
-constexpr int kWgEpiWarps = 8;
 constexpr int kWgMaxStages = 4;
 constexpr int kWgDzBox = 128 * 128;      // one 64-pixel box of 128 dZ rows (bf16)
 constexpr int kWgSmemLimit = 232448;
