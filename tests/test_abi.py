@@ -174,3 +174,24 @@ def test_slab_plan_rule_host():
     for s, ck, kc in declined:
         st, p = sadmm.sadmm_plan_init(sadmm.make_desc(s.desc16()), s.f, ck, s.k if ck == wl.COL_NONE else kc)
         assert st == 0 and p.xs_mode == 0, s
+
+
+def test_conv_fwd_phase_argument_checks_host():
+    """sadmm_conv_fwd_phase rejects on the host, before any device call: an
+    unknown phase, the rest of a gathered plan without x (it reads x itself),
+    and the input phase without x.  (The plan's buffer pointer is set to a
+    dummy: nothing is enqueued.)"""
+    import ctypes
+    from workloads import ConvShape
+    s = ConvShape(n=1, c=8, h=9, w=9, f=16, kh=3, kw=3, ph=1, pw=1)
+    st, p = sadmm.sadmm_plan_init(sadmm.make_desc(s.desc16()), s.f, wl.COL_SHAPE, 36)
+    assert st == 0 and p.xs_mode == 0
+    p.dev = ctypes.c_void_p(1 << 20)
+    y = 1 << 21
+    assert sadmm.sadmm_conv_fwd_phase(p, 1 << 22, None, 1, y, sadmm.SADMM_FP32, 7, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_conv_fwd_phase(p, None, None, 1, y, sadmm.SADMM_FP32, sadmm.SADMM_FWD_REST,
+                                      None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_conv_fwd_phase(p, None, None, 1, None, sadmm.SADMM_FP32, sadmm.SADMM_FWD_INPUT,
+                                      None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_conv_fwd_phase(p, 1 << 22, None, 1, None, sadmm.SADMM_FP32, sadmm.SADMM_FWD_ALL,
+                                      None) == sadmm.SADMM_EINVAL
