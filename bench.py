@@ -711,8 +711,9 @@ def run_gpu(args):
     if st != 0:
         raise RuntimeError(f"device status {st} after warm-up")
 
-    os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
-    clocks = ClockSampler(local, os.path.join(ROOT, "gpurun_out", f"bench_clocks_rank{rank}.csv"))
+    log_dir = args.log_dir if os.path.isabs(args.log_dir) else os.path.join(ROOT, args.log_dir)
+    os.makedirs(log_dir, exist_ok=True)
+    clocks = ClockSampler(local, os.path.join(log_dir, f"bench_clocks_rank{rank}.csv"))
     clocks.start()
     # clock soak: the same steps, untimed, so the sampler sees the load before the window
     t_end = time.time() + 1.0
@@ -843,6 +844,8 @@ def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--log-dir", default="bench_logs",
+                    help="directory (relative to the repo root unless absolute) for the raw clock samples")
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="alexnet", choices=sorted(wl.WORKLOADS))
