@@ -383,7 +383,14 @@ class ClockSampler:
                     reasons.add(nm)
         if not sm:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
-        loaded = [c for c, p in zip(sm, power)] if power else sm
+        # under load: samples drawing at least half the peak power seen (all of them when
+        # the power column was unreadable); the sampler also runs a little before and after
+        # the timed steps, where the GPU idles
+        if len(power) == len(sm):
+            top = max(power)
+            loaded = [c for c, p in zip(sm, power) if p >= 0.5 * top]
+        else:
+            loaded = sm
         return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": mx, "reasons": sorted(reasons),
                 "samples": len(sm), "power_w_max": max(power) if power else None}
 

@@ -1,0 +1,59 @@
+"""Host-side checks of bench.py's arithmetic (no GPU): the retained-MAC count
+that the TFLOP/s metric divides, and the parsing of the nvidia-smi clock
+samples that decide whether a timed run is kept."""
+import types
+
+import numpy as np
+import pytest
+
+import oracle
+import workloads as wl
+
+
+def _layers():
+    for name in sorted(wl.WORKLOADS):
+        for L in wl.get(name):
+            yield f"{name}/{L.name}", L
+
+
+@pytest.mark.parametrize("L", [L for _, L in _layers()], ids=[n for n, _ in _layers()])
+def test_flop_count_is_twice_the_kept_weights_times_output_pixels(L):
+    """The metric's numerator, 2 * M * F' * K', equals 2 * (output pixels per
+    filter) * (weights the projection keeps), counted from the oracle's mask;
+    the dense count is the same with nothing pruned."""
+    import bench
+    L = wl.subset_layer(L, 1)
+    s = L.shape
+    t = wl.gen_tensors(s, seed=L.seed)
+    rows, cols, _, _ = oracle.project(t["W"], s.taps, L.k_filters, L.colkind, L.k_cols)
+    kept = int(np.count_nonzero(oracle.masked_weights(np.ones(tuple(t["W"].shape)), rows, L.colkind, cols, s.taps)))
+    ref = 2.0 * s.m * kept  # s.m: output pixels of one filter over the batch
+    assert L.retained_flops() == ref
+    G = s.cg if L.colkind == wl.COL_CHANNEL else s.k
+    run = types.SimpleNamespace(s=s, k_filters=L.k_filters, colkind=L.colkind,
+                                k_cols=L.k_cols if L.colkind != wl.COL_NONE else 0)
+    assert bench.LayerRun.flops(run) == ref
+    dense = types.SimpleNamespace(s=s, k_filters=s.f, colkind=L.colkind, k_cols=G if L.colkind != wl.COL_NONE else 0)
+    assert bench.LayerRun.flops(dense) == 2.0 * s.m * int(np.prod(t["W"].shape)) == L.dense_flops()
+
+
+def _line(clk, mx=2070, power=900.0, reasons=("Not Active",) * 4):
+    return ", ".join(["2026/01/01 00:00:00.000", "0", str(clk), str(mx), str(power), "0x0"] + list(reasons))
+
+
+def test_clock_summary_reasons_and_loaded_median():
+    import bench
+    cs = bench.ClockSampler(0)
+    idle = [_line(345, power=120.0)] * 6
+    load = [_line(2070, power=1100.0)] * 5 + [_line(1995, power=1250.0)] * 2
+    cs.lines = idle + load + ["garbage", _line("[N/A]")]
+    s = cs.summary()
+    assert s["sm_mhz"] == 2070 and s["sm_max_mhz"] == 2070 and s["reasons"] == [] and s["samples"] == 13
+    assert s["power_w_max"] == 1250.0
+    cs.lines = load + [_line(1800, power=1300.0, reasons=("Not Active", "Active", "Not Active", "Active"))]
+    s = cs.summary()
+    assert s["reasons"] == ["hw_thermal_slowdown", "sw_power_cap"]
+    cs.lines = [_line(c, power="[N/A]") for c in (1000, 2000, 2070)]
+    assert cs.summary()["sm_mhz"] == 2000
+    cs.lines = []
+    assert cs.summary() == {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
