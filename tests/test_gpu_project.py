@@ -99,3 +99,49 @@ def test_large_group_count():
     t = wl.gen_tensors(s, seed=77)
     _check(s, t["W"], 1499, wl.COL_SHAPE, 2345)
     _check(s, t["W"], 1, wl.COL_SHAPE, s.k - 1)
+
+
+def _scaled(shape, seed, dtype):
+    """Random weights whose rows and columns span fp32's magnitudes: a per-row
+    power of two from 2^-70 to 2^70 times a per-column one from 2^-8 to 2^8,
+    plus 5 % exact zeros."""
+    g = torch.Generator().manual_seed(seed)
+    F = shape.f
+    W = torch.randn(shape.w_shape(), generator=g, dtype=torch.float64).reshape(F, -1)
+    K = W.shape[1]
+    er = torch.randint(-70, 71, (F, 1), generator=g).double()
+    ec = torch.randint(-8, 9, (1, K), generator=g).double()
+    W = W * torch.pow(2.0, er + ec)
+    W[torch.rand(W.shape, generator=g) < 0.05] = 0.0
+    return W.reshape(shape.w_shape()).to(dtype)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16], ids=["fp32", "bf16"])
+def test_keys_across_the_fp32_range(dtype):
+    """Groups whose elements span fp32's range, about 2^-85 to 2^79 (squares far
+    outside fp32's): keys within 1e-12 of the oracle's fp64 keys and index lists
+    exact, with and without U (U cancelling W exactly in some entries, tiny next
+    to W in others)."""
+    s = ConvShape(n=1, c=48, h=5, w=5, f=96, kh=3, kw=3, ph=1, pw=1)
+    W = _scaled(s, 11, dtype)
+    for kf, kc in ((48, 200), (95, 7), (3, 431)):
+        _check(s, W, kf, wl.COL_SHAPE, kc)
+        _check(s, W, kf, wl.COL_CHANNEL, min(kc, s.cg - 1))
+    g = torch.Generator().manual_seed(12)
+    U = (W.double() * torch.randn(W.shape, generator=g, dtype=torch.float64) * 2.0 ** -30).to(dtype)
+    flat = U.reshape(-1)
+    idx = torch.randperm(flat.numel(), generator=g)[: flat.numel() // 10]
+    flat[idx] = -W.reshape(-1)[idx]
+    _check(s, W, 40, wl.COL_SHAPE, 150, U=U)
+    _check(s, W, 70, wl.COL_CHANNEL, 20, U=U)
+
+
+def test_keys_of_long_rows_fp32_with_dual():
+    """36864 columns (144 elements per thread in the filter-key pass): the
+    partial sums keep the keys within 1e-12 of the oracle's sequential sums."""
+    s = ConvShape(n=1, c=4096, h=3, w=3, f=24, kh=3, kw=3, ph=1, pw=1)
+    t = wl.gen_tensors(s, seed=13)
+    W = t["W"].float() * 0.731
+    U = wl.gen_dual(s, seed=13, scale=0.3).float()
+    _check(s, W, 12, wl.COL_SHAPE, 9000, U=U)
+    _check(s, W, 23, wl.COL_CHANNEL, 1000, U=U)
