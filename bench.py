@@ -68,6 +68,14 @@ def workload_name(name, layers, out_dtype):
     return f"{desc} ({out_dtype} output)"
 
 
+def workload_config(args, layers):
+    """The config keys that name the workload, the same in both arms."""
+    return {"workload": workload_name(args.workload, layers, args.out_dtype),
+            "layers": [L.name for L in layers],
+            "out_dtype": args.out_dtype,
+            "parallelism": "one replica per GPU, batch per GPU fixed, no collective"}
+
+
 # --------------------------------------------------------------------------
 # Reference arm: the CPU oracle as it stands
 # --------------------------------------------------------------------------
@@ -142,10 +150,10 @@ def run_reference(args):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": tot / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": workload_name(args.workload, layers, "fp64"),
-                   "sample": "image 0 of every layer per step"},
+        "config": workload_config(args, layers),
         "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": oracle_threads(), "kind": "oracle",
-                         "sample": "image 0 of every layer per step"},
+                         "sample": "image 0 of every layer per step, through oracle.project + "
+                                   "oracle.pruned_conv (fp64 direct convolution over the full masked weights)"},
         "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
         "gpu_launches": 0,
     }
@@ -806,15 +814,12 @@ def run_gpu(args):
         "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": workload_name(args.workload, layers, args.out_dtype),
-                   "layers": [L.name for L in layers],
-                   "out_dtype": args.out_dtype,
+        "config": {**workload_config(args, layers),
                    "l2": "flushed before every timed step (256 MiB write, outside the timed window)",
                    "schedule": f"projection+pack of each layer on its own stream; convs back to back on the "
                                f"main stream; first conv on {first_ctas or n_sm} of {n_sm} SMs, its input-slab "
                                f"space-to-depth pass issued at the step's start beside the projections and packs",
-                   "breakdown": "per-conv times from separate steps with CUDA events around each whole forward call",
-                   "parallelism": "one replica per GPU, batch per GPU fixed, no collective"},
+                   "breakdown": "per-conv times from separate steps with CUDA events around each whole forward call"},
         "pct_bf16_peak": value / peaks["bf16_tflops"],
         "speedup_vs_dense": dense_step / pruned_step_med,
         "conv_speedup_vs_dense": sum(dense_conv_avg) / sum(conv_avg),

@@ -57,3 +57,31 @@ def test_clock_summary_reasons_and_loaded_median():
     assert cs.summary()["sm_mhz"] == 2000
     cs.lines = []
     assert cs.summary() == {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+
+
+def test_reference_arm_line_on_rank0(monkeypatch):
+    """`bench.py --impl reference` on one process: one JSON line with the GPU
+    arm's metric, unit, direction and workload config, the oracle described in
+    cpu_baseline, and an e2e entry with no host-device bytes."""
+    import contextlib
+    import io
+    import json
+
+    import bench
+    monkeypatch.setenv("RANK", "0")
+    monkeypatch.setenv("WORLD_SIZE", "1")
+    monkeypatch.setenv("LOCAL_RANK", "0")
+    args = types.SimpleNamespace(workload="single2d", steps=2, warmup=3, gpus=1, out_dtype="fp32")
+    buf = io.StringIO()
+    with contextlib.redirect_stdout(buf):
+        assert bench.run_reference(args) == 0
+    lines = [ln for ln in buf.getvalue().splitlines() if ln.strip()]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["unit"] == "TFLOP/s"
+    assert d["higher_is_better"] is True and d["n_gpus"] == 1 and d["steps"] == 2 and d["warmup"] == 3
+    assert d["value"] > 0 and d["ms_per_step"] > 0
+    assert d["config"] == bench.workload_config(args, wl.get("single2d"))
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
+    assert d["e2e"] == {"value": d["value"], "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
