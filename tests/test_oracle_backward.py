@@ -71,3 +71,33 @@ def test_zero_upstream_gradient():
     dy = np.zeros((s.n, s.f, s.oh, s.ow))
     dx, dW, db = oracle.pruned_conv_backward(t["x"], t["W"], t["bias"], s.desc16(), s.taps, rows, ck, cols, dy)
     assert not dx.any() and not dW.any() and not db.any()
+
+
+@pytest.mark.parametrize("stride", [1, 2])
+def test_pointwise_layer_reduces_to_matrix_products(stride):
+    """A 1x1 conv without ReLU is y[:, p] = Wm x[:, q(p)] + bm at every output
+    pixel p (input pixel q(p) = stride * p), so its gradients are matrix
+    products: dW = (dY X^T) on the kept entries, dX[:, q(p)] = Wm^T dY[:, p]
+    (zero at the input pixels the stride skips), db = the sum of dY over the
+    pixels and the batch for kept filters.  Checked to 1e-12 relative."""
+    s = ConvShape(n=3, c=7, h=6, w=8, f=9, kh=1, kw=1, sh=stride, sw=stride)
+    t = wl.gen_tensors(s, seed=31)
+    x, W, bias = t["x"].double(), t["W"].double(), t["bias"].double()
+    rows, cols, _, _ = oracle.project(t["W"], s.taps, 6, wl.COL_CHANNEL, 4)
+    rng = np.random.default_rng(8)
+    dy = rng.standard_normal((s.n, s.f, s.oh, s.ow))
+    dx, dW, db = oracle.pruned_conv_backward(x, W, bias, s.desc16(), s.taps, rows, wl.COL_CHANNEL, cols, dy,
+                                             relu=False)
+    Wm = oracle.masked_weights(W, rows, wl.COL_CHANNEL, cols, s.taps).reshape(s.f, s.c)
+    keep = oracle.masked_weights(np.ones(W.shape), rows, wl.COL_CHANNEL, cols, s.taps).reshape(s.f, s.c) != 0
+    xs = x.numpy()[:, :, ::stride, ::stride][:, :, :s.oh, :s.ow]      # [n][c][oh][ow]
+    X = xs.transpose(1, 0, 2, 3).reshape(s.c, -1)                      # [c][n*oh*ow]
+    D = dy.transpose(1, 0, 2, 3).reshape(s.f, -1)                      # [f][n*oh*ow]
+    dW_ref = (D @ X.T) * keep
+    assert np.allclose(dW.reshape(s.f, s.c), dW_ref, rtol=1e-12, atol=1e-12 * np.abs(dW_ref).max())
+    dx_ref = np.zeros(x.shape)
+    dx_ref[:, :, ::stride, ::stride][:, :, :s.oh, :s.ow] = (Wm.T @ D).reshape(s.c, s.n, s.oh, s.ow).transpose(1, 0, 2, 3)
+    assert np.allclose(dx, dx_ref, rtol=1e-12, atol=1e-12 * np.abs(dx_ref).max())
+    bkeep = np.isin(np.arange(s.f), rows)
+    assert np.allclose(db, D.sum(axis=1) * bkeep, rtol=1e-12, atol=1e-12)
+    assert np.all(db[~bkeep] == 0.0) and np.all(dW.reshape(s.f, s.c)[~keep] == 0.0)
