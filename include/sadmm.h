@@ -417,7 +417,9 @@ size_t sadmm_conv_bwd_workspace_size_chunk(const sadmm_plan* plan, long long chu
  *   y      device forward output of dtype ydt (bf16/fp32), read when relu != 0.
  *   dW     device fp32 [F][K] (OIDHW) or NULL; db fp32 [F] or NULL;
  *          dx fp32 [N][C][T][H][W] or NULL.  Every element of each is written.
- *   workspace  sadmm_conv_bwd_workspace_size(plan) bytes, 1024-byte aligned.
+ *   workspace  ws_bytes of device scratch, 1024-byte aligned: at least
+ *          sadmm_conv_bwd_workspace_size_chunk(plan, 256) (else SADMM_EINVAL);
+ *          sadmm_conv_bwd_workspace_size(plan) gives the largest chunks.
  */
 sadmm_status sadmm_conv_bwd(const sadmm_plan* plan, const void* x, const void* dy, const void* y, int ydt,
                             int relu, float* dW, float* db, float* dx, void* workspace, size_t ws_bytes,
