@@ -85,3 +85,21 @@ def test_reference_arm_line_on_rank0(monkeypatch):
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
     assert d["e2e"] == {"value": d["value"], "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+
+
+def test_traffic_reported_only_for_the_profiled_kernel_sources(monkeypatch, tmp_path):
+    """The roofline's `traffic` comes from the committed ncu summary only while
+    the forward kernels' sources hash to the sha1 recorded in it, and only for
+    the workload it was captured on; otherwise it is null."""
+    import bench
+    assert bench.conv_traffic("alexnet", "bf16") is None and bench.conv_traffic("resnet50", "fp32") is None
+    good = tmp_path / "good.txt"
+    good.write_text(f"# comment: 1\nkernel_source_sha1: {bench.conv_source_sha1()}\ndram_bytes_per_call_avg: 123\n")
+    monkeypatch.setattr(bench, "TRAFFIC_FILE", str(good))
+    assert bench.conv_traffic("alexnet", "fp32") == 123.0
+    stale = tmp_path / "stale.txt"
+    stale.write_text("kernel_source_sha1: " + "0" * 40 + "\ndram_bytes_per_call_avg: 123\n")
+    monkeypatch.setattr(bench, "TRAFFIC_FILE", str(stale))
+    assert bench.conv_traffic("alexnet", "fp32") is None
+    monkeypatch.setattr(bench, "TRAFFIC_FILE", str(tmp_path / "missing.txt"))
+    assert bench.conv_traffic("alexnet", "fp32") is None
