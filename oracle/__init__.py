@@ -197,11 +197,11 @@ def project(W, taps: int, k_filters: int, colkind: int, k_cols: int, U=None):
 
 def expand_columns(colkind: int, cols, taps: int, K: int) -> np.ndarray:
     """GEMM column indices kept: channel b keeps columns b*taps .. b*taps+taps-1."""
+    if colkind == COL_NONE:
+        return np.arange(K, dtype=np.int64)
     cols = np.asarray(cols, dtype=np.int64)
     if colkind == COL_CHANNEL:
         return (cols[:, None] * taps + np.arange(taps)[None, :]).reshape(-1)
-    if colkind == COL_NONE:
-        return np.arange(K, dtype=np.int64)
     return cols
 
 
