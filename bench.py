@@ -57,6 +57,15 @@ def dist_env():
     return ranks.dist_env()
 
 
+def check_gpus(gpus, world_size):
+    """None when --gpus matches the launch, else the error to print: one process
+    per GPU, so N > 1 GPUs need N ranks (torchrun sets WORLD_SIZE)."""
+    if gpus == world_size:
+        return None
+    return (f"bench.py: --gpus {gpus} but {world_size} rank(s) running; launch N > 1 GPUs as "
+            f"python -m torch.distributed.run --nproc-per-node N bench.py --gpus N")
+
+
 def workload_name(name, layers, out_dtype):
     desc = {
         "alexnet": "AlexNet CONV1-5, batch 128, filter-wise + shape-wise pruning, retained 1.0/0.5/0.25/0.2/0.2",
@@ -872,6 +881,10 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
+    err = check_gpus(args.gpus, dist_env()[0])
+    if err:
+        print(err, file=sys.stderr, flush=True)
+        return 2
     if args.impl == "reference":
         return run_reference(args)
     return run_gpu(args)

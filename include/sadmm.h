@@ -304,7 +304,10 @@ sadmm_status sadmm_plan_init_ctas(sadmm_plan* plan, const sadmm_conv_desc* d,
  * Writes the TMA descriptor of Wp into plan->tmap.  For a slab plan it also
  * packs the weights in slab column order (plan->off_wps, plan->tmap_ws) and
  * writes the TMA map of the space-to-depth input (plan->tmap_xs).  Index lists
- * that are not ascending or out of range give undefined (but in-bounds) plans.
+ * are checked on the device: a list that is not strictly ascending or holds an
+ * index out of range gives a plan with every filter pruned and every column
+ * dropped (its forward writes an all-zero output) and raises the device status
+ * word, which the next sadmm_last_device_status returns as SADMM_EINVAL.
  */
 sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt,
                         const int* filt_idx, const int* col_idx,
@@ -367,12 +370,16 @@ sadmm_status sadmm_conv_fwd_phase(const sadmm_plan* plan, const void* x, const f
  * compiled into the library, SADMM_NOALLOC_SCRATCH_BYTES (256 KiB) on every
  * GPU that loads the library, held until the process exits.  A layer
  * whose keys need more (sadmm_workspace_size() above that) is rejected with
- * SADMM_EUNSUPPORTED before anything is enqueued; F + K up to about 16000
- * groups fit.  The call allocates nothing: no cudaMalloc, no cudaFree.
+ * SADMM_EUNSUPPORTED before anything is enqueued.  Exactly: a layer fits when
+ * round_up(F, 32) + round_up(K, 32) <= 16352, K = Cg*KT*KH*KW, whatever the
+ * column kind (e.g. F = 192 filters with K = 16160 columns, or F = 16320 with
+ * K = 32).  The call allocates nothing: no cudaMalloc, no cudaFree.
  *
  * The first call on a device looks up the array's device address (a host-side
  * CUDA runtime query, once per device, with that device current); make that
- * first call before any stream capture.  Every call shares the array.  Nothing
+ * first call before any stream capture.  The address is kept for the life of
+ * the process: after cudaDeviceReset the array is gone and the kept address is
+ * stale, so do not call this entry point on a device that has been reset.  Every call shares the array.  Nothing
  * in it needs to start at zero (each key is written before it is read), but
  * calls that overlap on the GPU -- on different streams with no ordering
  * between them -- race on it and can return wrong index lists.

@@ -2,6 +2,7 @@
 // plan sizing and the device status word.  Every entry point checks its
 // arguments before enqueuing anything and never synchronises, except
 // sadmm_last_device_status.
+#include <nvtx3/nvToolsExt.h>
 #include <string.h>
 
 #include "common.cuh"
@@ -91,6 +92,25 @@ sadmm_status check_desc(const sadmm_conv_desc* d, Geometry* g)
     return SADMM_OK;
 }
 
+sadmm_status check_project_args(const Geometry& g, const void* W, int wdt, int k_filters, int colkind, int k_cols,
+                                const int* filt_idx, const int* col_idx, const double* keys_out)
+{
+    if (!W || !filt_idx) return SADMM_EINVAL;
+    if (wdt != SADMM_BF16 && wdt != SADMM_FP32) return SADMM_EINVAL;
+    if (colkind != SADMM_COL_NONE && colkind != SADMM_COL_SHAPE && colkind != SADMM_COL_CHANNEL)
+        return SADMM_EINVAL;
+    if (k_filters < 0 || k_filters > g.f) return SADMM_EINVAL;
+    if (colkind != SADMM_COL_NONE) {
+        const long long G = (colkind == SADMM_COL_SHAPE) ? g.k : g.cg;
+        if (k_cols < 0 || k_cols > G || !col_idx) return SADMM_EINVAL;
+    }
+    if (keys_out && (reinterpret_cast<uintptr_t>(keys_out) & 7) != 0) return SADMM_EINVAL;
+    return SADMM_OK;
+}
+
+NvtxRange::NvtxRange(const char* name) { nvtxRangePushA(name); }
+NvtxRange::~NvtxRange() { nvtxRangePop(); }
+
 }  // namespace sadmm
 
 using namespace sadmm;
@@ -124,21 +144,15 @@ sadmm_status sadmm_project_groups(const sadmm_conv_desc* d, const void* W, const
                                   int k_filters, int colkind, int k_cols, int* filt_idx, int* col_idx,
                                   double* keys_out, void* workspace, size_t ws_bytes, void* stream)
 {
+    NvtxRange range("sadmm_project_groups");
     Geometry g;
     sadmm_status st = check_desc(d, &g);
     if (st != SADMM_OK) return st;
-    if (!W || !filt_idx || !workspace) return SADMM_EINVAL;
-    if (wdt != SADMM_BF16 && wdt != SADMM_FP32) return SADMM_EINVAL;
-    if (colkind != SADMM_COL_NONE && colkind != SADMM_COL_SHAPE && colkind != SADMM_COL_CHANNEL)
-        return SADMM_EINVAL;
-    if (k_filters < 0 || k_filters > g.f) return SADMM_EINVAL;
-    if (colkind != SADMM_COL_NONE) {
-        const long long G = (colkind == SADMM_COL_SHAPE) ? g.k : g.cg;
-        if (k_cols < 0 || k_cols > G || !col_idx) return SADMM_EINVAL;
-    }
+    st = check_project_args(g, W, wdt, k_filters, colkind, k_cols, filt_idx, col_idx, keys_out);
+    if (st != SADMM_OK) return st;
+    if (!workspace) return SADMM_EINVAL;
     if (ws_bytes < project_workspace_bytes(g, colkind)) return SADMM_EINVAL;
     if ((reinterpret_cast<uintptr_t>(workspace) & 7) != 0) return SADMM_EINVAL;
-    if (keys_out && (reinterpret_cast<uintptr_t>(keys_out) & 7) != 0) return SADMM_EINVAL;
     return launch_project(g, W, U, wdt, k_filters, colkind, k_cols, filt_idx, col_idx, keys_out, workspace,
                           static_cast<cudaStream_t>(stream));
 }
@@ -154,21 +168,15 @@ sadmm_status sadmm_admm_update(const sadmm_conv_desc* d, const void* W, void* U,
                                int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out,
                                void* workspace, size_t ws_bytes, void* stream)
 {
+    NvtxRange range("sadmm_admm_update");
     Geometry g;
     sadmm_status st = check_desc(d, &g);
     if (st != SADMM_OK) return st;
-    if (!W || !U || !Z || !filt_idx || !workspace) return SADMM_EINVAL;
-    if (wdt != SADMM_BF16 && wdt != SADMM_FP32) return SADMM_EINVAL;
-    if (colkind != SADMM_COL_NONE && colkind != SADMM_COL_SHAPE && colkind != SADMM_COL_CHANNEL)
-        return SADMM_EINVAL;
-    if (k_filters < 0 || k_filters > g.f) return SADMM_EINVAL;
-    if (colkind != SADMM_COL_NONE) {
-        const long long G = (colkind == SADMM_COL_SHAPE) ? g.k : g.cg;
-        if (k_cols < 0 || k_cols > G || !col_idx) return SADMM_EINVAL;
-    }
+    st = check_project_args(g, W, wdt, k_filters, colkind, k_cols, filt_idx, col_idx, keys_out);
+    if (st != SADMM_OK) return st;
+    if (!U || !Z || !workspace) return SADMM_EINVAL;
     if (ws_bytes < admm_workspace_bytes(g, colkind)) return SADMM_EINVAL;
     if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0) return SADMM_EINVAL;
-    if (keys_out && (reinterpret_cast<uintptr_t>(keys_out) & 7) != 0) return SADMM_EINVAL;
     const size_t esz = (wdt == SADMM_FP32) ? 4 : 2;
     const uintptr_t bytes = (uintptr_t)(g.f * g.k) * esz;
     const uintptr_t w = reinterpret_cast<uintptr_t>(W), u = reinterpret_cast<uintptr_t>(U),
@@ -380,6 +388,7 @@ sadmm_status sadmm_plan_init_ctas(sadmm_plan* plan, const sadmm_conv_desc* d, in
 sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt, const int* filt_idx, const int* col_idx,
                         void* dev, size_t dev_bytes, void* stream)
 {
+    NvtxRange range("sadmm_pack");
     if (!plan || !W || !dev) return SADMM_EINVAL;
     Geometry g;
     sadmm_status st = check_desc(&plan->desc, &g);
@@ -404,6 +413,7 @@ sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt, const int* fil
 sadmm_status sadmm_conv_fwd_phase(const sadmm_plan* plan, const void* x, const float* bias, int relu, void* y,
                                   int ydt, int phase, void* stream)
 {
+    NvtxRange range("sadmm_conv_fwd");
     if (!plan || !plan->dev) return SADMM_EINVAL;
     if (phase != SADMM_FWD_ALL && phase != SADMM_FWD_INPUT && phase != SADMM_FWD_REST) return SADMM_EINVAL;
     const bool needs_x = phase != SADMM_FWD_REST || !plan->xs_mode;  // the rest of a slab plan reads its copy

@@ -19,6 +19,23 @@ struct Geometry {
 // Checks a descriptor; fills `g` on success.
 sadmm_status check_desc(const sadmm_conv_desc* d, Geometry* g);
 
+// The argument checks every projection entry point shares (sadmm_project_groups,
+// its no-workspace variant, sadmm_admm_update): W and filt_idx present, a known
+// dtype and column kind, k_filters in [0, F], k_cols in [0, G] with col_idx
+// present when columns are pruned, keys_out 8-byte aligned.  Each entry point
+// then checks its own workspace.
+sadmm_status check_project_args(const Geometry& g, const void* W, int wdt, int k_filters, int colkind, int k_cols,
+                                const int* filt_idx, const int* col_idx, const double* keys_out);
+
+// A named NVTX range around one entry point (seen by nsys / ncu range filters;
+// costs one branch when no tool is attached).
+struct NvtxRange {
+    explicit NvtxRange(const char* name);
+    ~NvtxRange();
+    NvtxRange(const NvtxRange&) = delete;
+    NvtxRange& operator=(const NvtxRange&) = delete;
+};
+
 // Address of the device status word on the current device (cached per device).
 int* device_status_ptr();
 

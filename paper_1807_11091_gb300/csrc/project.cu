@@ -16,6 +16,7 @@
 // Keys are non-negative fp64 values, so their IEEE bit patterns order like the
 // values; selection compares bit patterns (a NaN key would rank above +Inf).
 #include <algorithm>
+#include <atomic>
 
 #include "common.cuh"
 #include "internal.h"
@@ -370,7 +371,10 @@ constexpr size_t kNoAllocScratchBytes = SADMM_NOALLOC_SCRATCH_BYTES;
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 constexpr int kNoAllocMaxDevices = 64;
-void* g_noalloc_ptr[kNoAllocMaxDevices];
+// Per device, the array's address once looked up.  Atomic: host threads that
+// make their first call on one device at the same time may both look it up
+// (they find the same address); neither reads a half-written pointer.
+std::atomic<void*> g_noalloc_ptr[kNoAllocMaxDevices];
 
 // Device address of the array on the current device; looked up once per device
 // (host code only sees a stand-in for the array, never its device address).
@@ -380,13 +384,13 @@ cudaError_t noalloc_scratch(void** out)
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= kNoAllocMaxDevices) return cudaErrorInvalidDevice;
-    if (!g_noalloc_ptr[dev]) {
-        void* p = nullptr;
+    void* p = g_noalloc_ptr[dev].load(std::memory_order_acquire);
+    if (!p) {
         e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
         if (e != cudaSuccess) return e;
-        g_noalloc_ptr[dev] = p;
+        g_noalloc_ptr[dev].store(p, std::memory_order_release);
     }
-    *out = g_noalloc_ptr[dev];
+    *out = p;
     return cudaSuccess;
 }
 
@@ -399,19 +403,12 @@ extern "C" sadmm_status sadmm_project_groups_noalloc(const sadmm_conv_desc* d, c
                                                      void* stream)
 {
     using namespace sadmm;
+    NvtxRange range("sadmm_project_groups_noalloc");
     Geometry g;
     sadmm_status st = check_desc(d, &g);
     if (st != SADMM_OK) return st;
-    if (!W || !filt_idx) return SADMM_EINVAL;
-    if (wdt != SADMM_BF16 && wdt != SADMM_FP32) return SADMM_EINVAL;
-    if (colkind != SADMM_COL_NONE && colkind != SADMM_COL_SHAPE && colkind != SADMM_COL_CHANNEL)
-        return SADMM_EINVAL;
-    if (k_filters < 0 || k_filters > g.f) return SADMM_EINVAL;
-    if (colkind != SADMM_COL_NONE) {
-        const long long G = (colkind == SADMM_COL_SHAPE) ? g.k : g.cg;
-        if (k_cols < 0 || k_cols > G || !col_idx) return SADMM_EINVAL;
-    }
-    if (keys_out && (reinterpret_cast<uintptr_t>(keys_out) & 7) != 0) return SADMM_EINVAL;
+    st = check_project_args(g, W, wdt, k_filters, colkind, k_cols, filt_idx, col_idx, keys_out);
+    if (st != SADMM_OK) return st;
     // the layer's keys must fit the fixed array
     if (project_workspace_bytes(g, colkind) > kNoAllocScratchBytes) return SADMM_EUNSUPPORTED;
     void* ws = nullptr;

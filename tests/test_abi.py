@@ -195,3 +195,24 @@ def test_conv_fwd_phase_argument_checks_host():
                                       None) == sadmm.SADMM_EINVAL
     assert sadmm.sadmm_conv_fwd_phase(p, 1 << 22, None, 1, None, sadmm.SADMM_FP32, sadmm.SADMM_FWD_ALL,
                                       None) == sadmm.SADMM_EINVAL
+
+
+def test_noalloc_array_size_matches_header():
+    """The binding's copy of SADMM_NOALLOC_SCRATCH_BYTES equals the header's #define."""
+    import re
+    with open(os.path.join(ROOT, "include", "sadmm.h")) as fh:
+        m = re.search(r"#define\s+SADMM_NOALLOC_SCRATCH_BYTES\s+\(([^)]*)\)", fh.read())
+    assert m, "define not found"
+    assert eval(m.group(1), {"__builtins__": {}}) == sadmm.SADMM_NOALLOC_SCRATCH_BYTES
+
+
+def test_noalloc_size_rule_host():
+    """The fit rule the header states (round_up(F, 32) + round_up(K, 32) <= 16352)
+    is exactly where the projection's workspace reaches the fixed array."""
+    limit = sadmm.SADMM_NOALLOC_SCRATCH_BYTES
+    r32 = lambda v: (v + 31) // 32 * 32
+    for f, c in ((192, 16160), (193, 16160), (16320, 32), (16321, 32), (16384, 1), (1, 16352), (64, 16288)):
+        desc = sadmm.make_desc([1, c, 1, 1, 1, f, 1, 1, 1, 1, 1, 1, 1, 0, 0, 0])
+        for ck in (0, 1, 2):
+            fits = sadmm.sadmm_workspace_size(desc, ck) <= limit
+            assert fits == (r32(f) + r32(c) <= 16352), (f, c, ck)

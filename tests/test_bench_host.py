@@ -103,3 +103,10 @@ def test_traffic_reported_only_for_the_profiled_kernel_sources(monkeypatch, tmp_
     assert bench.conv_traffic("alexnet", "fp32") is None
     monkeypatch.setattr(bench, "TRAFFIC_FILE", str(tmp_path / "missing.txt"))
     assert bench.conv_traffic("alexnet", "fp32") is None
+
+
+def test_gpus_flag_must_match_the_ranks():
+    import bench
+    assert bench.check_gpus(1, 1) is None and bench.check_gpus(4, 4) is None
+    assert "torch.distributed.run" in bench.check_gpus(8, 1)
+    assert bench.check_gpus(1, 2) is not None

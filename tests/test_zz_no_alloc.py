@@ -62,3 +62,32 @@ def test_noalloc_rejects_layers_beyond_the_fixed_array():
     st = sadmm.sadmm_project_groups_noalloc(desc, fake, None, sadmm.SADMM_BF16, 4, wl.COL_SHAPE, 4, fake, fake,
                                             None, None)
     assert st == sadmm.SADMM_EUNSUPPORTED
+
+
+def test_noalloc_rejects_many_filters_without_column_pruning():
+    """The filter keys alone can overflow the array: F = 16384 with no column pruning."""
+    from paper_1807_11091_gb300 import sadmm
+    s = ConvShape(n=1, c=1, h=3, w=3, f=16384, kh=3, kw=3, ph=1, pw=1)
+    desc = sadmm.make_desc(s.desc16())
+    assert sadmm.sadmm_workspace_size(desc, wl.COL_NONE) > sadmm.SADMM_NOALLOC_SCRATCH_BYTES
+    fake = 1 << 20  # never dereferenced: rejected on the host
+    st = sadmm.sadmm_project_groups_noalloc(desc, fake, None, sadmm.SADMM_BF16, 100, wl.COL_NONE, 0, fake, None,
+                                            None, None)
+    assert st == sadmm.SADMM_EUNSUPPORTED
+
+
+@pytest.mark.parametrize("f,c,kf,ck,kc", [(192, 16160, 96, wl.COL_SHAPE, 4000),   # exactly at the limit
+                                          (192, 16160, 192, wl.COL_CHANNEL, 5000),
+                                          (16320, 32, 4000, wl.COL_NONE, 0)])
+def test_noalloc_layers_at_the_limit_match_workspace_path(f, c, kf, ck, kc):
+    """Layers whose keys fill the array exactly run and equal the workspace path."""
+    from paper_1807_11091_gb300 import sadmm
+    s = ConvShape(n=1, c=c, h=1, w=1, f=f, kh=1, kw=1)
+    desc = sadmm.make_desc(s.desc16())
+    assert sadmm.sadmm_workspace_size(desc, ck) == sadmm.SADMM_NOALLOC_SCRATCH_BYTES
+    W = wl.gen_tensors(s, seed=77)["W"].cuda()
+    ref = _run("workspace", s, W, kf, ck, kc)
+    for _ in range(2):
+        got = _run("noalloc", s, W, kf, ck, kc)
+        assert np.array_equal(got[0], ref[0]) and np.array_equal(got[1], ref[1])
+        np.testing.assert_allclose(got[2], ref[2], rtol=1e-12, atol=0)
