@@ -442,6 +442,19 @@ sadmm_status sadmm_gemm_bf16(const void* A, const void* B, float* C, long long M
                              long long ldc, int accumulate, void* stream);
 
 /*
+ * Failure-detection self-test; the paper has no counterpart.  Runs, in one
+ * CTA on `stream`, the bounded mbarrier wait every pipelined kernel here uses,
+ * with a limit of `limit_us` microseconds (1 .. 1000000) instead of the
+ * kernels' 4 s.  With `arrive` = 0 nothing ever arrives on the barrier: the
+ * wait gives up after the limit, raises the device status word (so the next
+ * sadmm_last_device_status returns SADMM_ETIMEOUT) and the kernel returns,
+ * leaving the context usable.  With `arrive` != 0 the barrier completes first
+ * and the wait succeeds.  `result` (device int, optional): 1 when the wait saw
+ * its phase complete, 0 when it gave up.  Nothing here faults or hangs.
+ */
+sadmm_status sadmm_selftest_wait(unsigned int limit_us, int arrive, int* result, void* stream);
+
+/*
  * Synchronises `stream`, then reports and clears the device status word that
  * the kernels set when a bounded wait expires (SADMM_ETIMEOUT) or a
  * device-side check fails (SADMM_EINVAL).  SADMM_OK when clear.

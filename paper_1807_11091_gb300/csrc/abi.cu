@@ -111,6 +111,30 @@ sadmm_status check_project_args(const Geometry& g, const void* W, int wdt, int k
 NvtxRange::NvtxRange(const char* name) { nvtxRangePushA(name); }
 NvtxRange::~NvtxRange() { nvtxRangePop(); }
 
+namespace {
+// One CTA runs the kernels' bounded mbarrier wait (mbar_wait_for) on a barrier
+// of one expected arrival.  With `arrive` set, thread 0 arrives first and the
+// wait must succeed at once; otherwise nothing ever arrives and the wait must
+// give up after limit_ns, raise the status word and return.  The result of the
+// wait (1 completed, 0 gave up) goes to `out` when it is not NULL.
+__global__ void k_selftest_wait(int* status, unsigned long long limit_ns, int arrive, int* out)
+{
+    __shared__ uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        if (arrive) mbar_arrive(&bar);
+        const bool ok = mbar_wait_for(&bar, 0, &abort_flag, status, limit_ns);
+        if (out) *out = ok ? 1 : 0;
+    }
+}
+}  // namespace
+
 }  // namespace sadmm
 
 using namespace sadmm;
@@ -483,6 +507,17 @@ sadmm_status sadmm_gemm_bf16(const void* A, const void* B, float* C, long long M
     if (bn < 16) return SADMM_EINVAL;
     if (device_cc_major() < 10) return SADMM_EUNSUPPORTED;
     return launch_gemm(A, B, C, M, N, K, ldc, bn, accumulate != 0, static_cast<cudaStream_t>(stream));
+}
+
+sadmm_status sadmm_selftest_wait(unsigned int limit_us, int arrive, int* result, void* stream)
+{
+    if (limit_us < 1 || limit_us > 1000000) return SADMM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(result) & 3) != 0) return SADMM_EINVAL;
+    int* status = device_status_ptr();
+    if (!status) return SADMM_ECUDA;
+    k_selftest_wait<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(status, 1000ull * limit_us, arrive ? 1 : 0,
+                                                                     result);
+    return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
 }
 
 sadmm_status sadmm_last_device_status(void* stream)

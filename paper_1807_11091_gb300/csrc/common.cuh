@@ -168,20 +168,27 @@ SADMM_DEV bool mbar_try_wait_suspend(uint64_t* bar, uint32_t parity)
 
 // Waits until the phase with the given parity of `bar` has completed.
 // Returns false (and raises the abort flag and the status word) when the wait
-// runs past kWaitLimitNs, or false at once when another role aborted.
-SADMM_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* status)
+// runs past `limit_ns`, or false at once when another role aborted.
+SADMM_DEV bool mbar_wait_for(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* status,
+                             unsigned long long limit_ns)
 {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = globaltimer();
     for (;;) {
         if (mbar_try_wait_suspend(bar, parity)) return true;
         if (*abort_flag) return false;
-        if (globaltimer() - t0 > kWaitLimitNs) {
+        if (globaltimer() - t0 > limit_ns) {
             *abort_flag = 1;
             raise_status(status, kDevTimeout);
             return false;
         }
     }
+}
+
+// mbar_wait_for with the kernels' limit, kWaitLimitNs.
+SADMM_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* status)
+{
+    return mbar_wait_for(bar, parity, abort_flag, status, kWaitLimitNs);
 }
 
 // --------------------------------------------------------------------- TMA --

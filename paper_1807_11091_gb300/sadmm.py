@@ -137,6 +137,8 @@ def load():
     lib.sadmm_gemm_bf16.argtypes = [vp, vp, vp, ll, ll, ll, ll, ci, vp]
     lib.sadmm_last_device_status.restype = ci
     lib.sadmm_last_device_status.argtypes = [vp]
+    lib.sadmm_selftest_wait.restype = ci
+    lib.sadmm_selftest_wait.argtypes = [ctypes.c_uint, ci, vp, vp]
     lib.sadmm_project_groups_noalloc.restype = ci
     lib.sadmm_project_groups_noalloc.argtypes = [P(ConvDesc), vp, vp, ci, ci, ci, ci, vp, vp, vp, vp]
     if lib.sadmm_plan_struct_size() != ctypes.sizeof(Plan):
@@ -277,6 +279,10 @@ def sadmm_gemm_bf16(A: int, B: int, C: int, M: int, N: int, K: int, ldc: int, ac
 
 def sadmm_last_device_status(stream: Optional[int]) -> int:
     return load().sadmm_last_device_status(stream)
+
+
+def sadmm_selftest_wait(limit_us: int, arrive: int, result: Optional[int], stream: Optional[int]) -> int:
+    return load().sadmm_selftest_wait(int(limit_us), int(arrive), result, stream)
 
 
 # --------------------------------------------------------------------------

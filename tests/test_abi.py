@@ -216,3 +216,9 @@ def test_noalloc_size_rule_host():
         for ck in (0, 1, 2):
             fits = sadmm.sadmm_workspace_size(desc, ck) <= limit
             assert fits == (r32(f) + r32(c) <= 16352), (f, c, ck)
+
+
+def test_selftest_wait_rejects_bad_arguments_on_host():
+    assert sadmm.sadmm_selftest_wait(0, 0, None, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_selftest_wait(1000001, 0, None, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_selftest_wait(1000, 0, (1 << 20) + 2, None) == sadmm.SADMM_EINVAL

@@ -219,3 +219,22 @@ def test_backward_weight_gradient_on_the_slab(case):
     assert np.all(dW[rdW == 0.0] == 0.0)
     (dW2, _, _), _, _, _ = _backward(s, t, kf, ck, kc)
     assert np.array_equal(dW, dW2)
+
+
+@pytest.mark.parametrize("li,batch", [(0, 16), (1, 72)], ids=["conv1_b16_slab_many_runs", "conv2_b72_full_chunks"])
+def test_backward_alexnet_at_benchmarked_paths(li, batch):
+    """The paths the benchmark's batch-128 backward takes, at batches the fp64
+    oracle finishes in seconds: CONV1's weight gradient on the slab over 378
+    output tiles (2.5 runs per CTA, one fp32 slice each, summed in CTA order);
+    CONV2 (two conv groups) in a full 32768-pixel chunk, with the benchmark's
+    weight-gradient split for that chunk, then a ragged second chunk."""
+    L = wl.subset_layer(wl.alexnet()[li], batch)
+    s = L.shape
+    t = wl.gen_tensors(s, seed=L.seed)
+    if li == 1:
+        assert s.n * s.oh * s.ow > 32768
+    (dW, db, dx), (rdW, rdb, rdx), rows, cols = _backward(s, t, L.k_filters, L.colkind, L.k_cols, seed=li)
+    assert_close(dW, rdW, what=f"{L.name} batch {batch} dW")
+    assert_close(db, rdb, what=f"{L.name} batch {batch} db")
+    assert_close(dx, rdx, what=f"{L.name} batch {batch} dx")
+    assert np.all(dW[rdW == 0.0] == 0.0)

@@ -56,3 +56,38 @@ def test_full_size_layer(layer):
         ref = oracle.pruned_conv(t["x"], t["W"], t["bias"], s.desc16(), s.taps, rows, layer.colkind, cols,
                                  relu=True, n0=n, n1=n + 1)
         assert_close(y[n:n + 1].cpu().numpy(), ref, what=f"{layer.name} image {n}")
+
+
+BF16_LAYERS = [wl.alexnet()[0], wl.alexnet()[1], wl.alexnet()[4], wl.c3d()[0],
+               wl.sweep(col_fracs=(0.25,), filt_fracs=(0.5,))[0]]
+
+
+@pytest.mark.parametrize("layer", BF16_LAYERS, ids=lambda l: l.name)
+def test_full_size_layer_bf16_output(layer):
+    """The bf16-output forward at full size: within one bf16 ulp of the oracle
+    rounded to bf16 on the first and last image; every element written; pruned
+    planes exactly zero over the whole tensor."""
+    from paper_1807_11091_gb300 import sadmm
+    s = layer.shape
+    t = wl.gen_tensors(s, seed=layer.seed)
+    dev = torch.device("cuda", 0)
+    W, x, bias = t["W"].to(dev), t["x"].to(dev), t["bias"].to(dev)
+    fi, ci, _ = sadmm.project_groups(s.desc16(), W, layer.k_filters, layer.colkind, layer.k_cols)
+    pc = sadmm.PrunedConv(s.desc16(), W, fi if layer.k_filters < s.f else None, layer.colkind, ci,
+                          layer.k_filters, layer.k_cols if layer.colkind != wl.COL_NONE else s.k)
+    y = torch.full(pc.out_shape(), float("nan"), dtype=torch.bfloat16, device=dev)
+    pc.forward(x, bias, relu=True, out=y)
+    assert sadmm.device_status() == 0
+    rows = fi.cpu().numpy().astype(np.int64)
+    cols = ci.cpu().numpy().astype(np.int64)
+    assert bool(torch.isfinite(y).all()), "unwritten or non-finite outputs"
+    pr = torch.as_tensor(pruned_filters(s.f, rows), device=dev)
+    if pr.numel():
+        assert bool((y.index_select(1, pr) == 0).all()), "pruned planes not zero"
+    for n in sorted({0, s.n - 1}):
+        ref = oracle.pruned_conv(t["x"], t["W"], t["bias"], s.desc16(), s.taps, rows, layer.colkind, cols,
+                                 relu=True, n0=n, n1=n + 1)
+        ref_b = torch.from_numpy(ref).to(torch.bfloat16).float().numpy()
+        got = y[n:n + 1].float().cpu().numpy().reshape(ref.shape)
+        ulp = np.abs(ref_b) * 2.0 ** -7 + 1e-30
+        assert np.all(np.abs(got - ref_b) <= ulp + 1e-6 * np.abs(ref).max()), f"{layer.name} image {n}"
