@@ -449,7 +449,103 @@ def conv_traffic(workload, out_dtype):
         return None
 
 
-def sweep_report(dev, out_dtype, reps=5):
+def time_steps(rs, ss, flush, k, with_conv_events):
+    """k steps of the layers `rs`, L2 flushed before each (outside the window):
+    the step times (ms) and, with events around each forward call, the per-call
+    times."""
+    import torch
+    step_ms, conv_ms = [], [[] for _ in rs]
+    for _ in range(k):
+        flush.fill_(1)
+        torch.cuda._sleep(3_000_000)  # ~1.5-2 ms: host enqueues the step meanwhile
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in rs] \
+            if with_conv_events else None
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        enqueue_step(rs, ss, ev)
+        e1.record()
+        torch.cuda.synchronize()
+        step_ms.append(e0.elapsed_time(e1))
+        if ev:
+            for i, (a, b) in enumerate(ev):
+                conv_ms[i].append(a.elapsed_time(b))
+    return step_ms, conv_ms
+
+
+def forward_roofline(runs, t_conv_s, peaks):
+    """Roofline of the forward calls of a step: the binding roof (HBM bytes or
+    bf16 tensor flops, algorithmic) and the fraction of it reached."""
+    nbytes = sum(r.conv_bytes() for r in runs)
+    flops = sum(r.flops() for r in runs)
+    t_mem = nbytes / (peaks["hbm_gbs"] * 1e9)
+    t_cmp = flops / (peaks["bf16_tflops"] * 1e12)
+    if t_mem >= t_cmp:
+        a = nbytes / t_conv_s / 1e9
+        roof = {"bound": "hbm", "achieved": a, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": a / peaks["hbm_gbs"]}
+    else:
+        a = flops / t_conv_s / 1e12
+        roof = {"bound": "tensor", "achieved": a, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                "frac": a / peaks["bf16_tflops"]}
+    roof["combined_roofline_frac"] = max(t_mem, t_cmp) / t_conv_s
+    return roof
+
+
+WORKLOAD_LABELS = {
+    "c3d": "C3D layer N8 C128 T8 28x28 F256 3x3x3 p1, shape-wise 30%",
+    "resnet50": "ResNet-50 bottleneck CONV layers (16), batch 64, filter-wise 50% x channel-wise 50%",
+    "single2d": "single 2-D CONV N8 C64 32x32 F64 3x3 p1, shape-wise 50%",
+}
+
+
+def configs_report(dev, out_dtype, peaks, steps=10, names=("c3d", "resnet50", "single2d")):
+    """The other workloads through the same step as the headline line
+    (projection + pack + forward of every layer, L2 flushed before each step):
+    TFLOP/s on retained MACs, the forward calls' roofline (whichever of HBM and
+    the bf16 tensor peak binds) and the speedup over the same step at 0%
+    sparsity."""
+    import torch
+    out = {}
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    for name in names:
+        layers = wl.get(name)
+        tensors = [wl.gen_tensors(L.shape, seed=L.seed) for L in layers]
+        runs = [LayerRun(L, t, dev, out_dtype) for L, t in zip(layers, tensors)]
+        dense = [LayerRun(L, t, dev, out_dtype, dense=True) for L, t in zip(layers, tensors)]
+        ss = StepStreams(len(runs))
+        for _ in range(3):
+            enqueue_step(runs, ss)
+            enqueue_step(dense, ss)
+        torch.cuda.synchronize()
+        step_ms, _ = time_steps(runs, ss, flush, steps, False)
+        _, conv_ms = time_steps(runs, ss, flush, steps, True)
+        dense_ms, _ = time_steps(dense, ss, flush, steps, False)
+        _, dconv_ms = time_steps(dense, ss, flush, steps, True)
+        from paper_1807_11091_gb300 import sadmm
+        if sadmm.sadmm_last_device_status(int(torch.cuda.current_stream().cuda_stream)) != 0:
+            raise RuntimeError(f"device status set after the {name} steps")
+        flops = sum(r.flops() for r in runs)
+        t_step = statistics.median(step_ms)
+        t_conv = sum(statistics.median(c) for c in conv_ms)
+        t_dconv = sum(statistics.median(c) for c in dconv_ms)
+        tf = flops / (t_step * 1e-3) / 1e12
+        out[name] = {
+            "workload": WORKLOAD_LABELS[name], "layers": len(runs), "ms_per_step": t_step,
+            "tflops_retained": tf, "pct_bf16_peak": tf / peaks["bf16_tflops"],
+            "conv_us": t_conv * 1e3, "conv_tflops": flops / (t_conv * 1e-3) / 1e12,
+            "speedup_vs_dense": statistics.median(dense_ms) / t_step,
+            "conv_speedup_vs_dense": t_dconv / t_conv,
+            "roofline": forward_roofline(runs, t_conv * 1e-3, peaks),
+        }
+        del runs, dense, tensors, ss
+        torch.cuda.empty_cache()
+    del flush
+    torch.cuda.empty_cache()
+    return out
+
+
+def sweep_report(dev, out_dtype, reps=5, peak_tflops=None):
     """sadmm_conv_fwd alone on the large sweep layer (N128 C256 28x28 F512 3x3)
     at every retained fraction, against the same kernel at 0% sparsity."""
     import torch
@@ -484,12 +580,76 @@ def sweep_report(dev, out_dtype, reps=5):
     dense_us = times[0] * 1e3
     out = {"layer": "N128 C256 28x28 F512 3x3 p1, shape-wise x filter-wise", "dense_conv_us": dense_us,
            "dense_tflops": runs[0].flops() / (times[0] * 1e-3) / 1e12, "variants": []}
+    if peak_tflops:
+        out["dense_pct_bf16_peak"] = out["dense_tflops"] / peak_tflops
     for L, r, ms in zip(layers, runs[1:], times[1:]):
         out["variants"].append({"filters": L.filt_frac, "columns": L.col_frac, "conv_us": ms * 1e3,
                                 "tflops_retained": r.flops() / (ms * 1e-3) / 1e12,
                                 "speedup_vs_dense": times[0] / ms,
                                 "retained_fraction": r.flops() / runs[0].flops()})
+        if peak_tflops:
+            out["variants"][-1]["pct_bf16_peak"] = out["variants"][-1]["tflops_retained"] / peak_tflops
     del runs, flush
+    torch.cuda.empty_cache()
+    return out
+
+
+def sparse_report(dev, out_dtype, sweep, reps=3, densities=(0.5, 0.25, 0.1, 0.05)):
+    """The paper's non-structured comparison (Sec. 5) on this GPU: the sweep
+    layer pruned element by element (sadmm_project_elements keeps the largest
+    |W|) and run by the sparse forward (sadmm_sparse_conv_fwd, CSR rows on the
+    CUDA cores), beside the structured kernel at the same retained fraction
+    (filters kept, that fraction of the columns) and the dense run."""
+    import torch
+    from paper_1807_11091_gb300 import sadmm
+    L0 = wl.sweep()[0]
+    s = L0.shape
+    t = wl.gen_tensors(s, seed=L0.seed)
+    W, x, b = t["W"].to(dev), t["x"].to(dev), t["bias"].to(dev)
+    ytype = torch.bfloat16 if out_dtype == "bf16" else torch.float32
+    y = torch.empty(s.y_shape(), dtype=ytype, device=dev)
+    ydt = sadmm.SADMM_BF16 if out_dtype == "bf16" else sadmm.SADMM_FP32
+    desc = sadmm.make_desc(s.desc16())
+    sp = int(torch.cuda.current_stream().cuda_stream)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    structured = {(v["filters"], v["columns"]): v for v in sweep["variants"]}
+    out = {"what": "sweep layer N128 C256 28x28 F512 3x3 pruned element by element (largest |W| kept), "
+                   "sadmm_sparse_conv_fwd (CSR rows, CUDA cores) vs sadmm_conv_fwd at the same retained "
+                   "fraction, L2 flushed, median of " + str(reps), "variants": []}
+    for d in densities:
+        k = wl.retained(d, s.f * s.k)
+        keep = sadmm.project_elements(s.desc16(), W, k)
+        nbytes = sadmm.sadmm_sparse_plan_size(desc, k)
+        plan = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+        st = sadmm.sadmm_sparse_pack(desc, W.data_ptr(), sadmm.SADMM_BF16, keep.data_ptr(), k, plan.data_ptr(),
+                                     nbytes, sp)
+        assert st == 0, st
+        ms = []
+        for _ in range(reps + 1):
+            flush.fill_(1)
+            torch.cuda._sleep(1_000_000)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+            st = sadmm.sadmm_sparse_conv_fwd(desc, plan.data_ptr(), x.data_ptr(), b.data_ptr(), 1, y.data_ptr(),
+                                             ydt, sp)
+            e1.record()
+            torch.cuda.synchronize()
+            assert st == 0, st
+            ms.append(e0.elapsed_time(e1))
+        t_ms = statistics.median(ms[1:])
+        fl = 2.0 * s.m * k
+        v = {"density": d, "sparse_us": t_ms * 1e3, "sparse_tflops_retained": fl / (t_ms * 1e-3) / 1e12,
+             "sparse_speedup_vs_dense": sweep["dense_conv_us"] / (t_ms * 1e3)}
+        st_v = structured.get((1.0, d))
+        if st_v:
+            v["structured_us"] = st_v["conv_us"]
+            v["structured_over_sparse"] = t_ms * 1e3 / st_v["conv_us"]
+        out["variants"].append(v)
+        del keep, plan
+    if sadmm.sadmm_last_device_status(sp) != 0:
+        raise RuntimeError("device status set after the sparse forwards")
+    del flush, y, W, x, b
     torch.cuda.empty_cache()
     return out
 
@@ -708,23 +868,7 @@ def run_gpu(args):
     peaks, peak_src = load_peaks()
 
     def timed_steps(rs, k, with_conv_events):
-        step_ms, conv_ms = [], [[] for _ in rs]
-        for _ in range(k):
-            flush.fill_(1)
-            torch.cuda._sleep(3_000_000)  # ~1.5-2 ms: host enqueues the step meanwhile
-            ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in rs] \
-                if with_conv_events else None
-            e0 = torch.cuda.Event(enable_timing=True)
-            e1 = torch.cuda.Event(enable_timing=True)
-            e0.record()
-            enqueue_step(rs, ss, ev)
-            e1.record()
-            torch.cuda.synchronize()
-            step_ms.append(e0.elapsed_time(e1))
-            if ev:
-                for i, (a, b) in enumerate(ev):
-                    conv_ms[i].append(a.elapsed_time(b))
-        return step_ms, conv_ms
+        return time_steps(rs, ss, flush, k, with_conv_events)
 
     # warm-up (also the first-call setup of every kernel)
     for _ in range(max(args.warmup, 3)):
@@ -843,8 +987,12 @@ def run_gpu(args):
         "gpu_launches": sum(r.launches for r in runs) * args.steps,
         "clocks": clocks.summary(),
     }
+    if rank == 0 and not args.no_configs and args.workload == "alexnet":
+        line["configs"] = configs_report(dev, args.out_dtype, peaks)
     if rank == 0 and not args.no_sweep:
-        line["sweep"] = sweep_report(dev, args.out_dtype)
+        line["sweep"] = sweep_report(dev, args.out_dtype, peak_tflops=peaks["bf16_tflops"])
+        if not args.no_sparse:
+            line["non_structured"] = sparse_report(dev, args.out_dtype, line["sweep"])
     if rank == 0 and not args.no_batch1:
         line["batch1"] = batch1_report(dev, args.out_dtype)
     if rank == 0 and not args.no_backward:
@@ -873,6 +1021,10 @@ def main():
     ap.add_argument("--out-dtype", default="fp32", choices=["fp32", "bf16"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--no-sparse", action="store_true",
+                    help="skip the element-wise (non-structured) sparse forward beside the sweep")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the C3D, ResNet-50 and single 2-D steps reported beside the headline")
     ap.add_argument("--no-admm", action="store_true")
     ap.add_argument("--no-batch1", action="store_true")
     ap.add_argument("--no-backward", action="store_true")

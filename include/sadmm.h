@@ -211,7 +211,7 @@ size_t sadmm_elements_workspace_size(const sadmm_conv_desc* d);
  *   keep_out  device uint8 [F*K]: 1 for a kept entry, 0 otherwise.
  *   workspace sadmm_elements_workspace_size() bytes, 256-byte aligned.
  * The paper finds this sparsity hard to speed up on a GPU (Sec. 5, cuSPARSE);
- * the library offers the projection (for ADMM training), not a sparse conv.
+ * sadmm_sparse_conv_fwd below runs such a layer, for that comparison.
  */
 sadmm_status sadmm_project_elements(const sadmm_conv_desc* d, const void* W, const void* U, int wdt,
                                     long long k_elems, unsigned char* keep_out, void* workspace,
@@ -225,6 +225,37 @@ sadmm_status sadmm_project_elements(const sadmm_conv_desc* d, const void* W, con
  */
 sadmm_status sadmm_admm_update_elements(const sadmm_conv_desc* d, const void* W, void* U, void* Z, int wdt,
                                         long long k_elems, void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * Forward of a layer pruned element by element (non-structured sparsity, Sec. 4;
+ * the comparison of the paper's speed tests, Sec. 5, where such layers run
+ * through a sparse library and gain little or lose on a GPU).  The kept
+ * weights are stored per filter in compressed rows (CSR) and the forward runs
+ * on the CUDA cores, one thread per output pixel and filter: a sparse matrix
+ * has no dense tile for the tensor cores.  It exists to measure that contrast
+ * on this GPU beside sadmm_conv_fwd at the same density.
+ *
+ * sadmm_sparse_plan_size: device bytes of a plan holding up to `capacity` kept
+ *   weights (0 .. F*K): row pointers [F + 1] int32 (rounded up to 256 B), then
+ *   `capacity` 16-byte entries {x offset of the column, tap bits, fp32 weight}.
+ *   0 on a bad descriptor or capacity.
+ * sadmm_sparse_pack: builds the plan from W (bf16 or fp32, OIDHW) and a keep
+ *   mask (device uint8 [F][K], nonzero = kept; e.g. from
+ *   sadmm_project_elements).  plan: device, 256-byte aligned, at least
+ *   sadmm_sparse_plan_size bytes.  More kept weights than `capacity` give an
+ *   empty plan (its forward writes ReLU(bias)) and raise the device status
+ *   word (SADMM_EINVAL from sadmm_last_device_status).  F above 65535 gives
+ *   SADMM_EUNSUPPORTED.
+ * sadmm_sparse_conv_fwd: y[n, f, o] = ReLU(bias[f] + sum over the kept (f, col)
+ *   of W[f][col] * x at col's tap, zero outside the input), fp32 accumulation
+ *   in column order; x, bias, relu, y and ydt as in sadmm_conv_fwd.  No filter
+ *   is pruned as a whole here, so the bias is never masked.
+ */
+size_t sadmm_sparse_plan_size(const sadmm_conv_desc* d, long long capacity);
+sadmm_status sadmm_sparse_pack(const sadmm_conv_desc* d, const void* W, int wdt, const unsigned char* keep,
+                               long long capacity, void* plan, size_t plan_bytes, void* stream);
+sadmm_status sadmm_sparse_conv_fwd(const sadmm_conv_desc* d, const void* plan, const void* x, const float* bias,
+                                   int relu, void* y, int ydt, void* stream);
 
 /*
  * Sizes a plan for `n_filt` kept filters and `n_colgroups` kept column groups

@@ -22,7 +22,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libsadmm.so")
 
 SOURCES = ["abi.cu", "project.cu", "pack.cu", "conv_fwd.cu", "conv_slab.cu", "admm.cu", "elements.cu", "gemm.cu",
-           "bwd.cu", "bwd_slab.cu"]
+           "bwd.cu", "bwd_slab.cu", "sparse.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

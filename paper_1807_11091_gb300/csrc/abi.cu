@@ -509,6 +509,45 @@ sadmm_status sadmm_gemm_bf16(const void* A, const void* B, float* C, long long M
     return launch_gemm(A, B, C, M, N, K, ldc, bn, accumulate != 0, static_cast<cudaStream_t>(stream));
 }
 
+size_t sadmm_sparse_plan_size(const sadmm_conv_desc* d, long long capacity)
+{
+    Geometry g;
+    if (check_desc(d, &g) != SADMM_OK) return 0;
+    if (capacity < 0 || capacity > g.f * g.k) return 0;
+    return sparse_plan_bytes(g, capacity);
+}
+
+sadmm_status sadmm_sparse_pack(const sadmm_conv_desc* d, const void* W, int wdt, const unsigned char* keep,
+                               long long capacity, void* plan, size_t plan_bytes, void* stream)
+{
+    NvtxRange range("sadmm_sparse_pack");
+    Geometry g;
+    sadmm_status st = check_desc(d, &g);
+    if (st != SADMM_OK) return st;
+    if (!W || !keep || !plan) return SADMM_EINVAL;
+    if (wdt != SADMM_BF16 && wdt != SADMM_FP32) return SADMM_EINVAL;
+    if (capacity < 0 || capacity > g.f * g.k) return SADMM_EINVAL;
+    if (plan_bytes < sparse_plan_bytes(g, capacity)) return SADMM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(plan) & 255) != 0) return SADMM_EINVAL;
+    if (g.f > 65535) return SADMM_EUNSUPPORTED;
+    return launch_sparse_pack(g, W, wdt, keep, plan, capacity, static_cast<cudaStream_t>(stream));
+}
+
+sadmm_status sadmm_sparse_conv_fwd(const sadmm_conv_desc* d, const void* plan, const void* x, const float* bias,
+                                   int relu, void* y, int ydt, void* stream)
+{
+    NvtxRange range("sadmm_sparse_conv_fwd");
+    Geometry g;
+    sadmm_status st = check_desc(d, &g);
+    if (st != SADMM_OK) return st;
+    if (!plan || !x || !y) return SADMM_EINVAL;
+    if (ydt != SADMM_BF16 && ydt != SADMM_FP32) return SADMM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(plan) & 255) != 0 || (reinterpret_cast<uintptr_t>(x) & 1) != 0) return SADMM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(y) & (ydt == SADMM_FP32 ? 3 : 1)) != 0) return SADMM_EINVAL;
+    if (bias && (reinterpret_cast<uintptr_t>(bias) & 3) != 0) return SADMM_EINVAL;
+    return launch_sparse_conv(g, plan, x, bias, relu, y, ydt, static_cast<cudaStream_t>(stream));
+}
+
 sadmm_status sadmm_selftest_wait(unsigned int limit_us, int arrive, int* result, void* stream)
 {
     if (limit_us < 1 || limit_us > 1000000) return SADMM_EINVAL;

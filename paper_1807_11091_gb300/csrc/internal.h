@@ -67,6 +67,14 @@ size_t elements_workspace_bytes(const Geometry& g);
 sadmm_status launch_elements(const Geometry& g, const void* W, void* U, void* Z, int wdt, long long k,
                              uint8_t* keep_out, void* ws, cudaStream_t s);
 
+// ---- non-structured sparse forward (sparse.cu) ----
+// Plan buffer: row pointers [F + 1] int32 (to 256 B), then `capacity` entries of 16 B.
+size_t sparse_plan_bytes(const Geometry& g, long long capacity);
+sadmm_status launch_sparse_pack(const Geometry& g, const void* W, int wdt, const uint8_t* keep, void* buf,
+                                long long capacity, cudaStream_t s);
+sadmm_status launch_sparse_conv(const Geometry& g, const void* buf, const void* x, const float* bias, int relu,
+                                void* y, int ydt, cudaStream_t s);
+
 // ---- generic bf16 GEMM on the tensor cores (gemm.cu) ----
 // C[M][N] (fp32, row stride ldc floats) = (accumulate ? C : 0) + A[M][K] * B[N][K]^T,
 // A and B bf16 row-major (K contiguous, row stride K).  M % 128 == 0,

@@ -137,6 +137,12 @@ def load():
     lib.sadmm_gemm_bf16.argtypes = [vp, vp, vp, ll, ll, ll, ll, ci, vp]
     lib.sadmm_last_device_status.restype = ci
     lib.sadmm_last_device_status.argtypes = [vp]
+    lib.sadmm_sparse_plan_size.restype = sz
+    lib.sadmm_sparse_plan_size.argtypes = [P(ConvDesc), ll]
+    lib.sadmm_sparse_pack.restype = ci
+    lib.sadmm_sparse_pack.argtypes = [P(ConvDesc), vp, ci, vp, ll, vp, sz, vp]
+    lib.sadmm_sparse_conv_fwd.restype = ci
+    lib.sadmm_sparse_conv_fwd.argtypes = [P(ConvDesc), vp, vp, vp, ci, vp, ci, vp]
     lib.sadmm_selftest_wait.restype = ci
     lib.sadmm_selftest_wait.argtypes = [ctypes.c_uint, ci, vp, vp]
     lib.sadmm_project_groups_noalloc.restype = ci
@@ -279,6 +285,21 @@ def sadmm_gemm_bf16(A: int, B: int, C: int, M: int, N: int, K: int, ldc: int, ac
 
 def sadmm_last_device_status(stream: Optional[int]) -> int:
     return load().sadmm_last_device_status(stream)
+
+
+def sadmm_sparse_plan_size(desc: ConvDesc, capacity: int) -> int:
+    return load().sadmm_sparse_plan_size(ctypes.byref(desc), int(capacity))
+
+
+def sadmm_sparse_pack(desc: ConvDesc, W: int, wdt: int, keep: int, capacity: int, plan: int, plan_bytes: int,
+                      stream: Optional[int]) -> int:
+    return load().sadmm_sparse_pack(ctypes.byref(desc), W, int(wdt), keep, int(capacity), plan, int(plan_bytes),
+                                    stream)
+
+
+def sadmm_sparse_conv_fwd(desc: ConvDesc, plan: int, x: int, bias: Optional[int], relu: int, y: int, ydt: int,
+                          stream: Optional[int]) -> int:
+    return load().sadmm_sparse_conv_fwd(ctypes.byref(desc), plan, x, bias, int(relu), y, int(ydt), stream)
 
 
 def sadmm_selftest_wait(limit_us: int, arrive: int, result: Optional[int], stream: Optional[int]) -> int:

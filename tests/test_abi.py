@@ -222,3 +222,20 @@ def test_selftest_wait_rejects_bad_arguments_on_host():
     assert sadmm.sadmm_selftest_wait(0, 0, None, None) == sadmm.SADMM_EINVAL
     assert sadmm.sadmm_selftest_wait(1000001, 0, None, None) == sadmm.SADMM_EINVAL
     assert sadmm.sadmm_selftest_wait(1000, 0, (1 << 20) + 2, None) == sadmm.SADMM_EINVAL
+
+
+def test_sparse_entry_points_reject_bad_arguments_on_host():
+    desc = sadmm.make_desc([1, 4, 1, 6, 6, 8, 1, 1, 3, 3, 1, 1, 1, 0, 1, 1])
+    full = 8 * 36
+    assert sadmm.sadmm_sparse_plan_size(desc, full) == 256 + full * 16
+    assert sadmm.sadmm_sparse_plan_size(desc, full + 1) == 0
+    assert sadmm.sadmm_sparse_plan_size(desc, -1) == 0
+    fake = 1 << 20
+    nb = sadmm.sadmm_sparse_plan_size(desc, 10)
+    assert sadmm.sadmm_sparse_pack(desc, fake, sadmm.SADMM_BF16, fake, 10, fake, nb - 1, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_sparse_pack(desc, fake, sadmm.SADMM_BF16, fake, 10, fake + 16, nb, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_sparse_pack(desc, fake, 7, fake, 10, fake, nb, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_sparse_pack(desc, None, sadmm.SADMM_BF16, fake, 10, fake, nb, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_sparse_conv_fwd(desc, fake, fake, None, 1, fake, 9, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_sparse_conv_fwd(desc, fake + 16, fake, None, 1, fake, 1, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_sparse_conv_fwd(desc, fake, fake, None, 1, fake + 2, 1, None) == sadmm.SADMM_EINVAL
