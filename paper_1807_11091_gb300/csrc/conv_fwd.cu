@@ -18,10 +18,11 @@
 //               ReLU, coalesced stores to the NCHW output (consecutive lanes
 //               write consecutive pixels of one filter plane), and zero-fill of
 //               the pruned filters' planes for the tile's pixels
-//   warps 12-27 gather, in two sets that fill alternate stages: in a set, two
-//               threads per pixel of the tile, each building four 16-byte
-//               K-major chunks of A through the gather table, with zero fill
-//               outside the input, into the 128-byte-swizzled stage buffer
+//   warps 12-27 gather, in two sets that fill alternate stages: in a set, each
+//               thread builds two 16-byte K-major chunks of A for two pixels
+//               of the tile (rows pp and pp + 64) through the gather table,
+//               with zero fill outside the input, into the 128-byte-swizzled
+//               stage buffer
 // Shared-memory stages are guarded by mbarriers; the accumulator is double
 // buffered in TMEM so the epilogue of one tile overlaps the MMAs of the next.
 #include <cuda.h>
@@ -45,9 +46,16 @@ constexpr int kGatherThreads = kGatherWarps * 32;
 // stage overlaps the loads of the next.
 constexpr int kGatherSets = 2;
 constexpr int kSetThreads = kGatherThreads / kGatherSets;
-constexpr int kSetGroups = kSetThreads / kBM;       // threads of a set per pixel
-constexpr int kChunksPerThread = 8 / kSetGroups;    // 16-byte chunks of a stage row per thread
-static_assert(kSetThreads % kBM == 0 && 8 % kSetGroups == 0, "a gather set must split a 64-column row evenly");
+// A gather thread builds kPixPerThread pixel rows (pp, pp + kPixStride, ...) of
+// kChunksPerThread 16-byte column chunks each.  More pixels per thread mean
+// fewer reads of the (broadcast) gather table per element: a 16-byte shared
+// load takes four wavefronts of the L1 data pipe whatever its addresses, and
+// that pipe also carries the gather's global loads.
+constexpr int kPixPerThread = 2;
+constexpr int kPixStride = kBM / kPixPerThread;                         // 64 pixel slots
+constexpr int kChunksPerThread = 8 * kPixStride / kSetThreads;          // 2 chunks of 8 columns
+static_assert(kSetThreads % kPixStride == 0 && kChunksPerThread * kSetThreads == 8 * kPixStride,
+              "a gather set must split a 128 x 64 stage evenly");
 constexpr int kATileBytes = kBM * kBK * 2;  // 16 KB
 constexpr int kMaxStages = 8;        // A stages (and B stages when B streams)
 constexpr int kStreamStages = 4;     // stages when B streams with A
@@ -655,8 +663,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int gt = threadIdx.x - (4 + kEpiWarps) * 32;
         const int set = gt / kSetThreads;
         const int st = gt - set * kSetThreads;
-        const int prow = st & (kBM - 1);
-        const int chunk0 = st >> 7;  // this thread builds chunks chunk0 + kSetGroups * i
+        const int pp = st % kPixStride;                        // first pixel row of this thread
+        const int chunk0 = (st / kPixStride) * kChunksPerThread;  // its chunks chunk0 .. + kChunksPerThread - 1
         const unsigned short* xs = reinterpret_cast<const unsigned short*>(a.x);
         int s = 0;
         uint32_t ph = 0;
@@ -666,65 +674,80 @@ __global__ void __launch_bounds__(kThreads, 1)
         int p, g, sp, ks0, ks1, mt;
         while (ok && work_next<SK>(a, wk, p, g, mt, sp, ks0, ks1)) {
             if (s_counts[2 * g] <= p * a.nacc * a.bn) continue;
-            const int m = mt * kBM + prow;
-            uint32_t M = 0;
-            const unsigned short* xb = xs;
-            if (m < a.M) {
-                const long long n_img = fdiv((uint32_t)m, a.plane_div);
-                const int pix = (int)(m - n_img * a.plane);
-                const int ot = (int)fdiv((uint32_t)pix, a.ohw_div);
-                const int r2 = pix - ot * a.OHW;
-                const int oh = (int)fdiv((uint32_t)r2, a.ow_div);
-                const int ow = r2 - oh * a.OW;
-                const int it0 = ot * a.st - a.pt, ih0 = oh * a.sh - a.ph, iw0 = ow * a.sw - a.pw;
-                M = pixel_mask(a, it0, ih0, iw0);
-                xb = xs + (n_img * a.x_chw + (long long)g * a.Cg * a.thw + (long long)it0 * a.hw +
-                           (long long)ih0 * a.W + iw0);
+            uint32_t M[kPixPerThread];
+            const unsigned short* xb[kPixPerThread];
+            bool full = true;
+#pragma unroll
+            for (int r = 0; r < kPixPerThread; ++r) {
+                const int m = mt * kBM + pp + r * kPixStride;
+                M[r] = 0;
+                xb[r] = xs;
+                if (m < a.M) {
+                    const long long n_img = fdiv((uint32_t)m, a.plane_div);
+                    const int pix = (int)(m - n_img * a.plane);
+                    const int ot = (int)fdiv((uint32_t)pix, a.ohw_div);
+                    const int r2 = pix - ot * a.OHW;
+                    const int oh = (int)fdiv((uint32_t)r2, a.ow_div);
+                    const int ow = r2 - oh * a.OW;
+                    const int it0 = ot * a.st - a.pt, ih0 = oh * a.sh - a.ph, iw0 = ow * a.sw - a.pw;
+                    M[r] = pixel_mask(a, it0, ih0, iw0);
+                    xb[r] = xs + (n_img * a.x_chw + (long long)g * a.Cg * a.thw + (long long)it0 * a.hw +
+                                  (long long)ih0 * a.W + iw0);
+                }
+                full = full && M[r] == a.full_mask;
             }
-            // Every lane's pixel sees every tap: no bounds test is needed.
-            const bool interior = __all_sync(0xffffffffu, M == a.full_mask);
+            // Every lane's pixels see every tap: no bounds test is needed.
+            const bool interior = __all_sync(0xffffffffu, full);
             for (int ks = ks0; ks < ks1; ++ks) {
                 if (turn == set) {
                     // Issue every load of this thread's columns first (they
                     // read only x), then wait for the stage buffer and store.
                     const uint2* te = s_table + (size_t)ks * kBK;
-                    uint32_t v[8 * kChunksPerThread];
-                    // two table entries per 16-byte shared-memory load
+                    uint32_t v[8 * kChunksPerThread * kPixPerThread];  // [pixel][chunk][column]
+                    // two table entries per 16-byte shared-memory load, used for every pixel of the thread
                     const uint4* te4 = reinterpret_cast<const uint4*>(te);
                     if (interior && (ks + 1) * kBK <= a.n_cols) {
 #pragma unroll
                         for (int ci = 0; ci < kChunksPerThread; ++ci) {
-                            const int c = chunk0 + kSetGroups * ci;
 #pragma unroll
                             for (int e = 0; e < 8; e += 2) {
-                                const uint4 t = te4[(c * 8 + e) >> 1];
-                                v[ci * 8 + e] = __ldg(xb + (int)t.x);
-                                v[ci * 8 + e + 1] = __ldg(xb + (int)t.z);
+                                const uint4 t = te4[((chunk0 + ci) * 8 + e) >> 1];
+#pragma unroll
+                                for (int r = 0; r < kPixPerThread; ++r) {
+                                    v[(r * kChunksPerThread + ci) * 8 + e] = __ldg(xb[r] + (int)t.x);
+                                    v[(r * kChunksPerThread + ci) * 8 + e + 1] = __ldg(xb[r] + (int)t.z);
+                                }
                             }
                         }
                     } else {
 #pragma unroll
                         for (int ci = 0; ci < kChunksPerThread; ++ci) {
-                            const int c = chunk0 + kSetGroups * ci;
 #pragma unroll
                             for (int e = 0; e < 8; e += 2) {
-                                const uint4 t = te4[(c * 8 + e) >> 1];
-                                v[ci * 8 + e] = ldg_u16_if(xb + (int)t.x, t.y, M);
-                                v[ci * 8 + e + 1] = ldg_u16_if(xb + (int)t.z, t.w, M);
+                                const uint4 t = te4[((chunk0 + ci) * 8 + e) >> 1];
+#pragma unroll
+                                for (int r = 0; r < kPixPerThread; ++r) {
+                                    v[(r * kChunksPerThread + ci) * 8 + e] = ldg_u16_if(xb[r] + (int)t.x, t.y, M[r]);
+                                    v[(r * kChunksPerThread + ci) * 8 + e + 1] =
+                                        ldg_u16_if(xb[r] + (int)t.z, t.w, M[r]);
+                                }
                             }
                         }
                     }
                     if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, a.status)) { ok = false; break; }
                     uint8_t* tile = sA + (size_t)s * kATileBytes;
 #pragma unroll
-                    for (int ci = 0; ci < kChunksPerThread; ++ci) {
-                        const int c = chunk0 + kSetGroups * ci;
-                        const uint32_t* q = v + ci * 8;
-                        *reinterpret_cast<uint4*>(tile + sw128_offset((uint32_t)prow, (uint32_t)c)) =
-                            make_uint4(__byte_perm(q[0], q[1], 0x5410), __byte_perm(q[2], q[3], 0x5410),
-                                       __byte_perm(q[4], q[5], 0x5410), __byte_perm(q[6], q[7], 0x5410));
+                    for (int r = 0; r < kPixPerThread; ++r) {
+#pragma unroll
+                        for (int ci = 0; ci < kChunksPerThread; ++ci) {
+                            const uint32_t* q = v + (r * kChunksPerThread + ci) * 8;
+                            *reinterpret_cast<uint4*>(
+                                tile + sw128_offset((uint32_t)(pp + r * kPixStride), (uint32_t)(chunk0 + ci))) =
+                                make_uint4(__byte_perm(q[0], q[1], 0x5410), __byte_perm(q[2], q[3], 0x5410),
+                                           __byte_perm(q[4], q[5], 0x5410), __byte_perm(q[6], q[7], 0x5410));
+                        }
                     }
-                    // every lane's stores are visible to the tensor core's async
+                // every lane's stores are visible to the tensor core's async
                     // proxy, then one arrival for the warp
                     fence_proxy_async_smem();
                     __syncwarp();
