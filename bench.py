@@ -654,6 +654,55 @@ def sparse_report(dev, out_dtype, sweep, reps=3, densities=(0.5, 0.25, 0.1, 0.05
     return out
 
 
+def projection_batch_report(dev, peak_gbs, reps=5):
+    """The projection of every ResNet-50 bottleneck layer (16 layers, bf16 W,
+    filter-wise 50 % + channel-wise 50 %, Sec. 4) as one
+    sadmm_project_groups_batch call, against the same 16 projections as
+    separate sadmm_project_groups calls back to back; L2 flushed before each.
+    Algorithmic bytes: W read once per key family (filter keys over all rows,
+    column keys over the kept rows) plus the keys and index lists."""
+    import torch
+    from paper_1807_11091_gb300 import sadmm
+    layers = wl.resnet50()
+    Ws = [wl.gen_tensors(L.shape.with_batch(1), seed=L.seed)["W"].to(dev) for L in layers]
+    args = [(L.shape.desc16(), W, L.k_filters, L.colkind, L.k_cols, None) for L, W in zip(layers, Ws)]
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    nbytes = 0
+    for L in layers:
+        s = L.shape
+        G = s.cg if L.colkind == wl.COL_CHANNEL else s.k
+        nbytes += 2 * s.f * s.k + 2 * L.k_filters * s.k + 8 * (s.f + G) + 4 * (L.k_filters + L.k_cols)
+
+    def timed(fn):
+        fn()
+        torch.cuda.synchronize()
+        ms = []
+        for _ in range(reps):
+            flush.fill_(1)
+            torch.cuda._sleep(2_000_000)  # the host enqueues the calls meanwhile
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+            fn()
+            e1.record()
+            torch.cuda.synchronize()
+            ms.append(e0.elapsed_time(e1))
+        return statistics.median(ms)
+
+    pb = sadmm.ProjectBatch(args)
+    singles = [sadmm.ProjectBatch([a]) for a in args]  # the same work as 16 separate calls
+    t_batch = timed(lambda: pb())
+    t_each = timed(lambda: [p() for p in singles])
+    if sadmm.device_status() != 0:
+        raise RuntimeError("device status set after the projections")
+    del flush, Ws, pb, singles
+    torch.cuda.empty_cache()
+    gbs = nbytes / (t_batch * 1e-3) / 1e9
+    return {"what": "projection of the 16 ResNet-50 bottleneck layers (bf16 W), one batched call vs 16 calls",
+            "batch_us": t_batch * 1e3, "separate_us": t_each * 1e3, "bytes": nbytes, "batch_gbs": gbs,
+            "batch_hbm_frac": gbs / peak_gbs if peak_gbs else None}
+
+
 def batch1_report(dev, out_dtype, reps=7):
     """The paper's timing setting (Sec. 5): every AlexNet CONV layer at batch 1,
     sadmm_conv_fwd alone (projection and pack done once), against the same
@@ -836,7 +885,27 @@ def admm_report(dev, peak_gbs, reps=5):
     out["total_us"] = tot_ms * 1e3
     out["gbs"] = tot_bytes / (tot_ms * 1e-3) / 1e9
     out["hbm_frac"] = out["gbs"] / peak_gbs if peak_gbs else None
-    del bufs, steps, flush
+    # the five updates as one sadmm_admm_update_batch call (one launch per phase for all layers)
+    batch = sadmm.AdmmBatch([(L.shape.desc16(), L.k_filters, L.colkind, L.k_cols) for L in layers], dev)
+    Ws, Us, Zs = [b[0] for b in bufs], [b[1] for b in bufs], [b[2] for b in bufs]
+    batch(Ws, Us, Zs)
+    torch.cuda.synchronize()
+    ms = []
+    for _ in range(reps):
+        flush.fill_(1)
+        torch.cuda._sleep(1_000_000)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        batch(Ws, Us, Zs)
+        e1.record()
+        torch.cuda.synchronize()
+        ms.append(e0.elapsed_time(e1))
+    tb = statistics.median(ms)
+    out["batch"] = {"what": "the five layers' updates in one sadmm_admm_update_batch call", "us": tb * 1e3,
+                    "gbs": tot_bytes / (tb * 1e-3) / 1e9,
+                    "hbm_frac": tot_bytes / (tb * 1e-3) / 1e9 / peak_gbs if peak_gbs else None}
+    del bufs, steps, flush, batch
     torch.cuda.empty_cache()
     return out
 
@@ -999,6 +1068,7 @@ def run_gpu(args):
         line["backward"] = backward_report(dev, args.out_dtype)
     if rank == 0 and not args.no_admm:
         line["admm"] = admm_report(dev, peaks.get("hbm_gbs"))
+        line["projection_batch"] = projection_batch_report(dev, peaks.get("hbm_gbs"))
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(layers, [wl.gen_tensors(L.shape.with_batch(64), seed=L.seed)
                                                      for L in layers])

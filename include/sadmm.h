@@ -47,6 +47,10 @@ extern "C" {
 
 #define SADMM_ABI_VERSION 5
 
+/* Most layers one batched call (sadmm_project_groups_batch,
+ * sadmm_admm_update_batch) takes. */
+#define SADMM_MAX_BATCH 64
+
 /* Bytes of the fixed device array of sadmm_project_groups_noalloc. */
 #define SADMM_NOALLOC_SCRATCH_BYTES (256 * 1024)
 
@@ -166,6 +170,35 @@ sadmm_status sadmm_project_groups(const sadmm_conv_desc* d, const void* W, const
                                   int* filt_idx, int* col_idx, double* keys_out,
                                   void* workspace, size_t ws_bytes, void* stream);
 
+/*
+ * One layer of a batched projection (sadmm_project_groups_batch): the
+ * arguments of sadmm_project_groups for that layer, its own workspace
+ * included.
+ */
+typedef struct {
+    sadmm_conv_desc desc;
+    const void* W;
+    const void* U;         /* may be NULL */
+    int k_filters, colkind, k_cols;
+    int* filt_idx;
+    int* col_idx;
+    double* keys_out;      /* may be NULL */
+    void* workspace;
+    size_t ws_bytes;
+} sadmm_project_item;
+
+/*
+ * sadmm_project_groups for n layers at once (1 <= n <= SADMM_MAX_BATCH), all
+ * of dtype `wdt` (Sec. 4: an ADMM iteration projects every layer).  Results
+ * are those of n separate calls, bit for bit; the work of all layers shares
+ * each launch (filter keys, the layers' row selects side by side, column
+ * keys, the column selects side by side), so a batch costs about what one
+ * small layer does.  Each item is checked as sadmm_project_groups checks its
+ * arguments; any bad item gives SADMM_EINVAL and nothing is enqueued.  The
+ * items' outputs and workspaces must not overlap.
+ */
+sadmm_status sadmm_project_groups_batch(const sadmm_project_item* items, int n, int wdt, void* stream);
+
 /* Device bytes of scratch sadmm_admm_update needs for this layer and column
  * kind (the projection's keys plus row and column keep flags).  0 on a bad
  * descriptor. */
@@ -194,6 +227,33 @@ size_t sadmm_admm_workspace_size(const sadmm_conv_desc* d, int colkind);
 sadmm_status sadmm_admm_update(const sadmm_conv_desc* d, const void* W, void* U, void* Z, int wdt,
                                int k_filters, int colkind, int k_cols, int* filt_idx, int* col_idx,
                                double* keys_out, void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * One layer of a batched ADMM update (sadmm_admm_update_batch): the
+ * arguments of sadmm_admm_update for that layer.
+ */
+typedef struct {
+    sadmm_conv_desc desc;
+    const void* W;
+    void* U;
+    void* Z;
+    int k_filters, colkind, k_cols;
+    int* filt_idx;
+    int* col_idx;
+    double* keys_out;      /* may be NULL */
+    void* workspace;       /* sadmm_admm_workspace_size() bytes, 256-byte aligned */
+    size_t ws_bytes;
+} sadmm_admm_item;
+
+/*
+ * sadmm_admm_update for n layers at once (1 <= n <= SADMM_MAX_BATCH), all of
+ * dtype `wdt`: one ADMM Z- and U-update of every layer of a network (Sec. 4).
+ * Results equal those of n separate calls bit for bit; the batch shares the
+ * projection's launches (see sadmm_project_groups_batch) and one apply pass.
+ * Each item is checked as sadmm_admm_update checks its arguments (SADMM_EINVAL
+ * before anything is enqueued).  Tensors of different items must not overlap.
+ */
+sadmm_status sadmm_admm_update_batch(const sadmm_admm_item* items, int n, int wdt, void* stream);
 
 /* Device bytes of scratch the non-structured projection needs for this
  * layer (selection state, a 2048-bin histogram, one counter per 4096

@@ -181,6 +181,38 @@ sadmm_status sadmm_project_groups(const sadmm_conv_desc* d, const void* W, const
                           static_cast<cudaStream_t>(stream));
 }
 
+sadmm_status sadmm_project_groups_batch(const sadmm_project_item* items, int n, int wdt, void* stream)
+{
+    NvtxRange range("sadmm_project_groups_batch");
+    if (!items || n < 1 || n > SADMM_MAX_BATCH) return SADMM_EINVAL;
+    ProjItem pit[SADMM_MAX_BATCH];
+    for (int l = 0; l < n; ++l) {
+        const sadmm_project_item& it = items[l];
+        Geometry g;
+        sadmm_status st = check_desc(&it.desc, &g);
+        if (st != SADMM_OK) return st;
+        st = check_project_args(g, it.W, wdt, it.k_filters, it.colkind, it.k_cols, it.filt_idx, it.col_idx,
+                                it.keys_out);
+        if (st != SADMM_OK) return st;
+        if (!it.workspace || it.ws_bytes < project_workspace_bytes(g, it.colkind)) return SADMM_EINVAL;
+        if ((reinterpret_cast<uintptr_t>(it.workspace) & 7) != 0) return SADMM_EINVAL;
+        pit[l].g = g;
+        pit[l].W = it.W;
+        pit[l].U = it.U;
+        pit[l].Z = nullptr;
+        pit[l].k_filters = it.k_filters;
+        pit[l].colkind = it.colkind;
+        pit[l].k_cols = it.k_cols;
+        pit[l].filt_idx = it.filt_idx;
+        pit[l].col_idx = it.col_idx;
+        pit[l].keys_out = it.keys_out;
+        pit[l].ws = it.workspace;
+        pit[l].rkeep = nullptr;
+        pit[l].ckeep = nullptr;
+    }
+    return launch_project_batch(pit, n, wdt, static_cast<cudaStream_t>(stream));
+}
+
 size_t sadmm_admm_workspace_size(const sadmm_conv_desc* d, int colkind)
 {
     Geometry g;
@@ -188,11 +220,12 @@ size_t sadmm_admm_workspace_size(const sadmm_conv_desc* d, int colkind)
     return admm_workspace_bytes(g, colkind);
 }
 
-sadmm_status sadmm_admm_update(const sadmm_conv_desc* d, const void* W, void* U, void* Z, int wdt, int k_filters,
-                               int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out,
-                               void* workspace, size_t ws_bytes, void* stream)
+// The checks of one layer of an ADMM update (sadmm_admm_update and each item
+// of sadmm_admm_update_batch).
+static sadmm_status check_admm_item(const sadmm_conv_desc* d, const void* W, const void* U, const void* Z, int wdt,
+                                    int k_filters, int colkind, int k_cols, const int* filt_idx, const int* col_idx,
+                                    const double* keys_out, const void* workspace, size_t ws_bytes, Geometry* gout)
 {
-    NvtxRange range("sadmm_admm_update");
     Geometry g;
     sadmm_status st = check_desc(d, &g);
     if (st != SADMM_OK) return st;
@@ -209,6 +242,47 @@ sadmm_status sadmm_admm_update(const sadmm_conv_desc* d, const void* W, void* U,
     auto overlap = [bytes](uintptr_t p, uintptr_t q) { return p < q + bytes && q < p + bytes; };
     if (overlap(w, u) || overlap(w, z) || overlap(u, z)) return SADMM_EINVAL;
     if (g.f > 65535) return SADMM_EUNSUPPORTED;
+    *gout = g;
+    return SADMM_OK;
+}
+
+sadmm_status sadmm_admm_update_batch(const sadmm_admm_item* items, int n, int wdt, void* stream)
+{
+    NvtxRange range("sadmm_admm_update_batch");
+    if (!items || n < 1 || n > SADMM_MAX_BATCH) return SADMM_EINVAL;
+    ProjItem pit[SADMM_MAX_BATCH];
+    for (int l = 0; l < n; ++l) {
+        const sadmm_admm_item& it = items[l];
+        Geometry g;
+        const sadmm_status st = check_admm_item(&it.desc, it.W, it.U, it.Z, wdt, it.k_filters, it.colkind, it.k_cols,
+                                                it.filt_idx, it.col_idx, it.keys_out, it.workspace, it.ws_bytes, &g);
+        if (st != SADMM_OK) return st;
+        pit[l].g = g;
+        pit[l].W = it.W;
+        pit[l].U = it.U;
+        pit[l].Z = it.Z;
+        pit[l].k_filters = it.k_filters;
+        pit[l].colkind = it.colkind;
+        pit[l].k_cols = it.k_cols;
+        pit[l].filt_idx = it.filt_idx;
+        pit[l].col_idx = it.col_idx;
+        pit[l].keys_out = it.keys_out;
+        pit[l].ws = it.workspace;
+        pit[l].rkeep = nullptr;
+        pit[l].ckeep = nullptr;
+    }
+    return launch_admm_batch(pit, n, wdt, static_cast<cudaStream_t>(stream));
+}
+
+sadmm_status sadmm_admm_update(const sadmm_conv_desc* d, const void* W, void* U, void* Z, int wdt, int k_filters,
+                               int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out,
+                               void* workspace, size_t ws_bytes, void* stream)
+{
+    NvtxRange range("sadmm_admm_update");
+    Geometry g;
+    const sadmm_status st = check_admm_item(d, W, U, Z, wdt, k_filters, colkind, k_cols, filt_idx, col_idx,
+                                            keys_out, workspace, ws_bytes, &g);
+    if (st != SADMM_OK) return st;
     return launch_admm_update(g, W, U, Z, wdt, k_filters, colkind, k_cols, filt_idx, col_idx, keys_out,
                               workspace, static_cast<cudaStream_t>(stream));
 }

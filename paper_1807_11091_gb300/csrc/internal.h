@@ -50,6 +50,30 @@ inline long long round_up(long long x, long long a) { return (x + a - 1) / a * a
 
 // ---- projection (project.cu) ----
 size_t project_workspace_bytes(const Geometry& g, int colkind);
+
+// One layer of a batched projection or ADMM update: its geometry, tensors,
+// selection, index lists and workspace; rkeep / ckeep (optional) get a byte
+// per filter / column group; Z is the ADMM update's output (NULL otherwise).
+struct ProjItem {
+    Geometry g;
+    const void* W;
+    const void* U;
+    void* Z;
+    int k_filters, colkind, k_cols;
+    int* filt_idx;
+    int* col_idx;
+    double* keys_out;
+    void* ws;
+    uint8_t* rkeep;
+    uint8_t* ckeep;
+};
+constexpr int kMaxBatch = SADMM_MAX_BATCH;
+// The projection of items[0..n) (checked arguments, one dtype): one launch per
+// phase for the whole batch.
+sadmm_status launch_project_batch(const ProjItem* items, int n, int wdt, cudaStream_t s);
+// The ADMM update of items[0..n): the batched projection with keep flags in
+// each item's workspace, then one apply pass over every layer.
+sadmm_status launch_admm_batch(const ProjItem* items, int n, int wdt, cudaStream_t s);
 // rkeep / ckeep (optional): a byte per filter / per column group, 1 when kept.
 sadmm_status launch_project(const Geometry& g, const void* W, const void* U, int wdt, int k_filters,
                             int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out,

@@ -2,19 +2,25 @@
 // solution of the Z-subproblem, Eq. 4): squared Frobenius norms of the filter,
 // channel or shape groups of V = W (+U), then an exact top-k.
 //
-// Kernels:
+// Every launch serves a batch of layers (a single call is a batch of one):
+// the layers' parameters travel in kernel parameter space, and a block finds
+// its layer by its index.
 //   k_filter_keys   one block per GEMM row (filter): fp64 sums of squares in
 //                   four independent partials per thread, warp-shuffle and
 //                   fixed-order block reduction.
 //   k_column_keys   32 columns per block, 8 warps over the (kept) rows, fixed
 //                   order shared-memory reduction: one key per GEMM column.
-//   k_select        one block: optional channel sums of column keys, an MSB-
-//                   first radix select over the fp64 key bit patterns (exact
-//                   k-th largest key), then an ordered compaction that keeps
-//                   every key above it and the lowest-index keys equal to it.
+//   k_select_rows / k_select_cols
+//                   one block per layer: optional channel sums of column keys,
+//                   an MSB-first radix select over the fp64 key bit patterns
+//                   (exact k-th largest key), then an ordered compaction that
+//                   keeps every key above it and the lowest-index keys equal
+//                   to it.  The layers' selects run side by side.
 //
 // Keys are non-negative fp64 values, so their IEEE bit patterns order like the
 // values; selection compares bit patterns (a NaN key would rank above +Inf).
+#include <string.h>
+
 #include <algorithm>
 #include <atomic>
 
@@ -40,15 +46,62 @@ SADMM_DEV double v_elem(const T* __restrict__ W, const T* __restrict__ U, long l
     return v;
 }
 
+// Per-layer parameters of a batched projection (kernel parameter space; a
+// block finds its layer by its first-block offsets).
+struct BLayer {
+    const void* W;
+    const void* U;
+    const int* krows;  // kept-row list the column keys sum over (NULL: every row)
+    int* filt_idx;
+    int* col_idx;
+    double* keys_out;
+    double* fkeys;  // filter keys [F]
+    double* ckeys;  // column-group keys [G]
+    double* parts;  // partial column keys [R][K]
+    uint8_t* rkeep;
+    uint8_t* ckeep;
+    int F, K, taps, G, k_filters, k_cols;
+    int do_rows, do_cols;  // 1: keys and select of this kind run
+    int R, cblocks, nrows;
+    int fk0, ck0, ka0, ka_n;  // first block in the filter-key, column-key, keep-all grids; keep-all length
+    int rows_all, cols_all;   // lists written whole by the keep-all pass
+};
+
+struct BatchArgs {
+    int n;
+    BLayer L[kMaxBatch];
+};
+
+// The layer whose block range of one grid holds block b: the last layer with
+// first block <= b (the ranges are ascending; empty ranges are skipped by the
+// callers' bounds checks).
+template <int BLayer::*Start>
+SADMM_DEV int find_layer(const BatchArgs& a, int b)
+{
+    int lo = 0, hi = a.n - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (a.L[mid].*Start <= b) lo = mid;
+        else hi = mid - 1;
+    }
+    return lo;
+}
+
 // O_a = sum_k V[a,k]^2 for every row a (filter-wise groups): one block per
-// row, strided fp64 partial sums, fixed-order block reduction.
+// row of every layer that needs them, strided fp64 partial sums, fixed-order
+// block reduction.
 template <typename T>
-__global__ void __launch_bounds__(256) k_filter_keys(const T* __restrict__ W, const T* __restrict__ U, int F,
-                                                     int K, double* __restrict__ keys)
+__global__ void __launch_bounds__(256) k_filter_keys(const __grid_constant__ BatchArgs ba)
 {
     pdl_wait();  // after the kernel before it in the stream
     __shared__ double part[8];
-    const int a = blockIdx.x;
+    const int l = find_layer<&BLayer::fk0>(ba, blockIdx.x);
+    const BLayer& L = ba.L[l];
+    const int a = blockIdx.x - L.fk0;
+    if (!L.do_rows || a >= L.F) return;
+    const T* W = static_cast<const T*>(L.W);
+    const T* U = static_cast<const T*>(L.U);
+    const int K = L.K;
     const int lane = threadIdx.x & 31, wy = threadIdx.x >> 5;
     const long long base = (long long)a * K;
     // four independent partial sums per thread (loads and fp64 FMAs overlap),
@@ -74,29 +127,33 @@ __global__ void __launch_bounds__(256) k_filter_keys(const T* __restrict__ W, co
     if (threadIdx.x == 0) {
         double t = 0.0;
         for (int q = 0; q < 8; ++q) t += part[q];
-        keys[a] = t;
+        L.fkeys[a] = t;
     }
 }
 
-// Partial column keys: block (bx, by) sums V[a,j]^2 over rows by, by + R, ...
-// of the kept-row list for the 32 columns j of bx, and writes
-// part[by][j].  rows == NULL means rows 0..nrows-1.  The select kernel adds the
-// R partials of a column in fixed order.
+// Partial column keys: block (bx, by) of a layer sums V[a,j]^2 over rows by,
+// by + R, ... of the kept-row list for the 32 columns j of bx, and writes
+// part[by][j].  The select adds the R partials of a column in fixed order.
 template <typename T>
-__global__ void __launch_bounds__(256) k_column_keys(const T* __restrict__ W, const T* __restrict__ U, int K,
-                                                     const int* __restrict__ rows, int nrows,
-                                                     double* __restrict__ part_out)
+__global__ void __launch_bounds__(256) k_column_keys(const __grid_constant__ BatchArgs ba)
 {
-    pdl_wait();  // after the kernel before it in the stream
+    pdl_wait();  // after the kernel before it in the stream (the kept rows)
     __shared__ double part[8][33];
+    const int l = find_layer<&BLayer::ck0>(ba, blockIdx.x);
+    const BLayer& L = ba.L[l];
+    const int local = blockIdx.x - L.ck0;
+    if (!L.do_cols || local >= L.cblocks * L.R) return;
+    const int bx = local % L.cblocks, by = local / L.cblocks;
+    const T* W = static_cast<const T*>(L.W);
+    const T* U = static_cast<const T*>(L.U);
+    const int K = L.K, R = L.R;
     const int lane = threadIdx.x & 31;
     const int wy = threadIdx.x >> 5;
-    const int j = blockIdx.x * 32 + lane;
-    const int R = gridDim.y;
+    const int j = bx * 32 + lane;
     double s = 0.0;
     if (j < K) {
-        for (int r = blockIdx.y + R * wy; r < nrows; r += 8 * R) {
-            const int a = rows ? rows[r] : r;
+        for (int r = by + R * wy; r < L.nrows; r += 8 * R) {
+            const int a = L.krows ? L.krows[r] : r;
             const double v = v_elem(W, U, (long long)a * K + j);
             s = fma(v, v, s);
         }
@@ -106,7 +163,7 @@ __global__ void __launch_bounds__(256) k_column_keys(const T* __restrict__ W, co
     if (wy == 0 && j < K) {
         double t = 0.0;
         for (int q = 0; q < 8; ++q) t += part[q][lane];
-        part_out[(long long)blockIdx.y * K + j] = t;
+        L.parts[(long long)by * K + j] = t;
     }
 }
 
@@ -138,16 +195,15 @@ SADMM_DEV int block_excl_count(bool pred, int* warp_tot, int* total)
     return r;
 }
 
-// Exact top-k of G fp64 keys (ties to the lower index), ascending index list.
-// When taps > 1 the keys are first formed as sums of `taps` consecutive source
-// keys (channel-wise groups from column keys).  keep_out (optional) gets a
-// byte per group: 1 when kept.
-__global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict__ src, int G, int taps, int k,
-                                                        int nparts, long long part_stride,
-                                                        double* __restrict__ keys, double* __restrict__ keys_out,
-                                                        int* __restrict__ out_idx, uint8_t* __restrict__ keep_out)
+// Exact top-k of G fp64 keys (ties to the lower index), ascending index list,
+// by one block.  When taps > 1 the keys are first formed as sums of `taps`
+// consecutive source keys (channel-wise groups from column keys), each the sum
+// of its nparts partial sums.  keep_out (optional) gets a byte per group: 1
+// when kept.
+SADMM_DEV void select_block(const double* __restrict__ src, int G, int taps, int k, int nparts,
+                            long long part_stride, double* __restrict__ keys, double* __restrict__ keys_out,
+                            int* __restrict__ out_idx, uint8_t* __restrict__ keep_out)
 {
-    pdl_wait();  // after the kernel before it in the stream
     __shared__ unsigned int hist[256];
     __shared__ unsigned long long s_prefix;
     __shared__ int s_kk;
@@ -258,15 +314,27 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const double* __restrict
     }
 }
 
-void launch_select(const double* src, int G, int taps, int k, int nparts, long long part_stride, double* keys,
-                   double* keys_out, int* out_idx, uint8_t* keep_out, cudaStream_t s)
+// Row (filter) selects: one block per layer of the batch.
+__global__ void __launch_bounds__(kSelThreads) k_select_rows(const __grid_constant__ BatchArgs ba)
 {
-    launch_pdl(k_select, dim3(1), dim3(kSelThreads), 0, s, src, G, taps, k, nparts, part_stride, keys, keys_out,
-               out_idx, keep_out);
+    pdl_wait();  // after the kernel before it in the stream (the filter keys)
+    const BLayer& L = ba.L[blockIdx.x];
+    if (!L.do_rows) return;
+    select_block(L.fkeys, L.F, 1, L.k_filters, 1, 0, L.fkeys, L.keys_out, L.filt_idx, L.rkeep);
 }
 
-// Row chunks of the column-key pass: enough blocks to fill the GPU, with the
-// partial sums bounded to 16384 doubles.
+// Column-group selects: one block per layer of the batch.
+__global__ void __launch_bounds__(kSelThreads) k_select_cols(const __grid_constant__ BatchArgs ba)
+{
+    pdl_wait();  // after the kernel before it in the stream (the column keys)
+    const BLayer& L = ba.L[blockIdx.x];
+    if (!L.do_cols) return;
+    select_block(L.parts, L.G, L.taps, L.k_cols, L.R, L.K, L.ckeys, L.keys_out ? L.keys_out + L.F : nullptr,
+                 L.col_idx, L.ckeep);
+}
+
+// Row-chunk count of the column-key pass of one layer: enough blocks to fill
+// the GPU, with the partial sums bounded to 16384 doubles.
 int column_parts(long long K, long long nrows)
 {
     long long r = (304 + (K + 31) / 32 - 1) / ((K + 31) / 32);
@@ -275,56 +343,87 @@ int column_parts(long long K, long long nrows)
     return (int)std::max(r, 1ll);
 }
 
-// Index lists 0..n-1 and keep flags of one for the kinds kept whole (a null
-// list is skipped).
-__global__ void __launch_bounds__(256) k_keep_all(int* idx_a, int na, uint8_t* keep_a, int* idx_b, int nb,
-                                                  uint8_t* keep_b)
+// Index lists 0..n-1 and keep flags of one for the kinds kept whole.
+__global__ void __launch_bounds__(256) k_keep_all(const __grid_constant__ BatchArgs ba)
 {
     pdl_wait();  // after the kernel before it in the stream
-    const int i = blockIdx.x * 256 + threadIdx.x;
-    if (idx_a && i < na) {
-        idx_a[i] = i;
-        if (keep_a) keep_a[i] = 1;
+    const int l = find_layer<&BLayer::ka0>(ba, blockIdx.x);
+    const BLayer& L = ba.L[l];
+    const int i = (blockIdx.x - L.ka0) * 256 + threadIdx.x;
+    if (i >= L.ka_n) return;
+    if (L.rows_all && i < L.F) {
+        L.filt_idx[i] = i;
+        if (L.rkeep) L.rkeep[i] = 1;
     }
-    if (idx_b && i < nb) {
-        idx_b[i] = i;
-        if (keep_b) keep_b[i] = 1;
+    if (L.cols_all && i < L.G) {
+        L.col_idx[i] = i;
+        if (L.ckeep) L.ckeep[i] = 1;
     }
 }
 
 template <typename T>
-sadmm_status run_project(const Geometry& g, const T* W, const T* U, int k_filters, int colkind, int k_cols,
-                         int* filt_idx, int* col_idx, double* keys_out, void* ws, uint8_t* rkeep, uint8_t* ckeep,
-                         cudaStream_t s)
+sadmm_status run_project_batch(const ProjItem* items, int n, cudaStream_t s)
 {
-    const int F = (int)g.f, K = (int)g.k;
-    double* fkeys = reinterpret_cast<double*>(ws);
-    double* ckeys = fkeys + round_up(F, 32);                   // column keys
-    double* parts = ckeys + round_up(K, 32);                   // [R][K] partial column keys
-
-    // Keeping every group of a kind needs no keys: the top-G of G keys is the
-    // whole ascending index list.  Unless the caller asked for the keys, such
-    // lists (and keep flags) are written directly, in one launch for both kinds.
-    const int taps = (colkind == SADMM_COL_CHANNEL) ? (int)g.taps : 1;
-    const int G = (colkind == SADMM_COL_CHANNEL) ? (int)g.cg : K;
-    const bool rows_all = (k_filters == F) && !keys_out;
-    const bool cols_all = (colkind != SADMM_COL_NONE) && (k_cols == G) && !keys_out;
-    if (rows_all || cols_all) {
-        const int n = (rows_all ? F : 0) > (cols_all ? G : 0) ? F : (cols_all ? G : 0);
-        launch_pdl(k_keep_all, dim3((n + 255) / 256), dim3(256), 0, s, rows_all ? filt_idx : nullptr, F,
-                   rows_all ? rkeep : nullptr, cols_all ? col_idx : nullptr, G, cols_all ? ckeep : nullptr);
+    BatchArgs ba;
+    memset(&ba, 0, sizeof(ba));
+    ba.n = n;
+    int fk = 0, ck = 0, ka = 0;
+    bool any_rows = false, any_cols = false;
+    for (int l = 0; l < n; ++l) {
+        const ProjItem& it = items[l];
+        const Geometry& g = it.g;
+        BLayer& L = ba.L[l];
+        const int F = (int)g.f, K = (int)g.k;
+        double* fkeys = reinterpret_cast<double*>(it.ws);
+        L.W = it.W;
+        L.U = it.U;
+        L.filt_idx = it.filt_idx;
+        L.col_idx = it.col_idx;
+        L.keys_out = it.keys_out;
+        L.fkeys = fkeys;
+        L.ckeys = fkeys + round_up(F, 32);
+        L.parts = L.ckeys + round_up(K, 32);
+        L.rkeep = it.rkeep;
+        L.ckeep = it.colkind == SADMM_COL_NONE ? nullptr : it.ckeep;
+        L.F = F;
+        L.K = K;
+        L.taps = (it.colkind == SADMM_COL_CHANNEL) ? (int)g.taps : 1;
+        L.G = (it.colkind == SADMM_COL_CHANNEL) ? (int)g.cg : K;
+        L.k_filters = it.k_filters;
+        L.k_cols = it.k_cols;
+        // Keeping every group of a kind needs no keys: the top-G of G keys is
+        // the whole ascending index list.  Unless the caller asked for the
+        // keys, such lists (and keep flags) are written by the keep-all pass.
+        L.rows_all = (it.k_filters == F) && !it.keys_out;
+        L.cols_all = (it.colkind != SADMM_COL_NONE) && (it.k_cols == L.G) && !it.keys_out;
+        L.do_rows = !L.rows_all;
+        L.do_cols = it.colkind != SADMM_COL_NONE && !L.cols_all;
+        const bool all_rows = (it.k_filters == F);
+        L.krows = all_rows ? nullptr : it.filt_idx;
+        L.nrows = all_rows ? F : it.k_filters;
+        L.R = L.do_cols ? column_parts(K, L.nrows) : 0;
+        L.cblocks = (K + 31) / 32;
+        L.fk0 = fk;
+        L.ck0 = ck;
+        L.ka0 = ka;
+        L.ka_n = std::max(L.rows_all ? F : 0, L.cols_all ? L.G : 0);
+        fk += L.do_rows ? F : 0;
+        ck += L.do_cols ? L.cblocks * L.R : 0;
+        ka += (L.ka_n + 255) / 256;
+        any_rows = any_rows || L.do_rows;
+        any_cols = any_cols || L.do_cols;
     }
-    if (!rows_all) {
-        launch_pdl(k_filter_keys<T>, dim3(F), dim3(256), 0, s, W, U, F, K, fkeys);
-        launch_select(fkeys, F, 1, k_filters, 1, 0, fkeys, keys_out, filt_idx, rkeep, s);
+    // Row keys, row selects, column keys over the kept rows, column selects:
+    // one launch each for the whole batch (the column keys read the kept-row
+    // lists, so they follow the row selects).
+    if (ka > 0) launch_pdl(k_keep_all, dim3(ka), dim3(256), 0, s, ba);
+    if (any_rows) {
+        launch_pdl(k_filter_keys<T>, dim3(fk), dim3(256), 0, s, ba);
+        launch_pdl(k_select_rows, dim3(n), dim3(kSelThreads), 0, s, ba);
     }
-    if (colkind != SADMM_COL_NONE && !cols_all) {
-        const bool all_rows = (k_filters == F);
-        const int nrows = all_rows ? F : k_filters;
-        const int R = column_parts(K, nrows);
-        launch_pdl(k_column_keys<T>, dim3((K + 31) / 32, R), dim3(256), 0, s, W, U, K,
-                   all_rows ? nullptr : filt_idx, nrows, parts);
-        launch_select(parts, G, taps, k_cols, R, K, ckeys, keys_out ? keys_out + F : nullptr, col_idx, ckeep, s);
+    if (any_cols) {
+        launch_pdl(k_column_keys<T>, dim3(ck), dim3(256), 0, s, ba);
+        launch_pdl(k_select_cols, dim3(n), dim3(kSelThreads), 0, s, ba);
     }
     return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
 }
@@ -340,15 +439,32 @@ size_t project_workspace_bytes(const Geometry& g, int colkind)
     return (size_t)(round_up(g.f, 32) + round_up(g.k, 32) + parts) * sizeof(double) + 256;
 }
 
+sadmm_status launch_project_batch(const ProjItem* items, int n, int wdt, cudaStream_t s)
+{
+    if (n < 1 || n > kMaxBatch) return SADMM_EINVAL;
+    if (wdt == SADMM_BF16) return run_project_batch<__nv_bfloat16>(items, n, s);
+    return run_project_batch<float>(items, n, s);
+}
+
 sadmm_status launch_project(const Geometry& g, const void* W, const void* U, int wdt, int k_filters,
                             int colkind, int k_cols, int* filt_idx, int* col_idx, double* keys_out,
                             void* ws, cudaStream_t s, uint8_t* rkeep, uint8_t* ckeep)
 {
-    if (wdt == SADMM_BF16)
-        return run_project<__nv_bfloat16>(g, (const __nv_bfloat16*)W, (const __nv_bfloat16*)U, k_filters,
-                                          colkind, k_cols, filt_idx, col_idx, keys_out, ws, rkeep, ckeep, s);
-    return run_project<float>(g, (const float*)W, (const float*)U, k_filters, colkind, k_cols, filt_idx,
-                              col_idx, keys_out, ws, rkeep, ckeep, s);
+    ProjItem it;
+    it.g = g;
+    it.W = W;
+    it.U = U;
+    it.Z = nullptr;
+    it.k_filters = k_filters;
+    it.colkind = colkind;
+    it.k_cols = k_cols;
+    it.filt_idx = filt_idx;
+    it.col_idx = col_idx;
+    it.keys_out = keys_out;
+    it.ws = ws;
+    it.rkeep = rkeep;
+    it.ckeep = ckeep;
+    return launch_project_batch(&it, 1, wdt, s);
 }
 
 // ---------------------------------------------------------------------------

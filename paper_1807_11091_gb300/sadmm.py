@@ -36,6 +36,25 @@ class ConvDesc(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int) for n in DESC_FIELDS]
 
 
+class ProjectItem(ctypes.Structure):
+    """sadmm_project_item: one layer of sadmm_project_groups_batch."""
+    _fields_ = [("desc", ConvDesc), ("W", ctypes.c_void_p), ("U", ctypes.c_void_p),
+                ("k_filters", ctypes.c_int), ("colkind", ctypes.c_int), ("k_cols", ctypes.c_int),
+                ("filt_idx", ctypes.c_void_p), ("col_idx", ctypes.c_void_p), ("keys_out", ctypes.c_void_p),
+                ("workspace", ctypes.c_void_p), ("ws_bytes", ctypes.c_size_t)]
+
+
+class AdmmItem(ctypes.Structure):
+    """sadmm_admm_item: one layer of sadmm_admm_update_batch."""
+    _fields_ = [("desc", ConvDesc), ("W", ctypes.c_void_p), ("U", ctypes.c_void_p), ("Z", ctypes.c_void_p),
+                ("k_filters", ctypes.c_int), ("colkind", ctypes.c_int), ("k_cols", ctypes.c_int),
+                ("filt_idx", ctypes.c_void_p), ("col_idx", ctypes.c_void_p), ("keys_out", ctypes.c_void_p),
+                ("workspace", ctypes.c_void_p), ("ws_bytes", ctypes.c_size_t)]
+
+
+SADMM_MAX_BATCH = 64  # include/sadmm.h
+
+
 class Plan(ctypes.Structure):
     _fields_ = [
         ("desc", ConvDesc),
@@ -137,6 +156,10 @@ def load():
     lib.sadmm_gemm_bf16.argtypes = [vp, vp, vp, ll, ll, ll, ll, ci, vp]
     lib.sadmm_last_device_status.restype = ci
     lib.sadmm_last_device_status.argtypes = [vp]
+    lib.sadmm_project_groups_batch.restype = ci
+    lib.sadmm_project_groups_batch.argtypes = [P(ProjectItem), ci, ci, vp]
+    lib.sadmm_admm_update_batch.restype = ci
+    lib.sadmm_admm_update_batch.argtypes = [P(AdmmItem), ci, ci, vp]
     lib.sadmm_sparse_plan_size.restype = sz
     lib.sadmm_sparse_plan_size.argtypes = [P(ConvDesc), ll]
     lib.sadmm_sparse_pack.restype = ci
@@ -287,6 +310,16 @@ def sadmm_last_device_status(stream: Optional[int]) -> int:
     return load().sadmm_last_device_status(stream)
 
 
+def sadmm_project_groups_batch(items: Sequence[ProjectItem], wdt: int, stream: Optional[int]) -> int:
+    arr = (ProjectItem * len(items))(*items)
+    return load().sadmm_project_groups_batch(arr, len(items), int(wdt), stream)
+
+
+def sadmm_admm_update_batch(items: Sequence[AdmmItem], wdt: int, stream: Optional[int]) -> int:
+    arr = (AdmmItem * len(items))(*items)
+    return load().sadmm_admm_update_batch(arr, len(items), int(wdt), stream)
+
+
 def sadmm_sparse_plan_size(desc: ConvDesc, capacity: int) -> int:
     return load().sadmm_sparse_plan_size(ctypes.byref(desc), int(capacity))
 
@@ -385,6 +418,75 @@ def admm_update_elements(desc16: Sequence[int], W, U, Z, k_elems: int, stream=No
     _check(st, "sadmm_admm_update_elements")
 
 
+class ProjectBatch:
+    """Repeated sadmm_project_groups_batch calls over fixed layers: the index
+    lists, keys and workspaces are allocated once and the item array is built
+    once, so a call is one C entry point and nothing else."""
+
+    def __init__(self, layers, with_keys: bool = False):
+        """layers: (desc16, W, k_filters, colkind, k_cols, U or None) per layer."""
+        torch = _torch()
+        items, self.outs, self._keep = [], [], []
+        self.wdt = None
+        for desc16, W, k_filters, colkind, k_cols, U in layers:
+            desc = make_desc(desc16)
+            dev = W.device
+            self.wdt = _wdt(W) if self.wdt is None else self.wdt
+            ws_bytes = sadmm_workspace_size(desc, colkind)
+            if ws_bytes == 0:
+                raise SadmmError(SADMM_EINVAL, "sadmm_workspace_size")
+            ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+            f = int(desc16[5])
+            cg = int(desc16[1]) // int(desc16[6])
+            taps = int(desc16[7]) * int(desc16[8]) * int(desc16[9])
+            G = 0 if colkind == SADMM_COL_NONE else (cg * taps if colkind == SADMM_COL_SHAPE else cg)
+            fi = torch.empty(max(k_filters, 1), dtype=torch.int32, device=dev)
+            ci = torch.empty(max(k_cols, 1), dtype=torch.int32, device=dev) if colkind != SADMM_COL_NONE else None
+            keys = torch.empty(f + G, dtype=torch.float64, device=dev) if with_keys else None
+            items.append(ProjectItem(desc, _ptr(W), _ptr(U), int(k_filters), int(colkind), int(k_cols), _ptr(fi),
+                                     _ptr(ci), _ptr(keys), _ptr(ws), ws_bytes))
+            self._keep += [W, U, ws]
+            self.outs.append((fi[:k_filters], ci[:k_cols] if ci is not None else None, keys))
+        self.n = len(items)
+        self.arr = (ProjectItem * self.n)(*items)
+
+    def __call__(self, stream=None):
+        """Projects every layer; returns [(filt_idx, col_idx, keys or None)]."""
+        _check(load().sadmm_project_groups_batch(self.arr, self.n, int(self.wdt), _stream(stream)),
+               "sadmm_project_groups_batch")
+        return self.outs
+
+
+def project_groups_batch(layers, with_keys: bool = False, stream=None):
+    """Runs sadmm_project_groups_batch over layers given as (desc16, W,
+    k_filters, colkind, k_cols, U or None); returns [(filt_idx, col_idx, keys
+    or None)] per layer, device tensors."""
+    torch = _torch()
+    items, outs, keep = [], [], []
+    wdt = None
+    for desc16, W, k_filters, colkind, k_cols, U in layers:
+        desc = make_desc(desc16)
+        dev = W.device
+        wdt = _wdt(W) if wdt is None else wdt
+        ws_bytes = sadmm_workspace_size(desc, colkind)
+        if ws_bytes == 0:
+            raise SadmmError(SADMM_EINVAL, "sadmm_workspace_size")
+        ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+        f = int(desc16[5])
+        cg = int(desc16[1]) // int(desc16[6])
+        taps = int(desc16[7]) * int(desc16[8]) * int(desc16[9])
+        G = 0 if colkind == SADMM_COL_NONE else (cg * taps if colkind == SADMM_COL_SHAPE else cg)
+        fi = torch.empty(max(k_filters, 1), dtype=torch.int32, device=dev)
+        ci = torch.empty(max(k_cols, 1), dtype=torch.int32, device=dev) if colkind != SADMM_COL_NONE else None
+        keys = torch.empty(f + G, dtype=torch.float64, device=dev) if with_keys else None
+        items.append(ProjectItem(desc, _ptr(W), _ptr(U), int(k_filters), int(colkind), int(k_cols), _ptr(fi),
+                                 _ptr(ci), _ptr(keys), _ptr(ws), ws_bytes))
+        keep.append(ws)
+        outs.append((fi[:k_filters], ci[:k_cols] if ci is not None else None, keys))
+    _check(sadmm_project_groups_batch(items, wdt, _stream(stream)), "sadmm_project_groups_batch")
+    return outs
+
+
 class AdmmStep:
     """Device buffers for repeated sadmm_admm_update calls on one layer: the
     kept index lists, the optional keys and the workspace."""
@@ -416,6 +518,37 @@ class AdmmStep:
         _check(st, "sadmm_admm_update")
         ci = self.col_idx[:self.k_cols] if self.col_idx is not None else None
         return self.filt_idx[:self.k_filters], ci
+
+
+class AdmmBatch:
+    """Repeated sadmm_admm_update_batch calls over a list of layers: one
+    AdmmStep's buffers per layer, one call for all of them."""
+
+    def __init__(self, layers, device, with_keys: bool = False):
+        """layers: (desc16, k_filters, colkind, k_cols) per layer."""
+        self.steps = [AdmmStep(d, kf, ck, kc, device, with_keys=with_keys) for d, kf, ck, kc in layers]
+
+    def __call__(self, Ws, Us, Zs, stream=None):
+        """Z_l <- Proj_S(W_l + U_l); U_l <- (W_l + U_l) - Z_l for every layer.
+        Returns [(filt_idx, col_idx)] per layer.  The item array is built once
+        per set of tensor addresses."""
+        key = tuple(_ptr(t) for t in list(Ws) + list(Us) + list(Zs))
+        if getattr(self, "_key", None) != key:
+            items = []
+            for st, W, U, Z in zip(self.steps, Ws, Us, Zs):
+                items.append(AdmmItem(st.desc, _ptr(W), _ptr(U), _ptr(Z), st.k_filters, st.colkind, st.k_cols,
+                                      _ptr(st.filt_idx), _ptr(st.col_idx), _ptr(st.keys), _ptr(st.workspace),
+                                      st.ws_bytes))
+            self._arr = (AdmmItem * len(items))(*items)
+            self._wdt = _wdt(Ws[0])
+            self._key = key
+        _check(load().sadmm_admm_update_batch(self._arr, len(self.steps), int(self._wdt), _stream(stream)),
+               "sadmm_admm_update_batch")
+        out = []
+        for st in self.steps:
+            ci = st.col_idx[:st.k_cols] if st.col_idx is not None else None
+            out.append((st.filt_idx[:st.k_filters], ci))
+        return out
 
 
 class PrunedConv:

@@ -1,0 +1,98 @@
+"""GPU checks of the batched projection and ADMM update: sadmm_project_groups_batch
+and sadmm_admm_update_batch over a list of layers give, bit for bit, what one
+call per layer gives (index lists, keys, Z and U), for batches that mix layer
+shapes, column kinds, kinds kept whole and requested keys.  The per-layer calls
+are themselves checked against the oracle in test_gpu_project.py and
+test_gpu_admm.py; the batched ADMM update is also checked against the oracle
+directly on AlexNet CONV1-5."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+
+def _layers(name):
+    if name == "alexnet":
+        return wl.alexnet()
+    if name == "resnet50":
+        return wl.resnet50()
+    # a mix: shape-wise, channel-wise, filters only, kept whole, 3-D
+    return [wl.alexnet()[2], wl.resnet50()[3], wl.c3d()[0], wl.single2d()[0],
+            wl.Layer("filters_only", wl.alexnet()[4].shape, 0.3, wl.COL_NONE, 1.0, seed=3),
+            wl.Layer("whole", wl.alexnet()[3].shape, 1.0, wl.COL_SHAPE, 1.0, seed=4)]
+
+
+@pytest.mark.parametrize("name", ["alexnet", "resnet50", "mixed"])
+@pytest.mark.parametrize("with_keys", [False, True])
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_batched_projection_equals_per_layer_calls(name, with_keys, dtype):
+    from paper_1807_11091_gb300 import sadmm
+    layers = _layers(name)
+    dev = torch.device("cuda", 0)
+    Ws = [wl.gen_tensors(L.shape.with_batch(1), seed=L.seed)["W"].to(dtype).to(dev) for L in layers]
+    args = [(L.shape.desc16(), W, L.k_filters, L.colkind, L.k_cols, None) for L, W in zip(layers, Ws)]
+    got = sadmm.project_groups_batch(args, with_keys=with_keys)
+    for (d, W, kf, ck, kc, U), (fi, ci, keys) in zip(args, got):
+        fi1, ci1, keys1 = sadmm.project_groups(d, W, kf, ck, kc, with_keys=with_keys)
+        assert torch.equal(fi, fi1)
+        assert (ci is None) == (ci1 is None) and (ci is None or torch.equal(ci, ci1))
+        if with_keys:
+            assert torch.equal(keys, keys1)
+    assert sadmm.device_status() == 0
+
+
+def _bits(t):
+    return t.view(torch.int16 if t.dtype == torch.bfloat16 else torch.int32)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_batched_admm_update_equals_per_layer_and_oracle(dtype):
+    from paper_1807_11091_gb300 import sadmm
+    layers = _layers("alexnet") + [wl.resnet50()[15]]
+    dev = torch.device("cuda", 0)
+    states = [wl.gen_admm_state(L.shape, L.seed) for L in layers]
+    W = [st["W"].to(dtype).to(dev) for st in states]
+    U0 = [st["U"].to(dtype).to(dev) for st in states]
+    spec = [(L.shape.desc16(), L.k_filters, L.colkind, L.k_cols) for L in layers]
+    batch = sadmm.AdmmBatch(spec, dev)
+    steps = [sadmm.AdmmStep(d, kf, ck, kc, dev) for d, kf, ck, kc in spec]
+    Ub = [u.clone() for u in U0]
+    Us = [u.clone() for u in U0]
+    for it in range(2):  # twice in a row: the second update starts from the first one's U
+        Zb = [torch.full_like(w, float("nan")) for w in W]
+        Zs = [torch.full_like(w, float("nan")) for w in W]
+        outs = batch(W, Ub, Zb)
+        for step, w, u, z, (fi, ci) in zip(steps, W, Us, Zs, outs):
+            fi1, ci1 = step(w, u, z)
+            assert torch.equal(fi, fi1) and ((ci is None and ci1 is None) or torch.equal(ci, ci1))
+        for ub, zb, us, zs in zip(Ub, Zb, Us, Zs):
+            assert torch.equal(_bits(ub), _bits(us)) and torch.equal(_bits(zb), _bits(zs))
+        if it == 0:
+            # the first update against the oracle
+            for L, st, (fi, ci), ub, zb in zip(layers, states, outs, Ub, Zb):
+                s = L.shape
+                rows, cols, Zo, Uo = oracle.admm_update(st["W"].to(dtype), st["U"].to(dtype), s.taps, L.k_filters,
+                                                        L.colkind, L.k_cols)
+                assert np.array_equal(fi.cpu().numpy(), rows)
+                if ci is not None:
+                    assert np.array_equal(ci.cpu().numpy(), cols)
+                assert torch.equal(_bits(zb.cpu()), _bits(Zo.reshape(zb.shape)))
+                assert torch.equal(_bits(ub.cpu()), _bits(Uo.reshape(ub.shape)))
+    assert sadmm.device_status() == 0
+
+
+def test_batch_rejects_bad_items():
+    from paper_1807_11091_gb300 import sadmm
+    L = wl.alexnet()[2]
+    dev = torch.device("cuda", 0)
+    W = wl.gen_tensors(L.shape.with_batch(1), seed=L.seed)["W"].to(dev)
+    good = (L.shape.desc16(), W, L.k_filters, L.colkind, L.k_cols, None)
+    bad = (L.shape.desc16(), W, L.shape.f + 1, L.colkind, L.k_cols, None)
+    with pytest.raises(sadmm.SadmmError):
+        sadmm.project_groups_batch([good, bad])
+    with pytest.raises(sadmm.SadmmError):
+        sadmm.project_groups_batch([good] * (sadmm.SADMM_MAX_BATCH + 1))
