@@ -31,20 +31,97 @@ namespace sadmm {
 namespace {
 
 template <typename T>
-SADMM_DEV double to_f64(T v);
+SADMM_DEV float to_f32(T v);
 template <>
-SADMM_DEV double to_f64<__nv_bfloat16>(__nv_bfloat16 v) { return (double)__bfloat162float(v); }
+SADMM_DEV float to_f32<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
 template <>
-SADMM_DEV double to_f64<float>(float v) { return (double)v; }
+SADMM_DEV float to_f32<float>(float v) { return v; }
 
-// V = W (+U) element, exactly in fp64.
-template <typename T>
-SADMM_DEV double v_elem(const T* __restrict__ W, const T* __restrict__ U, long long i)
+// A sum of squares V_e^2 kept on the fp32 pipe (fp64 arithmetic is slow on
+// this GPU) without losing precision: V = W (+U) is formed as an exact pair
+// s + err (TwoSum), its square as p + e with p = s*s and
+// e = fma(s, s, -p) + 2*s*err (exact up to err^2 <= 2^-48 V^2); the running
+// sum hi collects p, each addition's exact rounding error (TwoSum) goes to lo
+// with e, and every 8 terms the pair is renormalised (hi + lo exactly, lo below
+// half an ulp of hi).  The lo additions between renormalisations bound the
+// relative error of a thread's sum by about 8^2 * 2^-48 = 2^-42; pair merges
+// across threads add about 2^-47 each.  Elements with |s| outside
+// [2^-40, 2^40] (whose squares or residuals could leave fp32's normal range)
+// are squared and added in fp64 (d) instead.
+SADMM_DEV void two_sum(float a, float b, float& s, float& e)
 {
-    double v = to_f64<T>(W[i]);
-    if (U) v += to_f64<T>(U[i]);
-    return v;
+    s = a + b;
+    const float bb = s - a;
+    e = (a - (s - bb)) + (b - bb);
 }
+
+struct SqSum {
+    float hi, lo;
+    double d;
+    int n;
+    SADMM_DEV void init()
+    {
+        hi = lo = 0.0f;
+        d = 0.0;
+        n = 0;
+    }
+    SADMM_DEV void renorm()
+    {
+        const float t = hi + lo;
+        lo = lo - (t - hi);
+        hi = t;
+    }
+    template <typename T>
+    SADMM_DEV void add(const T* __restrict__ W, const T* __restrict__ U, long long i)
+    {
+        const float w = to_f32<T>(W[i]);
+        float sv = w, err = 0.0f, u = 0.0f;
+        if (U) {
+            u = to_f32<T>(U[i]);
+            two_sum(w, u, sv, err);
+        }
+        const float as = fabsf(sv);
+        if (as >= 0x1p-40f && as <= 0x1p40f) {
+            const float p = sv * sv;
+            const float e = fmaf(sv, sv, -p) + 2.0f * sv * err;
+            float t, te;
+            two_sum(hi, p, t, te);
+            lo += te + e;
+            hi = t;
+            if (++n == 8) {
+                renorm();
+                n = 0;
+            }
+        } else if (sv != 0.0f || err != 0.0f) {
+            const double v = (double)w + (double)u;
+            d = fma(v, v, d);
+        }
+    }
+    // adds another sum given as its pair (and fp64 part)
+    SADMM_DEV void merge(float ohi, float olo, double od)
+    {
+        float t, te;
+        two_sum(hi, ohi, t, te);
+        lo += olo + te;
+        hi = t;
+        renorm();
+        d += od;
+    }
+    // the warp's sums merged into lane 0 in a fixed order (lane 0's result
+    // is the warp total; d is reduced only when some lane has an fp64 part)
+    SADMM_DEV void warp_reduce()
+    {
+        renorm();
+        const bool any_d = __any_sync(0xffffffffu, d != 0.0);
+        for (int o = 16; o > 0; o >>= 1) {
+            const float oh = __shfl_down_sync(0xffffffffu, hi, o);
+            const float ol = __shfl_down_sync(0xffffffffu, lo, o);
+            const double od = any_d ? __shfl_down_sync(0xffffffffu, d, o) : 0.0;
+            merge(oh, ol, od);
+        }
+    }
+    SADMM_DEV double value() const { return ((double)hi + (double)lo) + d; }
+};
 
 // Per-layer parameters of a batched projection (kernel parameter space; a
 // block finds its layer by its first-block offsets).
@@ -94,7 +171,8 @@ template <typename T>
 __global__ void __launch_bounds__(256) k_filter_keys(const __grid_constant__ BatchArgs ba)
 {
     pdl_wait();  // after the kernel before it in the stream
-    __shared__ double part[8];
+    __shared__ float part_h[8], part_l[8];
+    __shared__ double part_d[8];
     const int l = find_layer<&BLayer::fk0>(ba, blockIdx.x);
     const BLayer& L = ba.L[l];
     const int a = blockIdx.x - L.fk0;
@@ -104,30 +182,28 @@ __global__ void __launch_bounds__(256) k_filter_keys(const __grid_constant__ Bat
     const int K = L.K;
     const int lane = threadIdx.x & 31, wy = threadIdx.x >> 5;
     const long long base = (long long)a * K;
-    // four independent partial sums per thread (loads and fp64 FMAs overlap),
-    // added in a fixed order
-    double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
+    SqSum acc;
+    acc.init();
     int k = threadIdx.x;
     for (; k + 768 < K; k += 1024) {
-        const double v0 = v_elem(W, U, base + k), v1 = v_elem(W, U, base + k + 256);
-        const double v2 = v_elem(W, U, base + k + 512), v3 = v_elem(W, U, base + k + 768);
-        s0 = fma(v0, v0, s0);
-        s1 = fma(v1, v1, s1);
-        s2 = fma(v2, v2, s2);
-        s3 = fma(v3, v3, s3);
+        acc.add(W, U, base + k);
+        acc.add(W, U, base + k + 256);
+        acc.add(W, U, base + k + 512);
+        acc.add(W, U, base + k + 768);
     }
-    for (; k < K; k += 256) {
-        const double v = v_elem(W, U, base + k);
-        s0 = fma(v, v, s0);
+    for (; k < K; k += 256) acc.add(W, U, base + k);
+    acc.warp_reduce();
+    if (lane == 0) {
+        part_h[wy] = acc.hi;
+        part_l[wy] = acc.lo;
+        part_d[wy] = acc.d;
     }
-    double s = (s0 + s1) + (s2 + s3);
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_down_sync(0xffffffffu, s, o);
-    if (lane == 0) part[wy] = s;
     __syncthreads();
     if (threadIdx.x == 0) {
-        double t = 0.0;
-        for (int q = 0; q < 8; ++q) t += part[q];
-        L.fkeys[a] = t;
+        SqSum t;
+        t.init();
+        for (int q = 0; q < 8; ++q) t.merge(part_h[q], part_l[q], part_d[q]);
+        L.fkeys[a] = t.value();
     }
 }
 
@@ -138,7 +214,8 @@ template <typename T>
 __global__ void __launch_bounds__(256) k_column_keys(const __grid_constant__ BatchArgs ba)
 {
     pdl_wait();  // after the kernel before it in the stream (the kept rows)
-    __shared__ double part[8][33];
+    __shared__ float part_h[8][33], part_l[8][33];
+    __shared__ double part_d[8][33];
     const int l = find_layer<&BLayer::ck0>(ba, blockIdx.x);
     const BLayer& L = ba.L[l];
     const int local = blockIdx.x - L.ck0;
@@ -150,20 +227,24 @@ __global__ void __launch_bounds__(256) k_column_keys(const __grid_constant__ Bat
     const int lane = threadIdx.x & 31;
     const int wy = threadIdx.x >> 5;
     const int j = bx * 32 + lane;
-    double s = 0.0;
+    SqSum acc;
+    acc.init();
     if (j < K) {
         for (int r = by + R * wy; r < L.nrows; r += 8 * R) {
             const int a = L.krows ? L.krows[r] : r;
-            const double v = v_elem(W, U, (long long)a * K + j);
-            s = fma(v, v, s);
+            acc.add(W, U, (long long)a * K + j);
         }
     }
-    part[wy][lane] = s;
+    acc.renorm();
+    part_h[wy][lane] = acc.hi;
+    part_l[wy][lane] = acc.lo;
+    part_d[wy][lane] = acc.d;
     __syncthreads();
     if (wy == 0 && j < K) {
-        double t = 0.0;
-        for (int q = 0; q < 8; ++q) t += part[q][lane];
-        L.parts[(long long)by * K + j] = t;
+        SqSum t;
+        t.init();
+        for (int q = 0; q < 8; ++q) t.merge(part_h[q][lane], part_l[q][lane], part_d[q][lane]);
+        L.parts[(long long)by * K + j] = t.value();
     }
 }
 

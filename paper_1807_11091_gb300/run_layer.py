@@ -37,7 +37,16 @@ def main(argv=None) -> int:
     ap.add_argument("--elements", type=float, default=0.0,
                     help="time the non-structured ADMM update keeping this fraction of the weights")
     ap.add_argument("--backward", action="store_true", help="time sadmm_conv_bwd (dW, db, dx) after one forward")
+    ap.add_argument("--batch-all", action="store_true",
+                    help="with --admm: one sadmm_admm_update_batch over every layer of the workload; alone: one "
+                         "sadmm_project_groups_batch over every layer (bf16 W)")
+    ap.add_argument("--sparse", type=float, default=0.0,
+                    help="time sadmm_sparse_conv_fwd with the layer pruned element by element to this density")
     args = ap.parse_args(argv)
+    if args.batch_all:
+        return run_batch_all(args)
+    if args.sparse > 0:
+        return run_sparse(args)
     if args.admm:
         return run_admm(args)
     if args.elements > 0:
@@ -118,6 +127,77 @@ def run_elements(args) -> int:
         ms = e0.elapsed_time(e1)
         print(f"{L.name} elements {args.elements} run {i}: {ms * 1e3:.1f} us  {nbytes / ms / 1e6:.1f} GB/s "
               "(16 B per weight)")
+    return 1 if sadmm.device_status() != 0 else 0
+
+
+def run_batch_all(args) -> int:
+    """One batched projection (or, with --admm, ADMM update on fp32 state) of
+    every layer of the workload, `reps` times."""
+    import torch
+
+    import workloads as wl
+    from paper_1807_11091_gb300 import sadmm
+
+    layers = wl.get(args.workload)
+    dev = torch.device("cuda", 0)
+    if args.admm:
+        states = [wl.gen_admm_state(L.shape, L.seed) for L in layers]
+        Ws = [st["W"].to(dev) for st in states]
+        Us = [st["U"].to(dev) for st in states]
+        Zs = [torch.empty_like(w) for w in Ws]
+        batch = sadmm.AdmmBatch([(L.shape.desc16(), L.k_filters, L.colkind, L.k_cols) for L in layers], dev)
+        fn = lambda: batch(Ws, Us, Zs)  # noqa: E731
+        what = "admm batch"
+    else:
+        Ws = [wl.gen_tensors(L.shape.with_batch(1), seed=L.seed)["W"].to(dev) for L in layers]
+        pb = sadmm.ProjectBatch([(L.shape.desc16(), W, L.k_filters, L.colkind, L.k_cols, None)
+                                 for L, W in zip(layers, Ws)])
+        fn = pb
+        what = "projection batch"
+    for i in range(args.reps):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        torch.cuda._sleep(1_000_000)
+        e0.record()
+        fn()
+        e1.record()
+        torch.cuda.synchronize()
+        print(f"{args.workload} {what} of {len(layers)} layers run {i}: {e0.elapsed_time(e1) * 1e3:.1f} us")
+    return 1 if sadmm.device_status() != 0 else 0
+
+
+def run_sparse(args) -> int:
+    """sadmm_sparse_conv_fwd `reps` times with the layer pruned element by
+    element (sadmm_project_elements keeps the largest |W|)."""
+    import torch
+
+    import workloads as wl
+    from paper_1807_11091_gb300 import sadmm
+
+    L = wl.get(args.workload)[args.layer]
+    s = L.shape if args.batch == 0 else L.shape.with_batch(args.batch)
+    t = wl.gen_tensors(s, seed=L.seed, device="cuda")
+    k = wl.retained(args.sparse, s.f * s.k)
+    keep = sadmm.project_elements(s.desc16(), t["W"], k)
+    desc = sadmm.make_desc(s.desc16())
+    nbytes = sadmm.sadmm_sparse_plan_size(desc, k)
+    plan = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    sp = int(torch.cuda.current_stream().cuda_stream)
+    assert sadmm.sadmm_sparse_pack(desc, t["W"].data_ptr(), sadmm.SADMM_BF16, keep.data_ptr(), k, plan.data_ptr(),
+                                   nbytes, sp) == 0
+    y = torch.empty(s.y_shape(), dtype=torch.float32, device="cuda")
+    for i in range(args.reps):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        torch.cuda._sleep(200_000)
+        e0.record()
+        assert sadmm.sadmm_sparse_conv_fwd(desc, plan.data_ptr(), t["x"].data_ptr(), t["bias"].data_ptr(), 1,
+                                           y.data_ptr(), sadmm.SADMM_FP32, sp) == 0
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        print(f"{L.name} N={s.n} sparse {args.sparse} run {i}: {ms * 1e3:.1f} us  "
+              f"{2.0 * s.m * k / ms / 1e9:.2f} TFLOP/s")
     return 1 if sadmm.device_status() != 0 else 0
 
 
