@@ -204,12 +204,13 @@ class LayerRun:
         ytype = torch.bfloat16 if out_dtype == "bf16" else torch.float32
         self.y = torch.empty(s.y_shape(), dtype=ytype, device=dev)
         self.out_bytes = 2 if out_dtype == "bf16" else 4
-        # projection (keys + select per kind, one launch for the kinds kept whole),
-        # pack (meta + rows, the slab-ordered rows in the same launch), conv (+ split-K
-        # finalize, or after the input-slab path's space-to-depth pass)
+        # projection (filter keys, whose launch also writes the lists of kinds kept
+        # whole; the row select; column keys + select), pack (meta + rows, the
+        # slab-ordered rows in the same launch), conv (+ split-K finalize, or after
+        # the input-slab path's space-to-depth pass)
         rows_all = self.k_filters == s.f
         cols_all = self.colkind != wl.COL_NONE and self.k_cols == G
-        self.launches = ((1 if rows_all or cols_all else 0) + (0 if rows_all else 2)
+        self.launches = (1 + (0 if rows_all else 1)
                          + (2 if self.colkind != wl.COL_NONE and not cols_all else 0) + 2
                          + (2 if self.plan.splits > 1 or self.plan.xs_mode else 1))
 

@@ -146,6 +146,7 @@ struct BLayer {
 
 struct BatchArgs {
     int n;
+    int fk_total;  // blocks of the filter-key pass; the keep-all blocks follow them
     BLayer L[kMaxBatch];
 };
 
@@ -164,13 +165,36 @@ SADMM_DEV int find_layer(const BatchArgs& a, int b)
     return lo;
 }
 
+// Index lists 0..n-1 and keep flags of one for the kinds kept whole: block b
+// of the keep-all range.
+SADMM_DEV void keep_all_block(const BatchArgs& ba, int b)
+{
+    const int l = find_layer<&BLayer::ka0>(ba, b);
+    const BLayer& L = ba.L[l];
+    const int i = (b - L.ka0) * 256 + threadIdx.x;
+    if (i >= L.ka_n) return;
+    if (L.rows_all && i < L.F) {
+        L.filt_idx[i] = i;
+        if (L.rkeep) L.rkeep[i] = 1;
+    }
+    if (L.cols_all && i < L.G) {
+        L.col_idx[i] = i;
+        if (L.ckeep) L.ckeep[i] = 1;
+    }
+}
+
 // O_a = sum_k V[a,k]^2 for every row a (filter-wise groups): one block per
-// row of every layer that needs them, strided fp64 partial sums, fixed-order
-// block reduction.
+// row of every layer that needs them, a sum of squares per thread (SqSum),
+// fixed-order warp and block merges.  Blocks past the filter-key range write
+// the index lists of the kinds kept whole.
 template <typename T>
 __global__ void __launch_bounds__(256) k_filter_keys(const __grid_constant__ BatchArgs ba)
 {
     pdl_wait();  // after the kernel before it in the stream
+    if ((int)blockIdx.x >= ba.fk_total) {
+        keep_all_block(ba, (int)blockIdx.x - ba.fk_total);
+        return;
+    }
     __shared__ float part_h[8], part_l[8];
     __shared__ double part_d[8];
     const int l = find_layer<&BLayer::fk0>(ba, blockIdx.x);
@@ -424,24 +448,6 @@ int column_parts(long long K, long long nrows)
     return (int)std::max(r, 1ll);
 }
 
-// Index lists 0..n-1 and keep flags of one for the kinds kept whole.
-__global__ void __launch_bounds__(256) k_keep_all(const __grid_constant__ BatchArgs ba)
-{
-    pdl_wait();  // after the kernel before it in the stream
-    const int l = find_layer<&BLayer::ka0>(ba, blockIdx.x);
-    const BLayer& L = ba.L[l];
-    const int i = (blockIdx.x - L.ka0) * 256 + threadIdx.x;
-    if (i >= L.ka_n) return;
-    if (L.rows_all && i < L.F) {
-        L.filt_idx[i] = i;
-        if (L.rkeep) L.rkeep[i] = 1;
-    }
-    if (L.cols_all && i < L.G) {
-        L.col_idx[i] = i;
-        if (L.ckeep) L.ckeep[i] = 1;
-    }
-}
-
 template <typename T>
 sadmm_status run_project_batch(const ProjItem* items, int n, cudaStream_t s)
 {
@@ -494,14 +500,13 @@ sadmm_status run_project_batch(const ProjItem* items, int n, cudaStream_t s)
         any_rows = any_rows || L.do_rows;
         any_cols = any_cols || L.do_cols;
     }
-    // Row keys, row selects, column keys over the kept rows, column selects:
-    // one launch each for the whole batch (the column keys read the kept-row
-    // lists, so they follow the row selects).
-    if (ka > 0) launch_pdl(k_keep_all, dim3(ka), dim3(256), 0, s, ba);
-    if (any_rows) {
-        launch_pdl(k_filter_keys<T>, dim3(fk), dim3(256), 0, s, ba);
-        launch_pdl(k_select_rows, dim3(n), dim3(kSelThreads), 0, s, ba);
-    }
+    // Row keys (with the lists of the kinds kept whole), row selects, column
+    // keys over the kept rows, column selects: one launch each for the whole
+    // batch (the column keys read the kept-row lists, so they follow the row
+    // selects).
+    ba.fk_total = fk;
+    if (fk + ka > 0) launch_pdl(k_filter_keys<T>, dim3(fk + ka), dim3(256), 0, s, ba);
+    if (any_rows) launch_pdl(k_select_rows, dim3(n), dim3(kSelThreads), 0, s, ba);
     if (any_cols) {
         launch_pdl(k_column_keys<T>, dim3(ck), dim3(256), 0, s, ba);
         launch_pdl(k_select_cols, dim3(n), dim3(kSelThreads), 0, s, ba);
