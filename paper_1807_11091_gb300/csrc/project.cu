@@ -141,6 +141,7 @@ struct BLayer {
     int do_rows, do_cols;  // 1: keys and select of this kind run
     int R, cblocks, nrows;
     int fk0, ck0, ka0, ka_n;  // first block in the filter-key, column-key, keep-all grids; keep-all length
+    int rpb;                  // filter-key rows per block: 8 (a warp per row, K <= 1024) or 1
     int rows_all, cols_all;   // lists written whole by the keep-all pass
 };
 
@@ -199,12 +200,24 @@ __global__ void __launch_bounds__(256) k_filter_keys(const __grid_constant__ Bat
     __shared__ double part_d[8];
     const int l = find_layer<&BLayer::fk0>(ba, blockIdx.x);
     const BLayer& L = ba.L[l];
-    const int a = blockIdx.x - L.fk0;
-    if (!L.do_rows || a >= L.F) return;
     const T* W = static_cast<const T*>(L.W);
     const T* U = static_cast<const T*>(L.U);
     const int K = L.K;
     const int lane = threadIdx.x & 31, wy = threadIdx.x >> 5;
+    if (L.rpb == 8) {
+        // short rows: warp wy sums row 8 b + wy, lanes strided over its columns
+        const int a = (blockIdx.x - L.fk0) * 8 + wy;
+        if (!L.do_rows || a >= L.F) return;
+        const long long base = (long long)a * K;
+        SqSum acc;
+        acc.init();
+        for (int k = lane; k < K; k += 32) acc.add(W, U, base + k);
+        acc.warp_reduce();
+        if (lane == 0) L.fkeys[a] = acc.value();
+        return;
+    }
+    const int a = blockIdx.x - L.fk0;
+    if (!L.do_rows || a >= L.F) return;
     const long long base = (long long)a * K;
     SqSum acc;
     acc.init();
@@ -494,7 +507,8 @@ sadmm_status run_project_batch(const ProjItem* items, int n, cudaStream_t s)
         L.ck0 = ck;
         L.ka0 = ka;
         L.ka_n = std::max(L.rows_all ? F : 0, L.cols_all ? L.G : 0);
-        fk += L.do_rows ? F : 0;
+        L.rpb = K <= 1024 ? 8 : 1;
+        fk += L.do_rows ? (F + L.rpb - 1) / L.rpb : 0;
         ck += L.do_cols ? L.cblocks * L.R : 0;
         ka += (L.ka_n + 255) / 256;
         any_rows = any_rows || L.do_rows;
