@@ -26,8 +26,9 @@ def n_colgroups(colkind, k_cols, shape):
 
 
 def gpu_layer(shape: wl.ConvShape, t, k_filters, colkind, k_cols, relu=True, out_dtype=torch.float32,
-              use_bias=True, project=True, filt_idx=None, col_idx=None):
-    """Projection (unless index lists are given), pack and forward on cuda:0.
+              use_bias=True, project=True, filt_idx=None, col_idx=None, max_ctas=0):
+    """Projection (unless index lists are given), pack and forward on cuda:0
+    (max_ctas > 0: a plan for at most that many SMs).
     Returns (filt_idx, col_idx, y on the host, the PrunedConv)."""
     from paper_1807_11091_gb300 import sadmm
     dev = torch.device("cuda", 0)
@@ -40,7 +41,8 @@ def gpu_layer(shape: wl.ConvShape, t, k_filters, colkind, k_cols, relu=True, out
         fi_d = torch.as_tensor(np.asarray(filt_idx, dtype=np.int32), device=dev)
         ci_d = None if col_idx is None else torch.as_tensor(np.asarray(col_idx, dtype=np.int32), device=dev)
     pc = sadmm.PrunedConv(shape.desc16(), W, fi_d if k_filters < shape.f else None, colkind,
-                          ci_d if colkind != wl.COL_NONE else None, k_filters, n_colgroups(colkind, k_cols, shape))
+                          ci_d if colkind != wl.COL_NONE else None, k_filters, n_colgroups(colkind, k_cols, shape),
+                          max_ctas=max_ctas)
     y = torch.full(pc.out_shape(), float("nan"), dtype=out_dtype, device=dev)
     pc.forward(x, bias, relu=relu, out=y)
     st = sadmm.device_status()
