@@ -292,7 +292,15 @@ def enqueue_step(runs, ss, conv_events=None):
         if split and r.early_input:
             r.conv(mp, sadmm.SADMM_FWD_INPUT)
     for i, (r, done) in enumerate(zip(runs, ss.done)):
-        ss.main.wait_event(done)
+        # The later layers' packs finish beside the first conv; waiting for all
+        # of them before the second conv leaves the later convs back to back in
+        # the stream, so each is launched while the one before it drains
+        # (programmatic dependent launch; a wait between two kernels prevents it).
+        if i == 0:
+            ss.main.wait_event(done)
+        elif i == 1:
+            for d in ss.done[1:]:
+                ss.main.wait_event(d)
         if conv_events is not None:
             conv_events[i][0].record(ss.main)
         r.conv(mp, sadmm.SADMM_FWD_REST if split and r.early_input else sadmm.SADMM_FWD_ALL)
@@ -472,6 +480,37 @@ def time_steps(rs, ss, flush, k, with_conv_events):
             for i, (a, b) in enumerate(ev):
                 conv_ms[i].append(a.elapsed_time(b))
     return step_ms, conv_ms
+
+
+def calls_report(runs, flush, reps=50, warmup=10):
+    """sadmm_conv_fwd alone, per layer (the plans packed by the steps before):
+    10 warm-up calls, then the median of `reps` calls with the L2 flushed before
+    each (outside the window) and of `reps` back-to-back calls with a warm L2."""
+    import torch
+    sp = int(torch.cuda.current_stream().cuda_stream)
+    out = {}
+    for r in runs:
+        for _ in range(warmup):
+            r.conv(sp)
+        res = {}
+        for mode in ("flushed", "warm"):
+            evs = []
+            for _ in range(reps):
+                if mode == "flushed":
+                    flush.fill_(1)
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record()
+                r.conv(sp)
+                e1.record()
+                evs.append((e0, e1))
+            torch.cuda.synchronize()
+            us = statistics.median(a.elapsed_time(b) for a, b in evs) * 1e3
+            res[f"{mode}_us"] = us
+            res[f"{mode}_tflops"] = r.flops() / (us * 1e-6) / 1e12
+        out[r.L.name] = res
+    return {"what": f"sadmm_conv_fwd alone per layer: {warmup} warm-up calls, median of {reps} calls with the L2 "
+                    f"flushed before each and of {reps} back-to-back calls (warm L2)", "layers": out}
 
 
 def forward_roofline(runs, t_conv_s, peaks):
@@ -974,6 +1013,7 @@ def run_gpu(args):
     _, conv_ms = timed_steps(runs, n_aux, True)
     dense_ms, _ = timed_steps(dense, n_aux, False)
     _, dense_conv_ms = timed_steps(dense, n_aux, True)
+    calls = calls_report(runs, flush) if rank == 0 else None
 
     # end to end through the C ABI with host buffers: pinned H2D of every input,
     # the step, D2H of every output
@@ -1057,6 +1097,8 @@ def run_gpu(args):
         "gpu_launches": sum(r.launches for r in runs) * args.steps,
         "clocks": clocks.summary(),
     }
+    if calls is not None:
+        line["calls"] = calls
     if rank == 0 and not args.no_configs and args.workload == "alexnet":
         line["configs"] = configs_report(dev, args.out_dtype, peaks)
     if rank == 0 and not args.no_sweep:
