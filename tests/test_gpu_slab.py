@@ -37,6 +37,9 @@ CASES = [
      wl.COL_NONE, 1.0),
     ("wide_256_filters", ConvShape(n=2, c=3, h=40, w=41, f=256, kh=3, kw=3, sh=2, sw=2, ph=1, pw=1), 1.0,
      wl.COL_NONE, 1.0),
+    # stride 4 with padding on both sides and channel pruning
+    ("stride4_pads_channels", ConvShape(n=2, c=8, h=37, w=41, f=24, kh=7, kw=7, sh=4, sw=4, ph=2, pw=3), 1.0,
+     wl.COL_CHANNEL, 0.5),
 ]
 
 
@@ -95,6 +98,24 @@ def test_slab_repeated_launches_identical():
     y2 = torch.full(pc.out_shape(), float("nan"), device=dev)
     pc.forward(other, bias, out=y2)
     pc.forward(x, bias, out=y2)
+    assert sadmm.device_status() == 0
+    assert np.array_equal(y2.cpu().numpy(), y)
+
+
+@pytest.mark.parametrize("case", [CASES[0], CASES[-1]], ids=lambda c: c[0])
+def test_slab_input_off_the_16_byte_grid(case):
+    """x 2-byte aligned only (a view one element into a buffer, which the ABI
+    allows): the output equals the aligned call's bit for bit."""
+    s, t, rows, ck, cols, y, pc = _run(case, seed=309)
+    dev = torch.device("cuda", 0)
+    x = t["x"].to(dev)
+    big = torch.empty(x.numel() + 1, dtype=torch.bfloat16, device=dev)
+    big[1:].copy_(x.reshape(-1))
+    x_off = big[1:].view(x.shape)
+    assert x_off.data_ptr() % 16 == 2
+    y2 = torch.full(pc.out_shape(), float("nan"), device=dev)
+    pc.forward(x_off, t["bias"].to(dev), out=y2)
+    from paper_1807_11091_gb300 import sadmm
     assert sadmm.device_status() == 0
     assert np.array_equal(y2.cpu().numpy(), y)
 
