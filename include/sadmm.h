@@ -412,7 +412,8 @@ sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt,
  * x outside the input reads as zero.  bf16 x bf16 products accumulate in fp32
  * (tcgen05 MMA, TMEM accumulator).
  *
- *   x     device bf16 [N][C][T][H][W]; 16-byte aligned.
+ *   x     device bf16 [N][C][T][H][W]; element (2-byte) aligned (SADMM_EINVAL
+ *         otherwise): the kernels read x one element at a time.
  *   bias  device fp32 [F] or NULL (zero).
  *   relu  nonzero: apply ReLU.
  *   y     device [N][F][OT][OH][OW] of dtype `ydt` (fp32 or bf16, rounded
