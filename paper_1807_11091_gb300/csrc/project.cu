@@ -5,8 +5,9 @@
 // Every launch serves a batch of layers (a single call is a batch of one):
 // the layers' parameters travel in kernel parameter space, and a block finds
 // its layer by its index.
-//   k_filter_keys   one block per GEMM row (filter): fp64 sums of squares in
-//                   four independent partials per thread, warp-shuffle and
+//   k_filter_keys   one block per GEMM row (filter), or a warp per row for
+//                   rows of at most 1024 columns: error-free fp32 pair sums of
+//                   squares (SqSum) over 16-byte loads, warp-shuffle and
 //                   fixed-order block reduction.
 //   k_column_keys   32 columns per block, 8 warps over the (kept) rows, fixed
 //                   order shared-memory reduction: one key per GEMM column.
@@ -74,12 +75,13 @@ struct SqSum {
     template <typename T>
     SADMM_DEV void add(const T* __restrict__ W, const T* __restrict__ U, long long i)
     {
-        const float w = to_f32<T>(W[i]);
-        float sv = w, err = 0.0f, u = 0.0f;
-        if (U) {
-            u = to_f32<T>(U[i]);
-            two_sum(w, u, sv, err);
-        }
+        add_f(to_f32<T>(W[i]), U ? to_f32<T>(U[i]) : 0.0f, U != nullptr);
+    }
+    // adds V^2 for V = w (+ u when has_u)
+    SADMM_DEV void add_f(float w, float u, bool has_u)
+    {
+        float sv = w, err = 0.0f;
+        if (has_u) two_sum(w, u, sv, err);
         const float as = fabsf(sv);
         if (as >= 0x1p-40f && as <= 0x1p40f) {
             const float p = sv * sv;
@@ -122,6 +124,44 @@ struct SqSum {
     }
     SADMM_DEV double value() const { return ((double)hi + (double)lo) + d; }
 };
+
+// Eight consecutive elements as fp32, from a 16-byte aligned address.
+SADMM_DEV void load8(const __nv_bfloat16* p, float (&v)[8])
+{
+    const uint4 q = __ldg(reinterpret_cast<const uint4*>(p));
+    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        v[2 * i] = __uint_as_float(w[i] << 16);
+        v[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+    }
+}
+SADMM_DEV void load8(const float* p, float (&v)[8])
+{
+    const float4 a = __ldg(reinterpret_cast<const float4*>(p));
+    const float4 b = __ldg(reinterpret_cast<const float4*>(p) + 1);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+
+// Adds the squares of a row's K elements: thread t of nt takes the 8-element
+// runs t, t + nt, ... with 16-byte loads when the row (of W, and of U) starts
+// 16-byte aligned, then the last K % 8 elements one by one (K8 + t, ...);
+// every element one by one when the row is not aligned.
+template <typename T>
+SADMM_DEV void add_row(SqSum& acc, const T* __restrict__ Wr, const T* __restrict__ Ur, int K, int t, int nt)
+{
+    const bool vec = ((reinterpret_cast<uintptr_t>(Wr) | reinterpret_cast<uintptr_t>(Ur)) & 15) == 0;
+    const int K8 = vec ? (K & ~7) : 0;
+    for (int k = t * 8; k < K8; k += nt * 8) {
+        float w[8], u[8];
+        load8(Wr + k, w);
+        if (Ur) load8(Ur + k, u);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc.add_f(w[e], Ur ? u[e] : 0.0f, Ur != nullptr);
+    }
+    for (int k = K8 + t; k < K; k += nt) acc.add(Wr, Ur, k);
+}
 
 // Per-layer parameters of a batched projection (kernel parameter space; a
 // block finds its layer by its first-block offsets).
@@ -211,7 +251,7 @@ __global__ void __launch_bounds__(256) k_filter_keys(const __grid_constant__ Bat
         const long long base = (long long)a * K;
         SqSum acc;
         acc.init();
-        for (int k = lane; k < K; k += 32) acc.add(W, U, base + k);
+        add_row(acc, W + base, U ? U + base : nullptr, K, lane, 32);
         acc.warp_reduce();
         if (lane == 0) L.fkeys[a] = acc.value();
         return;
@@ -221,14 +261,7 @@ __global__ void __launch_bounds__(256) k_filter_keys(const __grid_constant__ Bat
     const long long base = (long long)a * K;
     SqSum acc;
     acc.init();
-    int k = threadIdx.x;
-    for (; k + 768 < K; k += 1024) {
-        acc.add(W, U, base + k);
-        acc.add(W, U, base + k + 256);
-        acc.add(W, U, base + k + 512);
-        acc.add(W, U, base + k + 768);
-    }
-    for (; k < K; k += 256) acc.add(W, U, base + k);
+    add_row(acc, W + base, U ? U + base : nullptr, K, (int)threadIdx.x, 256);
     acc.warp_reduce();
     if (lane == 0) {
         part_h[wy] = acc.hi;
