@@ -85,26 +85,30 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
     return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
 
+// Bits lo .. hi-1 of a word (none when hi <= lo; 0 <= lo and hi <= 31).
+SADMM_DEV uint32_t bits_between(int lo, int hi) { return hi > lo ? (1u << hi) - (1u << lo) : 0u; }
+
 // Tap-validity mask of one output pixel whose receptive window starts at
 // (it0, ih0, iw0) of a T x H x W input: a bit is set where a tap reads inside
 // the input.  One bit per tap t = (kt*KH + kh)*KW + kw when the kernel has at
 // most 31 taps (split = 0); otherwise (split = 1) bits 0..15 mark valid rows
 // kt*KH + kh and bits 16..30 valid kw.  Bit 31 is never set (the gather
-// tables mark padding columns with it).
+// tables mark padding columns with it).  Each kernel coordinate's valid range
+// (0 <= i0 + k < extent) is formed in closed form.
 SADMM_DEV uint32_t tap_mask(int it0, int ih0, int iw0, int KT, int KH, int KW, int T, int H, int W, int split)
 {
-    uint32_t rm = 0, cm = 0;
-    for (int kt = 0; kt < KT; ++kt) {
-        const bool vt = (unsigned)(it0 + kt) < (unsigned)T;
-        for (int kh = 0; kh < KH; ++kh)
-            if (vt && (unsigned)(ih0 + kh) < (unsigned)H) rm |= 1u << (kt * KH + kh);
+    const int t_lo = max(0, -it0), t_hi = min(KT, T - it0);
+    const int h_lo = max(0, -ih0), h_hi = min(KH, H - ih0);
+    const int w_lo = max(0, -iw0), w_hi = min(KW, W - iw0);
+    const uint32_t cm = bits_between(w_lo, w_hi), hm = bits_between(h_lo, h_hi);
+    if (split) {
+        uint32_t rm = 0;
+        for (int kt = t_lo; kt < t_hi; ++kt) rm |= hm << (kt * KH);
+        return rm | (cm << 16);
     }
-    for (int kw = 0; kw < KW; ++kw)
-        if ((unsigned)(iw0 + kw) < (unsigned)W) cm |= 1u << kw;
-    if (split) return rm | (cm << 16);
     uint32_t m = 0;
-    for (int r = 0; r < KT * KH; ++r)
-        if (rm & (1u << r)) m |= cm << (r * KW);
+    for (int kt = t_lo; kt < t_hi; ++kt)
+        for (int kh = h_lo; kh < h_hi; ++kh) m |= cm << ((kt * KH + kh) * KW);
     return m;
 }
 
