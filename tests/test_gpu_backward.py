@@ -45,6 +45,9 @@ CASES = [
     ("groups2_5x5", ConvShape(n=2, c=8, h=9, w=9, f=12, kh=5, kw=5, ph=2, pw=2, groups=2), 0.5, wl.COL_SHAPE, 0.5),
     ("stride4_11x11", ConvShape(n=2, c=3, h=35, w=35, f=16, kh=11, kw=11, sh=4, sw=4), 1.0, wl.COL_SHAPE, 0.8),
     ("c3d", ConvShape(n=2, c=4, t=5, h=6, w=7, f=20, kt=3, kh=3, kw=3, pt=1, ph=1, pw=1), 1.0, wl.COL_SHAPE, 0.3),
+    # 45 taps: the split tap-mask form (row bits kt*KH + kh, kw bits apart), frames and rows clipped
+    ("c3d_45_taps", ConvShape(n=2, c=4, t=6, h=7, w=8, f=16, kt=3, kh=3, kw=5, pt=1, ph=1, pw=2), 0.75, wl.COL_SHAPE,
+     0.4),
     ("channel_3x3", ConvShape(n=2, c=24, h=9, w=9, f=40, kh=3, kw=3, ph=1, pw=1), 0.5, wl.COL_CHANNEL, 0.5),
     ("two_filter_tiles", ConvShape(n=2, c=16, h=10, w=10, f=300, kh=3, kw=3, ph=1, pw=1), 1.0, wl.COL_SHAPE, 1.0),
 ]

@@ -26,6 +26,9 @@ SMALL = [
     ("groups2_5x5", ConvShape(n=2, c=8, h=9, w=9, f=12, kh=5, kw=5, ph=2, pw=2, groups=2), 0.5, wl.COL_SHAPE, 0.5),
     ("stride4_11x11", ConvShape(n=2, c=3, h=35, w=35, f=16, kh=11, kw=11, sh=4, sw=4), 1.0, wl.COL_SHAPE, 0.8),
     ("c3d", ConvShape(n=2, c=4, t=5, h=6, w=7, f=20, kt=3, kh=3, kw=3, pt=1, ph=1, pw=1), 1.0, wl.COL_SHAPE, 0.3),
+    # 45 taps: the split tap-mask form (row bits kt*KH + kh, kw bits apart), frames and rows clipped
+    ("c3d_45_taps", ConvShape(n=2, c=4, t=6, h=7, w=8, f=16, kt=3, kh=3, kw=5, pt=1, ph=1, pw=2), 0.75, wl.COL_SHAPE,
+     0.4),
     ("channel_1x1", ConvShape(n=2, c=32, h=8, w=8, f=48, kh=1, kw=1), 0.5, wl.COL_CHANNEL, 0.5),
     ("channel_3x3", ConvShape(n=2, c=24, h=9, w=9, f=40, kh=3, kw=3, ph=1, pw=1), 0.5, wl.COL_CHANNEL, 0.5),
     ("no_col_pruning", ConvShape(n=1, c=12, h=7, w=7, f=33, kh=3, kw=3, ph=1, pw=1, groups=3), 0.6, wl.COL_NONE, 1.0),
