@@ -434,7 +434,7 @@ class ClockSampler:
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "conv_fwd_alexnet_b128_dram.txt")
 # the forward kernels' sources: the gathered kernel, the input-slab kernels and what they share
 CONV_SRCS = [os.path.join(ROOT, "paper_1807_11091_gb300", "csrc", f)
-             for f in ("conv_fwd.cu", "conv_slab.cu", "conv_common.cuh")]
+             for f in ("conv_fwd.cu", "conv_slab.cu", "conv_common.cuh", "common.cuh")]
 
 
 def conv_source_sha1():

@@ -156,14 +156,16 @@ __global__ void __launch_bounds__(kWgThreads, 1)
         __syncwarp();
     } else if (warp == 1) {
         // ------------------------------------------------------- MMA issuer
-        if (lane == 0) {
+        // The whole warp runs the loop (warp-uniform descriptors); one elected
+        // lane issues the MMAs and the commits that track them.
+        {
             const uint32_t idesc = idesc_bf16_f32_bmn(128, a.cs);
             const uint32_t sbo = (uint32_t)a.sp * 16u;  // next 8-channel chunk (along N)
             int s = 0;
             uint32_t ph = 0;
             bool first = true, ok = true;
             for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
-                if (!mbar_wait(&full[s], ph, abort_flag, a.status)) { ok = false; break; }
+                if (!mbar_wait_warp(&full[s], ph, abort_flag, a.status)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t x0 = smem_u32(smem + (size_t)s * a.stage_stride);
                 const uint32_t d0 = x0 + (uint32_t)a.stage_stride - 2u * kWgDzBox;
@@ -177,18 +179,20 @@ __global__ void __launch_bounds__(kWgThreads, 1)
                             const uint64_t adesc =
                                 sdesc_kmajor_sw128(d0 + (uint32_t)(kk >> 2) * kWgDzBox + (uint32_t)(kk & 3) * 32u);
                             const uint64_t bdesc = sdesc_kmajor_none(xt + (uint32_t)kk * 256u, 128u, sbo);
-                            mma_bf16_ss(d, adesc, bdesc, idesc, (first && kk == 0) ? 0u : 1u);
+                            mma_bf16_ss_elect(d, adesc, bdesc, idesc, (first && kk == 0) ? 0u : 1u);
                         }
                     }
                 }
                 first = false;
-                mma_commit(&empty[s]);
+                mma_commit_elect(&empty[s]);
                 if (++s == a.stages) { s = 0; ph ^= 1u; }
             }
-            if (ok) mma_commit(acc_full);
-            mma_commit(drain);
-            const unsigned long long t0 = globaltimer();
-            while (!mbar_try_wait(drain, 0) && globaltimer() - t0 < kWaitLimitNs) {}
+            if (ok) mma_commit_elect(acc_full);
+            mma_commit_elect(drain);
+            if (lane == 0) {
+                const unsigned long long t0 = globaltimer();
+                while (!mbar_try_wait(drain, 0) && globaltimer() - t0 < kWaitLimitNs) {}
+            }
         }
         __syncwarp();
     } else {

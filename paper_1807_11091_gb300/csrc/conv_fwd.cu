@@ -384,7 +384,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();  // the whole warp reaches the block barrier below together
     } else if (warp == 1) {
         // ------------------------------------------------------- MMA issuer
-        if (lane == 0) {
+        // The whole warp runs the loop (warp-uniform descriptors); one elected
+        // lane issues the MMAs and the commits that track them.
+        {
             int s = 0;
             uint32_t ph = 0;
             int ab = 0;
@@ -401,8 +403,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (a.b_res) {
                     const long long key = (long long)g * a.upairs + p;
                     if (key != cur) {
-                        if (cur >= 0) mma_commit(b_empty);  // the old weights are free once these MMAs finish
-                        if (!mbar_wait(b_full, bf_ph, abort_flag, a.status)) break;
+                        if (cur >= 0) mma_commit_elect(b_empty);  // the old weights are free once these MMAs finish
+                        if (!mbar_wait_warp(b_full, bf_ph, abort_flag, a.status)) break;
                         bf_ph ^= 1u;
                         cur = key;
                     }
@@ -412,12 +414,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t idesc0 = idesc_bf16_f32(kBM, min(a.bn, (cnt + 15) & ~15));
                 const uint32_t idesc1 = idesc_bf16_f32(kBM, min(a.bn, (max(rows1, 16) + 15) & ~15));
                 const bool two = rows1 > 0;
-                if (!mbar_wait(&acc_empty[ab], acc_ph ^ 1u, abort_flag, a.status)) break;
+                if (!mbar_wait_warp(&acc_empty[ab], acc_ph ^ 1u, abort_flag, a.status)) break;
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + (uint32_t)(ab * a.nacc * a.tmem_stride);
                 for (int ks = ks0; ks < ks1; ++ks) {
-                    if (!mbar_wait(&full_a[s], ph, abort_flag, a.status) ||
-                        (!a.b_res && !mbar_wait(&full_b[s], ph, abort_flag, a.status))) {
+                    if (!mbar_wait_warp(&full_a[s], ph, abort_flag, a.status) ||
+                        (!a.b_res && !mbar_wait_warp(&full_b[s], ph, abort_flag, a.status))) {
                         ok = false;
                         break;
                     }
@@ -429,7 +431,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (!two) {
 #pragma unroll
                         for (int kk = 0; kk < kBK / 16; ++kk)
-                            mma_bf16_ss(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32), sdesc_kmajor_sw128(b0 + kk * 32),
+                            mma_bf16_ss_elect(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32), sdesc_kmajor_sw128(b0 + kk * 32),
                                         idesc0, (ks != ks0 || kk != 0) ? 1u : 0u);
                     } else {
                         const uint32_t d1 = d_tmem + (uint32_t)a.tmem_stride;
@@ -438,21 +440,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int kk = 0; kk < kBK / 16; ++kk) {
                             const uint64_t adesc = sdesc_kmajor_sw128(a0 + kk * 32);
                             const uint32_t acc = (ks != ks0 || kk != 0) ? 1u : 0u;
-                            mma_bf16_ss(d_tmem, adesc, sdesc_kmajor_sw128(b0 + kk * 32), idesc0, acc);
-                            mma_bf16_ss(d1, adesc, sdesc_kmajor_sw128(b1 + kk * 32), idesc1, acc);
+                            mma_bf16_ss_elect(d_tmem, adesc, sdesc_kmajor_sw128(b0 + kk * 32), idesc0, acc);
+                            mma_bf16_ss_elect(d1, adesc, sdesc_kmajor_sw128(b1 + kk * 32), idesc1, acc);
                         }
                     }
-                    mma_commit(&empty[s]);
+                    mma_commit_elect(&empty[s]);
                     if (++s == S) { s = 0; ph ^= 1u; }
                 }
                 if (!ok) break;
-                mma_commit(&acc_full[ab]);
+                mma_commit_elect(&acc_full[ab]);
                 if (++ab == a.acc_bufs) { ab = 0; acc_ph ^= 1u; }
             }
             // Every MMA this thread issued has completed before TMEM is freed.
-            mma_commit(drain);
-            const unsigned long long t0 = globaltimer();
-            while (!mbar_try_wait(drain, 0) && globaltimer() - t0 < kWaitLimitNs) {}
+            mma_commit_elect(drain);
+            if (lane == 0) {
+                const unsigned long long t0 = globaltimer();
+                while (!mbar_try_wait(drain, 0) && globaltimer() - t0 < kWaitLimitNs) {}
+            }
         }
         __syncwarp();
     } else if (warp >= 4 && warp < 4 + kEpiWarps) {

@@ -45,6 +45,7 @@ constexpr int kSlabTables = 2 * 256 * 4;  // plane offset and bias of each kept 
 constexpr int kSlabZcap = 1024;           // pruned filters whose plane offsets sit in shared memory
 constexpr int kSlabBars = 256;            // barriers, TMEM address, abort flag
 constexpr int kSlabSmemLimit = 232448;
+constexpr int kSlabMaxSteps = 128;  // MMAs per tile whose descriptor offsets travel in the parameters
 
 struct SlabArgs {
     void* y;
@@ -61,6 +62,8 @@ struct SlabArgs {
     int stages, stage_bytes, stage_stride;
     int tmem_stride, tmem_cols;
     int relu;
+    int nsteps;                     // MMAs per tile (R * Q * ksteps)
+    uint2 steps[kSlabMaxSteps];     // per MMA: A start (16-byte units from the slab), B start (from the weights)
 };
 
 struct XsArgs {
@@ -217,39 +220,38 @@ __global__ void __launch_bounds__(kSlabThreads, 1)
         __syncwarp();
     } else if (warp == 1) {
         // ------------------------------------------------------- MMA issuer
-        if (lane == 0) {
-            bool ok = mbar_wait(b_full, 0, abort_flag, a.status);
-            const uint32_t idesc = idesc_bf16_f32(128, a.bn);
-            const uint32_t lbo = (uint32_t)a.sp * 16u;  // next chunk (8 channels further along K)
-            const uint32_t sB0 = smem_u32(sB);
-            int s = 0, ab = 0;
-            uint32_t ph = 0, acc_ph = 0;
-            for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-                if (!mbar_wait(&acc_empty[ab], acc_ph ^ 1u, abort_flag, a.status)) break;
-                tc_fence_after();
-                if (!mbar_wait(&full[s], ph, abort_flag, a.status)) break;
-                tc_fence_after();
-                const uint32_t d = tmem_base + (uint32_t)(ab * a.tmem_stride);
-                const uint32_t a0 = smem_u32(sA + (size_t)s * a.stage_stride);
-                int step = 0;
-                for (int r = 0; r < a.R; ++r) {
-                    for (int q = 0; q < a.Q; ++q) {
-                        const uint32_t at = a0 + (uint32_t)(r * a.Wb + q) * 16u;
-                        for (int j = 0; j < a.ksteps; ++j, ++step) {
-                            const uint64_t adesc = sdesc_kmajor_none(at + 2u * (uint32_t)j * lbo, lbo, 128u);
-                            const uint64_t bdesc =
-                                sdesc_kmajor_sw128(sB0 + (uint32_t)(step >> 2) * bbox + (uint32_t)(step & 3) * 32u);
-                            mma_bf16_ss(d, adesc, bdesc, idesc, step > 0 ? 1u : 0u);
-                        }
-                    }
-                }
-                mma_commit(&empty[s]);
-                mma_commit(&acc_full[ab]);
-                if (++s == a.stages) { s = 0; ph ^= 1u; }
-                if (++ab == 2) { ab = 0; acc_ph ^= 1u; }
+        // The whole warp runs the loop, so the descriptors stay warp-uniform;
+        // one elected lane issues the MMAs and the commits that track them.
+        bool ok = mbar_wait_warp(b_full, 0, abort_flag, a.status);
+        const uint32_t idesc = idesc_bf16_f32(128, a.bn);
+        const uint64_t ad0 = sdesc_kmajor_none(smem_u32(sA), (uint32_t)a.sp * 16u, 128u);
+        const uint64_t bd0 = sdesc_kmajor_sw128(smem_u32(sB));
+        const uint32_t ahi = (uint32_t)(ad0 >> 32), bhi = (uint32_t)(bd0 >> 32), blo = (uint32_t)bd0;
+        int s = 0, ab = 0;
+        uint32_t ph = 0, acc_ph = 0;
+        for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
+            if (!mbar_wait_warp(&acc_empty[ab], acc_ph ^ 1u, abort_flag, a.status)) break;
+            tc_fence_after();
+            if (!mbar_wait_warp(&full[s], ph, abort_flag, a.status)) break;
+            tc_fence_after();
+            const uint32_t d = tmem_base + (uint32_t)(ab * a.tmem_stride);
+            // The low descriptor word starts with the start-address field (the
+            // shared address / 16, below 2^14), so offsets in 16-byte units add to it.
+            const uint32_t alo = (uint32_t)ad0 + ((uint32_t)(s * a.stage_stride) >> 4);
+#pragma unroll 4
+            for (int st = 0; st < a.nsteps; ++st) {
+                const uint2 e = a.steps[st];
+                mma_bf16_ss_elect(d, ((uint64_t)ahi << 32) | (alo + e.x), ((uint64_t)bhi << 32) | (blo + e.y), idesc,
+                                  st > 0 ? 1u : 0u);
             }
-            // Every MMA this thread issued has completed before TMEM is freed.
-            mma_commit(drain);
+            mma_commit_elect(&empty[s]);
+            mma_commit_elect(&acc_full[ab]);
+            if (++s == a.stages) { s = 0; ph ^= 1u; }
+            if (++ab == 2) { ab = 0; acc_ph ^= 1u; }
+        }
+        // Every MMA the elected lane issued has completed before TMEM is freed.
+        mma_commit_elect(drain);
+        if (lane == 0) {
             const unsigned long long t0 = globaltimer();
             while (!mbar_try_wait(drain, 0) && globaltimer() - t0 < kWaitLimitNs) {}
         }
@@ -341,7 +343,7 @@ cudaError_t launch_slab(const CUtensorMap& tw, const CUtensorMap& tx, const Slab
 
 int slab_stages(int bn, int kpad_s, int cs, int sp)
 {
-    if (bn < 16 || bn > 256 || bn % 16 || kpad_s % 64 || cs % 16 || sp % 8) return 0;
+    if (bn < 16 || bn > 256 || bn % 16 || kpad_s % 64 || cs % 16 || sp % 8 || kpad_s / 16 > kSlabMaxSteps) return 0;
     const long long room = (long long)kSlabSmemLimit - slab_fixed_bytes(bn, kpad_s);
     if (room <= 0) return 0;
     const long long st = room / slab_stage_stride(cs, sp);
@@ -418,6 +420,15 @@ sadmm_status launch_conv_slab(const sadmm_plan* plan, const Geometry& g, const v
     while (cols < 2 * a.tmem_stride) cols <<= 1;
     a.tmem_cols = cols;
     a.relu = relu ? 1 : 0;
+    a.nsteps = a.R * a.Q * a.ksteps;
+    {
+        int st = 0;
+        for (int r = 0; r < a.R; ++r)
+            for (int q = 0; q < a.Q; ++q)
+                for (int j = 0; j < a.ksteps; ++j, ++st)
+                    a.steps[st] = make_uint2((uint32_t)(r * a.Wb + q) + (uint32_t)j * (uint32_t)a.sp * 2u,
+                                             (uint32_t)(st >> 2) * (uint32_t)a.bn * 8u + (uint32_t)(st & 3) * 2u);
+    }
     const size_t smem = (size_t)slab_fixed_bytes(a.bn, plan->xs_kpad) + (size_t)stages * a.stage_stride;
     long long grid = plan->ctas > 0 ? plan->ctas : device_sm_count();
     if (grid > units) grid = units;

@@ -98,26 +98,29 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
         __syncwarp();
     } else if (warp == 1) {
-        if (lane == 0) {
+        // the whole warp runs the loop; one elected lane issues the MMAs and commits
+        {
             const uint32_t idesc = idesc_bf16_f32(128, a.bn);
             bool ok = true;
             for (int ks = 0; ks < a.nk; ++ks) {
                 const int s = ks % kGemmStages;
                 const uint32_t ph = (uint32_t)(ks / kGemmStages) & 1u;
-                if (!mbar_wait(&full[s], ph, abort_flag, a.status)) { ok = false; break; }
+                if (!mbar_wait_warp(&full[s], ph, abort_flag, a.status)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t a0 = smem_u32(sA + (size_t)s * kATile);
                 const uint32_t b0 = smem_u32(sB + (size_t)s * b_bytes);
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk)
-                    mma_bf16_ss(tmem_base, sdesc_kmajor_sw128(a0 + kk * 32), sdesc_kmajor_sw128(b0 + kk * 32), idesc,
+                    mma_bf16_ss_elect(tmem_base, sdesc_kmajor_sw128(a0 + kk * 32), sdesc_kmajor_sw128(b0 + kk * 32), idesc,
                                 (ks | kk) != 0 ? 1u : 0u);
-                mma_commit(&empty[s]);
+                mma_commit_elect(&empty[s]);
             }
-            if (ok) mma_commit(acc_full);
-            mma_commit(drain);
-            const unsigned long long t0 = globaltimer();
-            while (!mbar_try_wait(drain, 0) && globaltimer() - t0 < kWaitLimitNs) {}
+            if (ok) mma_commit_elect(acc_full);
+            mma_commit_elect(drain);
+            if (lane == 0) {
+                const unsigned long long t0 = globaltimer();
+                while (!mbar_try_wait(drain, 0) && globaltimer() - t0 < kWaitLimitNs) {}
+            }
         }
         __syncwarp();
     } else {

@@ -208,3 +208,21 @@ def test_slab_extreme_geometry(case):
     s, t, rows, ck, cols, y, pc = _run(case, seed=308)
     ref = oracle_layer(s, t, rows, ck, cols)
     assert_close(y, ref, what=case[0])
+
+
+def test_slab_mma_step_limit():
+    """A slab plan issues at most 128 MMAs per tile (their descriptor offsets travel
+    in the kernel parameters): 15 x 15 stride 2 over 8 channels is 64 block taps x 32
+    slab channels = 128 MMAs and takes the slab path; over 12 channels (192 MMAs) the
+    same kernel takes the gathered path.  Both match the oracle."""
+    at_cap = ("steps_128", ConvShape(n=2, c=8, h=40, w=40, f=16, kh=15, kw=15, sh=2, sw=2), 1.0, wl.COL_NONE, 1.0)
+    s, t, rows, ck, cols, y, pc = _run(at_cap, seed=309)
+    assert pc.plan.xs_r * pc.plan.xs_q * pc.plan.xs_cs // 16 == 128
+    assert_close(y, oracle_layer(s, t, rows, ck, cols), what="steps_128")
+    s = ConvShape(n=2, c=12, h=40, w=40, f=16, kh=15, kw=15, sh=2, sw=2)
+    t = wl.gen_tensors(s, seed=310)
+    fi, ci, y, pc = gpu_layer(s, t, s.f, wl.COL_NONE, 0)
+    assert pc.plan.xs_mode == 0
+    rows, cols, _, _ = oracle.project(t["W"], s.taps, s.f, wl.COL_NONE, 0)
+    assert np.array_equal(fi, rows)
+    assert_close(y, oracle_layer(s, t, rows, wl.COL_NONE, cols), what="steps_192")
