@@ -45,7 +45,7 @@
 extern "C" {
 #endif
 
-#define SADMM_ABI_VERSION 5
+#define SADMM_ABI_VERSION 6
 
 /* Most layers one batched call (sadmm_project_groups_batch,
  * sadmm_admm_update_batch) takes. */
@@ -59,7 +59,8 @@ typedef enum {
     SADMM_EINVAL = -1,       /* bad argument, shape or buffer size          */
     SADMM_ECUDA = -2,        /* a CUDA runtime call or launch failed        */
     SADMM_ETIMEOUT = -3,     /* a device-side wait ran past its limit       */
-    SADMM_EUNSUPPORTED = -4  /* valid request outside what the kernels do   */
+    SADMM_EUNSUPPORTED = -4, /* valid request outside what the kernels do   */
+    SADMM_EBOUNDS = -5       /* debug build: a device-side index check failed */
 } sadmm_status;
 
 typedef enum { SADMM_BF16 = 0, SADMM_FP32 = 1 } sadmm_dtype;
@@ -548,8 +549,11 @@ sadmm_status sadmm_selftest_wait(unsigned int limit_us, int arrive, int* result,
 
 /*
  * Synchronises `stream`, then reports and clears the device status word that
- * the kernels set when a bounded wait expires (SADMM_ETIMEOUT) or a
- * device-side check fails (SADMM_EINVAL).  SADMM_OK when clear.
+ * the kernels set when a bounded wait expires (SADMM_ETIMEOUT), a device-side
+ * check of an index list fails (SADMM_EINVAL) or, in a library built with
+ * -DSADMM_DEBUG, an index check of a global load or store fails
+ * (SADMM_EBOUNDS: the access was skipped, a load read zero).  SADMM_OK when
+ * clear.
  */
 sadmm_status sadmm_last_device_status(void* stream);
 

@@ -643,6 +643,7 @@ sadmm_status sadmm_last_device_status(void* stream)
         cudaMemcpyToSymbol(g_status_word, &zero, sizeof(int));
     }
     if (v == kDevTimeout) return SADMM_ETIMEOUT;
+    if (v == kDevBounds) return SADMM_EBOUNDS;
     if (v != 0) return SADMM_EINVAL;
     return SADMM_OK;
 }

@@ -44,6 +44,7 @@ struct BwdGeo {
     int split_mask;        // tap-mask encoding of the gather table (see tap_mask)
     const uint2* table;    // the plan's gather table: [k_pad] {x offset from the window origin, tap bits}
     size_t slab_wg_bytes;  // workspace of the slab weight gradient (0: gathered weight gradient)
+    int* status;           // device status word (the debug build's index checks)
 };
 
 inline void divisor(uint32_t d, uint32_t& mul, uint32_t& sh)
@@ -102,7 +103,10 @@ __global__ void __launch_bounds__(256) k_bwd_im2col(const BwdGeo b, int g, long 
         }
         for (int jj = 0; jj < nj; ++jj) {
             const uint2 t = s_t[jj];
-            as[(size_t)(j0 + jj) * b.mc + ml] = ((M & t.y) == t.y) ? __ldg(xs + base + (int)t.x) : (unsigned short)0;
+            as[(size_t)(j0 + jj) * b.mc + ml] =
+                ((M & t.y) == t.y && dbg_in(base + (int)t.x, (long long)b.N * b.x_chw, b.status))
+                    ? __ldg(xs + base + (int)t.x)
+                    : (unsigned short)0;
         }
     }
 }
@@ -205,7 +209,8 @@ __global__ void __launch_bounds__(256) k_bwd_col2im(const BwdGeo b, int g, long 
             const uint2 t = s_t[jj];
             if ((M & t.y) == t.y) {
                 const float v = dat[(size_t)(j0 + jj) * b.mc + ml];
-                if (v != 0.0f) atomicAdd(dx + base + (int)t.x, v);
+                if (v != 0.0f && dbg_in(base + (int)t.x, (long long)b.N * b.x_chw, b.status))
+                    atomicAdd(dx + base + (int)t.x, v);
             }
         }
     }
@@ -354,6 +359,7 @@ BwdGeo geometry(const sadmm_plan* plan, const Geometry& g, long long chunk)
     divisor((uint32_t)(b.OH * b.OW), b.ohw_mul, b.ohw_sh);
     divisor((uint32_t)b.OW, b.ow_mul, b.ow_sh);
     b.x_chw = g.c * g.t * g.h * g.w;
+    b.status = device_status_ptr();
     b.thw = g.t * g.h * g.w;
     b.hw = (int)(g.h * g.w);
     b.split_mask = tap_mask_mode(g);

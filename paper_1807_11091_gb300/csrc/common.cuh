@@ -20,6 +20,7 @@ namespace sadmm {
 // Device-side status codes (written into the library's status word).
 constexpr int kDevTimeout = 1;
 constexpr int kDevBadIndex = 2;
+constexpr int kDevBounds = 3;   // a debug build's index check failed
 
 // A bounded wait gives up after this much wall time.
 constexpr unsigned long long kWaitLimitNs = 4000000000ull;  // 4 s
@@ -116,6 +117,21 @@ SADMM_DEV void raise_status(int* status, int code)
 {
     if (status) atomicCAS(status, 0, code);
 }
+
+// Index checks of the debug build (-DSADMM_DEBUG): true when i lies in
+// [0, n); otherwise the status word gets kDevBounds and the caller skips the
+// access (a load then reads zero).  In the release build every check is the
+// constant true and compiles away.
+#ifdef SADMM_DEBUG
+SADMM_DEV bool dbg_in(long long i, long long n, int* status)
+{
+    if (i >= 0 && i < n) return true;
+    raise_status(status, kDevBounds);
+    return false;
+}
+#else
+SADMM_DEV bool dbg_in(long long, long long, int*) { return true; }
+#endif
 
 // ---------------------------------------------------------------- mbarrier --
 

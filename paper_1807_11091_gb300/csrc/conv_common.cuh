@@ -31,12 +31,20 @@ inline FastDiv make_fastdiv(uint32_t d)
 
 SADMM_DEV uint32_t fdiv(uint32_t n, const FastDiv& f) { return (__umulhi(n, f.mul) + n) >> f.shift; }
 
+// The output's extent for the debug build's store checks: yf / yh point at
+// element pix of y, which holds total elements.
+struct YCheck {
+    long long pix, total;
+    int* status;
+};
+SADMM_DEV bool y_ok(const YCheck& c, long long off) { return dbg_in(c.pix + off, c.total, c.status); }
+
 // Bias, ReLU and the stores of accumulator columns c0 .. c0+kEpiCols-1 of one
 // pixel (columns at or past nrows are skipped): t_off / t_bias give each
 // column's output-plane offset and bias, yf / yh point at the pixel in plane 0.
 template <bool OUT_BF16>
 SADMM_DEV void store_cols(const float (&v)[kEpiCols], int c0, int nrows, const int* t_off, const float* t_bias,
-                          int relu, float* yf, __nv_bfloat16* yh)
+                          int relu, float* yf, __nv_bfloat16* yh, const YCheck& yc)
 {
     if (c0 + kEpiCols <= nrows) {
 #pragma unroll
@@ -49,11 +57,15 @@ SADMM_DEV void store_cols(const float (&v)[kEpiCols], int c0, int nrows, const i
                 v2 = fmaxf(v2, 0.0f); v3 = fmaxf(v3, 0.0f);
             }
             if (OUT_BF16) {
-                yh[o.x] = __float2bfloat16_rn(v0); yh[o.y] = __float2bfloat16_rn(v1);
-                yh[o.z] = __float2bfloat16_rn(v2); yh[o.w] = __float2bfloat16_rn(v3);
+                if (y_ok(yc, o.x)) yh[o.x] = __float2bfloat16_rn(v0);
+                if (y_ok(yc, o.y)) yh[o.y] = __float2bfloat16_rn(v1);
+                if (y_ok(yc, o.z)) yh[o.z] = __float2bfloat16_rn(v2);
+                if (y_ok(yc, o.w)) yh[o.w] = __float2bfloat16_rn(v3);
             } else {
-                __stcs(yf + o.x, v0); __stcs(yf + o.y, v1);
-                __stcs(yf + o.z, v2); __stcs(yf + o.w, v3);
+                if (y_ok(yc, o.x)) __stcs(yf + o.x, v0);
+                if (y_ok(yc, o.y)) __stcs(yf + o.y, v1);
+                if (y_ok(yc, o.z)) __stcs(yf + o.z, v2);
+                if (y_ok(yc, o.w)) __stcs(yf + o.w, v3);
             }
         }
     } else {
@@ -62,10 +74,12 @@ SADMM_DEV void store_cols(const float (&v)[kEpiCols], int c0, int nrows, const i
             if (c0 + j < nrows) {
                 float x = v[j] + t_bias[c0 + j];
                 if (relu) x = fmaxf(x, 0.0f);
+                const int off = t_off[c0 + j];
+                if (!y_ok(yc, off)) continue;
                 if (OUT_BF16)
-                    yh[t_off[c0 + j]] = __float2bfloat16_rn(x);
+                    yh[off] = __float2bfloat16_rn(x);
                 else
-                    __stcs(yf + t_off[c0 + j], x);
+                    __stcs(yf + off, x);
             }
         }
     }

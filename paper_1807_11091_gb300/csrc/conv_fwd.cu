@@ -85,6 +85,7 @@ struct ConvArgs {
     const int* counts;
     int* status;
     int M;            // N * plane (below 2^31)
+    long long x_total, y_total;  // elements of x and y (the debug build's index checks)
     long long x_chw;  // elements per input image
     long long thw;    // elements per input channel
     int units;        // work items: m_tiles * groups * upairs * splits (below 2^31)
@@ -233,8 +234,11 @@ SADMM_DEV uint32_t pixel_mask(const ConvArgs& a, int it0, int ih0, int iw0)
 // input), else 0 (a predicated load).  Testing against zero lets the and and
 // the compare fold into one logic operation that writes the predicate
 // (measured 2-4 % faster than testing (mask & bits) == bits).
-SADMM_DEV uint32_t ldg_u16_if(const unsigned short* p, uint32_t bits, uint32_t nM)
+SADMM_DEV uint32_t ldg_u16_if(const unsigned short* p, uint32_t bits, uint32_t nM, const ConvArgs& a)
 {
+    if ((bits & nM) == 0 &&
+        !dbg_in(p - reinterpret_cast<const unsigned short*>(a.x), a.x_total, a.status))
+        return 0;  // debug build: an index outside x
     uint32_t v;
     asm("{\n\t.reg .pred q;\n\t.reg .b32 t;\n\t"
         "and.b32 t, %2, %3;\n\t"
@@ -518,6 +522,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const long long pix = valid ? m - n_img * a.plane : 0;
             float* yf = reinterpret_cast<float*>(a.y) + (n_img * (long long)a.F * a.plane + pix);
             __nv_bfloat16* yh = reinterpret_cast<__nv_bfloat16*>(a.y) + (n_img * (long long)a.F * a.plane + pix);
+            const YCheck yc{n_img * (long long)a.F * a.plane + pix, a.y_total, a.status};
             int chunks = 0;  // chunks of this unit so far (zero planes, then accumulator columns)
             if (zc > 0 && alive && a.splits == 1 && ks0 == 0) {
                 // Pruned filters of this conv group: their planes are zero.  They
@@ -533,6 +538,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                         for (int j = 0; j < kEpiCols; j += 4) {
                             const int4 o = *reinterpret_cast<const int4*>(u_zero + z0 + j);
+                            if (!(y_ok(yc, o.x) && y_ok(yc, o.y) && y_ok(yc, o.z) && y_ok(yc, o.w))) continue;
                             if (OUT_BF16) {
                                 const __nv_bfloat16 zb = __float2bfloat16_rn(0.0f);
                                 yh[o.x] = zb; yh[o.y] = zb; yh[o.z] = zb; yh[o.w] = zb;
@@ -544,6 +550,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     } else {
                         for (int z = z0; z < min(z0 + kEpiCols, zc); ++z) {
                             const int off = z < a.zcap ? u_zero[z] : __ldg(zmap + z) * a.plane;
+                            if (!y_ok(yc, off)) continue;
                             if (OUT_BF16)
                                 yh[off] = __float2bfloat16_rn(0.0f);
                             else
@@ -602,7 +609,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                             for (int j = 0; j < kEpiCols; ++j)
                                 v[j] = __uint_as_float(r[j]) + __ldcg(other + col0 + (size_t)j * kBM);
-                            if (valid) store_cols<OUT_BF16>(v, c0, nrows, t_off, t_bias, a.relu, yf, yh);
+                            if (valid) store_cols<OUT_BF16>(v, c0, nrows, t_off, t_bias, a.relu, yf, yh, yc);
                         } else if (valid && a.splits > 1) {
                             // split K': raw fp32 partial sums, [split][column][pixel]
                             float* pp = a.partial +
@@ -616,7 +623,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             float v[kEpiCols];
 #pragma unroll
                             for (int j = 0; j < kEpiCols; ++j) v[j] = __uint_as_float(r[j]);
-                            store_cols<OUT_BF16>(v, c0, nrows, t_off, t_bias, a.relu, yf, yh);
+                            store_cols<OUT_BF16>(v, c0, nrows, t_off, t_bias, a.relu, yf, yh, yc);
                         }
                     }
                     chunks += nch;
@@ -655,7 +662,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                             for (int j = 0; j < kEpiCols; ++j)
                                 v[j] = __uint_as_float(r[j]) + __ldcg(other + col0 + (size_t)j * kBM);
-                            if (valid) store_cols<OUT_BF16>(v, c0, nrows, t_off, t_bias, a.relu, yf, yh);
+                            if (valid) store_cols<OUT_BF16>(v, c0, nrows, t_off, t_bias, a.relu, yf, yh, yc);
                         }
                         ch += nch;
                     }
@@ -725,8 +732,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 const uint4 t = te4[((chunk0 + ci) * 8 + e) >> 1];
 #pragma unroll
                                 for (int r = 0; r < kPixPerThread; ++r) {
-                                    v[(r * kChunksPerThread + ci) * 8 + e] = __ldg(xb[r] + (int)t.x);
-                                    v[(r * kChunksPerThread + ci) * 8 + e + 1] = __ldg(xb[r] + (int)t.z);
+                                    v[(r * kChunksPerThread + ci) * 8 + e] =
+                                        dbg_in(xb[r] + (int)t.x - xs, a.x_total, a.status) ? __ldg(xb[r] + (int)t.x) : 0u;
+                                    v[(r * kChunksPerThread + ci) * 8 + e + 1] =
+                                        dbg_in(xb[r] + (int)t.z - xs, a.x_total, a.status) ? __ldg(xb[r] + (int)t.z) : 0u;
                                 }
                             }
                         }
@@ -738,9 +747,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 const uint4 t = te4[((chunk0 + ci) * 8 + e) >> 1];
 #pragma unroll
                                 for (int r = 0; r < kPixPerThread; ++r) {
-                                    v[(r * kChunksPerThread + ci) * 8 + e] = ldg_u16_if(xb[r] + (int)t.x, t.y, M[r]);
+                                    v[(r * kChunksPerThread + ci) * 8 + e] = ldg_u16_if(xb[r] + (int)t.x, t.y, M[r], a);
                                     v[(r * kChunksPerThread + ci) * 8 + e + 1] =
-                                        ldg_u16_if(xb[r] + (int)t.z, t.w, M[r]);
+                                        ldg_u16_if(xb[r] + (int)t.z, t.w, M[r], a);
                                 }
                             }
                         }
@@ -813,6 +822,7 @@ __global__ void __launch_bounds__(256) k_splitk_finalize(const ConvArgs a)
         }
         const int n_img = (int)fdiv((uint32_t)m, a.plane_div);
         const size_t off = ((size_t)n_img * a.F + f) * a.plane + (m - n_img * a.plane);
+        if (!dbg_in((long long)off, a.y_total, a.status)) continue;
         if (OUT_BF16)
             reinterpret_cast<__nv_bfloat16*>(a.y)[off] = __float2bfloat16_rn(v);
         else
@@ -877,6 +887,8 @@ sadmm_status launch_conv_fwd(const sadmm_plan* plan, const Geometry& g, const vo
     a.status = device_status_ptr();
     if (g.m >= (1ll << 31) - 256) return SADMM_EUNSUPPORTED;  // pixel indices stay in int
     a.M = (int)g.m;
+    a.x_total = g.n * g.c * g.t * g.h * g.w;
+    a.y_total = g.n * g.f * g.plane;
     a.x_chw = g.c * g.t * g.h * g.w;
     a.thw = g.t * g.h * g.w;
     a.hw = (int)(g.h * g.w);

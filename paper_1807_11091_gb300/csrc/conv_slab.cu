@@ -54,6 +54,7 @@ struct SlabArgs {
     const int* zeromap;  // pruned filters, ascending
     const int* counts;   // [kept, pruned]
     int* status;
+    long long y_total;  // elements of y (the debug build's store checks)
     int F, OH, OW, plane;
     int Wb, MT, units;     // block-pixel row width, tiles per image, tiles in all
     FastDiv mt_div, wb_div;
@@ -69,6 +70,8 @@ struct SlabArgs {
 struct XsArgs {
     int C, H, W, sh, sw, ph, pw;
     int nck, cs, Hb, Wb, pimg;
+    long long x_total, xs_total;  // elements of x and of the copy (the debug build's index checks)
+    int* status;
 };
 
 // Thread (tx, ty) of block (bw, bh, n) writes every chunk's 16-byte vector
@@ -101,8 +104,8 @@ __global__ void __launch_bounds__(kXsPix * kXsRows) k_slab_input(const __nv_bflo
         const int pad = b.pimg - b.Hb * b.Wb;
         for (int v = tid; v < chunks * pad; v += kXsPix * kXsRows) {
             const int k = v / pad, j = v - k * pad;
-            *reinterpret_cast<uint4*>(xs + (((long long)n * chunks + k) * b.pimg + (long long)b.Hb * b.Wb + j) * 8) =
-                make_uint4(0u, 0u, 0u, 0u);
+            const long long o = (((long long)n * chunks + k) * b.pimg + (long long)b.Hb * b.Wb + j) * 8;
+            if (dbg_in(o + 7, b.xs_total, b.status)) *reinterpret_cast<uint4*>(xs + o) = make_uint4(0u, 0u, 0u, 0u);
         }
     }
     const int wb = blockIdx.x * kXsPix + threadIdx.x;
@@ -118,12 +121,14 @@ __global__ void __launch_bounds__(kXsPix * kXsRows) k_slab_input(const __nv_bflo
         for (int e = 0; e < 8; ++e) {
             const int4 d = s_dec[8 * k + e];
             const int ih = ih0 + d.y, iw = iw0 + d.z;
-            h[e] = (d.x >= 0 && (unsigned)ih < (unsigned)b.H && (unsigned)iw < (unsigned)b.W)
+            h[e] = (d.x >= 0 && (unsigned)ih < (unsigned)b.H && (unsigned)iw < (unsigned)b.W &&
+                    dbg_in(xi - reinterpret_cast<const unsigned short*>(x) + d.x + ih * b.W + iw, b.x_total, b.status))
                        ? (uint32_t)__ldg(xi + d.x + ih * b.W + iw)
                        : 0u;
         }
-        *reinterpret_cast<uint4*>(dst0 + (long long)k * b.pimg * 8) =
-            make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16), h[6] | (h[7] << 16));
+        if (dbg_in(dst0 - xs + (long long)k * b.pimg * 8 + 7, b.xs_total, b.status))
+            *reinterpret_cast<uint4*>(dst0 + (long long)k * b.pimg * 8) =
+                make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16), h[6] | (h[7] << 16));
     }
 }
 
@@ -276,10 +281,12 @@ __global__ void __launch_bounds__(kSlabThreads, 1)
             const long long pix = (long long)n * a.F * a.plane + (long long)oh * a.OW + ow;
             float* yf = reinterpret_cast<float*>(a.y) + pix;
             __nv_bfloat16* yh = reinterpret_cast<__nv_bfloat16*>(a.y) + pix;
+            const YCheck yc{pix, a.y_total, a.status};
             // pruned filters' planes: zero, while the tile's MMAs run
             if (alive && valid) {
                 for (int z = h; z < pruned; z += 2) {
                     const long long off = z < kSlabZcap ? z_off[z] : (long long)__ldg(a.zeromap + z) * a.plane;
+                    if (!y_ok(yc, off)) continue;
                     if (OUT_BF16)
                         yh[off] = __float2bfloat16_rn(0.0f);
                     else
@@ -300,7 +307,7 @@ __global__ void __launch_bounds__(kSlabThreads, 1)
                     float v[kEpiCols];
 #pragma unroll
                     for (int j = 0; j < kEpiCols; ++j) v[j] = __uint_as_float(r[j]);
-                    if (valid) store_cols<OUT_BF16>(v, c0, kept, t_off, t_bias, a.relu, yf, yh);
+                    if (valid) store_cols<OUT_BF16>(v, c0, kept, t_off, t_bias, a.relu, yf, yh, yc);
                 }
                 tc_fence_before();
                 __syncwarp();
@@ -375,6 +382,9 @@ sadmm_status launch_conv_slab(const sadmm_plan* plan, const Geometry& g, const v
     b.Hb = plan->xs_hb;
     b.Wb = plan->xs_wb;
     b.pimg = plan->xs_pimg;
+    b.x_total = g.n * g.c * g.h * g.w;
+    b.xs_total = g.n * (long long)(plan->xs_cs / 8) * plan->xs_pimg * 8;
+    b.status = device_status_ptr();
     // without channel pruning the kept channels are 0 .. C-1: the pass then
     // reads nothing sadmm_pack writes (it may overlap the layer's pack)
     const int* chan = plan->colkind == SADMM_COL_CHANNEL
@@ -397,6 +407,7 @@ sadmm_status launch_conv_slab(const sadmm_plan* plan, const Geometry& g, const v
     a.zeromap = reinterpret_cast<const int*>(base + plan->off_zeromap);
     a.counts = reinterpret_cast<const int*>(base + plan->off_counts);
     a.status = device_status_ptr();
+    a.y_total = g.n * g.f * g.plane;
     a.F = (int)g.f;
     a.OH = (int)g.oh;
     a.OW = (int)g.ow;

@@ -146,6 +146,8 @@ struct SparseConvArgs {
     int T, H, W, KT, KH, KW, st, sh, sw, pt, ph, pw, split;
     long long x_chw, thw;
     int hw, relu;
+    long long x_total, y_total;  // elements of x and y (the debug build's index checks)
+    int* status;
 };
 
 template <bool OUT_BF16>
@@ -168,7 +170,7 @@ __global__ void __launch_bounds__(kSparseThreads) k_sparse_conv(const SparseConv
     for (int e = e0; e < e1; ++e) {
         const int4 t = __ldg(a.entries + e);
         const uint32_t bits = (uint32_t)t.y;
-        if ((M & bits) == bits) {
+        if ((M & bits) == bits && dbg_in(xb + t.x - a.x, a.x_total, a.status)) {
             const float xv = __uint_as_float((uint32_t)__ldg(xb + t.x) << 16);
             acc = fmaf(__int_as_float(t.z), xv, acc);
         }
@@ -176,6 +178,7 @@ __global__ void __launch_bounds__(kSparseThreads) k_sparse_conv(const SparseConv
     float v = acc + (a.bias ? __ldg(a.bias + f) : 0.0f);
     if (a.relu) v = fmaxf(v, 0.0f);
     const long long off = ((long long)n * a.F + f) * a.plane + pix;
+    if (!dbg_in(off, a.y_total, a.status)) return;
     if (OUT_BF16)
         reinterpret_cast<__nv_bfloat16*>(a.y)[off] = __float2bfloat16_rn(v);
     else
@@ -258,6 +261,9 @@ sadmm_status launch_sparse_conv(const Geometry& g, const void* buf, const void* 
     a.x_chw = g.c * g.t * g.h * g.w;
     a.thw = g.t * g.h * g.w;
     a.hw = (int)(g.h * g.w);
+    a.x_total = g.n * g.c * g.t * g.h * g.w;
+    a.y_total = g.n * g.f * g.plane;
+    a.status = device_status_ptr();
     a.relu = relu ? 1 : 0;
     if (g.f > 65535) return SADMM_EUNSUPPORTED;
     const dim3 grid((unsigned)((g.m + kSparseThreads - 1) / kSparseThreads), (unsigned)g.f);

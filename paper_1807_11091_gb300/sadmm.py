@@ -16,7 +16,7 @@ from typing import Optional, Sequence, Tuple
 
 from . import build as _build
 
-SADMM_OK, SADMM_EINVAL, SADMM_ECUDA, SADMM_ETIMEOUT, SADMM_EUNSUPPORTED = 0, -1, -2, -3, -4
+SADMM_OK, SADMM_EINVAL, SADMM_ECUDA, SADMM_ETIMEOUT, SADMM_EUNSUPPORTED, SADMM_EBOUNDS = 0, -1, -2, -3, -4, -5
 SADMM_BF16, SADMM_FP32 = 0, 1
 SADMM_COL_NONE, SADMM_COL_SHAPE, SADMM_COL_CHANNEL = 0, 1, 2
 SADMM_FWD_ALL, SADMM_FWD_INPUT, SADMM_FWD_REST = 0, 1, 2
@@ -103,7 +103,8 @@ _lib = None
 
 
 def library_path() -> str:
-    return _build.LIB
+    """The library load() uses: the debug build when SADMM_DEBUG=1 is set."""
+    return _build.DEBUG_LIB if _build.debug_requested() else _build.LIB
 
 
 def load():

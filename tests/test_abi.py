@@ -33,7 +33,7 @@ def test_library_exports_every_declared_entry_point():
 
 
 def test_struct_layout_and_version():
-    assert sadmm.sadmm_abi_version() == 5
+    assert sadmm.sadmm_abi_version() == 6
     assert sadmm.sadmm_plan_struct_size() == ctypes.sizeof(sadmm.Plan)
     assert sadmm.sadmm_status_string(-1) == "invalid argument"
 
