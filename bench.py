@@ -743,14 +743,28 @@ def projection_batch_report(dev, peak_gbs, reps=5):
     singles = [sadmm.ProjectBatch([a]) for a in args]  # the same work as 16 separate calls
     t_batch = timed(lambda: pb())
     t_each = timed(lambda: [p() for p in singles])
+    # the 16 packs (sadmm_pack_batch vs 16 sadmm_pack calls) of the lists just
+    # made; algorithmic bytes: the kept weights read, the packed matrices written
+    convs, pbytes = [], 0
+    for L, W, (fi, ci, _) in zip(layers, Ws, pb.outs):
+        s = L.shape
+        pc = sadmm.PrunedConv(s.desc16(), W, fi, L.colkind, ci, L.k_filters, L.k_cols)
+        convs.append((pc, W, fi, ci))
+        pbytes += 2 * L.k_filters * pc.plan.n_cols + 2 * s.groups * pc.plan.n_pad * pc.plan.k_pad
+    t_pack = timed(lambda: sadmm.pack_batch(convs))
+    t_pack_each = timed(lambda: [pc.repack(W, fi, ci) for pc, W, fi, ci in convs])
     if sadmm.device_status() != 0:
-        raise RuntimeError("device status set after the projections")
-    del flush, Ws, pb, singles
+        raise RuntimeError("device status set after the projections and packs")
+    del flush, Ws, pb, singles, convs
     torch.cuda.empty_cache()
     gbs = nbytes / (t_batch * 1e-3) / 1e9
+    pgbs = pbytes / (t_pack * 1e-3) / 1e9
     return {"what": "projection of the 16 ResNet-50 bottleneck layers (bf16 W), one batched call vs 16 calls",
             "batch_us": t_batch * 1e3, "separate_us": t_each * 1e3, "bytes": nbytes, "batch_gbs": gbs,
-            "batch_hbm_frac": gbs / peak_gbs if peak_gbs else None}
+            "batch_hbm_frac": gbs / peak_gbs if peak_gbs else None,
+            "pack": {"what": "sadmm_pack of the same 16 layers: one sadmm_pack_batch call vs 16 sadmm_pack calls",
+                     "batch_us": t_pack * 1e3, "separate_us": t_pack_each * 1e3, "bytes": pbytes,
+                     "batch_gbs": pgbs, "batch_hbm_frac": pgbs / peak_gbs if peak_gbs else None}}
 
 
 def batch1_report(dev, out_dtype, reps=7):

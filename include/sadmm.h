@@ -406,6 +406,24 @@ sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt,
                         void* dev, size_t dev_bytes, void* stream);
 
 /*
+ * sadmm_pack for a batch of layers (1 .. SADMM_MAX_BATCH items, one plan each,
+ * every W of type wdt): the same plans, buffers, descriptors and device checks
+ * as n sadmm_pack calls, with two kernel launches for the whole batch (the
+ * meta data of every layer, then the packed rows of every layer).  Each item's
+ * fields are as the arguments of sadmm_pack; a bad item returns SADMM_EINVAL
+ * and enqueues nothing.
+ */
+typedef struct {
+    sadmm_plan* plan;
+    const void* W;
+    const int* filt_idx;
+    const int* col_idx;
+    void* dev;
+    size_t dev_bytes;
+} sadmm_pack_item;
+sadmm_status sadmm_pack_batch(sadmm_pack_item* items, int n, int wdt, void* stream);
+
+/*
  * Pruned CONV forward (Sec. 3: the pruned layer is a smaller full GEMM):
  *   y[n, f, o] = ReLU(bias[f] + sum_{j < K'} Wp[f][j] * x[n, g*Cg + c_j,
  *                ot*st-pt+kt_j, oh*sh-ph+kh_j, ow*sw-pw+kw_j])   f kept,

@@ -483,29 +483,60 @@ sadmm_status sadmm_plan_init_ctas(sadmm_plan* plan, const sadmm_conv_desc* d, in
     return SADMM_OK;
 }
 
-sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt, const int* filt_idx, const int* col_idx,
-                        void* dev, size_t dev_bytes, void* stream)
+namespace {
+
+// The host checks of one layer of sadmm_pack / sadmm_pack_batch.
+sadmm_status check_pack(const sadmm_plan* plan, const void* W, int wdt, const int* filt_idx, const int* col_idx,
+                        const void* dev, size_t dev_bytes, Geometry* g)
 {
-    NvtxRange range("sadmm_pack");
     if (!plan || !W || !dev) return SADMM_EINVAL;
-    Geometry g;
-    sadmm_status st = check_desc(&plan->desc, &g);
+    sadmm_status st = check_desc(&plan->desc, g);
     if (st != SADMM_OK) return st;
     if (wdt != SADMM_BF16 && wdt != SADMM_FP32) return SADMM_EINVAL;
     if (dev_bytes < plan->dev_bytes) return SADMM_EINVAL;
     if ((reinterpret_cast<uintptr_t>(dev) & 255) != 0) return SADMM_EINVAL;
-    if (plan->n_filt < (int)g.f && plan->n_filt > 0 && !filt_idx) return SADMM_EINVAL;
+    if (plan->n_filt < (int)g->f && plan->n_filt > 0 && !filt_idx) return SADMM_EINVAL;
     if (plan->colkind != SADMM_COL_NONE && plan->n_colgroups > 0 && !col_idx) return SADMM_EINVAL;
+    return SADMM_OK;
+}
+
+}  // namespace
+
+sadmm_status sadmm_pack(sadmm_plan* plan, const void* W, int wdt, const int* filt_idx, const int* col_idx,
+                        void* dev, size_t dev_bytes, void* stream)
+{
+    NvtxRange range("sadmm_pack");
+    PackJob job;
+    sadmm_status st = check_pack(plan, W, wdt, filt_idx, col_idx, dev, dev_bytes, &job.g);
+    if (st != SADMM_OK) return st;
     if (device_cc_major() < 10) return SADMM_EUNSUPPORTED;
     plan->dev = dev;
-    st = launch_pack(plan, g, W, wdt, filt_idx, col_idx, static_cast<cudaStream_t>(stream));
-    if (st != SADMM_OK) return st;
-    // stream-K arrival counters start at zero (each launch leaves them so)
-    if (plan->sk_len > 0 &&
-        cudaMemsetAsync(static_cast<char*>(dev) + plan->off_sk, 0, (size_t)plan->sk_grid * 4,
-                        static_cast<cudaStream_t>(stream)) != cudaSuccess)
-        return SADMM_ECUDA;
-    return SADMM_OK;
+    job.plan = plan;
+    job.W = W;
+    job.filt_idx = filt_idx;
+    job.col_idx = col_idx;
+    return launch_pack_batch(&job, 1, wdt, static_cast<cudaStream_t>(stream));
+}
+
+sadmm_status sadmm_pack_batch(sadmm_pack_item* items, int n, int wdt, void* stream)
+{
+    NvtxRange range("sadmm_pack_batch");
+    if (!items || n < 1 || n > SADMM_MAX_BATCH) return SADMM_EINVAL;
+    PackJob jobs[SADMM_MAX_BATCH];
+    for (int i = 0; i < n; ++i) {
+        const sadmm_pack_item& it = items[i];
+        sadmm_status st = check_pack(it.plan, it.W, wdt, it.filt_idx, it.col_idx, it.dev, it.dev_bytes, &jobs[i].g);
+        if (st != SADMM_OK) return st;
+        for (int j = 0; j < i; ++j)
+            if (items[j].plan == it.plan) return SADMM_EINVAL;  // one plan per item
+        jobs[i].plan = it.plan;
+        jobs[i].W = it.W;
+        jobs[i].filt_idx = it.filt_idx;
+        jobs[i].col_idx = it.col_idx;
+    }
+    if (device_cc_major() < 10) return SADMM_EUNSUPPORTED;
+    for (int i = 0; i < n; ++i) items[i].plan->dev = items[i].dev;
+    return launch_pack_batch(jobs, n, wdt, static_cast<cudaStream_t>(stream));
 }
 
 sadmm_status sadmm_conv_fwd_phase(const sadmm_plan* plan, const void* x, const float* bias, int relu, void* y,

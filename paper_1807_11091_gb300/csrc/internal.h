@@ -133,8 +133,18 @@ sadmm_status launch_wgrad_slab(const sadmm_plan* plan, const Geometry& g, const 
                                const void* y, int ydt, int relu, float* dW, void* ws, cudaStream_t s);
 
 // ---- pack (pack.cu) ----
-sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* filt_idx,
-                         const int* col_idx, cudaStream_t s);
+// One layer of a pack launch: its plan (dev bound), geometry, weights and
+// index lists (validated on the host as for sadmm_pack).
+struct PackJob {
+    sadmm_plan* plan;
+    Geometry g;
+    const void* W;
+    const int* filt_idx;
+    const int* col_idx;
+};
+// Packs n layers (1 .. kMaxBatch) with two kernel launches, then encodes each
+// plan's TMA descriptors on the host.
+sadmm_status launch_pack_batch(const PackJob* jobs, int n, int wdt, cudaStream_t s);
 
 // TMA descriptors of a slab plan's weights and space-to-depth input (host only).
 sadmm_status launch_pack_slab(sadmm_plan* plan, const Geometry& g);

@@ -3,11 +3,15 @@
 // pruning and channel-/shape-wise sparsity is column pruning; what remains is a
 // smaller full matrix).
 //
-//   k_pack_meta  one block: per conv group the kept and pruned filter lists and
-//                counts, the kept-column list and the gather table (channel
-//                offset of each kept column in x plus its tap bits).
-//   k_pack_wp    one block per packed row: Wp[g][i][j] = bf16(W[f_i][col_j]),
-//                zero outside the kept counts, 16-byte stores.
+//   k_pack_meta  one block per layer: per conv group the kept and pruned
+//                filter lists and counts, the kept-column list and the gather
+//                table (channel offset of each kept column in x plus its tap
+//                bits); it also zeroes the plan's stream-K arrival counters.
+//   k_pack_wp    one block per packed row of every layer:
+//                Wp[g][i][j] = bf16(W[f_i][col_j]), zero outside the kept
+//                counts, 16-byte stores.
+// A call packs a batch of layers (sadmm_pack_batch; sadmm_pack is the batch of
+// one): two launches whatever the batch size.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <string.h>
@@ -38,6 +42,33 @@ struct PackArgs {
     int* scol;   // [xs_kpad] slab column -> GEMM column (-1: zero)
     int* chan;   // [xs_cs] kept input channels (-1 past them)
     int C, xs_cs, xs_kpad, xs_r, xs_q, sh, sw;
+    int* skcnt;         // stream-K arrival counters, zeroed here
+    int sk_n;
+    int lists_in_smem;  // 1: the filter and column lists are staged in shared memory
+};
+
+// The layers of one pack launch, in kernel parameter space.
+template <int N>
+struct PackBatch {
+    PackArgs L[N];
+};
+
+// One layer's rows for k_pack_wp: blocks first .. first + rows + srows - 1.
+struct WpLayer {
+    const void* W;
+    const int* rowmap;
+    const int* colidx;
+    const int* scol;
+    __nv_bfloat16* wp;
+    __nv_bfloat16* wps;
+    long long rows, first;
+    int K, k_pad, kpad_s;
+};
+
+template <int N>
+struct WpBatch {
+    WpLayer L[N];
+    int n;
 };
 
 // First position p in the ascending list a[0..n) with a[p] >= v.
@@ -54,14 +85,14 @@ SADMM_DEV int lower_bound(const int* a, int n, int v)
 
 // Dynamic shared memory (when the host passes enough): the filter and column
 // lists, so the binary searches below read shared memory, not HBM.
-__global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status, int lists_in_smem)
+SADMM_DEV void pack_meta(PackArgs a, int* status)
 {
-    pdl_wait();  // after the kernel before it in the stream
     __shared__ int s_start[65];
     __shared__ int s_bad;
     extern __shared__ int s_lists[];
     const int tid = threadIdx.x;
-    if (lists_in_smem) {
+    for (int i = tid; i < a.sk_n; i += blockDim.x) a.skcnt[i] = 0;
+    if (a.lists_in_smem) {
         int* fl = s_lists;
         int* cl = s_lists + (a.all_kept ? 0 : a.n_filt);
         if (!a.all_kept)
@@ -191,6 +222,14 @@ __global__ void __launch_bounds__(1024) k_pack_meta(PackArgs a, int* status, int
     }
 }
 
+// Block b packs the meta data of layer b of the batch.
+template <int N>
+__global__ void __launch_bounds__(1024) k_pack_meta(const __grid_constant__ PackBatch<N> pb, int* status)
+{
+    pdl_wait();  // after the kernel before it in the stream
+    pack_meta(pb.L[blockIdx.x], status);
+}
+
 template <typename T>
 SADMM_DEV float load_f32(const T* p);
 template <>
@@ -198,23 +237,22 @@ SADMM_DEV float load_f32<__nv_bfloat16>(const __nv_bfloat16* p) { return __bfloa
 template <>
 SADMM_DEV float load_f32<float>(const float* p) { return *p; }
 
-// Blocks past `rows` pack the input-slab plan's weights: row r - rows of
-// conv group 0 through the slab column map scol, into wps [bn][kpad_s].
+// Row r of a layer: rows past `rows` pack the input-slab plan's weights, row
+// r - rows of conv group 0 through the slab column map scol, into wps [bn][kpad_s].
 template <typename T>
-__global__ void __launch_bounds__(128) k_pack_wp(const T* __restrict__ W, int K, const int* __restrict__ rowmap,
-                                                 const int* __restrict__ colidx, int k_pad,
-                                                 __nv_bfloat16* __restrict__ wp, long long rows,
-                                                 const int* __restrict__ scol, int kpad_s, __nv_bfloat16* wps)
+SADMM_DEV void pack_wp_row(const WpLayer& L, long long r)
 {
-    pdl_wait();  // after the kernel before it in the stream
-    long long r = blockIdx.x;
-    if (r >= rows) {
-        r -= rows;
-        colidx = scol;
-        k_pad = kpad_s;
-        wp = wps;
+    const T* W = static_cast<const T*>(L.W);
+    const int* colidx = L.colidx;
+    int k_pad = L.k_pad;
+    __nv_bfloat16* wp = L.wp;
+    if (r >= L.rows) {
+        r -= L.rows;
+        colidx = L.scol;
+        k_pad = L.kpad_s;
+        wp = L.wps;
     }
-    const int f = rowmap[r];
+    const int f = L.rowmap[r];
     uint4* dst = reinterpret_cast<uint4*>(wp + r * k_pad);
     for (int j8 = threadIdx.x; j8 < k_pad / 8; j8 += blockDim.x) {
         uint32_t w[4];
@@ -222,13 +260,28 @@ __global__ void __launch_bounds__(128) k_pack_wp(const T* __restrict__ W, int K,
         for (int e = 0; e < 4; ++e) {
             const int j0 = j8 * 8 + 2 * e;
             const int c0 = colidx[j0], c1 = colidx[j0 + 1];
-            const float v0 = (f >= 0 && c0 >= 0) ? load_f32<T>(W + (long long)f * K + c0) : 0.0f;
-            const float v1 = (f >= 0 && c1 >= 0) ? load_f32<T>(W + (long long)f * K + c1) : 0.0f;
+            const float v0 = (f >= 0 && c0 >= 0) ? load_f32<T>(W + (long long)f * L.K + c0) : 0.0f;
+            const float v1 = (f >= 0 && c1 >= 0) ? load_f32<T>(W + (long long)f * L.K + c1) : 0.0f;
             const __nv_bfloat162 p = __floats2bfloat162_rn(v0, v1);  // .x = v0 (low half)
             w[e] = *reinterpret_cast<const uint32_t*>(&p);
         }
         dst[j8] = make_uint4(w[0], w[1], w[2], w[3]);
     }
+}
+
+// Block b packs one row of the layer whose block range holds b.
+template <typename T, int N>
+__global__ void __launch_bounds__(128) k_pack_wp(const __grid_constant__ WpBatch<N> wb)
+{
+    pdl_wait();  // after the kernel before it in the stream
+    const long long b = blockIdx.x;
+    int lo = 0, hi = wb.n - 1;
+    while (lo < hi) {  // the last layer whose first block is <= b
+        const int mid = (lo + hi + 1) >> 1;
+        if (wb.L[mid].first <= b) lo = mid;
+        else hi = mid - 1;
+    }
+    pack_wp_row<T>(wb.L[lo], b - wb.L[lo].first);
 }
 
 }  // namespace
@@ -248,11 +301,14 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn()
     return fn;
 }
 
-sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int wdt, const int* filt_idx,
-                         const int* col_idx, cudaStream_t s)
+namespace {
+
+// The kernel arguments of one layer's meta data (plan->dev bound).
+PackArgs pack_args(const sadmm_plan* plan, const Geometry& g, const int* filt_idx, const int* col_idx)
 {
     char* base = static_cast<char*>(plan->dev);
     PackArgs a;
+    memset(&a, 0, sizeof(a));
     a.all_kept = (plan->n_filt == (int)g.f) ? 1 : 0;
     a.filt_idx = a.all_kept ? nullptr : filt_idx;
     a.col_idx = col_idx;
@@ -280,8 +336,6 @@ sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int
     a.rowmap = reinterpret_cast<int*>(base + plan->off_rowmap);
     a.zeromap = reinterpret_cast<int*>(base + plan->off_zeromap);
     a.counts = reinterpret_cast<int*>(base + plan->off_counts);
-    a.scol = nullptr;
-    a.chan = nullptr;
     a.C = (int)g.c;
     if (plan->xs_mode) {
         a.scol = reinterpret_cast<int*>(base + plan->off_scol);
@@ -293,29 +347,31 @@ sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int
         a.sh = (int)g.sh;
         a.sw = (int)g.sw;
     }
-    const size_t list_bytes =
-        (size_t)((a.all_kept ? 0 : a.n_filt) + ((col_idx && a.colkind != SADMM_COL_NONE) ? a.n_colgroups : 0)) * 4;
-    const bool in_smem = list_bytes <= 40 * 1024;
-    launch_pdl(k_pack_meta, dim3(1), dim3(1024), in_smem ? list_bytes : 0, s, a, device_status_ptr(),
-               in_smem ? 1 : 0);
+    if (plan->sk_len > 0) {
+        a.skcnt = reinterpret_cast<int*>(base + plan->off_sk);
+        a.sk_n = plan->sk_grid;
+    }
+    return a;
+}
 
-    __nv_bfloat16* wp = reinterpret_cast<__nv_bfloat16*>(base + plan->off_wp);
-    const unsigned rows = (unsigned)(g.groups * plan->n_pad);
-    // a slab plan also packs its weights in slab column order, in the same launch
-    __nv_bfloat16* wps = plan->xs_mode ? reinterpret_cast<__nv_bfloat16*>(base + plan->off_wps) : nullptr;
-    const unsigned srows = plan->xs_mode ? (unsigned)plan->bn : 0u;
-    if (wdt == SADMM_BF16)
-        launch_pdl(k_pack_wp<__nv_bfloat16>, dim3(rows + srows), dim3(128), 0, s, (const __nv_bfloat16*)W, (int)g.k,
-                   a.rowmap, a.colidx, plan->k_pad, wp, (long long)rows, (const int*)a.scol, plan->xs_kpad, wps);
-    else
-        launch_pdl(k_pack_wp<float>, dim3(rows + srows), dim3(128), 0, s, (const float*)W, (int)g.k, a.rowmap,
-                   a.colidx, plan->k_pad, wp, (long long)rows, (const int*)a.scol, plan->xs_kpad, wps);
-    if (cudaGetLastError() != cudaSuccess) return SADMM_ECUDA;
+// Bytes of the filter and column lists k_pack_meta stages in shared memory.
+size_t list_bytes(const PackArgs& a)
+{
+    return (size_t)((a.all_kept ? 0 : a.n_filt) + ((a.col_idx && a.colkind != SADMM_COL_NONE) ? a.n_colgroups : 0)) *
+           4;
+}
 
-    // TMA descriptor of Wp: [groups*n_pad rows][k_pad bf16], boxes of 64 x bn,
-    // 128-byte swizzle (the layout the tensor-core operand descriptor expects).
+constexpr size_t kListSmemCap = 40 * 1024;
+
+// TMA descriptor of Wp: [groups*n_pad rows][k_pad bf16], boxes of 64 x bn,
+// 128-byte swizzle (the layout the tensor-core operand descriptor expects);
+// then those of a slab plan.
+sadmm_status encode_maps(sadmm_plan* plan, const Geometry& g)
+{
     PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
     if (!enc) return SADMM_ECUDA;
+    __nv_bfloat16* wp = reinterpret_cast<__nv_bfloat16*>(static_cast<char*>(plan->dev) + plan->off_wp);
+    const unsigned rows = (unsigned)(g.groups * plan->n_pad);
     alignas(64) CUtensorMap map;
     memset(&map, 0, sizeof(map));
     const cuuint64_t gdim[2] = {(cuuint64_t)plan->k_pad, (cuuint64_t)rows};
@@ -330,6 +386,64 @@ sadmm_status launch_pack(sadmm_plan* plan, const Geometry& g, const void* W, int
     memcpy(plan->tmap, &map, sizeof(map));
     if (plan->xs_mode) return launch_pack_slab(plan, g);
     return SADMM_OK;
+}
+
+template <int N>
+sadmm_status launch_batch(const PackJob* jobs, int n, int wdt, cudaStream_t s)
+{
+    PackBatch<N> pb;
+    WpBatch<N> wb;
+    memset(&pb, 0, sizeof(pb));
+    memset(&wb, 0, sizeof(wb));
+    size_t smem = 0;
+    for (int i = 0; i < n; ++i) {
+        pb.L[i] = pack_args(jobs[i].plan, jobs[i].g, jobs[i].filt_idx, jobs[i].col_idx);
+        const size_t lb = list_bytes(pb.L[i]);
+        if (lb <= kListSmemCap && lb > smem) smem = lb;
+    }
+    for (int i = 0; i < n; ++i) pb.L[i].lists_in_smem = list_bytes(pb.L[i]) <= smem ? 1 : 0;
+    if (launch_pdl(k_pack_meta<N>, dim3((unsigned)n), dim3(1024), smem, s, pb, device_status_ptr()) != cudaSuccess)
+        return SADMM_ECUDA;
+    long long blocks = 0;
+    for (int i = 0; i < n; ++i) {
+        const sadmm_plan* plan = jobs[i].plan;
+        const Geometry& g = jobs[i].g;
+        char* base = static_cast<char*>(plan->dev);
+        WpLayer& L = wb.L[i];
+        L.W = jobs[i].W;
+        L.K = (int)g.k;
+        L.rowmap = pb.L[i].rowmap;
+        L.colidx = pb.L[i].colidx;
+        L.k_pad = plan->k_pad;
+        L.wp = reinterpret_cast<__nv_bfloat16*>(base + plan->off_wp);
+        L.rows = g.groups * plan->n_pad;
+        // a slab plan also packs its weights in slab column order, in the same launch
+        L.scol = pb.L[i].scol;
+        L.kpad_s = plan->xs_kpad;
+        L.wps = plan->xs_mode ? reinterpret_cast<__nv_bfloat16*>(base + plan->off_wps) : nullptr;
+        L.first = blocks;
+        blocks += L.rows + (plan->xs_mode ? plan->bn : 0);
+    }
+    wb.n = n;
+    if (blocks >= (1ll << 31)) return SADMM_EUNSUPPORTED;
+    const cudaError_t e =
+        (wdt == SADMM_BF16)
+            ? launch_pdl(k_pack_wp<__nv_bfloat16, N>, dim3((unsigned)blocks), dim3(128), 0, s, wb)
+            : launch_pdl(k_pack_wp<float, N>, dim3((unsigned)blocks), dim3(128), 0, s, wb);
+    if (e != cudaSuccess || cudaGetLastError() != cudaSuccess) return SADMM_ECUDA;
+    for (int i = 0; i < n; ++i) {
+        const sadmm_status st = encode_maps(jobs[i].plan, jobs[i].g);
+        if (st != SADMM_OK) return st;
+    }
+    return SADMM_OK;
+}
+
+}  // namespace
+
+sadmm_status launch_pack_batch(const PackJob* jobs, int n, int wdt, cudaStream_t s)
+{
+    if (n < 1 || n > kMaxBatch) return SADMM_EINVAL;
+    return n == 1 ? launch_batch<1>(jobs, n, wdt, s) : launch_batch<kMaxBatch>(jobs, n, wdt, s);
 }
 
 sadmm_status launch_pack_slab(sadmm_plan* plan, const Geometry& g)

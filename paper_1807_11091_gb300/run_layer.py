@@ -40,9 +40,14 @@ def main(argv=None) -> int:
     ap.add_argument("--batch-all", action="store_true",
                     help="with --admm: one sadmm_admm_update_batch over every layer of the workload; alone: one "
                          "sadmm_project_groups_batch over every layer (bf16 W)")
+    ap.add_argument("--pack-all", action="store_true",
+                    help="sadmm_pack of every layer of the workload (after one batched projection), `reps` times "
+                         "as separate calls and as one sadmm_pack_batch call")
     ap.add_argument("--sparse", type=float, default=0.0,
                     help="time sadmm_sparse_conv_fwd with the layer pruned element by element to this density")
     args = ap.parse_args(argv)
+    if args.pack_all:
+        return run_pack_all(args)
     if args.batch_all:
         return run_batch_all(args)
     if args.sparse > 0:
@@ -163,6 +168,49 @@ def run_batch_all(args) -> int:
         e1.record()
         torch.cuda.synchronize()
         print(f"{args.workload} {what} of {len(layers)} layers run {i}: {e0.elapsed_time(e1) * 1e3:.1f} us")
+    return 1 if sadmm.device_status() != 0 else 0
+
+
+def run_pack_all(args) -> int:
+    """sadmm_pack of every layer of the workload (bf16 W; the index lists from one
+    batched projection), `reps` times as separate calls, then `reps` times as one
+    sadmm_pack_batch call; prints the time of all packs and their algorithmic
+    bytes (the kept weights read, the packed matrices written)."""
+    import torch
+
+    import workloads as wl
+    from paper_1807_11091_gb300 import sadmm
+
+    layers = wl.get(args.workload)
+    dev = torch.device("cuda", 0)
+    Ws = [wl.gen_tensors(L.shape.with_batch(1), seed=L.seed)["W"].to(dev) for L in layers]
+    pb = sadmm.ProjectBatch([(L.shape.desc16(), W, L.k_filters, L.colkind, L.k_cols, None)
+                             for L, W in zip(layers, Ws)])
+    lists = pb()
+    pcs = []
+    nbytes = 0
+    for L, W, (fi, ci, _) in zip(layers, Ws, lists):
+        s = L.shape
+        pc = sadmm.PrunedConv(s.desc16(), W, fi if L.k_filters < s.f else None, L.colkind,
+                              ci if L.colkind != wl.COL_NONE else None, L.k_filters,
+                              L.k_cols if L.colkind != wl.COL_NONE else s.k)
+        pcs.append((pc, W, fi if L.k_filters < s.f else None, ci if L.colkind != wl.COL_NONE else None))
+        kc = pc.plan.n_cols
+        nbytes += L.k_filters * kc * 2 + s.groups * pc.plan.n_pad * pc.plan.k_pad * 2
+    torch.cuda.synchronize()
+    for what, fn in (("separate calls", lambda: [pc.repack(W, fi, ci) for pc, W, fi, ci in pcs]),
+                     ("one batched call", lambda: sadmm.pack_batch(pcs))):
+        for i in range(args.reps):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            torch.cuda._sleep(1_000_000)
+            e0.record()
+            fn()
+            e1.record()
+            torch.cuda.synchronize()
+            us = e0.elapsed_time(e1) * 1e3
+            print(f"{args.workload} pack of {len(layers)} layers, {what}, run {i}: {us:.1f} us, "
+                  f"{nbytes / 1e6:.2f} MB ({nbytes / us / 1e3:.0f} GB/s)")
     return 1 if sadmm.device_status() != 0 else 0
 
 

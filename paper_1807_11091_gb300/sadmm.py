@@ -99,6 +99,12 @@ class Plan(ctypes.Structure):
     ]
 
 
+class PackItem(ctypes.Structure):
+    """sadmm_pack_item: one layer of sadmm_pack_batch."""
+    _fields_ = [("plan", ctypes.POINTER(Plan)), ("W", ctypes.c_void_p), ("filt_idx", ctypes.c_void_p),
+                ("col_idx", ctypes.c_void_p), ("dev", ctypes.c_void_p), ("dev_bytes", ctypes.c_size_t)]
+
+
 _lib = None
 
 
@@ -132,6 +138,8 @@ def load():
     lib.sadmm_plan_init_ctas.argtypes = [P(Plan), P(ConvDesc), ci, ci, ci, ci]
     lib.sadmm_pack.restype = ci
     lib.sadmm_pack.argtypes = [P(Plan), vp, ci, vp, vp, vp, sz, vp]
+    lib.sadmm_pack_batch.restype = ci
+    lib.sadmm_pack_batch.argtypes = [P(PackItem), ci, ci, vp]
     lib.sadmm_conv_fwd_phase.restype = ci
     lib.sadmm_conv_fwd_phase.argtypes = [P(Plan), vp, vp, ci, vp, ci, ci, vp]
     lib.sadmm_conv_fwd.restype = ci
@@ -314,6 +322,11 @@ def sadmm_last_device_status(stream: Optional[int]) -> int:
 def sadmm_project_groups_batch(items: Sequence[ProjectItem], wdt: int, stream: Optional[int]) -> int:
     arr = (ProjectItem * len(items))(*items)
     return load().sadmm_project_groups_batch(arr, len(items), int(wdt), stream)
+
+
+def sadmm_pack_batch(items: Sequence[PackItem], wdt: int, stream: Optional[int]) -> int:
+    arr = (PackItem * len(items))(*items)
+    return load().sadmm_pack_batch(arr, len(items), int(wdt), stream)
 
 
 def sadmm_admm_update_batch(items: Sequence[AdmmItem], wdt: int, stream: Optional[int]) -> int:
@@ -615,6 +628,15 @@ class PrunedConv:
         st = sadmm_conv_fwd(self.plan, _ptr(x), _ptr(bias), 1 if relu else 0, _ptr(out), ydt, _stream(stream))
         _check(st, "sadmm_conv_fwd")
         return out
+
+
+def pack_batch(convs, stream=None) -> None:
+    """Repacks PrunedConv layers with one sadmm_pack_batch call: convs is a
+    sequence of (PrunedConv, W, filt_idx or None, col_idx or None), every W of
+    one dtype."""
+    items = [PackItem(ctypes.pointer(pc.plan), _ptr(W), _ptr(fi), _ptr(ci), _ptr(pc.buf), pc.plan.dev_bytes)
+             for pc, W, fi, ci in convs]
+    _check(sadmm_pack_batch(items, _wdt(convs[0][1]), _stream(stream)), "sadmm_pack_batch")
 
 
 def device_status(stream=None) -> int:

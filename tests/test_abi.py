@@ -239,3 +239,27 @@ def test_sparse_entry_points_reject_bad_arguments_on_host():
     assert sadmm.sadmm_sparse_conv_fwd(desc, fake, fake, None, 1, fake, 9, None) == sadmm.SADMM_EINVAL
     assert sadmm.sadmm_sparse_conv_fwd(desc, fake + 16, fake, None, 1, fake, 1, None) == sadmm.SADMM_EINVAL
     assert sadmm.sadmm_sparse_conv_fwd(desc, fake, fake, None, 1, fake + 2, 1, None) == sadmm.SADMM_EINVAL
+
+
+def test_pack_batch_rejects_bad_items_on_host():
+    s = wl.single2d()[0].shape
+    st, p = sadmm.sadmm_plan_init(sadmm.make_desc(s.desc16()), s.f, wl.COL_SHAPE, 100)
+    assert st == 0
+    st, q = sadmm.sadmm_plan_init(sadmm.make_desc(s.desc16()), s.f, wl.COL_SHAPE, 100)
+    fake = 1 << 20
+
+    def item(plan, W=fake, col=fake, dev=fake, nbytes=None):
+        return sadmm.PackItem(ctypes.pointer(plan), W, None, col, dev, plan.dev_bytes if nbytes is None else nbytes)
+
+    assert sadmm.sadmm_pack_batch([], 0, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_pack_batch([item(p)], 7, None) == sadmm.SADMM_EINVAL  # no such weight type
+    assert sadmm.sadmm_pack_batch([item(p), item(p)], 0, None) == sadmm.SADMM_EINVAL  # one plan twice
+    assert sadmm.sadmm_pack_batch([item(p), item(q, W=None)], 0, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_pack_batch([item(p), item(q, col=None)], 0, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_pack_batch([item(p), item(q, dev=fake + 8)], 0, None) == sadmm.SADMM_EINVAL
+    assert sadmm.sadmm_pack_batch([item(p), item(q, nbytes=q.dev_bytes - 1)], 0, None) == sadmm.SADMM_EINVAL
+    plans = [sadmm.sadmm_plan_init(sadmm.make_desc(s.desc16()), s.f, wl.COL_SHAPE, 100)[1]
+             for _ in range(sadmm.SADMM_MAX_BATCH + 1)]
+    assert sadmm.sadmm_pack_batch([item(pl) for pl in plans], 0, None) == sadmm.SADMM_EINVAL
+    # nothing was bound: every rejected call enqueues nothing
+    assert not p.dev and not q.dev

@@ -96,3 +96,52 @@ def test_batch_rejects_bad_items():
         sadmm.project_groups_batch([good, bad])
     with pytest.raises(sadmm.SadmmError):
         sadmm.project_groups_batch([good] * (sadmm.SADMM_MAX_BATCH + 1))
+
+
+def _pack_layers():
+    """Plans of every kind: gathered shape-wise, channel-wise, grouped, 3-D,
+    filters only, kept whole on the input-slab path, split K' (batch 1) and
+    stream-K (AlexNet CONV3 at batch 128)."""
+    return [wl.Layer("first", wl.alexnet()[0].shape.with_batch(2), 1.0, wl.COL_SHAPE, 1.0, seed=100),
+            wl.Layer("conv2_b3", wl.alexnet()[1].shape.with_batch(3), 0.5, wl.COL_SHAPE, 0.5, seed=101),
+            wl.alexnet()[2],
+            wl.Layer("conv4_b1", wl.alexnet()[3].shape.with_batch(1), 0.2, wl.COL_SHAPE, 0.2, seed=103),
+            wl.resnet50()[3], wl.resnet50()[6], wl.c3d()[0], wl.single2d()[0],
+            wl.Layer("filters_only", wl.alexnet()[4].shape.with_batch(4), 0.3, wl.COL_NONE, 1.0, seed=3)]
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_batched_pack_equals_per_layer_packs(dtype):
+    """sadmm_pack_batch gives each plan the packed weights, tables and forward
+    output that its own sadmm_pack gives, bit for bit."""
+    from paper_1807_11091_gb300 import sadmm
+    dev = torch.device("cuda", 0)
+    layers = _pack_layers()
+    one, batch, tensors = [], [], []
+    for L in layers:
+        s = L.shape
+        t = wl.gen_tensors(s, seed=L.seed)
+        W = t["W"].to(dev).to(dtype)
+        fi, ci, _ = sadmm.project_groups(s.desc16(), W, L.k_filters, L.colkind, L.k_cols)
+        fi = fi if L.k_filters < s.f else None
+        ci = ci if L.colkind != wl.COL_NONE else None
+        ncg = L.k_cols if L.colkind != wl.COL_NONE else s.k
+        one.append(sadmm.PrunedConv(s.desc16(), W, fi, L.colkind, ci, L.k_filters, ncg))
+        pc = sadmm.PrunedConv(s.desc16(), W, fi, L.colkind, ci, L.k_filters, ncg)
+        pc.buf.zero_()
+        batch.append((pc, W, fi, ci))
+        tensors.append(t)
+    kinds = {(pc.plan.xs_mode, pc.plan.splits > 1, pc.plan.sk_len > 0) for pc, _, _, _ in batch}
+    assert (1, False, False) in kinds and any(k[1] for k in kinds) and any(k[2] for k in kinds), kinds
+    sadmm.pack_batch(batch)
+    for L, a, (b, _, _, _), t in zip(layers, one, batch, tensors):
+        pa, pb = a.plan, b.plan
+        end = pa.off_wp + pa.desc.groups * pa.n_pad * pa.k_pad * 2
+        for lo, hi in ((pa.off_wp, end), (pa.off_gather, pa.off_gather + pa.k_pad * 8),
+                       (pa.off_rowmap, pa.off_rowmap + pa.desc.groups * pa.n_pad * 4),
+                       (pa.off_counts, pa.off_counts + pa.desc.groups * 8),
+                       (pa.off_wps, pa.off_wps + (pa.bn * pa.xs_kpad * 2 if pa.xs_mode else 0))):
+            assert torch.equal(a.buf[lo:hi], b.buf[lo:hi]), (L.name, lo, hi)
+        x, bias = t["x"].to(dev), t["bias"].to(dev)
+        assert torch.equal(a.forward(x, bias), b.forward(x, bias)), L.name
+    assert sadmm.device_status() == 0
