@@ -259,8 +259,8 @@ class LayerRun:
 class StepStreams:
     """One side stream per layer: each layer's projection and pack run on its own
     stream (the layers are independent), forked from and joined back to the main
-    stream, where the convolutions run back to back.  The first layer's side
-    stream has the higher priority (its pack gates the first conv); the first
+    stream (high priority), where the convolutions run back to back.  The first
+    layer's side stream has the main stream's priority (its pack gates the first conv); the first
     conv's plan leaves a few SMs free so the other layers' projection and pack
     run beside it instead of after it."""
 
@@ -984,6 +984,10 @@ def run_gpu(args):
     dev = torch.device("cuda", local)
     from paper_1807_11091_gb300 import sadmm
     sadmm.load()
+    # The forwards run on a high-priority stream: the projections and packs on
+    # the side streams then take the SMs only when the critical path leaves
+    # them (first layer's input pass, the four SMs the first conv leaves free).
+    torch.cuda.set_stream(torch.cuda.Stream(priority=-1))
     stream = torch.cuda.current_stream()
     sp = int(stream.cuda_stream)
 
@@ -1105,7 +1109,7 @@ def run_gpu(args):
         "config": {**workload_config(args, layers),
                    "l2": "flushed before every timed step (256 MiB write, outside the timed window)",
                    "schedule": f"projection+pack of each layer on its own stream; convs back to back on the "
-                               f"main stream; first conv on {first_ctas or n_sm} of {n_sm} SMs, its input-slab "
+                               f"main stream (high priority); first conv on {first_ctas or n_sm} of {n_sm} SMs, its input-slab "
                                f"space-to-depth pass issued at the step's start beside the projections and packs",
                    "breakdown": "per-conv times from separate steps with CUDA events around each whole forward call"},
         "pct_bf16_peak": value / peaks["bf16_tflops"],
