@@ -9,7 +9,9 @@
 // x[n][chan[ci]][hb*sh + a - ph][wb*sw + b - pw], zero outside.  Output pixel
 // (oh, ow) and kernel tap (kh, kw) = (r*sh + a, q*sw + b) read block pixel
 // (oh + r, ow + q), phase (a, b): the layer becomes a stride-1 R x Q conv over
-// cs slab channels (R = ceil(KH/sh), Q = ceil(KW/sw)).
+// cs slab channels (R = ceil(KH/sh), Q = ceil(KW/sw)).  k_slab_input_rows
+// writes the same copy when sw divides 8 (each input row's offset and
+// validity formed once per row, not per element).
 //
 // k_conv_slab: GEMM row i of tile t of image n is block pixel p = 128t + i of
 // that image's output grid laid out in rows of Wb = OW + Q - 1 block pixels
@@ -125,6 +127,77 @@ __global__ void __launch_bounds__(kXsPix * kXsRows) k_slab_input(const __nv_bflo
                     dbg_in(xi - reinterpret_cast<const unsigned short*>(x) + d.x + ih * b.W + iw, b.x_total, b.status))
                        ? (uint32_t)__ldg(xi + d.x + ih * b.W + iw)
                        : 0u;
+        }
+        if (dbg_in(dst0 - xs + (long long)k * b.pimg * 8 + 7, b.xs_total, b.status))
+            *reinterpret_cast<uint4*>(dst0 + (long long)k * b.pimg * 8) =
+                make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16), h[6] | (h[7] << 16));
+    }
+}
+
+// The same copy when the column stride SW divides 8: a chunk's 8 slab
+// channels cc = (ci*sh + a)*SW + b are then 8/SW input rows rho = ci*sh + a
+// (channel chan[ci], row hb*sh + a - ph) of SW consecutive columns
+// wb*SW + b - pw each.  A thread forms each row's offset and validity once
+// and each column's validity once, so an element costs a predicated load at
+// a constant offset from its row (the generic kernel decodes every element).
+// Thread t of block (bx, n) writes block pixel p = 256*bx + t of image n
+// (hb = p / Wb, wb = p % Wb): no lanes idle at the end of a block row.
+constexpr int kXsFlat = 256;  // block pixels per block
+template <int SW>
+__global__ void __launch_bounds__(kXsFlat) k_slab_input_rows(const __nv_bfloat16* __restrict__ x,
+                                                            const int* __restrict__ chan, const XsArgs b,
+                                                            const FastDiv wb_div, __nv_bfloat16* __restrict__ xs)
+{
+    constexpr int kRows = 8 / SW;  // input rows per chunk
+    __shared__ int2 s_row[64];     // per row rho < cs/SW: {channel plane offset (-1: zero), a - ph}
+    pdl_wait();  // after the kernel before it in the stream
+    const int n = blockIdx.y;
+    const int tid = threadIdx.x;
+    if (tid < b.cs / SW) {
+        const int ci = tid / b.sh;
+        const int ch = ci < b.nck ? (chan ? __ldg(chan + ci) : ci) : -1;
+        s_row[tid] = make_int2(ch >= 0 ? ch * b.H * b.W : -1, tid - ci * b.sh - b.ph);
+    }
+    __syncthreads();
+    const int chunks = b.cs / 8;
+    const int npix = b.Hb * b.Wb;
+    if (blockIdx.x == 0) {
+        // the pixels past Hb*Wb up to pimg (fewer than 8 per chunk row) are zero:
+        // they are read by the GEMM rows past the output, and the weight gradient
+        // multiplies them by those rows' zero dZ
+        const int pad = b.pimg - npix;
+        for (int v = tid; v < chunks * pad; v += kXsFlat) {
+            const int k = v / pad, j = v - k * pad;
+            const long long o = (((long long)n * chunks + k) * b.pimg + npix + j) * 8;
+            if (dbg_in(o + 7, b.xs_total, b.status)) *reinterpret_cast<uint4*>(xs + o) = make_uint4(0u, 0u, 0u, 0u);
+        }
+    }
+    const int p = blockIdx.x * kXsFlat + tid;
+    if (p >= npix) return;
+    const int hb = (int)fdiv((uint32_t)p, wb_div);
+    const int wb = p - hb * b.Wb;
+    const int ih0 = hb * b.sh, iw0 = wb * SW - b.pw;
+    bool col_ok[SW];
+#pragma unroll
+    for (int c = 0; c < SW; ++c) col_ok[c] = (unsigned)(iw0 + c) < (unsigned)b.W;
+    const long long img = (long long)n * b.C * b.H * b.W;
+    const unsigned short* xi = reinterpret_cast<const unsigned short*>(x);
+    __nv_bfloat16* dst0 = xs + ((long long)n * chunks * b.pimg + p) * 8;
+#pragma unroll 2
+    for (int k = 0; k < chunks; ++k) {
+        uint32_t h[8];
+#pragma unroll
+        for (int r = 0; r < kRows; ++r) {
+            const int2 s = s_row[k * kRows + r];
+            const int ih = ih0 + s.y;
+            const bool row_ok = s.x >= 0 && (unsigned)ih < (unsigned)b.H;
+            // element offset of column 0 of this row (only read where the row and column are inside x)
+            const long long e0 = img + s.x + (long long)ih * b.W + iw0;
+#pragma unroll
+            for (int c = 0; c < SW; ++c)
+                h[r * SW + c] = (row_ok && col_ok[c] && dbg_in(e0 + c, b.x_total, b.status))
+                                    ? (uint32_t)__ldg(xi + e0 + c)
+                                    : 0u;
         }
         if (dbg_in(dst0 - xs + (long long)k * b.pimg * 8 + 7, b.xs_total, b.status))
             *reinterpret_cast<uint4*>(dst0 + (long long)k * b.pimg * 8) =
@@ -391,12 +464,24 @@ sadmm_status launch_conv_slab(const sadmm_plan* plan, const Geometry& g, const v
                           ? reinterpret_cast<const int*>(base + plan->off_scol) + plan->xs_kpad
                           : nullptr;
     __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(const_cast<char*>(base) + plan->off_xs);
-    if (phase != SADMM_FWD_REST &&
-        launch_pdl(k_slab_input,
-                   dim3((unsigned)((plan->xs_wb + kXsPix - 1) / kXsPix), (unsigned)((plan->xs_hb + kXsRows - 1) / kXsRows),
-                        (unsigned)g.n),
-                   dim3(kXsPix, kXsRows), 0, s, static_cast<const __nv_bfloat16*>(x), chan, b, xs) != cudaSuccess)
-        return SADMM_ECUDA;
+    if (phase != SADMM_FWD_REST) {
+        const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
+        const dim3 flat((unsigned)((plan->xs_hb * plan->xs_wb + kXsFlat - 1) / kXsFlat), (unsigned)g.n);
+        const FastDiv wdiv = make_fastdiv((uint32_t)plan->xs_wb);
+        cudaError_t e;
+        switch (g.sw) {
+        case 1: e = launch_pdl(k_slab_input_rows<1>, flat, dim3(kXsFlat), 0, s, xb, chan, b, wdiv, xs); break;
+        case 2: e = launch_pdl(k_slab_input_rows<2>, flat, dim3(kXsFlat), 0, s, xb, chan, b, wdiv, xs); break;
+        case 4: e = launch_pdl(k_slab_input_rows<4>, flat, dim3(kXsFlat), 0, s, xb, chan, b, wdiv, xs); break;
+        case 8: e = launch_pdl(k_slab_input_rows<8>, flat, dim3(kXsFlat), 0, s, xb, chan, b, wdiv, xs); break;
+        default:
+            e = launch_pdl(k_slab_input,
+                           dim3((unsigned)((plan->xs_wb + kXsPix - 1) / kXsPix),
+                                (unsigned)((plan->xs_hb + kXsRows - 1) / kXsRows), (unsigned)g.n),
+                           dim3(kXsPix, kXsRows), 0, s, xb, chan, b, xs);
+        }
+        if (e != cudaSuccess) return SADMM_ECUDA;
+    }
 
     if (phase == SADMM_FWD_INPUT) return cudaGetLastError() == cudaSuccess ? SADMM_OK : SADMM_ECUDA;
     SlabArgs a;

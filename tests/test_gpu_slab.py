@@ -40,6 +40,15 @@ CASES = [
     # stride 4 with padding on both sides and channel pruning
     ("stride4_pads_channels", ConvShape(n=2, c=8, h=37, w=41, f=24, kh=7, kw=7, sh=4, sw=4, ph=2, pw=3), 1.0,
      wl.COL_CHANNEL, 0.5),
+    # column stride 3 (does not divide 8): the space-to-depth copy decodes every element
+    ("stride3_generic_copy", ConvShape(n=2, c=3, h=25, w=26, f=16, kh=7, kw=7, sh=3, sw=3, ph=1, pw=2), 1.0,
+     wl.COL_NONE, 1.0),
+    # column stride 8: one input row of 8 columns per chunk
+    ("stride8_one_channel", ConvShape(n=2, c=1, h=67, w=70, f=16, kh=12, kw=12, sh=8, sw=8, ph=3, pw=5), 1.0,
+     wl.COL_NONE, 1.0),
+    # row stride 3, column stride 2: rows (channel, phase) decoded with sh = 3
+    ("rows_sh3_sw2", ConvShape(n=2, c=5, h=29, w=22, f=24, kh=6, kw=5, sh=3, sw=2, ph=2, pw=1), 0.75,
+     wl.COL_NONE, 1.0),
 ]
 
 
@@ -102,7 +111,12 @@ def test_slab_repeated_launches_identical():
     assert np.array_equal(y2.cpu().numpy(), y)
 
 
-@pytest.mark.parametrize("case", [CASES[0], CASES[-1]], ids=lambda c: c[0])
+_BY_NAME = {c[0]: c for c in CASES}
+
+
+@pytest.mark.parametrize("case", [_BY_NAME[n] for n in ("stride4_11x11", "stride4_pads_channels",
+                                                       "stride3_generic_copy", "stride8_one_channel")],
+                         ids=lambda c: c[0])
 def test_slab_input_off_the_16_byte_grid(case):
     """x 2-byte aligned only (a view one element into a buffer, which the ABI
     allows): the output equals the aligned call's bit for bit."""
