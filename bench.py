@@ -256,6 +256,55 @@ class LayerRun:
         return bool(self.plan.xs_mode) and self.colkind != wl.COL_CHANNEL
 
 
+class FirstLayerChunks:
+    """The first layer's forward over n_chunks equal slices of its batch, with a
+    plan of its own for the slice (the same projection lists, packed again for
+    that plan).  Used by the end-to-end step only: the first slice's output can
+    go back to the host while the later slices' inputs still upload, instead of
+    after the whole first input has crossed the link.  Every image's output is
+    the one the whole-batch plan gives."""
+
+    def __init__(self, r, n_chunks, dev, max_ctas=0):
+        import torch
+        from paper_1807_11091_gb300 import sadmm
+        s = r.s
+        assert n_chunks > 1 and s.n % n_chunks == 0
+        self.r = r
+        self.n_chunks = n_chunks
+        self.nb = s.n // n_chunks
+        d16 = s.desc16()
+        d16[0] = self.nb
+        self.desc = sadmm.make_desc(d16)
+        st, self.plan = sadmm.sadmm_plan_init_ctas(self.desc, r.k_filters, r.colkind, r.n_cg, max_ctas)
+        assert st == 0, st
+        self.buf = torch.empty(self.plan.dev_bytes, dtype=torch.uint8, device=dev)
+        self.x_bytes = self.nb * s.c * s.t * s.h * s.w * 2
+        self.y_bytes = self.nb * s.f * s.plane * r.out_bytes
+
+    def pack(self, stream):
+        from paper_1807_11091_gb300 import sadmm
+        r = self.r
+        st = sadmm.sadmm_pack(self.plan, r.W.data_ptr(), sadmm.SADMM_BF16,
+                              r.fi.data_ptr() if r.k_filters < r.s.f else None,
+                              r.ci.data_ptr() if r.colkind != wl.COL_NONE else None,
+                              self.buf.data_ptr(), self.plan.dev_bytes, stream)
+        assert st == 0, st
+
+    def conv(self, stream, j, phase=0):
+        from paper_1807_11091_gb300 import sadmm
+        r = self.r
+        st = sadmm.sadmm_conv_fwd_phase(self.plan, r.x.data_ptr() + j * self.x_bytes, r.bias.data_ptr(), 1,
+                                        r.y.data_ptr() + j * self.y_bytes, r.ydt, phase, stream)
+        assert st == 0, st
+
+    @property
+    def early_input(self):
+        return bool(self.plan.xs_mode) and self.r.colkind != wl.COL_CHANNEL
+
+    def rows(self, j):
+        return slice(j * self.nb, (j + 1) * self.nb)
+
+
 class StepStreams:
     """One side stream per layer: each layer's projection and pack run on its own
     stream (the layers are independent), forked from and joined back to the main
@@ -308,20 +357,22 @@ def enqueue_step(runs, ss, conv_events=None):
             conv_events[i][1].record(ss.main)
 
 
-def enqueue_step_e2e(runs, ss, copy_stream, h_x, h_w, h_b, h_y, up_stream):
+def enqueue_step_e2e(runs, ss, copy_stream, h_x, h_w, h_b, h_y, up_stream, first=None):
     """The step with its host transfers overlapped.  The inputs go host -> device
     on one upload stream, the layers' weights and biases first (small: every
     projection and pack can start), then x layer by layer, so the first conv's
     input arrives at the link's full rate; each output goes device -> host on
     `copy_stream` as soon as its conv has run, while the later inputs still
-    upload (the link carries both directions at once).  The main stream joins
-    the copy stream at the end, so an event recorded after this call covers
-    every copy."""
+    upload (the link carries both directions at once).  With `first` (a
+    FirstLayerChunks) the first layer's input, forward and output go slice by
+    slice, so its first output slice starts back while the rest still uploads.
+    The main stream joins the copy stream at the end, so an event recorded
+    after this call covers every copy."""
     import torch
     from paper_1807_11091_gb300 import sadmm
     ss.fork.record(ss.main)
     up_stream.wait_event(ss.fork)
-    w_ready, x_ready = [], []
+    w_ready, x_ready, xc_ready = [], [], []
     with torch.cuda.stream(up_stream):
         for r, b, c in zip(runs, h_w, h_b):
             r.W.copy_(b, non_blocking=True)
@@ -329,31 +380,56 @@ def enqueue_step_e2e(runs, ss, copy_stream, h_x, h_w, h_b, h_y, up_stream):
             ev = torch.cuda.Event()
             ev.record(up_stream)
             w_ready.append(ev)
-        for r, a in zip(runs, h_x):
+        for i, (r, a) in enumerate(zip(runs, h_x)):
+            if i == 0 and first is not None:
+                for j in range(first.n_chunks):
+                    r.x[first.rows(j)].copy_(a[first.rows(j)], non_blocking=True)
+                    ev = torch.cuda.Event()
+                    ev.record(up_stream)
+                    xc_ready.append(ev)
+                x_ready.append(xc_ready[-1])
+                continue
             r.x.copy_(a, non_blocking=True)
             ev = torch.cuda.Event()
             ev.record(up_stream)
             x_ready.append(ev)
-    for r, side, done, wr in zip(runs, ss.side, ss.done, w_ready):
+    for i, (r, side, done, wr) in enumerate(zip(runs, ss.side, ss.done, w_ready)):
         side.wait_event(wr)
         sp = int(side.cuda_stream)
         r.project(sp)
-        r.pack(sp)
+        (first if i == 0 and first is not None else r).pack(sp)
         done.record(side)
     mp = int(ss.main.cuda_stream)
-    early = runs[0].early_input
-    if early:
-        ss.main.wait_event(x_ready[0])
-        runs[0].conv(mp, sadmm.SADMM_FWD_INPUT)
-    for i, (r, done, hy, xr) in enumerate(zip(runs, ss.done, h_y, x_ready)):
-        ss.main.wait_event(done)
-        ss.main.wait_event(xr)
-        r.conv(mp, sadmm.SADMM_FWD_REST if (i == 0 and early) else sadmm.SADMM_FWD_ALL)
+
+    def copy_back(hy, y):
         ev = torch.cuda.Event()
         ev.record(ss.main)
         copy_stream.wait_event(ev)
         with torch.cuda.stream(copy_stream):
-            hy.copy_(r.y, non_blocking=True)
+            hy.copy_(y, non_blocking=True)
+
+    if first is not None:
+        early = first.early_input
+        for j in range(first.n_chunks):
+            ss.main.wait_event(xc_ready[j])
+            if early:
+                first.conv(mp, j, sadmm.SADMM_FWD_INPUT)
+            if j == 0:
+                ss.main.wait_event(ss.done[0])
+            first.conv(mp, j, sadmm.SADMM_FWD_REST if early else sadmm.SADMM_FWD_ALL)
+            copy_back(h_y[0][first.rows(j)], runs[0].y[first.rows(j)])
+    else:
+        early = runs[0].early_input
+        if early:
+            ss.main.wait_event(x_ready[0])
+            runs[0].conv(mp, sadmm.SADMM_FWD_INPUT)
+    for i, (r, done, hy, xr) in enumerate(zip(runs, ss.done, h_y, x_ready)):
+        if i == 0 and first is not None:
+            continue
+        ss.main.wait_event(done)
+        ss.main.wait_event(xr)
+        r.conv(mp, sadmm.SADMM_FWD_REST if (i == 0 and early) else sadmm.SADMM_FWD_ALL)
+        copy_back(hy, r.y)
     end = torch.cuda.Event()
     end.record(copy_stream)
     ss.main.wait_event(end)
@@ -1053,6 +1129,12 @@ def run_gpu(args):
     d2h = sum(a.numel() * a.element_size() for a in h_y)
     copy_stream = torch.cuda.Stream()
     up_stream = torch.cuda.Stream()
+    # the first layer in slices of its batch (its output is the largest and
+    # the first to go back); the device step's output checks the host's copy
+    nc = args.e2e_chunks
+    first = (FirstLayerChunks(runs[0], nc, dev, first_ctas)
+             if nc > 1 and runs[0].s.n % nc == 0 else None)
+    y_first = runs[0].y.cpu()
     e2e_ms = []
     for _ in range(max(2, min(args.steps, 10))):
         flush.fill_(1)
@@ -1060,13 +1142,17 @@ def run_gpu(args):
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record()
-        enqueue_step_e2e(runs, ss, copy_stream, h_x, h_w, h_b, h_y, up_stream)
+        enqueue_step_e2e(runs, ss, copy_stream, h_x, h_w, h_b, h_y, up_stream, first)
         e1.record()
         torch.cuda.synchronize()
         e2e_ms.append(e0.elapsed_time(e1))
     st = sadmm.sadmm_last_device_status(sp)
     if st != 0:
         raise RuntimeError(f"device status {st} after the timed steps")
+    if not torch.equal(h_y[0], y_first):
+        raise RuntimeError("the end-to-end step's first output differs from the device step's")
+    e2e_slices = first.n_chunks if first is not None else 1
+    del first
 
     # max over ranks of the timed totals
     tot_ms = ranks.max_over_ranks(sum(step_ms), device=dev)
@@ -1122,7 +1208,9 @@ def run_gpu(args):
         "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "transfers": "pinned host buffers; inputs uploaded on one stream (weights and biases first, then "
                              "x layer by layer), each output copied back as soon as its conv has run (overlapped "
-                             "with the later uploads and convs)",
+                             "with the later uploads and convs)" +
+                             (f"; the first layer in {e2e_slices} slices of its batch (a plan for the slice), each "
+                              "slice's output copied back as soon as it is written" if e2e_slices > 1 else ""),
                 "ms_per_step": e2e_med},
         "gpu_launches": sum(r.launches for r in runs) * args.steps,
         "clocks": clocks.summary(),
@@ -1171,6 +1259,8 @@ def main():
     ap.add_argument("--no-admm", action="store_true")
     ap.add_argument("--no-batch1", action="store_true")
     ap.add_argument("--no-backward", action="store_true")
+    ap.add_argument("--e2e-chunks", type=int, default=4,
+                    help="end-to-end step: the first layer's batch in this many slices (1: whole)")
     ap.add_argument("--reserve-sms", type=int, default=4,
                     help="SMs the first conv leaves to the other layers' projection and pack (0: none)")
     args = ap.parse_args()
