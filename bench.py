@@ -301,6 +301,14 @@ class FirstLayerChunks:
     def early_input(self):
         return bool(self.plan.xs_mode) and self.r.colkind != wl.COL_CHANNEL
 
+    @staticmethod
+    def plan_whole_tiles(plan):
+        """Every output tile summed by one CTA in K' order (no split-K, no stream-K)."""
+        return plan.splits == 1 and plan.sk_len == 0
+
+    def whole_tiles(self):
+        return self.plan_whole_tiles(self.plan)
+
     def rows(self, j):
         return slice(j * self.nb, (j + 1) * self.nb)
 
@@ -1134,6 +1142,8 @@ def run_gpu(args):
     nc = args.e2e_chunks
     first = (FirstLayerChunks(runs[0], nc, dev, first_ctas)
              if nc > 1 and runs[0].s.n % nc == 0 else None)
+    if first is not None and not (first.whole_tiles() and FirstLayerChunks.plan_whole_tiles(runs[0].plan)):
+        first = None  # split or stream-K sums: a slice's output need not match the whole batch's bit for bit
     y_first = runs[0].y.cpu()
     e2e_ms = []
     for _ in range(max(2, min(args.steps, 10))):
