@@ -145,3 +145,47 @@ def test_batched_pack_equals_per_layer_packs(dtype):
         x, bias = t["x"].to(dev), t["bias"].to(dev)
         assert torch.equal(a.forward(x, bias), b.forward(x, bias)), L.name
     assert sadmm.device_status() == 0
+
+
+@pytest.mark.parametrize("case", [
+    # input-slab plan (stride 4, kept whole) and a gathered whole-tile plan (shape-wise, grouped)
+    ("slab_stride4", wl.ConvShape(n=8, c=3, h=67, w=67, f=32, kh=11, kw=11, sh=4, sw=4), 1.0, wl.COL_NONE, 1.0),
+    ("gathered_groups", wl.ConvShape(n=8, c=32, h=27, w=27, f=64, kh=5, kw=5, ph=2, pw=2, groups=2), 0.5,
+     wl.COL_SHAPE, 0.5),
+], ids=lambda c: c[0])
+def test_batch_slices_match_the_whole_batch(case):
+    """A plan for a quarter of the batch, run on each quarter of x (the same
+    projection lists), writes each image's output bit for bit as the
+    whole-batch plan does, when both plans sum every tile in one CTA (no split
+    K', no stream-K) -- the property the end-to-end benchmark's sliced first
+    layer relies on."""
+    from paper_1807_11091_gb300 import sadmm
+    name, s, ff, ck, cf = case
+    dev = torch.device("cuda", 0)
+    t = wl.gen_tensors(s, seed=77)
+    kf = wl.retained(ff, s.f)
+    kc = wl.retained(cf, s.k) if ck != wl.COL_NONE else 0
+    W, x, bias = t["W"].to(dev), t["x"].to(dev), t["bias"].to(dev)
+    fi, ci, _ = sadmm.project_groups(s.desc16(), W, kf, ck, kc)
+    ncg = kc if ck != wl.COL_NONE else s.k
+    nb = s.n // 4
+
+    def ctas(n):
+        # a gathered plan on exactly as many CTAs as it has units neither splits K' nor runs stream-K
+        return 0 if name.startswith("slab") else s.groups * -(-(n * s.oh * s.ow) // 128)
+
+    whole = sadmm.PrunedConv(s.desc16(), W, fi if kf < s.f else None, ck, ci if ck != wl.COL_NONE else None, kf, ncg,
+                             max_ctas=ctas(s.n))
+    d16 = s.desc16()
+    d16[0] = nb
+    part = sadmm.PrunedConv(d16, W, fi if kf < s.f else None, ck, ci if ck != wl.COL_NONE else None, kf, ncg,
+                            max_ctas=ctas(nb))
+    for pc in (whole, part):
+        assert pc.plan.splits == 1 and pc.plan.sk_len == 0, name
+    assert whole.plan.xs_mode == part.plan.xs_mode == (1 if name.startswith("slab") else 0)
+    y = whole.forward(x, bias)
+    y4 = torch.full_like(y, float("nan"))
+    for j in range(4):
+        part.forward(x[j * nb:(j + 1) * nb].contiguous(), bias, out=y4[j * nb:(j + 1) * nb])
+    assert sadmm.device_status() == sadmm.SADMM_OK
+    assert torch.equal(y, y4), name
