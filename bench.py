@@ -552,10 +552,24 @@ def conv_traffic(workload, out_dtype):
         return None
 
 
-def time_steps(rs, ss, flush, k, with_conv_events):
+def capture_step(rs, ss):
+    """The step of the layers `rs` captured once (after warm-up) into a CUDA
+    graph: the same launches, streams' dependencies and programmatic launches,
+    replayed with one graph launch per step instead of one host call per
+    kernel."""
+    import torch
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=ss.main):
+        enqueue_step(rs, ss)
+    torch.cuda.synchronize()
+    return g
+
+
+def time_steps(rs, ss, flush, k, with_conv_events, graph=None):
     """k steps of the layers `rs`, L2 flushed before each (outside the window):
     the step times (ms) and, with events around each forward call, the per-call
-    times."""
+    times.  With `graph` (capture_step) each step without per-call events is
+    one replay of it."""
     import torch
     step_ms, conv_ms = [], [[] for _ in rs]
     for _ in range(k):
@@ -566,7 +580,10 @@ def time_steps(rs, ss, flush, k, with_conv_events):
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record()
-        enqueue_step(rs, ss, ev)
+        if graph is not None and not with_conv_events:
+            graph.replay()
+        else:
+            enqueue_step(rs, ss, ev)
         e1.record()
         torch.cuda.synchronize()
         step_ms.append(e0.elapsed_time(e1))
@@ -633,7 +650,7 @@ WORKLOAD_LABELS = {
 }
 
 
-def configs_report(dev, out_dtype, peaks, steps=10, names=("c3d", "resnet50", "single2d")):
+def configs_report(dev, out_dtype, peaks, steps=10, names=("c3d", "resnet50", "single2d"), graphs=True):
     """The other workloads through the same step as the headline line
     (projection + pack + forward of every layer, L2 flushed before each step):
     TFLOP/s on retained MACs, the forward calls' roofline (whichever of HBM and
@@ -652,10 +669,13 @@ def configs_report(dev, out_dtype, peaks, steps=10, names=("c3d", "resnet50", "s
             enqueue_step(runs, ss)
             enqueue_step(dense, ss)
         torch.cuda.synchronize()
-        step_ms, _ = time_steps(runs, ss, flush, steps, False)
+        g_runs = capture_step(runs, ss) if graphs else None
+        g_dense = capture_step(dense, ss) if graphs else None
+        step_ms, _ = time_steps(runs, ss, flush, steps, False, g_runs)
         _, conv_ms = time_steps(runs, ss, flush, steps, True)
-        dense_ms, _ = time_steps(dense, ss, flush, steps, False)
+        dense_ms, _ = time_steps(dense, ss, flush, steps, False, g_dense)
         _, dconv_ms = time_steps(dense, ss, flush, steps, True)
+        del g_runs, g_dense
         from paper_1807_11091_gb300 import sadmm
         if sadmm.sadmm_last_device_status(int(torch.cuda.current_stream().cuda_stream)) != 0:
             raise RuntimeError(f"device status set after the {name} steps")
@@ -1088,8 +1108,10 @@ def run_gpu(args):
     ss = StepStreams(len(runs))
     peaks, peak_src = load_peaks()
 
+    graphs = {}
+
     def timed_steps(rs, k, with_conv_events):
-        return time_steps(rs, ss, flush, k, with_conv_events)
+        return time_steps(rs, ss, flush, k, with_conv_events, graphs.get(id(rs)))
 
     # warm-up (also the first-call setup of every kernel)
     for _ in range(max(args.warmup, 3)):
@@ -1099,6 +1121,10 @@ def run_gpu(args):
     st = sadmm.sadmm_last_device_status(sp)
     if st != 0:
         raise RuntimeError(f"device status {st} after warm-up")
+    if not args.eager:
+        # each step one replay of the step captured here (the per-call breakdown stays eager)
+        graphs[id(runs)] = capture_step(runs, ss)
+        graphs[id(dense)] = capture_step(dense, ss)
 
     log_dir = args.log_dir if os.path.isabs(args.log_dir) else os.path.join(ROOT, args.log_dir)
     os.makedirs(log_dir, exist_ok=True)
@@ -1207,7 +1233,11 @@ def run_gpu(args):
                    "schedule": f"projection+pack of each layer on its own stream; convs back to back on the "
                                f"main stream (high priority); first conv on {first_ctas or n_sm} of {n_sm} SMs, its input-slab "
                                f"space-to-depth pass issued at the step's start beside the projections and packs",
-                   "breakdown": "per-conv times from separate steps with CUDA events around each whole forward call"},
+                   "launch": ("eager: one host call per kernel" if args.eager else
+                              "the step (every projection, pack and forward call and their streams) captured once "
+                              "after warm-up into a CUDA graph, one replay per timed step"),
+                   "breakdown": "per-conv times from separate eager steps with CUDA events around each whole "
+                                "forward call"},
         "pct_bf16_peak": value / peaks["bf16_tflops"],
         "speedup_vs_dense": dense_step / pruned_step_med,
         "conv_speedup_vs_dense": sum(dense_conv_avg) / sum(conv_avg),
@@ -1228,7 +1258,7 @@ def run_gpu(args):
     if calls is not None:
         line["calls"] = calls
     if rank == 0 and not args.no_configs and args.workload == "alexnet":
-        line["configs"] = configs_report(dev, args.out_dtype, peaks)
+        line["configs"] = configs_report(dev, args.out_dtype, peaks, graphs=not args.eager)
     if rank == 0 and not args.no_sweep:
         line["sweep"] = sweep_report(dev, args.out_dtype, peak_tflops=peaks["bf16_tflops"])
         if not args.no_sparse:
@@ -1269,6 +1299,8 @@ def main():
     ap.add_argument("--no-admm", action="store_true")
     ap.add_argument("--no-batch1", action="store_true")
     ap.add_argument("--no-backward", action="store_true")
+    ap.add_argument("--eager", action="store_true",
+                    help="time each step as host calls per kernel instead of replaying the step's CUDA graph")
     ap.add_argument("--e2e-chunks", type=int, default=4,
                     help="end-to-end step: the first layer's batch in this many slices (1: whole)")
     ap.add_argument("--reserve-sms", type=int, default=4,
